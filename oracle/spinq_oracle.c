@@ -1,0 +1,422 @@
+/*
+ * spinq_oracle.c -- plain, slow, double-precision CPU oracle for the rotated
+ * W4A4 hot path of SpinQuant (arXiv 2405.16406).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline / reference leg of bench.py may load this library.  It shares
+ * no code, header, table or constant with the CUDA library under
+ * paper_2405_16406_gb300/csrc, and the CUDA library never calls it.
+ *
+ * Every function computes the plain definition of what it names, in double,
+ * with no blocking, fusion or reordering beyond what that definition states.
+ * Rows are independent; OpenMP only splits independent rows across cores.
+ *
+ * Paper passages followed (section / equation of the paper):
+ *   - Eq. 1 (Sec. 2): min-max round-to-nearest quantizer, symmetric and
+ *     asymmetric forms, N bits.
+ *   - Sec. 2.2 footnote: a Hadamard matrix is a rotation whose entries all
+ *     share one magnitude; read here as R = H / sqrt(n) with H in {+1,-1}.
+ *   - Sec. 3.1 ("Additional unabsorbed rotations"): R4 is an online Hadamard
+ *     on the down_proj input, R3 an online Hadamard on Q/K over head_dim,
+ *     both computed with a fast Hadamard transform.
+ *   - Sec. 3.1 ("Rotating activations in residual"): rotational invariance,
+ *     x R (W R)^T = x W^T for orthonormal R, which fixes how a rotated weight
+ *     is merged (W' = W R).
+ *   - Appendix "Quantization choice": clipping ratio of the min-max range;
+ *     asymmetric quantization for activations and the KV cache.
+ *
+ * Readings where the paper is silent (each also listed in the design doc):
+ *   - Sylvester H_{2^k}[i][j] = (-1)^popcount(i & j) (natural order).
+ *   - Paley I for a prime power q = 3 mod 4, order q + 1: H = I + S with
+ *     S = [[0, 1^T], [-1, Q]], Q[i][j] = chi(a_i - a_j), chi the quadratic
+ *     character.  GF(p) for prime q (a_i = i); GF(27) = GF(3)[t]/(t^3+2t+1)
+ *     with a_i = c0 + c1 t + c2 t^2 for i = c0 + 3 c1 + 9 c2.
+ *   - Non-power-of-two sizes K = n_s * P use H_s (x) H_P with the small
+ *     factor on the slow index: k = i * P + j.  The rotation is the row-vector
+ *     product y = x (H_s (x) H_P) / sqrt(K).
+ *   - Rounding is round-half-to-even (nearbyint in the default mode).
+ *   - Symmetric codes clamp to [-2^(N-1), 2^(N-1)-1]; asymmetric to
+ *     [0, 2^N - 1]; a zero range gives alpha = 0 and all codes 0.
+ *   - Clipping scales max|x| (symmetric) or both min and max (asymmetric).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define OR_OK 0
+#define OR_EINVAL 1
+
+/* ------------------------------------------------------------------ */
+/* threads                                                             */
+/* ------------------------------------------------------------------ */
+int oracle_set_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+  return omp_get_max_threads();
+#else
+  (void)n;
+  return 1;
+#endif
+}
+
+/* ------------------------------------------------------------------ */
+/* IEEE 754 binary16 <-> double, written from the format definition    */
+/* ------------------------------------------------------------------ */
+double oracle_f16_to_double(uint16_t h) {
+  int s = (h >> 15) & 1, e = (h >> 10) & 0x1f, m = h & 0x3ff;
+  double v;
+  if (e == 0)
+    v = ldexp((double)m, -24); /* subnormal: m * 2^-24 */
+  else if (e == 31)
+    v = m ? NAN : INFINITY;
+  else
+    v = ldexp((double)(m + 1024), e - 25); /* (1 + m/1024) 2^(e-15) */
+  return s ? -v : v;
+}
+
+/* Round-to-nearest-even from double. */
+uint16_t oracle_double_to_f16(double d) {
+  uint16_t sign = signbit(d) ? 0x8000 : 0;
+  double a = fabs(d);
+  if (isnan(d)) return 0x7e00;
+  if (a >= 65520.0) return sign | 0x7c00; /* halfway to 2^16 and above -> inf */
+  if (a < ldexp(1.0, -14)) {
+    double q = nearbyint(ldexp(a, 24)); /* subnormal quantum 2^-24; q <= 1024 */
+    return sign | (uint16_t)q;
+  }
+  int e;
+  double f = frexp(a, &e);          /* a = f 2^e, f in [0.5, 1) */
+  double q = nearbyint(ldexp(f, 11)); /* significand with hidden bit, [1024, 2048] */
+  int E = e + 14;                   /* biased exponent */
+  if (q == 2048.0) {
+    q = 1024.0;
+    E += 1;
+  }
+  if (E >= 31) return sign | 0x7c00;
+  return (uint16_t)(sign | (E << 10) | ((int)q - 1024));
+}
+
+void oracle_f16_array_to_double(const uint16_t* h, double* d, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) d[i] = oracle_f16_to_double(h[i]);
+}
+
+void oracle_double_array_to_f16(const double* d, uint16_t* h, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) h[i] = oracle_double_to_f16(d[i]);
+}
+
+/* ------------------------------------------------------------------ */
+/* Hadamard constructions (Sec. 2.2 footnote; Sec. 3.1 R3/R4)           */
+/* ------------------------------------------------------------------ */
+static int is_pow2(int64_t n) { return n > 0 && (n & (n - 1)) == 0; }
+
+static int popcount_u64(uint64_t x) {
+  int c = 0;
+  while (x) {
+    c += (int)(x & 1u);
+    x >>= 1;
+  }
+  return c;
+}
+
+/* Sylvester: H_1 = [1], H_2n = [[H, H], [H, -H]], i.e. (-1)^popcount(i&j). */
+int oracle_sylvester(int64_t n, int8_t* H) {
+  if (!is_pow2(n)) return OR_EINVAL;
+  for (int64_t i = 0; i < n; ++i)
+    for (int64_t j = 0; j < n; ++j)
+      H[i * n + j] = (popcount_u64((uint64_t)(i & j)) & 1) ? -1 : 1;
+  return OR_OK;
+}
+
+/* GF(q) arithmetic for the Paley construction.  q prime: integers mod q.
+ * q = 27: polynomials over GF(3) modulo t^3 + 2t + 1, element index
+ * c0 + 3 c1 + 9 c2 for c0 + c1 t + c2 t^2.                              */
+static int gf_sub(int q, int a, int b) {
+  if (q != 27) return ((a - b) % q + q) % q;
+  int r = 0, p = 1;
+  for (int d = 0; d < 3; ++d) {
+    int da = a % 3, db = b % 3;
+    r += (((da - db) % 3 + 3) % 3) * p;
+    a /= 3;
+    b /= 3;
+    p *= 3;
+  }
+  return r;
+}
+
+static int gf_mul(int q, int a, int b) {
+  if (q != 27) return (a * b) % q;
+  int ca[3], cb[3], prod[5] = {0, 0, 0, 0, 0};
+  for (int d = 0; d < 3; ++d) {
+    ca[d] = a % 3;
+    cb[d] = b % 3;
+    a /= 3;
+    b /= 3;
+  }
+  for (int i = 0; i < 3; ++i)
+    for (int j = 0; j < 3; ++j) prod[i + j] += ca[i] * cb[j];
+  /* reduce degrees 4 and 3 with t^3 = -2t - 1 = t + 2 (mod 3) */
+  for (int d = 4; d >= 3; --d) {
+    int c = prod[d] % 3;
+    prod[d] = 0;
+    prod[d - 3 + 1] += c;     /* c * t^(d-3) * t   */
+    prod[d - 3] += 2 * c;     /* c * t^(d-3) * 2   */
+  }
+  return (prod[0] % 3) + 3 * (prod[1] % 3) + 9 * (prod[2] % 3);
+}
+
+/* quadratic character: a^((q-1)/2) is 1 for a nonzero square, -1 otherwise */
+static int gf_chi(int q, int a) {
+  if (a == 0) return 0;
+  int r = 1;
+  for (int e = 0; e < (q - 1) / 2; ++e) r = gf_mul(q, r, a);
+  if (r == 1) return 1;
+  /* -1 is q-1 for prime q and the constant 2 (index 2) in GF(27) */
+  if ((q != 27 && r == q - 1) || (q == 27 && r == 2)) return -1;
+  return -2; /* not a field: caller treats as error */
+}
+
+static int paley_q_supported(int q) {
+  if (q == 27) return 1;
+  if (q < 3 || q % 4 != 3) return 0;
+  for (int d = 2; d * d <= q; ++d)
+    if (q % d == 0) return 0;
+  return 1;
+}
+
+/* Paley I of order q + 1 (q = 3 mod 4 a prime power): H = I + S. */
+int oracle_paley1(int q, int8_t* H) {
+  if (!paley_q_supported(q)) return OR_EINVAL;
+  int n = q + 1;
+  for (int r = 0; r < n; ++r)
+    for (int c = 0; c < n; ++c) {
+      int s;
+      if (r == 0 && c == 0)
+        s = 0;
+      else if (r == 0)
+        s = 1;
+      else if (c == 0)
+        s = -1;
+      else {
+        s = gf_chi(q, gf_sub(q, r - 1, c - 1));
+        if (s == -2) return OR_EINVAL;
+      }
+      H[r * n + c] = (int8_t)((r == c ? 1 : 0) + s);
+    }
+  return OR_OK;
+}
+
+/* The small Kronecker factor H_s of order n_s: [1] for n_s = 1, Paley I of
+ * order n_s otherwise (n_s - 1 a supported prime power).                 */
+int oracle_small_hadamard(int n_s, int8_t* H) {
+  if (n_s == 1) {
+    H[0] = 1;
+    return OR_OK;
+  }
+  return oracle_paley1(n_s - 1, H);
+}
+
+/* ------------------------------------------------------------------ */
+/* Rotation y = x (H_s (x) H_P) / sqrt(K)   (Sec. 3.1, R3 and R4)      */
+/* ------------------------------------------------------------------ */
+
+/* In-place fast Walsh-Hadamard transform, natural order: v <- H_n v.  H_n
+ * (Sylvester) is symmetric, so this is also the row-vector product v H_n. */
+void oracle_fwht(double* v, int64_t n) {
+  for (int64_t h = 1; h < n; h <<= 1)
+    for (int64_t i = 0; i < n; i += 2 * h)
+      for (int64_t j = i; j < i + h; ++j) {
+        double a = v[j], b = v[j + h];
+        v[j] = a + b;
+        v[j + h] = a - b;
+      }
+}
+
+/* rows x K, K = n_s * n_pow2. */
+int oracle_rotate(const double* x, double* y, int64_t rows, int n_s, int64_t n_pow2) {
+  if (!is_pow2(n_pow2) || n_s < 1) return OR_EINVAL;
+  int8_t* Hs = (int8_t*)malloc((size_t)n_s * n_s);
+  if (!Hs) return OR_EINVAL;
+  if (oracle_small_hadamard(n_s, Hs) != OR_OK) {
+    free(Hs);
+    return OR_EINVAL;
+  }
+  const int64_t P = n_pow2, K = (int64_t)n_s * P;
+  const double inv = 1.0 / sqrt((double)K);
+  int err = 0;
+#pragma omp parallel
+  {
+    double* t = (double*)malloc(sizeof(double) * (size_t)K);
+    if (!t) {
+#pragma omp atomic write
+      err = 1;
+    }
+#pragma omp for schedule(static)
+    for (int64_t r = 0; r < rows; ++r) {
+      if (!t) continue;
+      const double* xr = x + r * K;
+      double* yr = y + r * K;
+      memcpy(t, xr, sizeof(double) * (size_t)K);
+      /* X[i][:] <- X[i][:] H_P for every slow index i */
+      for (int i = 0; i < n_s; ++i) oracle_fwht(t + (int64_t)i * P, P);
+      /* Y[i][j] = sum_i' X[i'][j] H_s[i'][i]  (row vector times H_s) */
+      for (int64_t j = 0; j < P; ++j)
+        for (int i = 0; i < n_s; ++i) {
+          double acc = 0.0;
+          for (int ip = 0; ip < n_s; ++ip) acc += t[(int64_t)ip * P + j] * (double)Hs[ip * n_s + i];
+          yr[(int64_t)i * P + j] = acc * inv;
+        }
+    }
+    free(t);
+  }
+  free(Hs);
+  return err ? OR_EINVAL : OR_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* Eq. 1 quantizer, per row (token / output channel / group)           */
+/* ------------------------------------------------------------------ */
+/* x: rows x K; each row is quantized with its own (alpha, beta).
+ * symmetric : alpha = clip max|x| / (2^(N-1) - 1), beta = 0,
+ *             q = clamp(rint(x / alpha), -2^(N-1), 2^(N-1) - 1)
+ * asymmetric: alpha = clip (max x - min x) / (2^N - 1), beta = clip min x,
+ *             u = clamp(rint((x - beta) / alpha), 0, 2^N - 1)
+ * Dequantized value is alpha * code + beta (Eq. 1).                     */
+int oracle_quantize_rows(const double* x, int64_t rows, int64_t K, int bits, int symmetric,
+                         double clip, int32_t* codes, double* alpha, double* beta) {
+  if (bits < 2 || bits > 8 || K <= 0 || !(clip > 0.0 && clip <= 1.0)) return OR_EINVAL;
+  const double smax = (double)((1 << (bits - 1)) - 1), smin = -(double)(1 << (bits - 1));
+  const double amax = (double)((1 << bits) - 1);
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < rows; ++r) {
+    const double* xr = x + r * K;
+    int32_t* cr = codes + r * K;
+    double a, b;
+    if (symmetric) {
+      double m = 0.0;
+      for (int64_t k = 0; k < K; ++k) m = fmax(m, fabs(xr[k]));
+      a = clip * m / smax;
+      b = 0.0;
+      for (int64_t k = 0; k < K; ++k) {
+        double q = a > 0.0 ? nearbyint(xr[k] / a) : 0.0;
+        cr[k] = (int32_t)fmin(fmax(q, smin), smax);
+      }
+    } else {
+      double hi = xr[0], lo = xr[0];
+      for (int64_t k = 1; k < K; ++k) {
+        hi = fmax(hi, xr[k]);
+        lo = fmin(lo, xr[k]);
+      }
+      hi *= clip;
+      lo *= clip;
+      a = (hi - lo) / amax;
+      b = lo;
+      for (int64_t k = 0; k < K; ++k) {
+        double u = a > 0.0 ? nearbyint((xr[k] - b) / a) : 0.0;
+        cr[k] = (int32_t)fmin(fmax(u, 0.0), amax);
+      }
+    }
+    alpha[r] = a;
+    beta[r] = b;
+  }
+  return OR_OK;
+}
+
+/* Dequantize codes back to reals: x_Q = alpha * code + beta (Eq. 1). */
+void oracle_dequantize_rows(const int32_t* codes, const double* alpha, const double* beta,
+                            int64_t rows, int64_t K, double* xq) {
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t k = 0; k < K; ++k)
+      xq[r * K + k] = alpha[r] * (double)codes[r * K + k] + (beta ? beta[r] : 0.0);
+}
+
+/* ------------------------------------------------------------------ */
+/* 4-bit packing: two codes per byte, even index in the low nibble.     */
+/* Signed codes are stored as two's complement nibbles.                 */
+/* ------------------------------------------------------------------ */
+void oracle_pack4(const int32_t* codes, int64_t n, uint8_t* packed) {
+  for (int64_t i = 0; i < n / 2; ++i)
+    packed[i] = (uint8_t)((codes[2 * i] & 0xF) | ((codes[2 * i + 1] & 0xF) << 4));
+}
+
+void oracle_unpack4(const uint8_t* packed, int64_t n, int is_signed, int32_t* codes) {
+  for (int64_t i = 0; i < n; ++i) {
+    int v = (packed[i / 2] >> (4 * (i & 1))) & 0xF;
+    if (is_signed && v >= 8) v -= 16;
+    codes[i] = v;
+  }
+}
+
+/* ------------------------------------------------------------------ */
+/* W4A4 linear: integer accumulator and dequantized output              */
+/* ------------------------------------------------------------------ */
+/* a_codes: M x K stored activation codes (q for symmetric, u for asymmetric)
+ * w_codes: N x K symmetric weight codes q_w.
+ * acc[m][n] = sum_k a_int * q_w with a_int = q (symmetric) or u - 2^(N-1)
+ *             (asymmetric, the zero-centred code); checked to fit int32.
+ * y[m][n]   = sum_k (alpha_m c_mk + beta_m) (s_n q_w,nk), the plain
+ *             dequantized product (Eq. 1 applied to both operands).       */
+static int gemm_one(const int32_t* a, const int32_t* w, int64_t K, int sym, double am, double bm,
+                    double sn, int32_t* acc_out, double* y_out) {
+  int64_t acc = 0;
+  double y = 0.0;
+  for (int64_t k = 0; k < K; ++k) {
+    const int64_t ai = sym ? a[k] : (int64_t)a[k] - 8;
+    acc += ai * (int64_t)w[k];
+    y += (am * (double)a[k] + bm) * (sn * (double)w[k]);
+  }
+  if (acc > INT32_MAX || acc < INT32_MIN) return OR_EINVAL;
+  *acc_out = (int32_t)acc;
+  *y_out = y;
+  return OR_OK;
+}
+
+int oracle_w4a4_gemm(const int32_t* a_codes, const double* a_scale, const double* a_zero,
+                     const int32_t* w_codes, const double* w_scale, int64_t M, int64_t N, int64_t K,
+                     int32_t* acc, double* y) {
+  const int sym = a_zero == NULL;
+  int err = 0;
+#pragma omp parallel for schedule(static) collapse(2)
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n) {
+      int e = gemm_one(a_codes + m * K, w_codes + n * K, K, sym, a_scale[m], sym ? 0.0 : a_zero[m],
+                       w_scale[n], acc + m * N + n, y + m * N + n);
+      if (e) {
+#pragma omp atomic write
+        err = 1;
+      }
+    }
+  return err ? OR_EINVAL : OR_OK;
+}
+
+/* Same definition at an explicit list of (m, n) output coordinates. */
+int oracle_w4a4_gemm_sampled(const int32_t* a_codes, const double* a_scale, const double* a_zero,
+                             const int32_t* w_codes, const double* w_scale, int64_t K,
+                             const int64_t* ms, const int64_t* ns, int64_t count, int32_t* acc,
+                             double* y) {
+  const int sym = a_zero == NULL;
+  int err = 0;
+#pragma omp parallel for schedule(static)
+  for (int64_t i = 0; i < count; ++i) {
+    const int64_t m = ms[i], n = ns[i];
+    int e = gemm_one(a_codes + m * K, w_codes + n * K, K, sym, a_scale[m], sym ? 0.0 : a_zero[m],
+                     w_scale[n], acc + i, y + i);
+    if (e) {
+#pragma omp atomic write
+      err = 1;
+    }
+  }
+  return err ? OR_EINVAL : OR_OK;
+}
+
+/* Integer row sums of codes: rowsum[r] = sum_k codes[r][k]. */
+void oracle_rowsum(const int32_t* codes, int64_t rows, int64_t K, int32_t* rowsum) {
+  for (int64_t r = 0; r < rows; ++r) {
+    int64_t s = 0;
+    for (int64_t k = 0; k < K; ++k) s += codes[r * K + k];
+    rowsum[r] = (int32_t)s;
+  }
+}
