@@ -1,0 +1,409 @@
+"""Benchmark of the rotated W4A4 hot path on GB300 (one JSON line on rank 0).
+
+A step is one pass of the hot path over one batch of 2048 tokens of a
+LLaMA-3-8B layer (synthetic inputs):
+  * R3 + KV4: spinq_rotate_quant_kv on Q/K/V of the 2048 tokens
+    (32 query heads, 8 KV heads, head_dim 128);
+  * act quant: spinq_rotate_quant_act on x [2048 x 4096] (gate/up input,
+    R1 merged so no online rotation, asymmetric per-token int4);
+  * W4A4 GEMM: spinq_w4a4_gemm, 2048 x 4096 -> 14336 (gate/up projection).
+The weight quantization (spinq_quant_weight) is offline and runs once before
+timing.  `value` counts the GEMM's 2*M*N*K integer ops per step over the whole
+step time.  Inputs rotate over 4 independent sets (4 layers' weights and
+activations, ~284 MB, larger than the 129 MB L2), so every step reads cold
+data.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (torchrun, one rank per GPU) every rank runs its own replica on its
+own tokens: the path shards by tokens with no collective ("replicas only").
+`--impl reference` times the CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "W4A4 rotated-linear TOPS and rotate+quant HBM GB/s (% of GB300 peak)"
+M, K, N = 2048, 4096, 14336
+B_KV, S_KV, HQ, HKV, D = 1, 2048, 32, 8, 128
+NSETS = 4
+# Measured GB300 peaks (generated MEASURED_PEAKS.json; fallbacks if absent)
+FALLBACK_HBM, FALLBACK_BF16 = 6800.0, 1900.0
+
+
+def peaks():
+    try:
+        p = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return FALLBACK_HBM, FALLBACK_BF16, "fallback"
+
+
+def step_bytes_rq():
+    # act quant: read fp16 x, write packed codes + alpha + beta
+    return M * K * 2 + M * K // 2 + 8 * M
+
+
+def step_bytes_kv():
+    rq, rkv = B_KV * S_KV * HQ, B_KV * S_KV * HKV
+    return rq * D * 4 + 2 * rkv * (D * 2 + D // 2 + 8)
+
+
+def gemm_ops():
+    return 2.0 * M * N * K
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while work runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev_index: int):
+        self.dev = dev_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[3:7]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------------------- ours
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2405_16406_gb300 import spinq
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    hbm_peak, bf16_peak, peak_kind = peaks()
+    fp8_peak = 2.0 * bf16_peak  # nominal e4m3 : bf16 dense ratio on GB300 is 2
+
+    g = torch.Generator(device=dev)
+    g.manual_seed(1000 + rank)
+
+    def acts(rows, cols, frac, factor):
+        x = torch.randn(rows, cols, generator=g, device=dev)
+        cols_idx = torch.randperm(cols, generator=g, device=dev)[: max(1, int(round(frac * cols)))]
+        x[:, cols_idx] *= factor
+        return x.half()
+
+    sets = []
+    for _ in range(NSETS):
+        x = acts(M, K, 0.01, 30.0)
+        w = (torch.randn(N, K, generator=g, device=dev) * 0.02).half()
+        qw = spinq.quant_weight(w, None)                       # offline, not timed
+        del w
+        q = torch.randn(B_KV, S_KV, HQ, D, generator=g, device=dev).half()
+        k = torch.randn(B_KV, S_KV, HKV, D, generator=g, device=dev).half()
+        v = torch.randn(B_KV, S_KV, HKV, D, generator=g, device=dev).half()
+        sets.append((x, qw, q, k, v))
+    qa_out = [spinq.ActCodes(torch.empty(M, K // 2, dtype=torch.uint8, device=dev),
+                             torch.empty(M, dtype=torch.float32, device=dev),
+                             torch.empty(M, dtype=torch.float32, device=dev)) for _ in range(NSETS)]
+    ys = [torch.empty(M, N, dtype=torch.float16, device=dev) for _ in range(NSETS)]
+    kv_out = [None] * NSETS
+    torch.cuda.synchronize()
+
+    n_ev = args.steps
+    ev = {k2: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(n_ev)] for k2 in ("kv", "rq", "gemm")}
+
+    def step(i, record=None):
+        x, qw, q, k, v = sets[i % NSETS]
+        j = i % NSETS
+        if record is not None:
+            ev["kv"][record][0].record(stream)
+        kv_out[j] = spinq.rotate_quant_kv(q, k, v, out=kv_out[j])
+        if record is not None:
+            ev["kv"][record][1].record(stream)
+            ev["rq"][record][0].record(stream)
+        spinq.rotate_quant_act(x, None, False, 1.0, out=qa_out[j])
+        if record is not None:
+            ev["rq"][record][1].record(stream)
+            ev["gemm"][record][0].record(stream)
+        spinq.w4a4_gemm(qa_out[j], qw, y=ys[j])
+        if record is not None:
+            ev["gemm"][record][1].record(stream)
+
+    for i in range(max(args.warmup, 3)):
+        step(i)
+    torch.cuda.synchronize()
+
+    # sustain ~1.5 s so the clock samples cover steady state, ending in the timed region
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    t_end = time.time() + 1.5
+    i = 0
+    while time.time() < t_end:
+        for _ in range(20):
+            step(i)
+            i += 1
+        torch.cuda.synchronize()
+
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for s in range(args.steps):
+        step(s, record=s)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    ms = t0.elapsed_time(t1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    def avg(key):
+        return statistics.mean(a.elapsed_time(b) for a, b in ev[key]) / 1e3  # seconds
+
+    t_gemm, t_rq, t_kv = avg("gemm"), avg("rq"), avg("kv")
+    gemm_tops = gemm_ops() / t_gemm / 1e12
+
+    # ---- end to end through the public API with host buffers
+    x_h = [sets[j][0].cpu().pin_memory() for j in range(NSETS)]
+    qkv_h = [tuple(t.cpu().pin_memory() for t in sets[j][2:]) for j in range(NSETS)]
+    y_h = torch.empty(M, N, dtype=torch.float16).pin_memory()
+    qo_h = torch.empty(B_KV, S_KV, HQ, D, dtype=torch.float16).pin_memory()
+    kc_h = torch.empty(B_KV, S_KV, HKV, D // 2, dtype=torch.uint8).pin_memory()
+    vc_h = torch.empty_like(kc_h).pin_memory()
+    sc_h = [torch.empty(B_KV, S_KV, HKV, dtype=torch.float32).pin_memory() for _ in range(4)]
+    x_d = torch.empty(M, K, dtype=torch.float16, device=dev)
+    q_d = torch.empty(B_KV, S_KV, HQ, D, dtype=torch.float16, device=dev)
+    k_d = torch.empty(B_KV, S_KV, HKV, D, dtype=torch.float16, device=dev)
+    v_d = torch.empty_like(k_d)
+
+    def e2e_step(i):
+        j = i % NSETS
+        x_d.copy_(x_h[j], non_blocking=True)
+        q_d.copy_(qkv_h[j][0], non_blocking=True)
+        k_d.copy_(qkv_h[j][1], non_blocking=True)
+        v_d.copy_(qkv_h[j][2], non_blocking=True)
+        o = spinq.rotate_quant_kv(q_d, k_d, v_d, out=kv_out[j])
+        spinq.rotate_quant_act(x_d, None, False, 1.0, out=qa_out[j])
+        spinq.w4a4_gemm(qa_out[j], sets[j][1], y=ys[j])
+        y_h.copy_(ys[j], non_blocking=True)
+        qo_h.copy_(o.q_out, non_blocking=True)
+        kc_h.copy_(o.k_codes, non_blocking=True)
+        vc_h.copy_(o.v_codes, non_blocking=True)
+        for dst, src in zip(sc_h, (o.k_scale, o.k_zero, o.v_scale, o.v_zero)):
+            dst.copy_(src, non_blocking=True)
+
+    for i in range(3):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.steps):
+        e2e_step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms_e2e = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms_e2e], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_e2e = float(t.item())
+    h2d = (M * K + B_KV * S_KV * (HQ + 2 * HKV) * D) * 2
+    d2h = M * N * 2 + B_KV * S_KV * HQ * D * 2 + 2 * B_KV * S_KV * HKV * D // 2 + B_KV * S_KV * HKV * 16
+
+    st, _ = spinq.spinq_device_status()
+    if st != spinq.SPINQ_OK:
+        raise RuntimeError(f"device status after bench: {spinq.spinq_status_string(st)}")
+
+    if rank != 0:
+        return None
+    value = world * gemm_ops() / (ms / 1e3) / 1e12
+    rq_gbs = step_bytes_rq() / t_rq / 1e9
+    kv_gbs = step_bytes_kv() / t_kv / 1e9
+    out = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "TOPS",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int4",
+        "data": "synthetic",
+        "config": {
+            "workload": "llama3_8b_gate_up_M2048_K4096_N14336 + R3/KV4 for the same 2048 tokens "
+                        "(32 q heads, 8 kv heads, head_dim 128)",
+            "M": M, "K": K, "N": N, "act_quant": "asymmetric per-token int4, no online rotation",
+            "weights": "symmetric per-channel int4 (quantized once, not timed)",
+            "l2": f"{NSETS} rotating input sets (~284 MB) > 129 MB L2",
+            "parallelism": f"replicas{world}",
+        },
+        "roofline": {
+            "bound": "tensor", "kernel": "w4a4_gemm_kernel",
+            "achieved": round(gemm_tops, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
+            "frac": round(gemm_tops / fp8_peak, 4), "traffic": None,
+            "peak_note": f"e4m3 dense = 2 x {peak_kind} bf16 ({bf16_peak} TFLOP/s); "
+                         "int4 codes carried as e4m3 on tcgen05 kind::f8f6f4",
+        },
+        "rotate_quant_roofline": {
+            "bound": "hbm", "kernel": "rotate_quant_rows_kernel (act, K=4096)",
+            "achieved": round(rq_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+            "frac": round(rq_gbs / hbm_peak, 4), "us": round(t_rq * 1e6, 2),
+        },
+        "kv_roofline": {
+            "bound": "hbm", "kernel": "rotate_quant_kv_kernel",
+            "achieved": round(kv_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+            "frac": round(kv_gbs / hbm_peak, 4), "us": round(t_kv * 1e6, 2),
+        },
+        "kernel_us": {"gemm": round(t_gemm * 1e6, 2), "act_quant": round(t_rq * 1e6, 2),
+                      "kv_quant": round(t_kv * 1e6, 2)},
+        "e2e": {"value": round(world * gemm_ops() / (ms_e2e / 1e3) / 1e12, 2), "unit": "TOPS",
+                "ms_per_step": round(ms_e2e, 4), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(sample_rows=args.cpu_rows)
+    return out
+
+
+# --------------------------------------------------------------------------- oracle on host cores
+def cpu_baseline(sample_rows=1024, threads=0):
+    """Time the oracle (as it stands) on a bounded sample of the same workload:
+    `sample_rows` tokens through act quant + GEMM (+ their KV rows)."""
+    import numpy as np
+
+    import oracle
+    from paper_2405_16406_gb300 import synth
+    cores = oracle.set_threads(threads)
+    rng = np.random.default_rng(0)
+    x = synth.activations(rng, sample_rows, K, outlier_frac=0.01, factor=30.0)
+    w = synth.weights(rng, N, K)
+    qw = oracle.quant_weight(w, None)       # offline, not timed
+    kv = synth.kv_case(seed=1, B=1, S=sample_rows, Hq=HQ, Hkv=HKV, D=D)
+    t0 = time.perf_counter()
+    oracle.rotate_quant_kv(kv.q, kv.k, kv.v, kv.had)
+    qa = oracle.rotate_quant_act(x, None, 4, False, 1.0)
+    oracle.w4a4_linear(qa, qw)
+    dt = time.perf_counter() - t0
+    ops = 2.0 * sample_rows * N * K
+    return {"value": round(ops / dt / 1e12, 6), "unit": "TOPS", "cores": cores, "kind": "oracle",
+            "sample": f"{sample_rows} of {M} tokens (KV rows for the same tokens, act quant, "
+                      f"GEMM {sample_rows}x{K}->{N}); {dt:.2f} s"}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    rows = args.ref_rows
+    for _ in range(args.warmup):
+        cpu_baseline(sample_rows=max(1, rows // 4))
+    vals = [cpu_baseline(sample_rows=rows) for _ in range(args.steps)]
+    v = statistics.mean(x["value"] for x in vals)
+    ms_per_step = 2.0 * M * N * K / (v * 1e12) * 1e3
+    cb = dict(vals[-1])
+    cb["value"] = round(v, 6)
+    return {
+        "metric": METRIC, "value": round(v, 6), "unit": "TOPS", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "impl": "reference",
+        "config": {"workload": "llama3_8b_gate_up_M2048_K4096_N14336 + R3/KV4 for the same 2048 tokens",
+                   "M": M, "K": K, "N": N, "note": "CPU oracle on a bounded token sample per step"},
+        "cpu_baseline": cb,
+        "e2e": {"value": round(v, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-rows", type=int, default=1024)
+    ap.add_argument("--ref-rows", type=int, default=128, help="tokens per --impl reference step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+    else:
+        import torch
+        import torch.distributed as dist
+        if world > 1:
+            torch.cuda.set_device(local_rank)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+        out = run_ours(args, rank, world, local_rank)
+        if world > 1:
+            dist.destroy_process_group()
+    if out is not None:
+        print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,173 @@
+/*
+ * spinq.h -- C ABI of the GB300 (sm_103a) rotated W4A4 hot path of SpinQuant
+ * (arXiv 2405.16406).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * Pointers.  Every data pointer is a DEVICE pointer owned by the caller; the
+ *   library never allocates, frees or keeps a pointer after the call returns.
+ *   `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
+ *   call is asynchronous: it validates its arguments on the host, enqueues
+ *   kernels on `stream` and returns; it never synchronizes.
+ * Layouts.  Row-major, the reduction dimension K (or head_dim D) contiguous.
+ *   4-bit codes are packed two per byte, the even index in the LOW nibble.
+ *   Symmetric codes are two's complement nibbles in [-8, 7]; asymmetric codes
+ *   are unsigned nibbles in [0, 15].  Scales and zeros are fp32.
+ * Rotation.  A Hadamard spec {n_small, n_pow2} names R = (H_s (x) H_P)/sqrt(K)
+ *   with K = n_small * n_pow2, H_P the natural-order Sylvester matrix of order
+ *   n_pow2 and H_s the small factor of order n_small: [1] for n_small = 1, else
+ *   the Paley I matrix of order n_small (n_small - 1 = q, a prime power with
+ *   q = 3 mod 4; GF(q) = integers mod q for prime q, GF(27) =
+ *   GF(3)[t]/(t^3 + 2t + 1) with element i = c0 + 3 c1 + 9 c2 <-> c0 + c1 t +
+ *   c2 t^2; H_s = I + S, S = [[0, 1..1], [-1.., Q]], Q[i][j] = chi(a_i - a_j)).
+ *   The small factor acts on the slow index (element k = i * n_pow2 + j) and
+ *   activations are rotated as row vectors: x' = x R (Sec. 3.1, R3 and R4;
+ *   Sec. 2.2 footnote for the Hadamard scaling).
+ * Quantizer.  Eq. 1 (Sec. 2): symmetric alpha = clip * max|x| / (2^(N-1)-1),
+ *   beta = 0, q = clamp(rint(x/alpha), -2^(N-1), 2^(N-1)-1); asymmetric
+ *   alpha = clip * (max x - min x) / (2^N - 1), beta = clip * min x,
+ *   u = clamp(rint((x - beta)/alpha), 0, 2^N - 1); a zero range stores
+ *   alpha = 0 and codes 0.  rint is round-half-to-even.  The clipping ratio
+ *   follows the appendix "Quantization choice".  Only N = 4 has kernels.
+ * Errors.  Invalid arguments return SPINQ_EINVAL before any launch (NULL
+ *   required pointer, non-positive or inconsistent size, K not even, a
+ *   pointer not 16-byte aligned where noted, clip_ratio outside (0, 1]).
+ *   A valid request with no compiled kernel (bits != 4, an unsupported
+ *   Hadamard order or granularity) returns SPINQ_EUNSUPPORTED.  A failed
+ *   launch returns SPINQ_ECUDA.  Device-side waits in the GEMM are bounded;
+ *   a wait that gives up records SPINQ_ETIMEOUT in a device status word that
+ *   spinq_device_status() reads back.
+ */
+#ifndef SPINQ_H_
+#define SPINQ_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SPINQ_OK = 0,
+  SPINQ_EINVAL = 1,
+  SPINQ_EUNSUPPORTED = 2,
+  SPINQ_ECUDA = 3,
+  SPINQ_ETIMEOUT = 4
+} spinq_status;
+
+typedef enum {
+  SPINQ_PER_TOKEN = 0,   /* one (alpha, beta) per row of activations      */
+  SPINQ_PER_CHANNEL = 1, /* one scale per output channel (row) of weights */
+  SPINQ_PER_GROUP = 2    /* one (alpha, beta) per group of group_size     */
+} spinq_gran;
+
+/* Quantizer of Eq. 1: bit width N, symmetric (1) or asymmetric (0),
+ * granularity, group size (PER_GROUP only) and clipping ratio in (0, 1]. */
+typedef struct {
+  int32_t bits;
+  int32_t symmetric;
+  int32_t granularity;
+  int32_t group_size;
+  float clip_ratio;
+} spinq_quant_cfg;
+
+/* Online Hadamard of size n_small * n_pow2 (Sec. 3.1, R3/R4). */
+typedef struct {
+  int32_t n_small; /* 1, 12, 20 or 28 */
+  int32_t n_pow2;  /* power of two, 1 .. 16384 */
+} spinq_had_cfg;
+
+/*
+ * spinq_rotate_quant_act -- online rotation R4 fused with per-token 4-bit
+ * activation quantization (Sec. 3.1 "Additional unabsorbed rotations" and
+ * Eq. 1).  For each row m: x'_m = x_m R (skipped when had == NULL), then
+ * Eq. 1 over the K values of x'_m with one (alpha_m, beta_m).  x' is kept in
+ * fp32 and never stored.
+ *   x_f16  [M][ldx] fp16, row m starts at x_f16 + m*ldx elements; 16-byte
+ *          aligned rows (ldx % 8 == 0, pointer 16-byte aligned).
+ *   had    NULL or a spec with n_small * n_pow2 == K.
+ *   q      bits = 4, granularity = SPINQ_PER_TOKEN.
+ *   codes  [M][K/2] packed codes (16-byte aligned).
+ *   scale  [M] alpha_m.   zero [M] beta_m (asymmetric) or NULL (symmetric).
+ * Supported K: 32 <= K <= 32768, K % 32 == 0 (with had: the spec's sizes).
+ */
+spinq_status spinq_rotate_quant_act(const void* x_f16, int64_t M, int64_t K, int64_t ldx,
+                                    const spinq_had_cfg* had, const spinq_quant_cfg* q,
+                                    uint8_t* codes, float* scale, float* zero, void* stream);
+
+/*
+ * spinq_quant_weight -- offline weight preparation: merge the rotation into
+ * the weight (Sec. 3.1 rotational invariance: x' W'^T = x R R^T W^T = x W^T
+ * with W' = W R, i.e. every output row rotated like an activation row), then
+ * symmetric Eq. 1 per output channel (round-to-nearest, the RTN weight
+ * quantizer of the appendix RTN-vs-GPTQ ablation), plus the integer row sum
+ * of the codes that the GEMM epilogue needs.
+ *   w_f16  [N][K] fp16 (16-byte aligned).   had NULL = no merge.
+ *   q      bits = 4, symmetric = 1, granularity = SPINQ_PER_CHANNEL.
+ *   codes  [N][K/2], scale [N] (s_n), rowsum [N] (sum_k q_nk).
+ */
+spinq_status spinq_quant_weight(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
+                                const spinq_quant_cfg* q, uint8_t* codes, float* scale,
+                                int32_t* rowsum, void* stream);
+
+/*
+ * spinq_w4a4_gemm -- the W4A4 linear on Eq. 1 codes with an exact integer
+ * accumulator and a fused per-token x per-channel dequantization epilogue.
+ *   acc[m][n] = sum_k a_mk * q_nk, a = q (symmetric activations) or u - 8
+ *               (asymmetric activations), exact in 32-bit integers;
+ *   y[m][n]   = fp16( s_n * (alpha_m * acc[m][n] + beta'_m * rowsum_n) ),
+ *               beta'_m = beta_m + 8 alpha_m (asymmetric) or 0 (symmetric),
+ *   which equals sum_k (alpha_m c_mk + beta_m)(s_n q_nk), the product of the
+ *   two dequantized operands of Eq. 1.
+ *   a_codes [M][K/2], a_scale [M], a_zero [M] or NULL (symmetric);
+ *   w_codes [N][K/2] symmetric, w_scale [N], w_rowsum [N];
+ *   y_f16 [M][N] fp16; acc_out [M][N] int32 or NULL (debug output).
+ *   Requirements: K % 128 == 0, N % 16 == 0, K <= 65536; code and output
+ *   pointers 16-byte aligned.
+ */
+spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
+                             const uint8_t* w_codes, const float* w_scale,
+                             const int32_t* w_rowsum, int64_t M, int64_t N, int64_t K,
+                             void* y_f16, int32_t* acc_out, void* stream);
+
+/*
+ * spinq_rotate_quant_kv -- R3 on Q and K over head_dim, then the 4-bit
+ * KV-cache quantizer (Sec. 3.1: R3 is an online Hadamard inserted for low-bit
+ * KV-cache quantization; appendix "Quantization choice": asymmetric).
+ * R2 is assumed merged into W_v / W_o, so V is quantized without rotation.
+ *   q_in  [B][S][Hq][D] fp16 -> q_out (same layout; may equal q_in):
+ *         q_out = fp16(q_in R).
+ *   k_in, v_in [B][S][Hkv][D] fp16.
+ *   K' = k_in R; K' and V quantized with kvq (bits = 4, symmetric = 0,
+ *         granularity = SPINQ_PER_GROUP, group_size = D) into
+ *   k_codes, v_codes [B][S][Hkv][D/2]; k_scale, k_zero, v_scale, v_zero
+ *         [B][S][Hkv] fp32.
+ *   had   {1, D}.  Supported D: 64 or 128.  All pointers 16-byte aligned.
+ */
+spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_in,
+                                   const void* v_in, int64_t B, int64_t S, int64_t Hq,
+                                   int64_t Hkv, int64_t D, const spinq_had_cfg* had,
+                                   const spinq_quant_cfg* kvq, uint8_t* k_codes, float* k_scale,
+                                   float* k_zero, uint8_t* v_codes, float* v_scale,
+                                   float* v_zero, void* stream);
+
+/* Human-readable name of a status code (static storage). */
+const char* spinq_status_string(spinq_status s);
+
+/*
+ * spinq_device_status -- read and clear the device status word that bounded
+ * waits in the kernels write when they give up (SPINQ_ETIMEOUT), for the
+ * current CUDA device.  Synchronizes the device.  Returns SPINQ_OK when no
+ * kernel recorded an error since the last call, SPINQ_ECUDA if the read
+ * itself failed.  `detail` (may be NULL) receives the recorded site code.
+ */
+spinq_status spinq_device_status(int32_t* detail);
+
+/* Library build identifier (static storage). */
+const char* spinq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPINQ_H_ */

@@ -1,0 +1,174 @@
+// spinq_api.cu -- the extern "C" entry points declared in include/spinq.h:
+// host-side argument validation, status codes and kernel dispatch.  No entry
+// point allocates memory or synchronizes (except spinq_device_status, which
+// documents that it does).
+#include <cuda_runtime.h>
+
+#include <cmath>
+
+#include "../../include/spinq.h"
+#include "spinq_internal.h"
+
+using namespace spinq;
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool is_pow2(int64_t v) { return v > 0 && (v & (v - 1)) == 0; }
+
+spinq_status from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return SPINQ_OK;
+  if (e == cudaErrorNotSupported) return SPINQ_EUNSUPPORTED;
+  return SPINQ_ECUDA;
+}
+
+bool clip_ok(float c) { return c > 0.f && c <= 1.f; }
+
+// Validates a Hadamard spec for a rotated dimension of size `dim` and fills
+// the small-factor table.  Returns SPINQ_OK, SPINQ_EINVAL or SPINQ_EUNSUPPORTED.
+spinq_status check_had(const spinq_had_cfg* had, int64_t dim, SmallHadamard* hs) {
+  if (had->n_small < 1 || had->n_pow2 < 1 || !is_pow2(had->n_pow2)) return SPINQ_EINVAL;
+  if ((int64_t)had->n_small * had->n_pow2 != dim) return SPINQ_EINVAL;
+  if (!build_small_hadamard(had->n_small, hs)) return SPINQ_EUNSUPPORTED;
+  if (had->n_pow2 > 16384) return SPINQ_EUNSUPPORTED;
+  return SPINQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* spinq_status_string(spinq_status s) {
+  switch (s) {
+    case SPINQ_OK: return "SPINQ_OK";
+    case SPINQ_EINVAL: return "SPINQ_EINVAL: invalid argument";
+    case SPINQ_EUNSUPPORTED: return "SPINQ_EUNSUPPORTED: no kernel for this configuration";
+    case SPINQ_ECUDA: return "SPINQ_ECUDA: CUDA launch or runtime error";
+    case SPINQ_ETIMEOUT: return "SPINQ_ETIMEOUT: a bounded device wait gave up";
+  }
+  return "SPINQ: unknown status";
+}
+
+const char* spinq_version(void) { return "spinq-gb300 sm_103a 0.1"; }
+
+spinq_status spinq_rotate_quant_act(const void* x_f16, int64_t M, int64_t K, int64_t ldx,
+                                    const spinq_had_cfg* had, const spinq_quant_cfg* q,
+                                    uint8_t* codes, float* scale, float* zero, void* stream) {
+  if (!q || M < 0 || K <= 0 || ldx < K) return SPINQ_EINVAL;
+  if (M > 0 && (!x_f16 || !codes || !scale)) return SPINQ_EINVAL;
+  if (!clip_ok(q->clip_ratio)) return SPINQ_EINVAL;
+  if (q->symmetric != 0 && q->symmetric != 1) return SPINQ_EINVAL;
+  if (!q->symmetric && M > 0 && !zero) return SPINQ_EINVAL;
+  if (K % 32 != 0 || ldx % 8 != 0 || !aligned16(x_f16) || !aligned16(codes)) return SPINQ_EINVAL;
+  if (q->bits != 4 || q->granularity != SPINQ_PER_TOKEN) return SPINQ_EUNSUPPORTED;
+  if (K > 32768) return SPINQ_EUNSUPPORTED;
+  RotQuantArgs a{};
+  if (had) {
+    spinq_status st = check_had(had, K, &a.hs);
+    if (st != SPINQ_OK) return st;
+    a.n_small = had->n_small;
+    a.n_pow2 = had->n_pow2;
+    a.norm = (float)(1.0 / std::sqrt((double)K));
+  } else {
+    a.n_small = 0;
+    a.n_pow2 = 1;
+    a.norm = 1.f;
+  }
+  if (M == 0) return SPINQ_OK;
+  a.x = x_f16;
+  a.rows = M;
+  a.K = K;
+  a.ldx = ldx;
+  a.symmetric = q->symmetric != 0;
+  a.clip = q->clip_ratio;
+  a.codes = codes;
+  a.scale = scale;
+  a.zero = q->symmetric ? nullptr : zero;
+  a.rowsum = nullptr;
+  return from_cuda(launch_rotate_quant_rows(a, static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_quant_weight(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
+                                const spinq_quant_cfg* q, uint8_t* codes, float* scale,
+                                int32_t* rowsum, void* stream) {
+  if (!q || N < 0 || K <= 0) return SPINQ_EINVAL;
+  if (N > 0 && (!w_f16 || !codes || !scale || !rowsum)) return SPINQ_EINVAL;
+  if (!clip_ok(q->clip_ratio)) return SPINQ_EINVAL;
+  if (K % 32 != 0 || !aligned16(w_f16) || !aligned16(codes)) return SPINQ_EINVAL;
+  if (q->bits != 4 || q->symmetric != 1 || q->granularity != SPINQ_PER_CHANNEL) return SPINQ_EUNSUPPORTED;
+  if (K > 32768) return SPINQ_EUNSUPPORTED;
+  RotQuantArgs a{};
+  if (had) {
+    spinq_status st = check_had(had, K, &a.hs);
+    if (st != SPINQ_OK) return st;
+    a.n_small = had->n_small;
+    a.n_pow2 = had->n_pow2;
+    a.norm = (float)(1.0 / std::sqrt((double)K));
+  } else {
+    a.n_small = 0;
+    a.n_pow2 = 1;
+    a.norm = 1.f;
+  }
+  if (N == 0) return SPINQ_OK;
+  a.x = w_f16;
+  a.rows = N;
+  a.K = K;
+  a.ldx = K;
+  a.symmetric = true;
+  a.clip = q->clip_ratio;
+  a.codes = codes;
+  a.scale = scale;
+  a.zero = nullptr;
+  a.rowsum = rowsum;
+  return from_cuda(launch_rotate_quant_rows(a, static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
+                             const uint8_t* w_codes, const float* w_scale,
+                             const int32_t* w_rowsum, int64_t M, int64_t N, int64_t K,
+                             void* y_f16, int32_t* acc_out, void* stream) {
+  if (M < 0 || N < 0 || K <= 0) return SPINQ_EINVAL;
+  if (M > 0 && N > 0 && (!a_codes || !a_scale || !w_codes || !w_scale || !w_rowsum || !y_f16))
+    return SPINQ_EINVAL;
+  if (K % 128 != 0 || N % 16 != 0) return SPINQ_EINVAL;
+  if (!aligned16(a_codes) || !aligned16(w_codes) || !aligned16(y_f16) || (acc_out && !aligned16(acc_out)))
+    return SPINQ_EINVAL;
+  if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
+  if (M == 0 || N == 0) return SPINQ_OK;
+  GemmArgs g{a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y_f16, acc_out};
+  return from_cuda(launch_w4a4_gemm(g, static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_in,
+                                   const void* v_in, int64_t B, int64_t S, int64_t Hq,
+                                   int64_t Hkv, int64_t D, const spinq_had_cfg* had,
+                                   const spinq_quant_cfg* kvq, uint8_t* k_codes, float* k_scale,
+                                   float* k_zero, uint8_t* v_codes, float* v_scale,
+                                   float* v_zero, void* stream) {
+  if (!had || !kvq || B < 0 || S < 0 || Hq < 0 || Hkv < 0 || D <= 0) return SPINQ_EINVAL;
+  const int64_t rows_q = B * S * Hq, rows_kv = B * S * Hkv;
+  if (rows_q > 0 && (!q_in || !q_out)) return SPINQ_EINVAL;
+  if (rows_kv > 0 && (!k_in || !v_in || !k_codes || !k_scale || !k_zero || !v_codes || !v_scale || !v_zero))
+    return SPINQ_EINVAL;
+  if (!clip_ok(kvq->clip_ratio)) return SPINQ_EINVAL;
+  if (had->n_small != 1 || had->n_pow2 != D) return SPINQ_EINVAL;
+  for (const void* p : {q_in, (const void*)q_out, k_in, v_in, (const void*)k_codes, (const void*)v_codes})
+    if (p && !aligned16(p)) return SPINQ_EINVAL;
+  if (kvq->bits != 4 || kvq->symmetric != 0 || kvq->granularity != SPINQ_PER_GROUP || kvq->group_size != D)
+    return SPINQ_EUNSUPPORTED;
+  if (D != 64 && D != 128) return SPINQ_EUNSUPPORTED;
+  if (rows_q == 0 && rows_kv == 0) return SPINQ_OK;
+  KVArgs a{q_in, q_out, k_in, v_in, rows_q, rows_kv, (int)D, kvq->clip_ratio,
+           (float)(1.0 / std::sqrt((double)D)), k_codes, k_scale, k_zero, v_codes, v_scale, v_zero};
+  return from_cuda(launch_rotate_quant_kv(a, static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_device_status(int32_t* detail) {
+  int32_t code = 0, d = 0;
+  if (read_and_clear_device_status(&code, &d) != cudaSuccess) return SPINQ_ECUDA;
+  if (detail) *detail = d;
+  return static_cast<spinq_status>(code);
+}
+
+}  // extern "C"

@@ -1,0 +1,79 @@
+// spinq_internal.h -- host-side launch interface between the C ABI layer
+// (spinq_api.cu) and the kernels.  Every launcher enqueues on `stream`, does
+// not synchronize and returns the launch status.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace spinq {
+
+// Small Kronecker factor H_s of order n (n <= 32) as sign bits:
+// bit i of neg[ip] is set when H_s[ip][i] == -1.
+struct SmallHadamard {
+  int n;
+  uint32_t neg[32];
+};
+
+// Builds H_s for n in {1, 12, 20, 28} (Paley I for n > 1).  Returns false
+// for an unsupported order.
+bool build_small_hadamard(int n, SmallHadamard* out);
+
+struct RotQuantArgs {
+  const void* x;      // fp16 [rows][ldx]
+  int64_t rows;
+  int64_t K;
+  int64_t ldx;
+  int n_small;        // 0 = no rotation
+  int n_pow2;
+  SmallHadamard hs;
+  bool symmetric;
+  float clip;
+  float norm;         // 1/sqrt(K) with a rotation, 1 without (applied to alpha and beta)
+  uint8_t* codes;     // [rows][K/2]
+  float* scale;       // [rows]
+  float* zero;        // [rows] or nullptr
+  int32_t* rowsum;    // [rows] or nullptr (weights)
+};
+
+cudaError_t launch_rotate_quant_rows(const RotQuantArgs& a, cudaStream_t stream);
+
+struct KVArgs {
+  const void* q_in;
+  void* q_out;
+  const void* k_in;
+  const void* v_in;
+  int64_t rows_q;     // B*S*Hq
+  int64_t rows_kv;    // B*S*Hkv
+  int D;
+  float clip;
+  float norm;         // 1/sqrt(D)
+  uint8_t* k_codes;
+  float* k_scale;
+  float* k_zero;
+  uint8_t* v_codes;
+  float* v_scale;
+  float* v_zero;
+};
+
+cudaError_t launch_rotate_quant_kv(const KVArgs& a, cudaStream_t stream);
+
+struct GemmArgs {
+  const uint8_t* a_codes;
+  const float* a_scale;
+  const float* a_zero;   // nullptr = symmetric activations
+  const uint8_t* w_codes;
+  const float* w_scale;
+  const int32_t* w_rowsum;
+  int64_t M, N, K;
+  void* y;               // fp16 [M][N]
+  int32_t* acc_out;      // optional
+};
+
+// Returns cudaErrorNotSupported when the TMA descriptor cannot be encoded.
+cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+
+// Device status word written by bounded waits that gave up.
+cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail);
+
+}  // namespace spinq

@@ -1,0 +1,225 @@
+"""Python binding of the C ABI in include/spinq.h (libspinq.so, sm_103a).
+
+Argument marshalling only: every step of the hot path runs in the library's
+CUDA kernels.  PyTorch supplies device memory and the current stream.  There
+is no fallback: importing this module raises if libspinq.so is missing, and
+every call raises ``SpinqError`` on a non-OK status.
+
+Low-level names mirror the C entry points (``spinq_rotate_quant_act`` ...) and
+take raw pointers; the tensor-level helpers below them (``rotate_quant_act``
+...) allocate the outputs with torch and call the same entry points.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional, Tuple
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libspinq.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(
+        f"libspinq.so not found at {LIB_PATH}; build it with "
+        "`python -m paper_2405_16406_gb300.build` (the CUDA path has no fallback)")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+SPINQ_OK, SPINQ_EINVAL, SPINQ_EUNSUPPORTED, SPINQ_ECUDA, SPINQ_ETIMEOUT = range(5)
+SPINQ_PER_TOKEN, SPINQ_PER_CHANNEL, SPINQ_PER_GROUP = range(3)
+
+EXPORTED = (
+    "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",
+    "spinq_status_string", "spinq_device_status", "spinq_version",
+)
+
+
+class QuantCfg(ctypes.Structure):
+    _fields_ = [("bits", ctypes.c_int32), ("symmetric", ctypes.c_int32),
+                ("granularity", ctypes.c_int32), ("group_size", ctypes.c_int32),
+                ("clip_ratio", ctypes.c_float)]
+
+
+class HadCfg(ctypes.Structure):
+    _fields_ = [("n_small", ctypes.c_int32), ("n_pow2", ctypes.c_int32)]
+
+
+class SpinqError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {_lib.spinq_status_string(status).decode()}")
+
+
+_P = ctypes.c_void_p
+_I64 = ctypes.c_int64
+_lib.spinq_status_string.restype = ctypes.c_char_p
+_lib.spinq_status_string.argtypes = [ctypes.c_int]
+_lib.spinq_version.restype = ctypes.c_char_p
+_lib.spinq_version.argtypes = []
+_lib.spinq_device_status.restype = ctypes.c_int
+_lib.spinq_device_status.argtypes = [ctypes.POINTER(ctypes.c_int32)]
+_lib.spinq_rotate_quant_act.restype = ctypes.c_int
+_lib.spinq_rotate_quant_act.argtypes = [_P, _I64, _I64, _I64, ctypes.POINTER(HadCfg),
+                                        ctypes.POINTER(QuantCfg), _P, _P, _P, _P]
+_lib.spinq_quant_weight.restype = ctypes.c_int
+_lib.spinq_quant_weight.argtypes = [_P, _I64, _I64, ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
+                                    _P, _P, _P, _P]
+_lib.spinq_w4a4_gemm.restype = ctypes.c_int
+_lib.spinq_w4a4_gemm.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
+_lib.spinq_rotate_quant_kv.restype = ctypes.c_int
+_lib.spinq_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
+                                       ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
+                                       _P, _P, _P, _P, _P, _P, _P]
+
+
+def _check(st: int, where: str) -> None:
+    if st != SPINQ_OK:
+        raise SpinqError(st, where)
+
+
+# ------------------------------------------------------------------ raw ABI
+def spinq_rotate_quant_act(x, M, K, ldx, had, q, codes, scale, zero, stream) -> int:
+    return _lib.spinq_rotate_quant_act(x, M, K, ldx, had, q, codes, scale, zero, stream)
+
+
+def spinq_quant_weight(w, N, K, had, q, codes, scale, rowsum, stream) -> int:
+    return _lib.spinq_quant_weight(w, N, K, had, q, codes, scale, rowsum, stream)
+
+
+def spinq_w4a4_gemm(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc, stream) -> int:
+    return _lib.spinq_w4a4_gemm(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc,
+                                stream)
+
+
+def spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k_codes, k_scale,
+                          k_zero, v_codes, v_scale, v_zero, stream) -> int:
+    return _lib.spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k_codes,
+                                      k_scale, k_zero, v_codes, v_scale, v_zero, stream)
+
+
+def spinq_status_string(st: int) -> str:
+    return _lib.spinq_status_string(st).decode()
+
+
+def spinq_version() -> str:
+    return _lib.spinq_version().decode()
+
+
+def spinq_device_status() -> Tuple[int, int]:
+    d = ctypes.c_int32(0)
+    st = _lib.spinq_device_status(ctypes.byref(d))
+    return st, d.value
+
+
+# ------------------------------------------------------------------ helpers
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream: Optional[torch.cuda.Stream]):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _had(had: Optional[Tuple[int, int]]):
+    return None if had is None else ctypes.byref(HadCfg(int(had[0]), int(had[1])))
+
+
+def quant_cfg(bits=4, symmetric=True, granularity=SPINQ_PER_TOKEN, group_size=0, clip=1.0) -> QuantCfg:
+    return QuantCfg(bits, int(bool(symmetric)), granularity, group_size, float(clip))
+
+
+@dataclass
+class ActCodes:
+    codes: torch.Tensor            # uint8 [M, K/2]
+    scale: torch.Tensor            # f32 [M]
+    zero: Optional[torch.Tensor]   # f32 [M] or None (symmetric)
+
+
+@dataclass
+class WeightCodes:
+    codes: torch.Tensor   # uint8 [N, K/2]
+    scale: torch.Tensor   # f32 [N]
+    rowsum: torch.Tensor  # int32 [N]
+
+
+def rotate_quant_act(x: torch.Tensor, had: Optional[Tuple[int, int]], symmetric: bool = True,
+                     clip: float = 1.0, out: Optional[ActCodes] = None,
+                     stream: Optional[torch.cuda.Stream] = None) -> ActCodes:
+    assert x.dtype == torch.float16 and x.dim() == 2 and x.stride(1) == 1
+    M, K = x.shape
+    if out is None:
+        out = ActCodes(torch.empty((M, K // 2), dtype=torch.uint8, device=x.device),
+                       torch.empty(M, dtype=torch.float32, device=x.device),
+                       None if symmetric else torch.empty(M, dtype=torch.float32, device=x.device))
+    q = quant_cfg(4, symmetric, SPINQ_PER_TOKEN, 0, clip)
+    _check(_lib.spinq_rotate_quant_act(_ptr(x), M, K, x.stride(0), _had(had), ctypes.byref(q),
+                                       _ptr(out.codes), _ptr(out.scale), _ptr(out.zero), _stream(stream)),
+           "spinq_rotate_quant_act")
+    return out
+
+
+def quant_weight(w: torch.Tensor, had: Optional[Tuple[int, int]], clip: float = 1.0,
+                 stream: Optional[torch.cuda.Stream] = None) -> WeightCodes:
+    assert w.dtype == torch.float16 and w.is_contiguous()
+    N, K = w.shape
+    out = WeightCodes(torch.empty((N, K // 2), dtype=torch.uint8, device=w.device),
+                      torch.empty(N, dtype=torch.float32, device=w.device),
+                      torch.empty(N, dtype=torch.int32, device=w.device))
+    q = quant_cfg(4, True, SPINQ_PER_CHANNEL, 0, clip)
+    _check(_lib.spinq_quant_weight(_ptr(w), N, K, _had(had), ctypes.byref(q), _ptr(out.codes),
+                                   _ptr(out.scale), _ptr(out.rowsum), _stream(stream)),
+           "spinq_quant_weight")
+    return out
+
+
+def w4a4_gemm(a: ActCodes, w: WeightCodes, want_acc: bool = False, y: Optional[torch.Tensor] = None,
+              stream: Optional[torch.cuda.Stream] = None):
+    M = a.codes.shape[0]
+    N, Kh = w.codes.shape
+    K = Kh * 2
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float16, device=a.codes.device)
+    acc = torch.empty((M, N), dtype=torch.int32, device=a.codes.device) if want_acc else None
+    _check(_lib.spinq_w4a4_gemm(_ptr(a.codes), _ptr(a.scale), _ptr(a.zero), _ptr(w.codes), _ptr(w.scale),
+                                _ptr(w.rowsum), M, N, K, _ptr(y), _ptr(acc), _stream(stream)),
+           "spinq_w4a4_gemm")
+    return (y, acc) if want_acc else y
+
+
+@dataclass
+class KVCodes:
+    q_out: torch.Tensor
+    k_codes: torch.Tensor
+    k_scale: torch.Tensor
+    k_zero: torch.Tensor
+    v_codes: torch.Tensor
+    v_scale: torch.Tensor
+    v_zero: torch.Tensor
+
+
+def rotate_quant_kv(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, clip: float = 1.0,
+                    in_place_q: bool = False, out: Optional[KVCodes] = None,
+                    stream: Optional[torch.cuda.Stream] = None) -> KVCodes:
+    B, S, Hq, D = q.shape
+    Hkv = k.shape[2]
+    dev = q.device
+    if out is None:
+        out = KVCodes(q if in_place_q else torch.empty_like(q),
+                      torch.empty((B, S, Hkv, D // 2), dtype=torch.uint8, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev),
+                      torch.empty((B, S, Hkv, D // 2), dtype=torch.uint8, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev))
+    kvq = quant_cfg(4, False, SPINQ_PER_GROUP, D, clip)
+    had = HadCfg(1, D)
+    _check(_lib.spinq_rotate_quant_kv(_ptr(q), _ptr(out.q_out), _ptr(k), _ptr(v), B, S, Hq, Hkv, D,
+                                      ctypes.byref(had), ctypes.byref(kvq), _ptr(out.k_codes),
+                                      _ptr(out.k_scale), _ptr(out.k_zero), _ptr(out.v_codes),
+                                      _ptr(out.v_scale), _ptr(out.v_zero), _stream(stream)),
+           "spinq_rotate_quant_kv")
+    return out

@@ -1,0 +1,104 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and
+loads, exports every entry point include/spinq.h declares, and rejects
+invalid arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2405_16406_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_entry_points():
+    names = []
+    for fn in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names += re.findall(r"\b(spinq_[a-z0-9_]+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_header_declares_the_four_hot_path_calls():
+    names = declared_entry_points()
+    for n in ("spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for n in declared_entry_points():
+        assert hasattr(lib, n), f"libspinq.so does not export {n}"
+
+
+def test_binding_names_match_header(lib):
+    from paper_2405_16406_gb300 import spinq
+    for n in declared_entry_points():
+        assert n in spinq.EXPORTED and hasattr(spinq, n)
+
+
+def test_status_strings(lib):
+    from paper_2405_16406_gb300 import spinq
+    for s in range(5):
+        assert spinq.spinq_status_string(s).startswith("SPINQ_")
+    assert "sm_103a" in spinq.spinq_version()
+
+
+def test_invalid_arguments_rejected_before_launch(lib):
+    from paper_2405_16406_gb300 import spinq as S
+    q = S.quant_cfg(4, True, S.SPINQ_PER_TOKEN, 0, 1.0)
+    fake = ctypes.c_void_p(1 << 20)   # never dereferenced: validation fails first
+    # NULL input
+    assert S.spinq_rotate_quant_act(None, 4, 256, 256, None, ctypes.byref(q), fake, fake, None, None) == S.SPINQ_EINVAL
+    # K not a multiple of 32
+    assert S.spinq_rotate_quant_act(fake, 4, 250, 256, None, ctypes.byref(q), fake, fake, None, None) == S.SPINQ_EINVAL
+    # misaligned pointer
+    assert S.spinq_rotate_quant_act(ctypes.c_void_p((1 << 20) + 2), 4, 256, 256, None, ctypes.byref(q), fake, fake,
+                                    None, None) == S.SPINQ_EINVAL
+    # Hadamard spec inconsistent with K
+    had = S.HadCfg(1, 128)
+    assert S.spinq_rotate_quant_act(fake, 4, 256, 256, ctypes.byref(had), ctypes.byref(q), fake, fake, None,
+                                    None) == S.SPINQ_EINVAL
+    # unsupported small Hadamard order (valid size, no kernel)
+    had = S.HadCfg(36, 64)
+    assert S.spinq_rotate_quant_act(fake, 4, 36 * 64, 36 * 64, ctypes.byref(had), ctypes.byref(q), fake, fake,
+                                    None, None) == S.SPINQ_EUNSUPPORTED
+    # clip outside (0, 1]
+    bad = S.quant_cfg(4, True, S.SPINQ_PER_TOKEN, 0, 1.5)
+    assert S.spinq_rotate_quant_act(fake, 4, 256, 256, None, ctypes.byref(bad), fake, fake, None, None) == S.SPINQ_EINVAL
+    # bits != 4 -> unsupported
+    b8 = S.quant_cfg(8, True, S.SPINQ_PER_TOKEN, 0, 1.0)
+    assert S.spinq_rotate_quant_act(fake, 4, 256, 256, None, ctypes.byref(b8), fake, fake, None, None) == S.SPINQ_EUNSUPPORTED
+    # asymmetric without a zero buffer
+    qa = S.quant_cfg(4, False, S.SPINQ_PER_TOKEN, 0, 1.0)
+    assert S.spinq_rotate_quant_act(fake, 4, 256, 256, None, ctypes.byref(qa), fake, fake, None, None) == S.SPINQ_EINVAL
+    # GEMM: K not a multiple of 128, N not a multiple of 16
+    assert S.spinq_w4a4_gemm(fake, fake, None, fake, fake, fake, 4, 32, 96, fake, None, None) == S.SPINQ_EINVAL
+    assert S.spinq_w4a4_gemm(fake, fake, None, fake, fake, fake, 4, 40, 128, fake, None, None) == S.SPINQ_EINVAL
+    # weight quantizer must be symmetric per-channel
+    qw = S.quant_cfg(4, False, S.SPINQ_PER_CHANNEL, 0, 1.0)
+    assert S.spinq_quant_weight(fake, 8, 256, None, ctypes.byref(qw), fake, fake, fake, None) == S.SPINQ_EUNSUPPORTED
+    # KV: group must equal head_dim, spec must be {1, D}
+    kvq = S.quant_cfg(4, False, S.SPINQ_PER_GROUP, 64, 1.0)
+    had = S.HadCfg(1, 128)
+    assert S.spinq_rotate_quant_kv(fake, fake, fake, fake, 1, 1, 4, 2, 128, ctypes.byref(had), ctypes.byref(kvq),
+                                   fake, fake, fake, fake, fake, fake, None) == S.SPINQ_EUNSUPPORTED
+    had = S.HadCfg(1, 64)
+    kvq = S.quant_cfg(4, False, S.SPINQ_PER_GROUP, 128, 1.0)
+    assert S.spinq_rotate_quant_kv(fake, fake, fake, fake, 1, 1, 4, 2, 128, ctypes.byref(had), ctypes.byref(kvq),
+                                   fake, fake, fake, fake, fake, fake, None) == S.SPINQ_EINVAL
+
+
+def test_empty_problems_are_ok_without_launch(lib):
+    from paper_2405_16406_gb300 import spinq as S
+    q = S.quant_cfg(4, True, S.SPINQ_PER_TOKEN, 0, 1.0)
+    fake = ctypes.c_void_p(1 << 20)
+    assert S.spinq_rotate_quant_act(fake, 0, 256, 256, None, ctypes.byref(q), fake, fake, None, None) == S.SPINQ_OK
+    assert S.spinq_w4a4_gemm(fake, fake, None, fake, fake, fake, 0, 32, 128, fake, None, None) == S.SPINQ_OK

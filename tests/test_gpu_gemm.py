@@ -1,0 +1,181 @@
+"""GPU parity: spinq_w4a4_gemm vs the oracle.
+
+Bars: the int32 accumulator is bit-exact given identical codes (the oracle's
+codes are fed to the GPU); the fp16 output is within 1e-2 relative Frobenius
+error of the oracle's double-precision dequantized product.  Full-size
+workloads are checked on sampled outputs the oracle computes one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2405_16406_gb300 import synth
+from tests import parity_util as pu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def S():
+    from paper_2405_16406_gb300 import spinq
+    return spinq
+
+
+def to_gpu_act(S, a_codes, alpha, beta):
+    packed = oracle.pack4(a_codes)
+    return S.ActCodes(torch.from_numpy(packed).cuda(),
+                      torch.from_numpy(alpha.astype(np.float32)).cuda(),
+                      None if beta is None else torch.from_numpy(beta.astype(np.float32)).cuda())
+
+
+def to_gpu_w(S, w_codes, scale):
+    return S.WeightCodes(torch.from_numpy(oracle.pack4(w_codes)).cuda(),
+                         torch.from_numpy(scale.astype(np.float32)).cuda(),
+                         torch.from_numpy(w_codes.sum(1).astype(np.int32)).cuda())
+
+
+def run(S, ac, al, be, wc, ws):
+    a = to_gpu_act(S, ac, al, be)
+    w = to_gpu_w(S, wc, ws)
+    y, acc = S.w4a4_gemm(a, w, want_acc=True)
+    torch.cuda.synchronize()
+    return y.cpu().numpy(), acc.cpu().numpy()
+
+
+def oracle_full(ac, al, be, wc, ws):
+    # alpha / beta / scale as the fp32 values the GPU receives
+    al32 = al.astype(np.float32).astype(np.float64)
+    be32 = None if be is None else be.astype(np.float32).astype(np.float64)
+    ws32 = ws.astype(np.float32).astype(np.float64)
+    a = oracle.QuantAct(ac, None, al32, be32, None)
+    w = oracle.QuantWeight(wc, None, ws32, wc.sum(1).astype(np.int32), None)
+    return oracle.w4a4_linear(a, w)
+
+
+def random_codes(rng, M, N, K, symmetric):
+    ac = (rng.integers(-8, 8, (M, K)) if symmetric else rng.integers(0, 16, (M, K))).astype(np.int32)
+    wc = rng.integers(-8, 8, (N, K)).astype(np.int32)
+    al = rng.uniform(0.01, 1.0, M)
+    be = None if symmetric else rng.uniform(-3.0, 0.0, M)
+    ws = rng.uniform(1e-3, 1e-2, N)
+    return ac, al, be, wc, ws
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 16, 128), (3, 48, 256), (128, 256, 128), (130, 272, 384),
+                                   (257, 512, 1024), (16, 512, 256), (200, 4096, 512)])
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_gemm_random_codes_exact(S, M, N, K, symmetric):
+    rng = np.random.default_rng(M * 7 + N + K + symmetric)
+    ac, al, be, wc, ws = random_codes(rng, M, N, K, symmetric)
+    y, acc = run(S, ac, al, be, wc, ws)
+    ref = oracle_full(ac, al, be, wc, ws)
+    assert np.array_equal(acc, ref.acc)
+    assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
+    # elementwise: fp32 epilogue then one fp16 rounding
+    assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
+
+
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_gemm_extreme_codes_long_k(S, symmetric):
+    # largest accumulator magnitudes: every product at its extreme, K = 65536
+    M, N, K = 130, 144, 65536
+    for aval, wval in ((7, 7), (-8, -8), (7, -8)):
+        ac = np.full((M, K), aval if symmetric else aval + 8, dtype=np.int32)
+        wc = np.full((N, K), wval, dtype=np.int32)
+        al, ws = np.full(M, 0.5), np.full(N, 0.25)
+        be = None if symmetric else np.full(M, -1.0)
+        y, acc = run(S, ac, al, be, wc, ws)
+        ref = oracle_full(ac, al, be, wc, ws)
+        assert np.array_equal(acc, ref.acc), (aval, wval)
+
+
+def test_gemm_alternating_and_sparse_codes(S):
+    M, N, K = 128, 256, 4096
+    k = np.arange(K)
+    ac = np.where(k % 2 == 0, 7, -8)[None, :].repeat(M, 0).astype(np.int32)
+    ac[::3] = -ac[::3]
+    ac = np.clip(ac, -8, 7)
+    wc = np.where((k // 3) % 2 == 0, -8, 7)[None, :].repeat(N, 0).astype(np.int32)
+    wc[:, ::5] = 0
+    rng = np.random.default_rng(0)
+    al, ws = rng.uniform(0.1, 1, M), rng.uniform(0.001, 0.01, N)
+    y, acc = run(S, ac, al, None, wc, ws)
+    assert np.array_equal(acc, oracle_full(ac, al, None, wc, ws).acc)
+
+
+FULL = [
+    ("gate_up", 2048, 4096, 14336, False),
+    ("down_proj", 2048, 14336, 4096, True),
+    ("l32_up_M8192", 8192, 3072, 8192, False),
+    ("l32_down_M8192", 8192, 8192, 3072, False),
+    ("l32_up_M1", 1, 3072, 8192, False),
+    ("l32_down_M16", 16, 8192, 3072, False),
+    ("l32_up_M128", 128, 3072, 8192, False),
+]
+
+
+@pytest.mark.parametrize("name,M,K,N,symmetric", FULL, ids=[f[0] for f in FULL])
+def test_gemm_full_size_sampled(S, name, M, K, N, symmetric):
+    rng = np.random.default_rng(len(name))
+    ac, al, be, wc, ws = random_codes(rng, M, N, K, symmetric)
+    y, acc = run(S, ac, al, be, wc, ws)
+    # sampled outputs (random + corners + tile edges)
+    ms = np.concatenate([rng.integers(0, M, 3000), [0, M - 1, min(127, M - 1), min(128, M - 1)]])
+    ns = np.concatenate([rng.integers(0, N, 3000), [N - 1, 0, min(255, N - 1), min(256, N - 1)]])
+    al32 = al.astype(np.float32).astype(np.float64)
+    be32 = None if be is None else be.astype(np.float32).astype(np.float64)
+    ws32 = ws.astype(np.float32).astype(np.float64)
+    racc, ry = oracle.w4a4_linear_sampled(ac, al32, be32, wc, ws32, ms, ns)
+    assert np.array_equal(acc[ms, ns], racc)
+    assert pu.rel_frob(y[ms, ns], ry) <= pu.Y_REL_FROB
+
+
+LINEAR = [
+    ("tiny", synth.tiny_linear, {}),
+    ("down_proj_M256", synth.llama3_8b_down_proj, {"M": 256}),
+    ("gate_up_M128", synth.llama3_8b_gate_up, {"M": 128}),
+    ("l32_up_M16", synth.llama32_3b_up, {"M": 16}),
+    ("l32_down_M128", synth.llama32_3b_down, {"M": 128}),
+]
+
+
+@pytest.mark.parametrize("name,builder,kw", LINEAR, ids=[c[0] for c in LINEAR])
+def test_rotated_linear_end_to_end(S, name, builder, kw):
+    """GPU rotate+quant -> GPU weight quant -> GPU GEMM vs the oracle chain."""
+    c = builder(**kw)
+    x = torch.from_numpy(c.x).cuda()
+    w = torch.from_numpy(c.w).cuda()
+    qa = S.rotate_quant_act(x, c.had, c.act_symmetric, c.clip)
+    qw = S.quant_weight(w, c.had)
+    y = S.w4a4_gemm(qa, qw)
+    torch.cuda.synchronize()
+    ra = oracle.rotate_quant_act(c.x, c.had, 4, c.act_symmetric, c.clip)
+    rw = oracle.quant_weight(c.w, c.had)
+    ref = oracle.w4a4_linear(ra, rw)
+    assert pu.rel_frob(y.cpu().numpy(), ref.y) <= pu.Y_REL_FROB
+    # and with the GPU's own codes, the accumulator is exact
+    got_a = pu.gpu_codes(qa.codes.cpu().numpy(), c.act_symmetric)
+    got_w = pu.gpu_codes(qw.codes.cpu().numpy(), True)
+    y2, acc2 = S.w4a4_gemm(qa, qw, want_acc=True)
+    ref2 = oracle.w4a4_linear(
+        oracle.QuantAct(got_a, None, qa.scale.cpu().numpy().astype(np.float64),
+                        None if qa.zero is None else qa.zero.cpu().numpy().astype(np.float64), None),
+        oracle.QuantWeight(got_w, None, qw.scale.cpu().numpy().astype(np.float64), got_w.sum(1), None))
+    assert np.array_equal(acc2.cpu().numpy(), ref2.acc)
+
+
+def test_rotated_linear_matches_full_precision(S):
+    """Sec. 3.1 invariance on the device: the rotated quantized layer stays close
+    to the unrotated full-precision product x W^T (quantization error only)."""
+    c = synth.llama3_8b_down_proj(M=64)
+    x = torch.from_numpy(c.x).cuda()
+    w = torch.from_numpy(c.w).cuda()
+    y = S.w4a4_gemm(S.rotate_quant_act(x, c.had, True), S.quant_weight(w, c.had))
+    ref = c.x.astype(np.float64) @ c.w.astype(np.float64).T
+    err_rot = pu.rel_frob(y.cpu().numpy(), ref)
+    y0 = S.w4a4_gemm(S.rotate_quant_act(x, None, True), S.quant_weight(w, None))
+    err_plain = pu.rel_frob(y0.cpu().numpy(), ref)
+    # per-token int4 on x100 outlier channels loses most of the signal without the
+    # rotation; with R4 the error is a fraction of it
+    assert err_rot < 0.5 * err_plain, (err_rot, err_plain)
