@@ -122,8 +122,8 @@ spinq_status spinq_quant_weight(const void* w_f16, int64_t N, int64_t K, const s
  *   a_codes [M][K/2], a_scale [M], a_zero [M] or NULL (symmetric);
  *   w_codes [N][K/2] symmetric, w_scale [N], w_rowsum [N];
  *   y_f16 [M][N] fp16; acc_out [M][N] int32 or NULL (debug output).
- *   Requirements: K % 128 == 0, N % 16 == 0, K <= 65536; code and output
- *   pointers 16-byte aligned.
+ *   Requirements: K % 128 == 0, N % 16 == 0, K <= 65536; code, output,
+ *   w_scale and w_rowsum pointers 16-byte aligned.
  */
 spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
                              const uint8_t* w_codes, const float* w_scale,

@@ -1,0 +1,56 @@
+// launch_util.h -- cached launch-configuration queries.  Each is computed once
+// per (device, kernel, dynamic shared memory) and then served from a table, so
+// launchers make no device queries on the hot path and stay usable while a
+// stream is being captured into a CUDA graph.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <map>
+#include <mutex>
+#include <tuple>
+
+namespace spinq {
+
+inline int device_sm_count() {
+  static int cache[64] = {0};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return 1;
+  if (cache[dev] == 0) {
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    cache[dev] = sms > 0 ? sms : 1;
+  }
+  return cache[dev];
+}
+
+// Raises the kernel's dynamic shared memory limit (once per size) and returns
+// the number of resident blocks per SM for this launch shape (at least 1).
+template <typename Kern>
+cudaError_t prepare_launch(Kern kern, int threads, size_t smem, int* blocks_per_sm) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, const void*, size_t, int>, int> occ;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const auto key = std::make_tuple(dev, reinterpret_cast<const void*>(kern), smem, threads);
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = occ.find(key);
+  if (it != occ.end()) {
+    *blocks_per_sm = it->second;
+    return cudaSuccess;
+  }
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  int per_sm = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) per_sm = 1;
+  occ[key] = per_sm;
+  *blocks_per_sm = per_sm;
+  return cudaSuccess;
+}
+
+}  // namespace spinq

@@ -1,0 +1,393 @@
+// rotate_quant_act.cu -- activation kernels of spinq_rotate_quant_act:
+// the online rotation R4 (Sec. 3.1) fused with the per-token Eq. 1 quantizer,
+// for a power-of-two rotation size 512 <= P <= 16384, and the quantizer alone
+// when there is no online rotation.
+//
+// One CTA of W warps owns one row at a time (persistent over rows).
+//
+// Phase 1 (registers).  Lane `lane` of warp w loads the 16-byte chunks
+// ch = lane + 32 (w + W v), v < V, so every load instruction is coalesced.
+// Element index bits: e (0..2, inside a chunk), c = lane & 3 (3..4),
+// g = lane >> 2 (5..7), w (8 .. 8+LW-1), v (8+LW ..).
+// A tensor-core m16n8k16 with B = the 16-point Sylvester matrix contracts the
+// bits {e0, e1, c0, c1} of the RAW fp16 input (entries +-1: exact products,
+// fp32 sums) and returns fp32 in the lane that supplied the data, at the same
+// element positions.  Radix-2 butterflies inside the lane then cover e2 and
+// the v bits.
+//
+// Transpose.  The rows go through shared memory once as fp32 (16-byte chunks
+// XOR-swizzled so that both the phase-1 stores and the phase-2 loads are free
+// of bank conflicts).
+//
+// Phase 2 (registers).  Thread t owns the remaining bits (g and w: 3 + LW
+// bits) for 2^L consecutive elements, finishes the butterflies, joins the
+// row-wide range reduction and writes its packed codes (2^L nibbles).
+//
+// Eq. 1 is applied to the unnormalised row; alpha and beta carry 1/sqrt(K).
+#include <cuda_fp16.h>
+#include <float.h>
+
+#include "launch_util.h"
+#include "spinq_device.cuh"
+#include "spinq_internal.h"
+
+namespace spinq {
+namespace {
+
+__device__ __forceinline__ uint32_t h16_entry_pair(int k0, int k1, int n, bool hadamard) {
+  float v0, v1;
+  if (hadamard) {
+    v0 = (__popc(k0 & n) & 1) ? -1.f : 1.f;
+    v1 = (__popc(k1 & n) & 1) ? -1.f : 1.f;
+  } else {
+    v0 = k0 == n ? 1.f : 0.f;
+    v1 = k1 == n ? 1.f : 0.f;
+  }
+  return pack_half2_bits(v0, v1);
+}
+
+// B fragments of the 16 x 16 Sylvester matrix (hadamard) or identity, for the
+// two n-tiles n = g and n = g + 8.
+__device__ __forceinline__ void make_b16(uint32_t b[2][2], bool hadamard) {
+  const int lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
+#pragma unroll
+  for (int nt = 0; nt < 2; ++nt) {
+    const int n = g + 8 * nt;
+    b[nt][0] = h16_entry_pair(2 * c, 2 * c + 1, n, hadamard);
+    b[nt][1] = h16_entry_pair(2 * c + 8, 2 * c + 9, n, hadamard);
+  }
+}
+
+// One 16-byte chunk (8 fp16) through the tensor core: y[e] for e = 0..7.
+__device__ __forceinline__ void chunk_mma(const uint4 in, const uint32_t b[2][2], float y[8]) {
+  const uint32_t A[4] = {in.x, in.z, in.y, in.w};
+  float d0[4], d1[4];
+  mma_16816_f16_f32(d0, A, b[0][0], b[0][1]);
+  mma_16816_f16_f32(d1, A, b[1][0], b[1][1]);
+  y[0] = d0[0];
+  y[1] = d0[1];
+  y[4] = d0[2];
+  y[5] = d0[3];
+  y[2] = d1[0];
+  y[3] = d1[1];
+  y[6] = d1[2];
+  y[7] = d1[3];
+}
+
+template <bool SYM>
+struct Range {
+  float hi, lo;
+  __device__ __forceinline__ Range() : hi(SYM ? 0.f : -FLT_MAX), lo(FLT_MAX) {}
+  __device__ __forceinline__ void add(float v) {
+    if (SYM) {
+      hi = fmaxf(hi, fabsf(v));
+    } else {
+      hi = fmaxf(hi, v);
+      lo = fminf(lo, v);
+    }
+  }
+  __device__ __forceinline__ void warp_reduce() {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+      if (!SYM) lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    }
+  }
+};
+
+// Row-wide range over the W warps of the CTA (red: 2*W floats).
+template <bool SYM, int W>
+__device__ __forceinline__ void block_range(Range<SYM>& r, float* red) {
+  r.warp_reduce();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (W > 1) {
+    if (lane == 0) {
+      red[w] = r.hi;
+      red[W + w] = r.lo;
+    }
+    __syncthreads();
+    r.hi = red[0];
+    r.lo = red[W];
+#pragma unroll
+    for (int i = 1; i < W; ++i) {
+      r.hi = fmaxf(r.hi, red[i]);
+      if (!SYM) r.lo = fminf(r.lo, red[W + i]);
+    }
+  }
+}
+
+// Quantizer constants of Eq. 1 for the (unnormalised) row range.
+template <bool SYM>
+struct QParams {
+  float inv, off, alpha, beta;
+  __device__ __forceinline__ QParams(const Range<SYM>& r, float clip) {
+    if (SYM) {
+      const float m = clip * r.hi;
+      alpha = m / 7.f;
+      inv = m > 0.f ? 7.f / m : 0.f;
+      off = 0.f;
+      beta = 0.f;
+    } else {
+      const float h2 = clip * r.hi, l2 = clip * r.lo;
+      alpha = (h2 - l2) / 15.f;
+      inv = h2 > l2 ? 15.f / (h2 - l2) : 0.f;
+      beta = l2;
+      off = -l2 * inv;
+    }
+  }
+  template <bool CLAMP>
+  __device__ __forceinline__ uint32_t code_bits(float v) const {
+    float t = fmaf(v, inv, off);
+    if (CLAMP) t = SYM ? fminf(fmaxf(t, -8.f), 7.f) : fminf(fmaxf(t, 0.f), 15.f);
+    return round_bits(t);
+  }
+};
+
+// ------------------------------------------------------------------------
+// power-of-two rotation
+// ------------------------------------------------------------------------
+template <int LW, int L>
+struct Pow2Shape {
+  static constexpr int W = 1 << LW;
+  static constexpr int T = 32 * W;
+  static constexpr int LV = LW + L;
+  static constexpr int V = 1 << LV;
+  static constexpr int P = 256 * W * V;
+  static constexpr int NG = 1 << (3 + LW);  // phase-2 groups per thread
+  static constexpr int GL = 1 << L;         // consecutive elements per group
+};
+
+// fp32 word index of element p in the swizzled row buffer
+template <int LW>
+__device__ __forceinline__ uint32_t swz_word(uint32_t p) {
+  const uint32_t q = p >> 2;
+  const uint32_t x = ((q >> 3) ^ (q >> (6 + LW))) & 1u;
+  return ((q ^ x) << 2) | (p & 3u);
+}
+
+template <int LW, int L, bool SYM, bool CLAMP>
+__global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
+  using S = Pow2Shape<LW, L>;
+  extern __shared__ __align__(16) float sm[];
+  __shared__ float red[2 * S::W];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  uint32_t bh[2][2];
+  make_b16(bh, true);
+  const __half* __restrict__ x = reinterpret_cast<const __half*>(a.x);
+
+  // phase-2 fixed element bits of this thread
+  const uint32_t t_lo = (uint32_t)tid & ((1u << (3 - L)) - 1u);
+  const uint32_t t_c = ((uint32_t)tid >> (3 - L)) & 3u;
+  const uint32_t t_v = (uint32_t)tid >> (5 - L);
+  const uint32_t fixed = (t_lo << L) | (t_c << 3) | (t_v << (8 + LW));
+
+  for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x) {
+    const uint4* src = reinterpret_cast<const uint4*>(x + row * a.ldx);
+    // ---------------- phase 1
+    uint4 in[S::V];
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) in[v] = __ldg(src + lane + 32 * (w + S::W * v));
+    float y[S::V][8];
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) chunk_mma(in[v], bh, y[v]);
+#pragma unroll
+    for (int v = 0; v < S::V; ++v)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float p0 = y[v][e], p1 = y[v][e + 4];
+        y[v][e] = p0 + p1;
+        y[v][e + 4] = p0 - p1;
+      }
+#pragma unroll
+    for (int bit = 1; bit < S::V; bit <<= 1)
+#pragma unroll
+      for (int v = 0; v < S::V; ++v)
+        if (!(v & bit)) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float p0 = y[v][e], p1 = y[v | bit][e];
+            y[v][e] = p0 + p1;
+            y[v | bit][e] = p0 - p1;
+          }
+        }
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) {
+      const uint32_t p = 8u * (uint32_t)(lane + 32 * (w + S::W * v));
+      *reinterpret_cast<float4*>(sm + swz_word<LW>(p)) = make_float4(y[v][0], y[v][1], y[v][2], y[v][3]);
+      *reinterpret_cast<float4*>(sm + swz_word<LW>(p + 4)) = make_float4(y[v][4], y[v][5], y[v][6], y[v][7]);
+    }
+    __syncthreads();
+
+    // ---------------- phase 2
+    float z[S::NG][S::GL];
+#pragma unroll
+    for (int m = 0; m < S::NG; ++m) {
+      const uint32_t p = fixed | ((uint32_t)(m & 7) << 5) | ((uint32_t)(m >> 3) << 8);
+      if constexpr (S::GL == 8) {
+        const float4 u0 = *reinterpret_cast<const float4*>(sm + swz_word<LW>(p));
+        const float4 u1 = *reinterpret_cast<const float4*>(sm + swz_word<LW>(p + 4));
+        z[m][0] = u0.x; z[m][1] = u0.y; z[m][2] = u0.z; z[m][3] = u0.w;
+        z[m][4 % S::GL] = u1.x; z[m][5 % S::GL] = u1.y; z[m][6 % S::GL] = u1.z; z[m][7 % S::GL] = u1.w;
+      } else if constexpr (S::GL == 4) {
+        const float4 u0 = *reinterpret_cast<const float4*>(sm + swz_word<LW>(p));
+        z[m][0] = u0.x; z[m][1 % S::GL] = u0.y; z[m][2 % S::GL] = u0.z; z[m][3 % S::GL] = u0.w;
+      } else {
+        const float2 u0 = *reinterpret_cast<const float2*>(sm + swz_word<LW>(p));
+        z[m][0] = u0.x; z[m][1 % S::GL] = u0.y;
+      }
+    }
+#pragma unroll
+    for (int bit = 1; bit < S::NG; bit <<= 1)
+#pragma unroll
+      for (int m = 0; m < S::NG; ++m)
+        if (!(m & bit)) {
+#pragma unroll
+          for (int j = 0; j < S::GL; ++j) {
+            const float p0 = z[m][j], p1 = z[m | bit][j];
+            z[m][j] = p0 + p1;
+            z[m | bit][j] = p0 - p1;
+          }
+        }
+    Range<SYM> r;
+#pragma unroll
+    for (int m = 0; m < S::NG; ++m)
+#pragma unroll
+      for (int j = 0; j < S::GL; ++j) r.add(z[m][j]);
+    block_range<SYM, S::W>(r, red);
+    const QParams<SYM> qp(r, a.clip);
+
+    uint8_t* out = a.codes + row * (a.K / 2);
+#pragma unroll
+    for (int m = 0; m < S::NG; ++m) {
+      const uint32_t p = fixed | ((uint32_t)(m & 7) << 5) | ((uint32_t)(m >> 3) << 8);
+      uint32_t rb[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) rb[j] = j < S::GL ? qp.template code_bits<CLAMP>(z[m][j % S::GL]) : 0u;
+      const uint32_t word = pack8_nibbles(rb);
+      if constexpr (S::GL == 8) *reinterpret_cast<uint32_t*>(out + p / 2) = word;
+      else if constexpr (S::GL == 4) *reinterpret_cast<uint16_t*>(out + p / 2) = (uint16_t)word;
+      else out[p / 2] = (uint8_t)word;
+    }
+    if (tid == 0) {
+      a.scale[row] = qp.alpha * a.norm;
+      if (!SYM) a.zero[row] = qp.beta * a.norm;
+    }
+    __syncthreads();  // the row buffer and `red` are reused by the next row
+  }
+}
+
+// ------------------------------------------------------------------------
+// quantizer only (no online rotation): W warps per row, up to 8 chunks a lane
+// ------------------------------------------------------------------------
+constexpr int kNoRotV = 8;
+
+template <bool SYM, bool CLAMP, int W>
+__global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
+  __shared__ float red[2 * W];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  uint32_t bi[2][2];
+  make_b16(bi, false);
+  const int nchunk = (int)(a.K / 8);
+  const __half* __restrict__ x = reinterpret_cast<const __half*>(a.x);
+  for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x) {
+    const uint4* src = reinterpret_cast<const uint4*>(x + row * a.ldx);
+    uint4 in[kNoRotV];
+#pragma unroll
+    for (int v = 0; v < kNoRotV; ++v) {
+      const int ch = lane + 32 * (w + W * v);
+      in[v] = ch < nchunk ? __ldg(src + ch) : make_uint4(0, 0, 0, 0);
+    }
+    float y[kNoRotV][8];
+    Range<SYM> r;
+#pragma unroll
+    for (int v = 0; v < kNoRotV; ++v) {
+      chunk_mma(in[v], bi, y[v]);  // exact fp16 -> fp32
+      if (lane + 32 * (w + W * v) < nchunk)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) r.add(y[v][e]);
+    }
+    block_range<SYM, W>(r, red);
+    const QParams<SYM> qp(r, a.clip);
+    uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
+#pragma unroll
+    for (int v = 0; v < kNoRotV; ++v) {
+      const int ch = lane + 32 * (w + W * v);
+      uint32_t rb[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) rb[e] = qp.template code_bits<CLAMP>(y[v][e]);
+      if (ch < nchunk) out[ch] = pack8_nibbles(rb);
+    }
+    if (tid == 0) {
+      a.scale[row] = qp.alpha * a.norm;
+      if (!SYM) a.zero[row] = qp.beta * a.norm;
+    }
+    if (W > 1) __syncthreads();
+  }
+}
+
+template <typename Kern>
+cudaError_t launch_rows(Kern kern, int threads, size_t smem, const RotQuantArgs& a, cudaStream_t stream) {
+  int per_sm = 0;
+  cudaError_t e = prepare_launch(kern, threads, smem, &per_sm);
+  if (e != cudaSuccess) return e;
+  const int64_t cap = (int64_t)device_sm_count() * per_sm;
+  const int64_t grid = a.rows < cap ? a.rows : cap;
+  kern<<<(unsigned)grid, threads, smem, stream>>>(a);
+  return cudaGetLastError();
+}
+
+template <int LW, int L, bool SYM, bool CLAMP>
+cudaError_t launch_pow2(const RotQuantArgs& a, cudaStream_t stream) {
+  using S = Pow2Shape<LW, L>;
+  return launch_rows(rq_pow2_kernel<LW, L, SYM, CLAMP>, S::T, sizeof(float) * S::P, a, stream);
+}
+
+template <bool SYM, bool CLAMP>
+cudaError_t launch_pow2_for(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = true;
+  switch (a.n_pow2) {
+    case 512: return launch_pow2<0, 1, SYM, CLAMP>(a, stream);
+    case 1024: return launch_pow2<0, 2, SYM, CLAMP>(a, stream);
+    case 2048: return launch_pow2<1, 1, SYM, CLAMP>(a, stream);
+    case 4096: return launch_pow2<1, 2, SYM, CLAMP>(a, stream);
+    case 8192: return launch_pow2<2, 1, SYM, CLAMP>(a, stream);
+    case 16384: return launch_pow2<2, 2, SYM, CLAMP>(a, stream);
+  }
+  *handled = false;
+  return cudaSuccess;
+}
+
+template <bool SYM, bool CLAMP>
+cudaError_t launch_norot_for(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  const int64_t nchunk = a.K / 8;
+  const int64_t warps = (nchunk + 32 * kNoRotV - 1) / (32 * kNoRotV);
+  *handled = true;
+  if (warps <= 1) return launch_rows(rq_norot_kernel<SYM, CLAMP, 1>, 32, 0, a, stream);
+  if (warps <= 2) return launch_rows(rq_norot_kernel<SYM, CLAMP, 2>, 64, 0, a, stream);
+  if (warps <= 4) return launch_rows(rq_norot_kernel<SYM, CLAMP, 4>, 128, 0, a, stream);
+  if (warps <= 8) return launch_rows(rq_norot_kernel<SYM, CLAMP, 8>, 256, 0, a, stream);
+  if (warps <= 16) return launch_rows(rq_norot_kernel<SYM, CLAMP, 16>, 512, 0, a, stream);
+  *handled = false;
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_rotate_quant_act_fast(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = false;
+  if (a.rows == 0 || a.rowsum) return cudaSuccess;
+  const bool clamp = a.clip < 1.0f;
+  if (a.n_small == 0) {
+    if (a.symmetric)
+      return clamp ? launch_norot_for<true, true>(a, stream, handled) : launch_norot_for<true, false>(a, stream, handled);
+    return clamp ? launch_norot_for<false, true>(a, stream, handled) : launch_norot_for<false, false>(a, stream, handled);
+  }
+  if (a.n_small == 1) {
+    if (a.symmetric)
+      return clamp ? launch_pow2_for<true, true>(a, stream, handled) : launch_pow2_for<true, false>(a, stream, handled);
+    return clamp ? launch_pow2_for<false, true>(a, stream, handled) : launch_pow2_for<false, false>(a, stream, handled);
+  }
+  return cudaSuccess;
+}
+
+}  // namespace spinq

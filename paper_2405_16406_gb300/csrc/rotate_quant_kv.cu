@@ -22,6 +22,7 @@
 #include <cuda_fp16.h>
 #include <float.h>
 
+#include "launch_util.h"
 #include "spinq_device.cuh"
 #include "spinq_internal.h"
 
@@ -194,9 +195,7 @@ __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) 
 template <int D, bool CLAMP>
 cudaError_t launch_t(const KVArgs& a, cudaStream_t stream) {
   const int64_t groups = (a.rows_q + 7) / 8 + 2 * ((a.rows_kv + 7) / 8);
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int sms = device_sm_count();
   int64_t blocks = (groups + kWarps - 1) / kWarps;
   const int64_t cap = (int64_t)sms * 16;  // persistent-style cap: 16 blocks of 8 warps per SM
   if (blocks > cap) blocks = cap;

@@ -13,6 +13,7 @@
 #include <cuda_fp16.h>
 #include <float.h>
 
+#include "launch_util.h"
 #include "spinq_device.cuh"
 #include "spinq_internal.h"
 
@@ -167,15 +168,11 @@ template <bool SYM, bool ROWSUM, bool CLAMP>
 cudaError_t launch_t(const RotQuantArgs& a, cudaStream_t stream) {
   const size_t smem = sizeof(float) * (size_t)a.K;
   auto kern = rotate_quant_rows_kernel<SYM, ROWSUM, CLAMP>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   int per_sm = 0;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
-  if (per_sm < 1) per_sm = 1;
-  const int64_t grid = a.rows < (int64_t)sms * per_sm * 4 ? a.rows : (int64_t)sms * per_sm * 4;
+  cudaError_t e = prepare_launch(kern, kThreads, smem, &per_sm);
+  if (e != cudaSuccess) return e;
+  const int64_t cap = (int64_t)device_sm_count() * per_sm * 4;
+  const int64_t grid = a.rows < cap ? a.rows : cap;
   kern<<<(unsigned)grid, kThreads, smem, stream>>>(a);
   return cudaGetLastError();
 }
@@ -184,6 +181,9 @@ cudaError_t launch_t(const RotQuantArgs& a, cudaStream_t stream) {
 
 cudaError_t launch_rotate_quant_rows(const RotQuantArgs& a, cudaStream_t stream) {
   if (a.rows == 0) return cudaSuccess;
+  bool handled = false;
+  cudaError_t e = launch_rotate_quant_act_fast(a, stream, &handled);
+  if (handled || e != cudaSuccess) return e;
   const bool clamp = a.clip < 1.0f;
   if (a.symmetric) {
     if (a.rowsum) return clamp ? launch_t<true, true, true>(a, stream) : launch_t<true, true, false>(a, stream);

@@ -132,7 +132,8 @@ spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const
   if (M > 0 && N > 0 && (!a_codes || !a_scale || !w_codes || !w_scale || !w_rowsum || !y_f16))
     return SPINQ_EINVAL;
   if (K % 128 != 0 || N % 16 != 0) return SPINQ_EINVAL;
-  if (!aligned16(a_codes) || !aligned16(w_codes) || !aligned16(y_f16) || (acc_out && !aligned16(acc_out)))
+  if (!aligned16(a_codes) || !aligned16(w_codes) || !aligned16(y_f16) || !aligned16(w_scale) ||
+      !aligned16(w_rowsum) || (acc_out && !aligned16(acc_out)))
     return SPINQ_EINVAL;
   if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
   if (M == 0 || N == 0) return SPINQ_OK;

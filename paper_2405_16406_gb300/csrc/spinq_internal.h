@@ -38,6 +38,10 @@ struct RotQuantArgs {
 
 cudaError_t launch_rotate_quant_rows(const RotQuantArgs& a, cudaStream_t stream);
 
+// Specialised activation kernels (no rotation, or a power-of-two rotation of
+// 512..16384).  Sets *handled = false when the shape has no such kernel.
+cudaError_t launch_rotate_quant_act_fast(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
+
 struct KVArgs {
   const void* q_in;
   void* q_out;

@@ -16,22 +16,28 @@
 // (sum_k u_w = rowsum_n + 8 K cancels the 64 K term).  sum_k u_a is counted
 // by the unpack warps while they expand the activation tiles.
 //
-// CTA tile 128 x BN (BN = 128 or 256), K step 128.  Warp roles:
-//   warp 0      TMA producer: packed A [128 x 64 B] and B [BN x 64 B] tiles,
-//               4-stage ring.
-//   warp 1      TMEM allocation and the single-thread MMA issuer
-//               (tcgen05.mma.cta_group::1.kind::f8f6f4, 4 x K=32 per stage).
-//   warps 4..7  unpack packed tiles into the 128-byte-swizzled K-major E4M3
-//               operand tiles (2-stage ring), then the epilogue: tcgen05.ld of
-//               the fp32 accumulator, integer recovery, scales, fp16 stores.
+// Persistent kernel: one CTA per SM walks the output tiles (128 x 256, M
+// fastest so that concurrently running CTAs share weight tiles in L2).  Warp
+// roles (448 threads):
+//   warp 0       TMA producer: packed A [128 x 64 B] and B [256 x 64 B] tiles
+//                for one K step of 128, ring of NP stages.
+//   warp 1       TMEM allocation (2 x 256 fp32 columns) and the single-thread
+//                MMA issuer: 4 x tcgen05.mma.cta_group::1.kind::f8f6f4 (K = 32)
+//                per stage into the accumulator buffer of the current tile.
+//   warps 2..5   epilogue, one TMEM lane quadrant each (warp % 4): tcgen05.ld
+//                of a finished accumulator, integer recovery, scales, fp16
+//                stores; runs while the MMA fills the other buffer.
+//   warps 6..13  unpack the packed tiles into the 128-byte-swizzled K-major
+//                E4M3 operand tiles (ring of NU stages) and count sum_k u_a.
 // Every mbarrier wait is bounded in time; a wait that gives up records
-// SPINQ_ETIMEOUT in the device status word and the CTA winds down.
+// SPINQ_ETIMEOUT in the device status word and every role winds down.
 #include <cuda.h>
 #include <cuda_fp16.h>
 
 #include <mutex>
 
 #include "../../include/spinq.h"
+#include "launch_util.h"
 #include "spinq_device.cuh"
 #include "spinq_internal.h"
 
@@ -43,8 +49,14 @@ __device__ int g_status_detail = 0;
 namespace {
 
 constexpr int BM = 128;
-constexpr int NP = 4;  // packed (TMA) stages
-constexpr int NU = 2;  // unpacked (MMA operand) stages
+constexpr int BN = 256;
+constexpr int NP = 3;   // packed (TMA) stages
+constexpr int NU = 3;   // unpacked (MMA operand) stages
+constexpr int kUnpackWarps = 8;
+constexpr int kEpiWarps = 4;
+constexpr int kThreads = (6 + kUnpackWarps) * 32;
+constexpr int kFirstUnpackWarp = 6;
+constexpr int kFirstEpiWarp = 2;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 __device__ __forceinline__ void record_timeout(int site) {
@@ -71,6 +83,8 @@ __device__ __forceinline__ uint32_t swz_off(int r, int chunk) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4));
 }
 
+// 32 packed codes (16 bytes) -> 32 unsigned E4M3 bytes: nibble n -> byte
+// (n ^ x) & 15; `lo` holds the even k of each byte group, `hi` the odd k.
 __device__ __forceinline__ void unpack16(const uint4 w, uint32_t x, uint4& lo, uint4& hi) {
   uint32_t t;
   t = w.x ^ x; lo.x = t & 0x0F0F0F0Fu; hi.x = (t >> 4) & 0x0F0F0F0Fu;
@@ -79,69 +93,67 @@ __device__ __forceinline__ void unpack16(const uint4 w, uint32_t x, uint4& lo, u
   t = w.w ^ x; lo.w = t & 0x0F0F0F0Fu; hi.w = (t >> 4) & 0x0F0F0F0Fu;
 }
 
-template <int BN>
 struct Layout {
   static constexpr uint32_t uA = 0;
   static constexpr uint32_t uB = uA + NU * BM * 128;
   static constexpr uint32_t pA = uB + NU * BN * 128;
   static constexpr uint32_t pB = pA + NP * BM * 64;
   static constexpr uint32_t bars = pB + NP * BN * 64;
-  static constexpr int nbars = 2 * NP + 2 * NU + 1;
-  static constexpr uint32_t misc = bars + nbars * 8;           // tmem slot, abort flag
-  static constexpr uint32_t col_scale = (misc + 16 + 15) & ~15u;
-  static constexpr uint32_t col_rowsum = col_scale + BN * 4;
-  static constexpr uint32_t rs_a = col_rowsum + BN * 4;
-  static constexpr uint32_t total = rs_a + BM * 4;
-  static constexpr size_t dyn_bytes = total + 1024;              // alignment slack
+  // full_p[NP] empty_p[NP] full_u[NU] empty_u[NU] acc_full[2] acc_empty[2] rs_full[2] rs_empty[2] drain
+  static constexpr int nbars = 2 * NP + 2 * NU + 9;
+  static constexpr uint32_t misc = bars + nbars * 8;   // tmem slot, abort flag
+  static constexpr uint32_t rs_a = (misc + 16 + 15) & ~15u;
+  static constexpr uint32_t total = rs_a + 2 * BM * 4;
+  static constexpr size_t dyn_bytes = total + 1024;
 };
 
-template <int BN, bool ASYM, bool ACC_OUT>
-__global__ void __launch_bounds__(256, 1)
+template <bool ASYM, bool ACC_OUT>
+__global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     GemmArgs args, int num_k) {
-  using L = Layout<BN>;
+                     GemmArgs args, int num_k, int m_tiles, int num_tiles) {
+  using L = Layout;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L::bars);
   uint64_t* full_p = bars;
-  uint64_t* empty_p = bars + NP;
-  uint64_t* full_u = bars + 2 * NP;
-  uint64_t* empty_u = bars + 2 * NP + NU;
-  uint64_t* acc_full = bars + 2 * NP + 2 * NU;
+  uint64_t* empty_p = full_p + NP;
+  uint64_t* full_u = empty_p + NP;
+  uint64_t* empty_u = full_u + NU;
+  uint64_t* acc_full = empty_u + NU;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* rs_full = acc_empty + 2;
+  uint64_t* rs_empty = rs_full + 2;
+  uint64_t* drain = rs_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + L::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + L::misc + 4);
-  float* col_scale = reinterpret_cast<float*>(base + L::col_scale);
-  int* col_rowsum = reinterpret_cast<int*>(base + L::col_rowsum);
   int* rs_a = reinterpret_cast<int*>(base + L::rs_a);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int64_t m0 = (int64_t)blockIdx.y * BM, n0 = (int64_t)blockIdx.x * BN;
 
   if (tid == 0) {
     for (int i = 0; i < NP; ++i) {
       mbar_init(&full_p[i], 1);
-      mbar_init(&empty_p[i], 4);
+      mbar_init(&empty_p[i], kUnpackWarps);
     }
     for (int i = 0; i < NU; ++i) {
-      mbar_init(&full_u[i], 4);
+      mbar_init(&full_u[i], kUnpackWarps);
       mbar_init(&empty_u[i], 1);
     }
-    mbar_init(acc_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], kEpiWarps);
+      mbar_init(&rs_full[i], kUnpackWarps);
+      mbar_init(&rs_empty[i], kEpiWarps);
+    }
+    mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, BN);
+    tmem_alloc(tmem_slot, 2 * BN);
     tmem_relinquish();
-  }
-  if (tid >= 128) {
-    for (int j = tid - 128; j < BN; j += 128) {
-      const int64_t n = n0 + j;
-      col_scale[j] = n < args.N ? args.w_scale[n] : 0.f;
-      col_rowsum[j] = n < args.N ? args.w_rowsum[n] : 0;
-    }
   }
   tc_fence_before();
   __syncthreads();
@@ -149,141 +161,202 @@ __global__ void __launch_bounds__(256, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
+    // ------------------------------------------------ TMA producer
     if (lane == 0) {
-      int issued = 0;
-      for (int kt = 0; kt < num_k; ++kt) {
-        const int s = kt % NP;
-        if (!wait_or_abort(&empty_p[s], ((kt / NP) & 1) ^ 1, abort_flag, 1)) break;
-        mbar_arrive_expect_tx(&full_p[s], (BM + BN) * 64);
-        tma_load_2d(base + L::pA + s * BM * 64, &tmA, &full_p[s], kt * 64, (int32_t)m0);
-        tma_load_2d(base + L::pB + s * BN * 64, &tmB, &full_p[s], kt * 64, (int32_t)n0);
-        issued = kt + 1;
+      int it = 0;
+      bool stop = false;
+      for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x) {
+        const int32_t m0 = (tile % m_tiles) * BM, n0 = (tile / m_tiles) * BN;
+        for (int kt = 0; kt < num_k; ++kt, ++it) {
+          const int s = it % NP;
+          if (!wait_or_abort(&empty_p[s], ((it / NP) & 1) ^ 1, abort_flag, 1)) {
+            stop = true;
+            break;
+          }
+          mbar_arrive_expect_tx(&full_p[s], (BM + BN) * 64);
+          tma_load_2d(base + L::pA + s * BM * 64, &tmA, &full_p[s], kt * 64, m0);
+          tma_load_2d(base + L::pB + s * BN * 64, &tmB, &full_p[s], kt * 64, n0);
+        }
       }
-      if (*abort_flag) {
-        // let the copies still in flight land before the CTA exits
-        for (int kt = issued - NP < 0 ? 0 : issued - NP; kt < issued; ++kt) {
+      if (stop) {
+        // let copies still in flight land before the CTA exits
+        for (int j = it - NP < 0 ? 0 : it - NP; j < it; ++j) {
           const uint64_t t0 = globaltimer_ns();
-          while (!mbar_try_wait(&full_p[kt % NP], (kt / NP) & 1) && globaltimer_ns() - t0 < kWaitLimitNs) {
+          while (!mbar_try_wait(&full_p[j % NP], (j / NP) & 1) && globaltimer_ns() - t0 < kWaitLimitNs) {
           }
         }
       }
     }
   } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = umma_idesc_e4m3_f32(BM, BN);
-      int kt = 0;
-      for (; kt < num_k; ++kt) {
-        const int su = kt % NU;
-        if (!wait_or_abort(&full_u[su], (kt / NU) & 1, abort_flag, 2)) break;
+      int it = 0, lt = 0;
+      bool stop = false;
+      for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x, ++lt) {
+        const int b = lt & 1;
+        if (!wait_or_abort(&acc_empty[b], ((lt >> 1) & 1) ^ 1, abort_flag, 2)) break;
         tc_fence_after();
-        const uint32_t a0 = smem_u32(base + L::uA + su * BM * 128);
-        const uint32_t b0 = smem_u32(base + L::uB + su * BN * 128);
+        const uint32_t d = tmem + (uint32_t)(b * BN);
+        for (int kt = 0; kt < num_k; ++kt, ++it) {
+          const int su = it % NU;
+          if (!wait_or_abort(&full_u[su], (it / NU) & 1, abort_flag, 3)) {
+            stop = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(base + L::uA + su * BM * 128);
+          const uint32_t b0 = smem_u32(base + L::uB + su * BN * 128);
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          tc_mma_f8f6f4(tmem, umma_desc_sw128(a0 + kk * 32), umma_desc_sw128(b0 + kk * 32), idesc,
-                        (kt | kk) != 0);
-        tc_commit(&empty_u[su]);
-      }
-      tc_commit(acc_full);
-      if (kt < num_k) {
-        // aborted: wait (bounded) until the issued MMAs have retired
-        const uint64_t t0 = globaltimer_ns();
-        while (!mbar_try_wait(acc_full, 0) && globaltimer_ns() - t0 < kWaitLimitNs) {
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_f8f6f4(d, umma_desc_sw128(a0 + kk * 32), umma_desc_sw128(b0 + kk * 32), idesc,
+                          (kt | kk) != 0);
+          tc_commit(&empty_u[su]);
         }
+        tc_commit(&acc_full[b]);
+      }
+      // every MMA issued by this thread has retired once `drain` fires, so the
+      // tensor memory can be released even when a role gave up early
+      tc_commit(drain);
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(drain, 0) && globaltimer_ns() - t0 < kWaitLimitNs) {
       }
     }
-  } else if (warp >= 4) {
-    const int u = tid - 128;
+  } else if (warp >= kFirstUnpackWarp) {
+    // ------------------------------------------------ unpack
+    const int u = tid - kFirstUnpackWarp * 32;   // 0..255
     const uint32_t xa = ASYM ? 0u : 0x88888888u;
-    int rsum[4] = {0, 0, 0, 0};
-    for (int kt = 0; kt < num_k; ++kt) {
-      const int s = kt % NP, su = kt % NU;
-      if (!wait_or_abort(&full_p[s], (kt / NP) & 1, abort_flag, 3)) break;
-      if (!wait_or_abort(&empty_u[su], ((kt / NU) & 1) ^ 1, abort_flag, 4)) break;
-      const uint8_t* PA = base + L::pA + s * BM * 64;
-      const uint8_t* PB = base + L::pB + s * BN * 64;
-      uint8_t* UA = base + L::uA + su * BM * 128;
-      uint8_t* UB = base + L::uB + su * BN * 128;
+    // fixed task assignment: 2 A chunks and 4 B chunks per thread per stage
+    uint32_t la[2], sa[2], ha[2], lb[4], sb[4], hb[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int i = u + 128 * j, r = i >> 2, ch = i & 3;
-        const uint4 w = *reinterpret_cast<const uint4*>(PA + r * 64 + ch * 16);
-        uint4 lo, hi;
-        unpack16(w, xa, lo, hi);
-        const uint32_t t = lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w;
-        rsum[j] = (int)__dp4a(t, 0x01010101u, (unsigned)rsum[j]);
-        *reinterpret_cast<uint4*>(UA + swz_off(r, 2 * ch)) = lo;
-        *reinterpret_cast<uint4*>(UA + swz_off(r, 2 * ch + 1)) = hi;
-      }
-#pragma unroll 4
-      for (int j = 0; j < BN / 32; ++j) {
-        const int i = u + 128 * j, r = i >> 2, ch = i & 3;
-        const uint4 w = *reinterpret_cast<const uint4*>(PB + r * 64 + ch * 16);
-        uint4 lo, hi;
-        unpack16(w, 0x88888888u, lo, hi);
-        *reinterpret_cast<uint4*>(UB + swz_off(r, 2 * ch)) = lo;
-        *reinterpret_cast<uint4*>(UB + swz_off(r, 2 * ch + 1)) = hi;
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&full_u[su]);
-        mbar_arrive(&empty_p[s]);
-      }
+    for (int j = 0; j < 2; ++j) {
+      const int i = u + 256 * j, r = i >> 2, ch = i & 3;
+      la[j] = r * 64 + ch * 16;
+      sa[j] = swz_off(r, 2 * ch);
+      ha[j] = swz_off(r, 2 * ch + 1);
     }
-    // row sums of the unsigned activation codes: lanes u..u^3 share a row
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      int v = rsum[j];
-      v += __shfl_xor_sync(0xffffffffu, v, 1);
-      v += __shfl_xor_sync(0xffffffffu, v, 2);
-      if ((u & 3) == 0) rs_a[(u >> 2) + 32 * j] = v;
+      const int i = u + 256 * j, r = i >> 2, ch = i & 3;
+      lb[j] = r * 64 + ch * 16;
+      sb[j] = swz_off(r, 2 * ch);
+      hb[j] = swz_off(r, 2 * ch + 1);
     }
-    asm volatile("bar.sync 1, 128;\n" ::: "memory");
-
-    // ---------------- epilogue ----------------
-    const bool ok = wait_or_abort(acc_full, 0, abort_flag, 5);
-    __syncwarp();
-    tc_fence_after();
+    const uint32_t sbase = smem_u32(base);
+    int it = 0, lt = 0;
+    bool stop = false;
+    for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x, ++lt) {
+      int rsum0 = 0, rsum1 = 0;
+      for (int kt = 0; kt < num_k; ++kt, ++it) {
+        const int s = it % NP, su = it % NU;
+        if (!wait_or_abort(&full_p[s], (it / NP) & 1, abort_flag, 4) ||
+            !wait_or_abort(&empty_u[su], ((it / NU) & 1) ^ 1, abort_flag, 5)) {
+          stop = true;
+          break;
+        }
+        const uint32_t PA = sbase + L::pA + s * BM * 64, PB = sbase + L::pB + s * BN * 64;
+        const uint32_t UA = sbase + L::uA + su * BM * 128, UB = sbase + L::uB + su * BN * 128;
+        uint4 wa0 = lds128(PA + la[0]), wa1 = lds128(PA + la[1]);
+        uint4 wb[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) wb[j] = lds128(PB + lb[j]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_p[s]);   // packed stage consumed
+        uint4 lo, hi;
+        unpack16(wa0, xa, lo, hi);
+        rsum0 = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u, (unsigned)rsum0);
+        sts128(UA + sa[0], lo);
+        sts128(UA + ha[0], hi);
+        unpack16(wa1, xa, lo, hi);
+        rsum1 = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u, (unsigned)rsum1);
+        sts128(UA + sa[1], lo);
+        sts128(UA + ha[1], hi);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          unpack16(wb[j], 0x88888888u, lo, hi);
+          sts128(UB + sb[j], lo);
+          sts128(UB + hb[j], hi);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&full_u[su]);
+      }
+      if (stop) break;
+      // row sums of the unsigned activation codes: 4 lanes share a row
+      rsum0 += __shfl_xor_sync(0xffffffffu, rsum0, 1);
+      rsum0 += __shfl_xor_sync(0xffffffffu, rsum0, 2);
+      rsum1 += __shfl_xor_sync(0xffffffffu, rsum1, 1);
+      rsum1 += __shfl_xor_sync(0xffffffffu, rsum1, 2);
+      const int b = lt & 1;
+      if (!wait_or_abort(&rs_empty[b], ((lt >> 1) & 1) ^ 1, abort_flag, 6)) break;
+      if ((u & 3) == 0) {
+        rs_a[b * BM + (u >> 2)] = rsum0;
+        rs_a[b * BM + (u >> 2) + 64] = rsum1;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&rs_full[b]);
+    }
+  } else if (warp >= kFirstEpiWarp && warp < kFirstEpiWarp + kEpiWarps) {
+    // ------------------------------------------------ epilogue
     const int q = warp & 3;
     const int row = q * 32 + lane;
-    const int64_t m = m0 + row;
-    const bool mvalid = ok && !*abort_flag && m < args.M;
-    float alpha = 0.f, bp = 0.f;
-    if (mvalid) {
-      alpha = args.a_scale[m];
-      if (ASYM) bp = args.a_zero[m] + 8.f * alpha;
-    }
-    const int rsa8 = 8 * rs_a[row];
-    __half* yrow = reinterpret_cast<__half*>(args.y) + m * args.N;
+    int lt = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
+      const int b = lt & 1;
+      const int64_t m = (int64_t)(tile % m_tiles) * BM + row;
+      const int64_t n0 = (int64_t)(tile / m_tiles) * BN;
+      bool ok = wait_or_abort(&acc_full[b], (lt >> 1) & 1, abort_flag, 7);
+      ok = ok && wait_or_abort(&rs_full[b], (lt >> 1) & 1, abort_flag, 8);
+      __syncwarp();
+      if (!ok) break;
+      tc_fence_after();
+      const int rsa8 = 8 * rs_a[b * BM + row];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&rs_empty[b]);
+      const bool mvalid = m < args.M;
+      float alpha = 0.f, bp = 0.f;
+      if (mvalid) {
+        alpha = __ldg(args.a_scale + m);
+        if (ASYM) bp = __ldg(args.a_zero + m) + 8.f * alpha;
+      }
+      __half* yrow = reinterpret_cast<__half*>(args.y) + m * args.N;
 #pragma unroll 1
-    for (int cc = 0; cc < BN / 32; ++cc) {
-      uint32_t r[32];
-      tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(cc * 32), r);
-      tmem_ld_wait();
-      if (!mvalid) continue;
-#pragma unroll
-      for (int g8 = 0; g8 < 4; ++g8) {
-        const int64_t n = n0 + cc * 32 + g8 * 8;
-        if (n >= args.N) break;
-        uint32_t h[4];
-        int accs[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int j = cc * 32 + g8 * 8 + e;
-          const int S = __float2int_rn(__uint_as_float(r[g8 * 8 + e]) * 262144.0f);
-          const int rsw = col_rowsum[j];
-          const int acc = S - rsa8 - 8 * rsw;
-          accs[e] = acc;
-          const float yv = col_scale[j] * fmaf(alpha, (float)acc, bp * (float)rsw);
-          if (e & 1) h[e >> 1] = pack_half2_bits(__uint_as_float(h[e >> 1]), yv);
-          else h[e >> 1] = __float_as_uint(yv);
+      for (int cc = 0; cc < BN / 32; ++cc) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN + cc * 32), r);
+        tmem_ld_wait();
+        if (cc == BN / 32 - 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[b]);   // accumulator buffer free again
         }
-        *reinterpret_cast<uint4*>(yrow + n) = make_uint4(h[0], h[1], h[2], h[3]);
-        if (ACC_OUT) {
-          int4* ap = reinterpret_cast<int4*>(args.acc_out + m * args.N + n);
-          ap[0] = make_int4(accs[0], accs[1], accs[2], accs[3]);
-          ap[1] = make_int4(accs[4], accs[5], accs[6], accs[7]);
+#pragma unroll
+        for (int g8 = 0; g8 < 4; ++g8) {
+          const int64_t n = n0 + cc * 32 + g8 * 8;
+          if (!mvalid || n >= args.N) continue;
+          const float4 s0 = __ldg(reinterpret_cast<const float4*>(args.w_scale + n));
+          const float4 s1 = __ldg(reinterpret_cast<const float4*>(args.w_scale + n) + 1);
+          const int4 q0 = __ldg(reinterpret_cast<const int4*>(args.w_rowsum + n));
+          const int4 q1 = __ldg(reinterpret_cast<const int4*>(args.w_rowsum + n) + 1);
+          const float sc[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+          const int rw[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+          float yv[8];
+          int accs[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int S = __float2int_rn(__uint_as_float(r[g8 * 8 + e]) * 262144.0f);
+            const int acc = S - rsa8 - 8 * rw[e];
+            accs[e] = acc;
+            yv[e] = sc[e] * fmaf(alpha, (float)acc, bp * (float)rw[e]);
+          }
+          *reinterpret_cast<uint4*>(yrow + n) =
+              make_uint4(pack_half2_bits(yv[0], yv[1]), pack_half2_bits(yv[2], yv[3]),
+                         pack_half2_bits(yv[4], yv[5]), pack_half2_bits(yv[6], yv[7]));
+          if (ACC_OUT) {
+            int4* ap = reinterpret_cast<int4*>(args.acc_out + m * args.N + n);
+            ap[0] = make_int4(accs[0], accs[1], accs[2], accs[3]);
+            ap[1] = make_int4(accs[4], accs[5], accs[6], accs[7]);
+          }
         }
       }
     }
@@ -294,7 +367,7 @@ __global__ void __launch_bounds__(256, 1)
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem, BN);
+    tmem_dealloc(tmem, 2 * BN);
   }
 }
 
@@ -333,37 +406,32 @@ bool encode_packed_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t 
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, bool ASYM, bool ACC_OUT>
+template <bool ASYM, bool ACC_OUT>
 cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   CUtensorMap tmA, tmB;
   if (!encode_packed_map(&tmA, a.a_codes, a.M, a.K, BM)) return cudaErrorNotSupported;
   if (!encode_packed_map(&tmB, a.w_codes, a.N, a.K, BN)) return cudaErrorNotSupported;
-  auto kern = w4a4_gemm_kernel<BN, ASYM, ACC_OUT>;
-  const size_t smem = Layout<BN>::dyn_bytes;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto kern = w4a4_gemm_kernel<ASYM, ACC_OUT>;
+  const size_t smem = Layout::dyn_bytes;
+  int per_sm = 0;
+  cudaError_t e = prepare_launch(kern, kThreads, smem, &per_sm);
   if (e != cudaSuccess) return e;
-  dim3 grid((unsigned)((a.N + BN - 1) / BN), (unsigned)((a.M + BM - 1) / BM));
-  kern<<<grid, 256, smem, stream>>>(tmA, tmB, a, (int)(a.K / 128));
+  const int sms = device_sm_count();
+  const int m_tiles = (int)((a.M + BM - 1) / BM);
+  const int n_tiles = (int)((a.N + BN - 1) / BN);
+  const int tiles = m_tiles * n_tiles;
+  const int grid = tiles < sms ? tiles : sms;
+  kern<<<grid, kThreads, smem, stream>>>(tmA, tmB, a, (int)(a.K / 128), m_tiles, tiles);
   return cudaGetLastError();
-}
-
-template <int BN>
-cudaError_t launch_bn(const GemmArgs& a, cudaStream_t stream) {
-  const bool asym = a.a_zero != nullptr, acc = a.acc_out != nullptr;
-  if (asym) return acc ? launch_t<BN, true, true>(a, stream) : launch_t<BN, true, false>(a, stream);
-  return acc ? launch_t<BN, false, true>(a, stream) : launch_t<BN, false, false>(a, stream);
 }
 
 }  // namespace
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t tiles256 = ((a.N + 255) / 256) * ((a.M + BM - 1) / BM);
-  if (tiles256 >= sms) return launch_bn<256>(a, stream);
-  return launch_bn<128>(a, stream);
+  const bool asym = a.a_zero != nullptr, acc = a.acc_out != nullptr;
+  if (asym) return acc ? launch_t<true, true>(a, stream) : launch_t<true, false>(a, stream);
+  return acc ? launch_t<false, true>(a, stream) : launch_t<false, false>(a, stream);
 }
 
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail) {
