@@ -184,6 +184,8 @@ cudaError_t launch_rotate_quant_rows(const RotQuantArgs& a, cudaStream_t stream)
   bool handled = false;
   cudaError_t e = launch_rotate_quant_act_fast(a, stream, &handled);
   if (handled || e != cudaSuccess) return e;
+  e = launch_rotate_quant_act_paley(a, stream, &handled);
+  if (handled || e != cudaSuccess) return e;
   const bool clamp = a.clip < 1.0f;
   if (a.symmetric) {
     if (a.rowsum) return clamp ? launch_t<true, true, true>(a, stream) : launch_t<true, true, false>(a, stream);

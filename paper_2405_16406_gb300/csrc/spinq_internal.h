@@ -42,6 +42,10 @@ cudaError_t launch_rotate_quant_rows(const RotQuantArgs& a, cudaStream_t stream)
 // 512..16384).  Sets *handled = false when the shape has no such kernel.
 cudaError_t launch_rotate_quant_act_fast(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
 
+// Activation kernel for a Paley factor (n_small in {12, 20, 28}, n_pow2 in
+// {128, 256, 512}).  Sets *handled = false for other shapes.
+cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
+
 struct KVArgs {
   const void* q_in;
   void* q_out;

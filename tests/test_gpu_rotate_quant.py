@@ -61,7 +61,9 @@ def test_act_full_configs(S, name, builder, kw):
     check_act(S, c.x, c.had, c.act_symmetric, c.clip, name)
 
 
-@pytest.mark.parametrize("had", [None, (1, 32), (1, 1024), (12, 64), (20, 128), (28, 64), (1, 16384)])
+@pytest.mark.parametrize("had", [None, (1, 32), (1, 256), (1, 512), (1, 1024), (1, 2048), (1, 4096), (1, 8192),
+                                 (1, 16384), (12, 64), (12, 128), (12, 256), (12, 512), (20, 128), (20, 256),
+                                 (20, 512), (28, 64), (28, 128), (28, 256), (28, 512)])
 @pytest.mark.parametrize("symmetric", [True, False])
 def test_act_shapes_and_modes(S, had, symmetric):
     K = 4096 if had is None else had[0] * had[1]
@@ -89,12 +91,14 @@ def test_act_degenerate_rows(S):
             check_act(S, x, had, sym, 1.0, f"degenerate sym={sym} had={had}")
 
 
-def test_act_strided_rows(S):
+@pytest.mark.parametrize("had", [None, (1, 512), (12, 256)])
+def test_act_strided_rows(S, had):
+    K = 4096 if had is None else had[0] * had[1]
     rng = np.random.default_rng(1)
-    big = synth.activations(rng, 19, 512 + 64, outlier_frac=0.01, factor=10.0)
-    x = torch.from_numpy(big).cuda()[:, :512]
-    out = S.rotate_quant_act(x, (1, 512), True, 1.0)
-    ref = oracle.rotate_quant_act(np.ascontiguousarray(big[:, :512]), (1, 512), 4, True, 1.0)
+    big = synth.activations(rng, 19, K + 64, outlier_frac=0.01, factor=10.0)
+    x = torch.from_numpy(big).cuda()[:, :K]
+    out = S.rotate_quant_act(x, had, True, 1.0)
+    ref = oracle.rotate_quant_act(np.ascontiguousarray(big[:, :K]), had, 4, True, 1.0)
     pu.assert_codes_close(pu.gpu_codes(out.codes.cpu().numpy(), True), ref.codes, "strided")
 
 
