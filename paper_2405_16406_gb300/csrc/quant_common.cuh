@@ -78,4 +78,69 @@ struct QParams {
   }
 };
 
+// ---------------------------------------------------------------------------
+// RowStream: rows of a row-major fp16 matrix streamed into shared memory with
+// TMA bulk copies, NST rows ahead, for a CTA that walks rows r0, r0 + G, ...
+// Thread 0 issues; every thread waits.  A stage is refilled (release) once
+// the CTA has read it.  Waits are bounded in time and set `*abort` on expiry.
+// ---------------------------------------------------------------------------
+template <int NST>
+struct RowStream {
+  uint8_t* stage0;      // NST stages of `stage_bytes`
+  uint32_t stage_bytes;
+  uint64_t* bars;       // NST mbarriers
+  const uint8_t* src;   // matrix base
+  int64_t row_bytes;    // pitch
+  uint32_t copy_bytes;  // bytes copied per row (multiple of 16)
+  int64_t rows, r0, G;
+  int issued;           // iterations issued so far (thread 0)
+
+  __device__ __forceinline__ void init() {
+    if (threadIdx.x == 0)
+      for (int s = 0; s < NST; ++s) mbar_init(&bars[s], 1);
+  }
+  __device__ __forceinline__ void issue(int iter) {
+    const int64_t row = r0 + (int64_t)iter * G;
+    if (row >= rows) return;
+    const int s = iter % NST;
+    fence_proxy_async_smem();
+    mbar_arrive_expect_tx(&bars[s], copy_bytes);
+    bulk_load(stage0 + (size_t)s * stage_bytes, src + row * row_bytes, copy_bytes, &bars[s]);
+    issued = iter + 1;
+  }
+  // thread 0, after init() and a CTA barrier
+  __device__ __forceinline__ void prologue() {
+    issued = 0;
+    if (threadIdx.x == 0)
+      for (int i = 0; i < NST; ++i) issue(i);
+  }
+  __device__ __forceinline__ uint8_t* stage(int iter) const { return stage0 + (size_t)(iter % NST) * stage_bytes; }
+  // every thread; false on timeout or abort
+  __device__ __forceinline__ bool wait(int iter, volatile int* abort, uint64_t limit_ns) {
+    const uint32_t par = (uint32_t)(iter / NST) & 1u;
+    if (mbar_try_wait(&bars[iter % NST], par)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(&bars[iter % NST], par)) {
+      if (*abort || globaltimer_ns() - t0 > limit_ns) {
+        *abort = 1;
+        return false;
+      }
+    }
+    return true;
+  }
+  // thread 0, after the CTA has finished reading stage(iter)
+  __device__ __forceinline__ void release(int iter) {
+    if (threadIdx.x == 0) issue(iter + NST);
+  }
+  // thread 0: let copies in flight land before the CTA exits (abort path)
+  __device__ __forceinline__ void drain(int iter, uint64_t limit_ns) {
+    if (threadIdx.x != 0) return;
+    for (int j = iter; j < issued; ++j) {
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(&bars[j % NST], (j / NST) & 1) && globaltimer_ns() - t0 < limit_ns) {
+      }
+    }
+  }
+};
+
 }  // namespace spinq

@@ -97,15 +97,42 @@ __device__ __forceinline__ uint32_t swz_word(uint32_t p) {
   return ((q ^ x) << 2) | (p & 3u);
 }
 
+constexpr uint64_t kRowWaitLimitNs = 2000000000ull;
+
+template <int LW, int L>
+struct Pow2Smem {
+  using S = Pow2Shape<LW, L>;
+  static constexpr int NST = S::P >= 4096 ? 1 : 2;     // fp16 rows staged ahead
+  static constexpr int OFF_F32 = 0;                     // P floats (transpose)
+  static constexpr int OFF_STAGE = S::P * 4;
+  static constexpr int OFF_BAR = OFF_STAGE + NST * S::P * 2;
+  static constexpr int OFF_MISC = OFF_BAR + NST * 8;   // abort flag + range scratch
+  static constexpr int BYTES = OFF_MISC + 16 + 2 * S::W * 4;
+};
+
 template <int LW, int L, bool SYM, bool CLAMP>
 __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
   using S = Pow2Shape<LW, L>;
-  extern __shared__ __align__(16) float sm[];
-  __shared__ float red[2 * S::W];
+  using SM = Pow2Smem<LW, L>;
+  extern __shared__ __align__(128) uint8_t smem[];
+  float* sm = reinterpret_cast<float*>(smem + SM::OFF_F32);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + SM::OFF_MISC);
+  float* red = reinterpret_cast<float*>(smem + SM::OFF_MISC + 16);
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   uint32_t bh[2][2];
   make_b16(bh, true);
-  const __half* __restrict__ x = reinterpret_cast<const __half*>(a.x);
+
+  RowStream<SM::NST> rs{smem + SM::OFF_STAGE, (uint32_t)(S::P * 2),
+                        reinterpret_cast<uint64_t*>(smem + SM::OFF_BAR),
+                        reinterpret_cast<const uint8_t*>(a.x), a.ldx * 2, (uint32_t)(S::P * 2),
+                        a.rows, (int64_t)blockIdx.x, (int64_t)gridDim.x, 0};
+  rs.init();
+  if (tid == 0) {
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  rs.prologue();
 
   // phase-2 fixed element bits of this thread
   const uint32_t t_lo = (uint32_t)tid & ((1u << (3 - L)) - 1u);
@@ -113,15 +140,16 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
   const uint32_t t_v = (uint32_t)tid >> (5 - L);
   const uint32_t fixed = (t_lo << L) | (t_c << 3) | (t_v << (8 + LW));
 
-  for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x) {
-    const uint4* src = reinterpret_cast<const uint4*>(x + row * a.ldx);
+  int it = 0;
+  for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x, ++it) {
+    rs.wait(it, abort_flag, kRowWaitLimitNs);
+    __syncthreads();
+    if (*abort_flag) break;
     // ---------------- phase 1
-    uint4 in[S::V];
-#pragma unroll
-    for (int v = 0; v < S::V; ++v) in[v] = __ldg(src + lane + 32 * (w + S::W * v));
+    const uint4* src = reinterpret_cast<const uint4*>(rs.stage(it));
     float y[S::V][8];
 #pragma unroll
-    for (int v = 0; v < S::V; ++v) chunk_mma(in[v], bh, y[v]);
+    for (int v = 0; v < S::V; ++v) chunk_mma(src[lane + 32 * (w + S::W * v)], bh, y[v]);
 #pragma unroll
     for (int v = 0; v < S::V; ++v)
 #pragma unroll
@@ -149,6 +177,7 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
       *reinterpret_cast<float4*>(sm + swz_word<LW>(p + 4)) = make_float4(y[v][4], y[v][5], y[v][6], y[v][7]);
     }
     __syncthreads();
+    rs.release(it);  // the staged row is consumed: the next copy overlaps phase 2
 
     // ---------------- phase 2
     float z[S::NG][S::GL];
@@ -204,8 +233,9 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
       a.scale[row] = qp.alpha * a.norm;
       if (!SYM) a.zero[row] = qp.beta * a.norm;
     }
-    __syncthreads();  // the row buffer and `red` are reused by the next row
+    __syncthreads();  // the transpose buffer and `red` are reused by the next row
   }
+  if (*abort_flag) rs.drain(it, kRowWaitLimitNs);
 }
 
 // ------------------------------------------------------------------------
@@ -213,31 +243,51 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
 // ------------------------------------------------------------------------
 constexpr int kNoRotV = 8;
 
+constexpr int kNoRotStages = 2;
+
 template <bool SYM, bool CLAMP, int W>
 __global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
-  __shared__ float red[2 * W];
+  extern __shared__ __align__(128) uint8_t smem[];
+  const uint32_t row_bytes = (uint32_t)(a.K * 2);
+  const uint32_t stage_bytes = (row_bytes + 127u) & ~127u;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kNoRotStages * stage_bytes);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + kNoRotStages);
+  float* red = reinterpret_cast<float*>(smem + kNoRotStages * stage_bytes + kNoRotStages * 8 + 16);
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   uint32_t bi[2][2];
   make_b16(bi, false);
   const int nchunk = (int)(a.K / 8);
-  const __half* __restrict__ x = reinterpret_cast<const __half*>(a.x);
-  for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x) {
-    const uint4* src = reinterpret_cast<const uint4*>(x + row * a.ldx);
-    uint4 in[kNoRotV];
+
+  RowStream<kNoRotStages> rs{smem, stage_bytes, bars, reinterpret_cast<const uint8_t*>(a.x), a.ldx * 2,
+                             row_bytes, a.rows, (int64_t)blockIdx.x, (int64_t)gridDim.x, 0};
+  rs.init();
+  if (tid == 0) {
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  rs.prologue();
+
+  int it = 0;
+  for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x, ++it) {
+    rs.wait(it, abort_flag, kRowWaitLimitNs);
+    __syncthreads();
+    if (*abort_flag) break;
+    const uint4* src = reinterpret_cast<const uint4*>(rs.stage(it));
+    float y[kNoRotV][8];
 #pragma unroll
     for (int v = 0; v < kNoRotV; ++v) {
       const int ch = lane + 32 * (w + W * v);
-      in[v] = ch < nchunk ? __ldg(src + ch) : make_uint4(0, 0, 0, 0);
+      chunk_mma(ch < nchunk ? src[ch] : make_uint4(0, 0, 0, 0), bi, y[v]);  // exact fp16 -> fp32
     }
-    float y[kNoRotV][8];
+    __syncthreads();
+    rs.release(it);
     Range<SYM> r;
 #pragma unroll
-    for (int v = 0; v < kNoRotV; ++v) {
-      chunk_mma(in[v], bi, y[v]);  // exact fp16 -> fp32
+    for (int v = 0; v < kNoRotV; ++v)
       if (lane + 32 * (w + W * v) < nchunk)
 #pragma unroll
         for (int e = 0; e < 8; ++e) r.add(y[v][e]);
-    }
     block_range<SYM, W>(r, red);
     const QParams<SYM> qp(r, a.clip);
     uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
@@ -255,6 +305,7 @@ __global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
     }
     if (W > 1) __syncthreads();
   }
+  if (*abort_flag) rs.drain(it, kRowWaitLimitNs);
 }
 
 template <typename Kern>
@@ -271,7 +322,7 @@ cudaError_t launch_rows(Kern kern, int threads, size_t smem, const RotQuantArgs&
 template <int LW, int L, bool SYM, bool CLAMP>
 cudaError_t launch_pow2(const RotQuantArgs& a, cudaStream_t stream) {
   using S = Pow2Shape<LW, L>;
-  return launch_rows(rq_pow2_kernel<LW, L, SYM, CLAMP>, S::T, sizeof(float) * S::P, a, stream);
+  return launch_rows(rq_pow2_kernel<LW, L, SYM, CLAMP>, S::T, Pow2Smem<LW, L>::BYTES, a, stream);
 }
 
 template <bool SYM, bool CLAMP>
@@ -293,12 +344,13 @@ template <bool SYM, bool CLAMP>
 cudaError_t launch_norot_for(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
   const int64_t nchunk = a.K / 8;
   const int64_t warps = (nchunk + 32 * kNoRotV - 1) / (32 * kNoRotV);
+  const size_t smem = kNoRotStages * (((size_t)a.K * 2 + 127) & ~(size_t)127) + kNoRotStages * 8 + 16 + 2 * 16 * 4;
   *handled = true;
-  if (warps <= 1) return launch_rows(rq_norot_kernel<SYM, CLAMP, 1>, 32, 0, a, stream);
-  if (warps <= 2) return launch_rows(rq_norot_kernel<SYM, CLAMP, 2>, 64, 0, a, stream);
-  if (warps <= 4) return launch_rows(rq_norot_kernel<SYM, CLAMP, 4>, 128, 0, a, stream);
-  if (warps <= 8) return launch_rows(rq_norot_kernel<SYM, CLAMP, 8>, 256, 0, a, stream);
-  if (warps <= 16) return launch_rows(rq_norot_kernel<SYM, CLAMP, 16>, 512, 0, a, stream);
+  if (warps <= 1) return launch_rows(rq_norot_kernel<SYM, CLAMP, 1>, 32, smem, a, stream);
+  if (warps <= 2) return launch_rows(rq_norot_kernel<SYM, CLAMP, 2>, 64, smem, a, stream);
+  if (warps <= 4) return launch_rows(rq_norot_kernel<SYM, CLAMP, 4>, 128, smem, a, stream);
+  if (warps <= 8) return launch_rows(rq_norot_kernel<SYM, CLAMP, 8>, 256, smem, a, stream);
+  if (warps <= 16) return launch_rows(rq_norot_kernel<SYM, CLAMP, 16>, 512, smem, a, stream);
   *handled = false;
   return cudaSuccess;
 }

@@ -48,7 +48,10 @@ struct PaleyShape {
   static constexpr int PS = P + 4;                 // fp32 row stride
   static constexpr int SEGB = 2 * P + 16;          // staged fp16 segment stride (bytes)
   static constexpr int ROWB = NS * SEGB;           // staged row (bytes)
-  static constexpr int NST = NS * P >= 8192 ? 3 : 4;   // rows in flight
+  // rows in flight: one staged row for the large shapes so that two CTAs fit
+  // on an SM; the next row is requested as soon as phase 1 has consumed the
+  // current one, so its copy overlaps phase 2
+  static constexpr int NST = NS * P >= 8192 ? 1 : 2;
   // shared memory layout (bytes)
   static constexpr int OFF_STAGE = 0;
   static constexpr int OFF_ZERO = NST * ROWB;
@@ -59,7 +62,7 @@ struct PaleyShape {
 };
 
 template <int NS, int LP, bool SYM, bool CLAMP>
-__global__ void __launch_bounds__(32 * ((1 << LP) / 64)) rq_paley_kernel(RotQuantArgs a) {
+__global__ void __launch_bounds__(32 * ((1 << LP) / 64), 16 / ((1 << LP) / 64)) rq_paley_kernel(RotQuantArgs a) {
   using S = PaleyShape<NS, LP>;
   constexpr int P = S::P, W = S::W;
   extern __shared__ __align__(128) uint8_t smem[];
@@ -110,7 +113,7 @@ __global__ void __launch_bounds__(32 * ((1 << LP) / 64)) rq_paley_kernel(RotQuan
   };
   int issued = 0;  // iterations whose row copy has been issued (thread 0 only)
   if (tid == 0) {
-    for (int s = 0; s < S::NST - 1; ++s)
+    for (int s = 0; s < S::NST; ++s)
       if (r0 + s * G < a.rows) {
         issue(r0 + s * G, s);
         issued = s + 1;
@@ -122,13 +125,6 @@ __global__ void __launch_bounds__(32 * ((1 << LP) / 64)) rq_paley_kernel(RotQuan
   int it = 0;
   for (int64_t row = r0; row < a.rows; row += G, ++it) {
     const int st = it % S::NST;
-    if (tid == 0) {
-      const int64_t nxt = row + (int64_t)(S::NST - 1) * G;
-      if (nxt < a.rows) {
-        issue(nxt, (it + S::NST - 1) % S::NST);
-        issued = it + S::NST;
-      }
-    }
     // wait for this row (bounded)
     {
       bool ok = mbar_try_wait(&full[st], (it / S::NST) & 1);
@@ -208,6 +204,14 @@ __global__ void __launch_bounds__(32 * ((1 << LP) / 64)) rq_paley_kernel(RotQuan
         }
       }
     __syncthreads();
+    // the staged row is consumed: request the row NST iterations ahead into it
+    if (tid == 0) {
+      const int64_t nxt = row + (int64_t)S::NST * G;
+      if (nxt < a.rows) {
+        issue(nxt, st);
+        issued = it + S::NST + 1;
+      }
+    }
 
     // ---------------- phase 2
     float z[S::NCB][W][8];

@@ -18,7 +18,7 @@
 //
 // Persistent kernel: one CTA per SM walks the output tiles (128 x 256, M
 // fastest so that concurrently running CTAs share weight tiles in L2).  Warp
-// roles (448 threads):
+// roles (704 threads):
 //   warp 0       TMA producer: packed A [128 x 64 B] and B [256 x 64 B] tiles
 //                for one K step of 128, ring of NP stages.
 //   warp 1       TMEM allocation (2 x 256 fp32 columns) and the single-thread
@@ -27,8 +27,10 @@
 //   warps 2..5   epilogue, one TMEM lane quadrant each (warp % 4): tcgen05.ld
 //                of a finished accumulator, integer recovery, scales, fp16
 //                stores; runs while the MMA fills the other buffer.
-//   warps 6..13  unpack the packed tiles into the 128-byte-swizzled K-major
-//                E4M3 operand tiles (ring of NU stages) and count sum_k u_a.
+//   warps 6..21  unpack the packed tiles into the 128-byte-swizzled K-major
+//                E4M3 operand tiles (ring of NU stages) and count sum_k u_a;
+//                two groups of 8 warps take alternate K stages so that one
+//                group's barrier and fence latency overlaps the other's work.
 // Every mbarrier wait is bounded in time; a wait that gives up records
 // SPINQ_ETIMEOUT in the device status word and every role winds down.
 #include <cuda.h>
@@ -52,9 +54,10 @@ constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int NP = 3;   // packed (TMA) stages
 constexpr int NU = 3;   // unpacked (MMA operand) stages
-constexpr int kUnpackWarps = 8;
+constexpr int kUnpackWarps = 8;   // per group; two groups take alternate K stages
+constexpr int kUnpackGroups = 2;
 constexpr int kEpiWarps = 4;
-constexpr int kThreads = (6 + kUnpackWarps) * 32;
+constexpr int kThreads = (6 + kUnpackGroups * kUnpackWarps) * 32;
 constexpr int kFirstUnpackWarp = 6;
 constexpr int kFirstEpiWarp = 2;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
@@ -103,7 +106,7 @@ struct Layout {
   static constexpr int nbars = 2 * NP + 2 * NU + 9;
   static constexpr uint32_t misc = bars + nbars * 8;   // tmem slot, abort flag
   static constexpr uint32_t rs_a = (misc + 16 + 15) & ~15u;
-  static constexpr uint32_t total = rs_a + 2 * BM * 4;
+  static constexpr uint32_t total = rs_a + 2 * kUnpackGroups * BM * 4;
   static constexpr size_t dyn_bytes = total + 1024;
 };
 
@@ -142,7 +145,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], kEpiWarps);
-      mbar_init(&rs_full[i], kUnpackWarps);
+      mbar_init(&rs_full[i], kUnpackGroups * kUnpackWarps);
       mbar_init(&rs_empty[i], kEpiWarps);
     }
     mbar_init(drain, 1);
@@ -223,8 +226,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp >= kFirstUnpackWarp) {
-    // ------------------------------------------------ unpack
-    const int u = tid - kFirstUnpackWarp * 32;   // 0..255
+    // ------------------------------------------------ unpack (group grp takes stages it % 2 == grp)
+    const int grp = (warp - kFirstUnpackWarp) / kUnpackWarps;
+    const int u = tid - (kFirstUnpackWarp + grp * kUnpackWarps) * 32;   // 0..255
     const uint32_t xa = ASYM ? 0u : 0x88888888u;
     // fixed task assignment: 2 A chunks and 4 B chunks per thread per stage
     uint32_t la[2], sa[2], ha[2], lb[4], sb[4], hb[4];
@@ -248,6 +252,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x, ++lt) {
       int rsum0 = 0, rsum1 = 0;
       for (int kt = 0; kt < num_k; ++kt, ++it) {
+        if ((it & 1) != grp) continue;
         const int s = it % NP, su = it % NU;
         if (!wait_or_abort(&full_p[s], (it / NP) & 1, abort_flag, 4) ||
             !wait_or_abort(&empty_u[su], ((it / NU) & 1) ^ 1, abort_flag, 5)) {
@@ -290,8 +295,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int b = lt & 1;
       if (!wait_or_abort(&rs_empty[b], ((lt >> 1) & 1) ^ 1, abort_flag, 6)) break;
       if ((u & 3) == 0) {
-        rs_a[b * BM + (u >> 2)] = rsum0;
-        rs_a[b * BM + (u >> 2) + 64] = rsum1;
+        rs_a[(b * kUnpackGroups + grp) * BM + (u >> 2)] = rsum0;
+        rs_a[(b * kUnpackGroups + grp) * BM + (u >> 2) + 64] = rsum1;
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&rs_full[b]);
@@ -310,15 +315,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (!ok) break;
       tc_fence_after();
-      const int rsa8 = 8 * rs_a[b * BM + row];
+      const int rsa = rs_a[(b * kUnpackGroups) * BM + row] + rs_a[(b * kUnpackGroups + 1) * BM + row];
       __syncwarp();
       if (lane == 0) mbar_arrive(&rs_empty[b]);
       const bool mvalid = m < args.M;
+      // y = s_n (alpha (S - 8 rs_a - 8 rw_n) + beta' rw_n), S = acc * 2^18, evaluated as
+      // y = s_n * fma(alpha * 2^18, acc, c + d * rw_n), c = -8 alpha rs_a, d = beta' - 8 alpha
       float alpha = 0.f, bp = 0.f;
       if (mvalid) {
         alpha = __ldg(args.a_scale + m);
         if (ASYM) bp = __ldg(args.a_zero + m) + 8.f * alpha;
       }
+      const float alpha_s = alpha * 262144.0f;
+      const float cm = -8.f * alpha * (float)rsa;
+      const float dm = bp - 8.f * alpha;
       __half* yrow = reinterpret_cast<__half*>(args.y) + m * args.N;
 #pragma unroll 1
       for (int cc = 0; cc < BN / 32; ++cc) {
@@ -341,18 +351,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float sc[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
           const int rw[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
           float yv[8];
-          int accs[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
-            const int S = __float2int_rn(__uint_as_float(r[g8 * 8 + e]) * 262144.0f);
-            const int acc = S - rsa8 - 8 * rw[e];
-            accs[e] = acc;
-            yv[e] = sc[e] * fmaf(alpha, (float)acc, bp * (float)rw[e]);
+            const float acc = __uint_as_float(r[g8 * 8 + e]);
+            yv[e] = sc[e] * fmaf(alpha_s, acc, fmaf(dm, (float)rw[e], cm));
           }
           *reinterpret_cast<uint4*>(yrow + n) =
               make_uint4(pack_half2_bits(yv[0], yv[1]), pack_half2_bits(yv[2], yv[3]),
                          pack_half2_bits(yv[4], yv[5]), pack_half2_bits(yv[6], yv[7]));
           if (ACC_OUT) {
+            int accs[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              accs[e] = __float2int_rn(__uint_as_float(r[g8 * 8 + e]) * 262144.0f) - 8 * rsa - 8 * rw[e];
             int4* ap = reinterpret_cast<int4*>(args.acc_out + m * args.N + n);
             ap[0] = make_int4(accs[0], accs[1], accs[2], accs[3]);
             ap[1] = make_int4(accs[4], accs[5], accs[6], accs[7]);
