@@ -16,8 +16,9 @@
 // (sum_k u_w = rowsum_n + 8 K cancels the 64 K term).  sum_k u_a is counted
 // by the unpack warps while they expand the activation tiles.
 //
-// Persistent kernel: one CTA per SM walks the output tiles (128 x 256, M
-// fastest so that concurrently running CTAs share weight tiles in L2).  Warp
+// Persistent kernel: one CTA per SM walks the output tiles (128 x 256 or
+// 256 x 256, M fastest so that concurrently running CTAs share weight tiles
+// in L2).  Warp
 // roles (704 threads):
 //   warp 0       TMA producer: packed A [128 x 64 B] and B [256 x 64 B] tiles
 //                for one K step of 128, ring of NP stages.
@@ -50,10 +51,7 @@ __device__ int g_status_detail = 0;
 
 namespace {
 
-constexpr int BM = 128;
 constexpr int BN = 256;
-constexpr int NP = 3;   // packed (TMA) stages
-constexpr int NU = 3;   // unpacked (MMA operand) stages
 constexpr int kUnpackWarps = 8;   // per group; two groups take alternate K stages
 constexpr int kUnpackGroups = 2;
 constexpr int kEpiWarps = 4;
@@ -96,25 +94,39 @@ __device__ __forceinline__ void unpack16(const uint4 w, uint32_t x, uint4& lo, u
   t = w.w ^ x; lo.w = t & 0x0F0F0F0Fu; hi.w = (t >> 4) & 0x0F0F0F0Fu;
 }
 
-struct Layout {
+// MT 128-row accumulators per output tile (tile = 128*MT x 256).  MT = 1
+// double-buffers the accumulator so the epilogue overlaps the next tile; MT = 2
+// uses all of tensor memory for the two accumulators of one tile and unpacks
+// each weight tile once for both.
+template <int MT>
+struct Cfg {
+  static constexpr int BMT = 128 * MT;
+  static constexpr int NACC = MT == 1 ? 2 : 1;
+  static constexpr int NP = MT == 1 ? 3 : 2;   // packed (TMA) stages
+  static constexpr int NU = MT == 1 ? 3 : 2;   // unpacked (MMA operand) stages
+  static constexpr int TA = BMT * 4 / (kUnpackWarps * 32);   // A chunks per unpack thread
+  static constexpr int TB = BN * 4 / (kUnpackWarps * 32);    // B chunks per unpack thread
   static constexpr uint32_t uA = 0;
-  static constexpr uint32_t uB = uA + NU * BM * 128;
+  static constexpr uint32_t uB = uA + NU * BMT * 128;
   static constexpr uint32_t pA = uB + NU * BN * 128;
-  static constexpr uint32_t pB = pA + NP * BM * 64;
+  static constexpr uint32_t pB = pA + NP * BMT * 64;
   static constexpr uint32_t bars = pB + NP * BN * 64;
-  // full_p[NP] empty_p[NP] full_u[NU] empty_u[NU] acc_full[2] acc_empty[2] rs_full[2] rs_empty[2] drain
-  static constexpr int nbars = 2 * NP + 2 * NU + 9;
+  // full_p[NP] empty_p[NP] full_u[NU] empty_u[NU] acc_full[NACC] acc_empty[NACC]
+  // rs_full[2] rs_empty[2] drain
+  static constexpr int nbars = 2 * NP + 2 * NU + 2 * NACC + 5;
   static constexpr uint32_t misc = bars + nbars * 8;   // tmem slot, abort flag
   static constexpr uint32_t rs_a = (misc + 16 + 15) & ~15u;
-  static constexpr uint32_t total = rs_a + 2 * kUnpackGroups * BM * 4;
+  static constexpr uint32_t cols = rs_a + 2 * kUnpackGroups * BMT * 4;   // s_n and (float) rowsum_n
+  static constexpr uint32_t total = cols + 2 * BN * 4;
   static constexpr size_t dyn_bytes = total + 1024;
 };
 
-template <bool ASYM, bool ACC_OUT>
+template <int MT, bool ASYM, bool ACC_OUT>
 __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      GemmArgs args, int num_k, int m_tiles, int num_tiles) {
-  using L = Layout;
+  using L = Cfg<MT>;
+  constexpr int BMT = L::BMT, NP = L::NP, NU = L::NU, NACC = L::NACC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L::bars);
@@ -123,13 +135,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* full_u = empty_p + NP;
   uint64_t* empty_u = full_u + NU;
   uint64_t* acc_full = empty_u + NU;
-  uint64_t* acc_empty = acc_full + 2;
-  uint64_t* rs_full = acc_empty + 2;
+  uint64_t* acc_empty = acc_full + NACC;
+  uint64_t* rs_full = acc_empty + NACC;
   uint64_t* rs_empty = rs_full + 2;
   uint64_t* drain = rs_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + L::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + L::misc + 4);
-  int* rs_a = reinterpret_cast<int*>(base + L::rs_a);
+  int* rs_a = reinterpret_cast<int*>(base + L::rs_a);   // [2][groups][BMT]
+  float* col_s = reinterpret_cast<float*>(base + L::cols);   // [BN] w_scale of the tile's columns
+  float* col_r = col_s + BN;                                  // [BN] w_rowsum as float
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -142,9 +156,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&full_u[i], kUnpackWarps);
       mbar_init(&empty_u[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < NACC; ++i) {
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], kEpiWarps);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(&rs_full[i], kUnpackGroups * kUnpackWarps);
       mbar_init(&rs_empty[i], kEpiWarps);
     }
@@ -155,7 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmB);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, 2 * BN);
+    tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -169,15 +185,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       int it = 0;
       bool stop = false;
       for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x) {
-        const int32_t m0 = (tile % m_tiles) * BM, n0 = (tile / m_tiles) * BN;
+        const int32_t m0 = (tile % m_tiles) * BMT, n0 = (tile / m_tiles) * BN;
         for (int kt = 0; kt < num_k; ++kt, ++it) {
           const int s = it % NP;
           if (!wait_or_abort(&empty_p[s], ((it / NP) & 1) ^ 1, abort_flag, 1)) {
             stop = true;
             break;
           }
-          mbar_arrive_expect_tx(&full_p[s], (BM + BN) * 64);
-          tma_load_2d(base + L::pA + s * BM * 64, &tmA, &full_p[s], kt * 64, m0);
+          mbar_arrive_expect_tx(&full_p[s], (BMT + BN) * 64);
+          tma_load_2d(base + L::pA + s * BMT * 64, &tmA, &full_p[s], kt * 64, m0);
           tma_load_2d(base + L::pB + s * BN * 64, &tmB, &full_p[s], kt * 64, n0);
         }
       }
@@ -193,14 +209,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = umma_idesc_e4m3_f32(BM, BN);
+      constexpr uint32_t idesc = umma_idesc_e4m3_f32(128, BN);
       int it = 0, lt = 0;
       bool stop = false;
       for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x, ++lt) {
-        const int b = lt & 1;
-        if (!wait_or_abort(&acc_empty[b], ((lt >> 1) & 1) ^ 1, abort_flag, 2)) break;
+        const int b = lt % NACC;
+        if (!wait_or_abort(&acc_empty[b], ((lt / NACC) & 1) ^ 1, abort_flag, 2)) break;
         tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(b * BN);
         for (int kt = 0; kt < num_k; ++kt, ++it) {
           const int su = it % NU;
           if (!wait_or_abort(&full_u[su], (it / NU) & 1, abort_flag, 3)) {
@@ -208,12 +223,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(base + L::uA + su * BM * 128);
+          const uint32_t a0 = smem_u32(base + L::uA + su * BMT * 128);
           const uint32_t b0 = smem_u32(base + L::uB + su * BN * 128);
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc_mma_f8f6f4(d, umma_desc_sw128(a0 + kk * 32), umma_desc_sw128(b0 + kk * 32), idesc,
-                          (kt | kk) != 0);
+          for (int mt = 0; mt < MT; ++mt) {
+            const uint32_t d = tmem + (uint32_t)((b * MT + mt) * BN);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc_mma_f8f6f4(d, umma_desc_sw128(a0 + mt * 128 * 128 + kk * 32), umma_desc_sw128(b0 + kk * 32),
+                            idesc, (kt | kk) != 0);
+          }
           tc_commit(&empty_u[su]);
         }
         tc_commit(&acc_full[b]);
@@ -230,17 +249,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int grp = (warp - kFirstUnpackWarp) / kUnpackWarps;
     const int u = tid - (kFirstUnpackWarp + grp * kUnpackWarps) * 32;   // 0..255
     const uint32_t xa = ASYM ? 0u : 0x88888888u;
-    // fixed task assignment: 2 A chunks and 4 B chunks per thread per stage
-    uint32_t la[2], sa[2], ha[2], lb[4], sb[4], hb[4];
+    uint32_t la[L::TA], sa[L::TA], ha[L::TA], lb[L::TB], sb[L::TB], hb[L::TB];
 #pragma unroll
-    for (int j = 0; j < 2; ++j) {
+    for (int j = 0; j < L::TA; ++j) {
       const int i = u + 256 * j, r = i >> 2, ch = i & 3;
       la[j] = r * 64 + ch * 16;
       sa[j] = swz_off(r, 2 * ch);
       ha[j] = swz_off(r, 2 * ch + 1);
     }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < L::TB; ++j) {
       const int i = u + 256 * j, r = i >> 2, ch = i & 3;
       lb[j] = r * 64 + ch * 16;
       sb[j] = swz_off(r, 2 * ch);
@@ -250,7 +268,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     int it = 0, lt = 0;
     bool stop = false;
     for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x, ++lt) {
-      int rsum0 = 0, rsum1 = 0;
+      int rsum[L::TA];
+#pragma unroll
+      for (int j = 0; j < L::TA; ++j) rsum[j] = 0;
       for (int kt = 0; kt < num_k; ++kt, ++it) {
         if ((it & 1) != grp) continue;
         const int s = it % NP, su = it % NU;
@@ -259,25 +279,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           stop = true;
           break;
         }
-        const uint32_t PA = sbase + L::pA + s * BM * 64, PB = sbase + L::pB + s * BN * 64;
-        const uint32_t UA = sbase + L::uA + su * BM * 128, UB = sbase + L::uB + su * BN * 128;
-        uint4 wa0 = lds128(PA + la[0]), wa1 = lds128(PA + la[1]);
-        uint4 wb[4];
+        const uint32_t PA = sbase + L::pA + s * BMT * 64, PB = sbase + L::pB + s * BN * 64;
+        const uint32_t UA = sbase + L::uA + su * BMT * 128, UB = sbase + L::uB + su * BN * 128;
+        uint4 wa[L::TA], wb[L::TB];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) wb[j] = lds128(PB + lb[j]);
+        for (int j = 0; j < L::TA; ++j) wa[j] = lds128(PA + la[j]);
+#pragma unroll
+        for (int j = 0; j < L::TB; ++j) wb[j] = lds128(PB + lb[j]);
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty_p[s]);   // packed stage consumed
-        uint4 lo, hi;
-        unpack16(wa0, xa, lo, hi);
-        rsum0 = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u, (unsigned)rsum0);
-        sts128(UA + sa[0], lo);
-        sts128(UA + ha[0], hi);
-        unpack16(wa1, xa, lo, hi);
-        rsum1 = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u, (unsigned)rsum1);
-        sts128(UA + sa[1], lo);
-        sts128(UA + ha[1], hi);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
+        for (int j = 0; j < L::TA; ++j) {
+          uint4 lo, hi;
+          unpack16(wa[j], xa, lo, hi);
+          rsum[j] = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u,
+                                (unsigned)rsum[j]);
+          sts128(UA + sa[j], lo);
+          sts128(UA + ha[j], hi);
+        }
+#pragma unroll
+        for (int j = 0; j < L::TB; ++j) {
+          uint4 lo, hi;
           unpack16(wb[j], 0x88888888u, lo, hi);
           sts128(UB + sb[j], lo);
           sts128(UB + hb[j], hi);
@@ -288,15 +310,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (stop) break;
       // row sums of the unsigned activation codes: 4 lanes share a row
-      rsum0 += __shfl_xor_sync(0xffffffffu, rsum0, 1);
-      rsum0 += __shfl_xor_sync(0xffffffffu, rsum0, 2);
-      rsum1 += __shfl_xor_sync(0xffffffffu, rsum1, 1);
-      rsum1 += __shfl_xor_sync(0xffffffffu, rsum1, 2);
+#pragma unroll
+      for (int j = 0; j < L::TA; ++j) {
+        rsum[j] += __shfl_xor_sync(0xffffffffu, rsum[j], 1);
+        rsum[j] += __shfl_xor_sync(0xffffffffu, rsum[j], 2);
+      }
       const int b = lt & 1;
       if (!wait_or_abort(&rs_empty[b], ((lt >> 1) & 1) ^ 1, abort_flag, 6)) break;
       if ((u & 3) == 0) {
-        rs_a[(b * kUnpackGroups + grp) * BM + (u >> 2)] = rsum0;
-        rs_a[(b * kUnpackGroups + grp) * BM + (u >> 2) + 64] = rsum1;
+#pragma unroll
+        for (int j = 0; j < L::TA; ++j) rs_a[(b * kUnpackGroups + grp) * BMT + (u >> 2) + 64 * j] = rsum[j];
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&rs_full[b]);
@@ -304,58 +327,74 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= kFirstEpiWarp && warp < kFirstEpiWarp + kEpiWarps) {
     // ------------------------------------------------ epilogue
     const int q = warp & 3;
-    const int row = q * 32 + lane;
+    const int et = tid - kFirstEpiWarp * 32;   // 0..127
     int lt = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
-      const int b = lt & 1;
-      const int64_t m = (int64_t)(tile % m_tiles) * BM + row;
+      const int b = lt % NACC, rb = lt & 1;
       const int64_t n0 = (int64_t)(tile / m_tiles) * BN;
-      bool ok = wait_or_abort(&acc_full[b], (lt >> 1) & 1, abort_flag, 7);
-      ok = ok && wait_or_abort(&rs_full[b], (lt >> 1) & 1, abort_flag, 8);
+      // column constants of this tile, staged once (the previous tile's epilogue is done)
+      named_bar_sync(1, kEpiWarps * 32);
+      for (int j = et; j < BN; j += kEpiWarps * 32) {
+        const int64_t n = n0 + j;
+        col_s[j] = n < args.N ? __ldg(args.w_scale + n) : 0.f;
+        col_r[j] = n < args.N ? (float)__ldg(args.w_rowsum + n) : 0.f;
+      }
+      named_bar_sync(1, kEpiWarps * 32);
+      bool ok = wait_or_abort(&acc_full[b], (lt / NACC) & 1, abort_flag, 7);
+      ok = ok && wait_or_abort(&rs_full[rb], (lt >> 1) & 1, abort_flag, 8);
       __syncwarp();
       if (!ok) break;
       tc_fence_after();
-      const int rsa = rs_a[(b * kUnpackGroups) * BM + row] + rs_a[(b * kUnpackGroups + 1) * BM + row];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&rs_empty[b]);
-      const bool mvalid = m < args.M;
-      // y = s_n (alpha (S - 8 rs_a - 8 rw_n) + beta' rw_n), S = acc * 2^18, evaluated as
-      // y = s_n * fma(alpha * 2^18, acc, c + d * rw_n), c = -8 alpha rs_a, d = beta' - 8 alpha
-      float alpha = 0.f, bp = 0.f;
-      if (mvalid) {
-        alpha = __ldg(args.a_scale + m);
-        if (ASYM) bp = __ldg(args.a_zero + m) + 8.f * alpha;
+      int rsa[MT];
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        const int row = mt * 128 + q * 32 + lane;
+        rsa[mt] = rs_a[(rb * kUnpackGroups) * BMT + row] + rs_a[(rb * kUnpackGroups + 1) * BMT + row];
       }
-      const float alpha_s = alpha * 262144.0f;
-      const float cm = -8.f * alpha * (float)rsa;
-      const float dm = bp - 8.f * alpha;
-      __half* yrow = reinterpret_cast<__half*>(args.y) + m * args.N;
-#pragma unroll 1
-      for (int cc = 0; cc < BN / 32; ++cc) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * BN + cc * 32), r);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&rs_empty[rb]);
+      // chunks of 16 accumulator columns, loads double-buffered across chunks
+      constexpr int NCH = MT * (BN / 16);
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * MT * BN);
+      uint32_t ra[16], rbuf[16];
+      auto step = [&](int ci, const uint32_t(&cur)[16], uint32_t(&nxt)[16]) {
         tmem_ld_wait();
-        if (cc == BN / 32 - 1) {
+        if (ci + 1 < NCH) {
+          tmem_ld_32x32b_x16(tbase + (uint32_t)((ci + 1) * 16), nxt);
+        } else {
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&acc_empty[b]);   // accumulator buffer free again
         }
+        const int mt = ci / (BN / 16), cc = ci % (BN / 16);
+        const int64_t m = (int64_t)(tile % m_tiles) * BMT + mt * 128 + q * 32 + lane;
+        const bool mvalid = m < args.M;
+        // y = s_n (alpha (S - 8 rs_a - 8 rw_n) + beta' rw_n), S = acc * 2^18, evaluated as
+        // y = s_n * fma(alpha * 2^18, acc, c + d * rw_n), c = -8 alpha rs_a, d = beta' - 8 alpha
+        float alpha = 0.f, bp = 0.f;
+        if (mvalid) {
+          alpha = __ldg(args.a_scale + m);
+          if (ASYM) bp = __ldg(args.a_zero + m) + 8.f * alpha;
+        }
+        const float alpha_s = alpha * 262144.0f;
+        const float cm = -8.f * alpha * (float)rsa[mt];
+        const float dm = bp - 8.f * alpha;
+        __half* yrow = reinterpret_cast<__half*>(args.y) + m * args.N;
 #pragma unroll
-        for (int g8 = 0; g8 < 4; ++g8) {
-          const int64_t n = n0 + cc * 32 + g8 * 8;
+        for (int g8 = 0; g8 < 2; ++g8) {
+          const int j0 = cc * 16 + g8 * 8;
+          const int64_t n = n0 + j0;
           if (!mvalid || n >= args.N) continue;
-          const float4 s0 = __ldg(reinterpret_cast<const float4*>(args.w_scale + n));
-          const float4 s1 = __ldg(reinterpret_cast<const float4*>(args.w_scale + n) + 1);
-          const int4 q0 = __ldg(reinterpret_cast<const int4*>(args.w_rowsum + n));
-          const int4 q1 = __ldg(reinterpret_cast<const int4*>(args.w_rowsum + n) + 1);
+          const float4 s0 = *reinterpret_cast<const float4*>(col_s + j0);
+          const float4 s1 = *reinterpret_cast<const float4*>(col_s + j0 + 4);
+          const float4 q0 = *reinterpret_cast<const float4*>(col_r + j0);
+          const float4 q1 = *reinterpret_cast<const float4*>(col_r + j0 + 4);
           const float sc[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-          const int rw[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+          const float rw[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
           float yv[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float acc = __uint_as_float(r[g8 * 8 + e]);
-            yv[e] = sc[e] * fmaf(alpha_s, acc, fmaf(dm, (float)rw[e], cm));
-          }
+          for (int e = 0; e < 8; ++e)
+            yv[e] = sc[e] * fmaf(alpha_s, __uint_as_float(cur[g8 * 8 + e]), fmaf(dm, rw[e], cm));
           *reinterpret_cast<uint4*>(yrow + n) =
               make_uint4(pack_half2_bits(yv[0], yv[1]), pack_half2_bits(yv[2], yv[3]),
                          pack_half2_bits(yv[4], yv[5]), pack_half2_bits(yv[6], yv[7]));
@@ -363,12 +402,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             int accs[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e)
-              accs[e] = __float2int_rn(__uint_as_float(r[g8 * 8 + e]) * 262144.0f) - 8 * rsa - 8 * rw[e];
+              accs[e] = __float2int_rn(__uint_as_float(cur[g8 * 8 + e]) * 262144.0f) - 8 * rsa[mt] -
+                        8 * (int)rw[e];
             int4* ap = reinterpret_cast<int4*>(args.acc_out + m * args.N + n);
             ap[0] = make_int4(accs[0], accs[1], accs[2], accs[3]);
             ap[1] = make_int4(accs[4], accs[5], accs[6], accs[7]);
           }
         }
+      };
+      tmem_ld_32x32b_x16(tbase, ra);
+#pragma unroll 1
+      for (int ci = 0; ci < NCH; ci += 2) {
+        step(ci, ra, rbuf);
+        step(ci + 1, rbuf, ra);
       }
     }
   }
@@ -378,7 +424,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem, 2 * BN);
+    tmem_dealloc(tmem, 512);
   }
 }
 
@@ -417,18 +463,19 @@ bool encode_packed_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t 
   return r == CUDA_SUCCESS;
 }
 
-template <bool ASYM, bool ACC_OUT>
+template <int MT, bool ASYM, bool ACC_OUT>
 cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
+  using L = Cfg<MT>;
   CUtensorMap tmA, tmB;
-  if (!encode_packed_map(&tmA, a.a_codes, a.M, a.K, BM)) return cudaErrorNotSupported;
+  if (!encode_packed_map(&tmA, a.a_codes, a.M, a.K, L::BMT)) return cudaErrorNotSupported;
   if (!encode_packed_map(&tmB, a.w_codes, a.N, a.K, BN)) return cudaErrorNotSupported;
-  auto kern = w4a4_gemm_kernel<ASYM, ACC_OUT>;
-  const size_t smem = Layout::dyn_bytes;
+  auto kern = w4a4_gemm_kernel<MT, ASYM, ACC_OUT>;
+  const size_t smem = L::dyn_bytes;
   int per_sm = 0;
   cudaError_t e = prepare_launch(kern, kThreads, smem, &per_sm);
   if (e != cudaSuccess) return e;
   const int sms = device_sm_count();
-  const int m_tiles = (int)((a.M + BM - 1) / BM);
+  const int m_tiles = (int)((a.M + L::BMT - 1) / L::BMT);
   const int n_tiles = (int)((a.N + BN - 1) / BN);
   const int tiles = m_tiles * n_tiles;
   const int grid = tiles < sms ? tiles : sms;
@@ -436,13 +483,21 @@ cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+template <int MT>
+cudaError_t launch_mt(const GemmArgs& a, cudaStream_t stream) {
+  const bool asym = a.a_zero != nullptr, acc = a.acc_out != nullptr;
+  if (asym) return acc ? launch_t<MT, true, true>(a, stream) : launch_t<MT, true, false>(a, stream);
+  return acc ? launch_t<MT, false, true>(a, stream) : launch_t<MT, false, false>(a, stream);
+}
+
 }  // namespace
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
-  const bool asym = a.a_zero != nullptr, acc = a.acc_out != nullptr;
-  if (asym) return acc ? launch_t<true, true>(a, stream) : launch_t<true, false>(a, stream);
-  return acc ? launch_t<false, true>(a, stream) : launch_t<false, false>(a, stream);
+  // 256-row tiles when they still give every SM at least two tiles
+  const int64_t tiles256 = ((a.M + 255) / 256) * ((a.N + BN - 1) / BN);
+  if (a.K >= 3072 && tiles256 >= 2 * (int64_t)device_sm_count()) return launch_mt<2>(a, stream);
+  return launch_mt<1>(a, stream);
 }
 
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail) {

@@ -112,6 +112,8 @@ FULL = [
     ("l32_up_M1", 1, 3072, 8192, False),
     ("l32_down_M16", 16, 8192, 3072, False),
     ("l32_up_M128", 128, 3072, 8192, False),
+    ("tile256_ragged_M2000", 2000, 1024, 10240, True),
+    ("tile256_ragged_M2001_asym", 2001, 512, 12288, False),
 ]
 
 
