@@ -63,6 +63,22 @@ def gemm_ops():
     return 2.0 * M * N * K
 
 
+def gemm_traffic_from_profile():
+    """DRAM bytes per GEMM launch from the committed ncu summary, or None when
+    the kernel source changed since the counters were taken."""
+    import hashlib
+    import re
+    try:
+        src = os.path.join(ROOT, "paper_2405_16406_gb300", "csrc", "w4a4_gemm.cu")
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        txt = open(os.path.join(ROOT, "profiles", "w4a4_gemm_gate_up_M2048_K4096_N14336.md")).read()
+        if re.search(r"sha256 \(first 16 hex\): ([0-9a-f]{16})", txt).group(1) != h:
+            return None
+        return int(re.search(r"traffic_bytes_per_launch: (\d+)", txt).group(1))
+    except Exception:
+        return None
+
+
 # --------------------------------------------------------------------------- clocks
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons while work runs."""
@@ -131,24 +147,24 @@ def run_ours(args, rank, world, local_rank):
     hbm_peak, bf16_peak, peak_kind = peaks()
     fp8_peak = 2.0 * bf16_peak  # nominal e4m3 : bf16 dense ratio on GB300 is 2
 
-    g = torch.Generator(device=dev)
-    g.manual_seed(1000 + rank)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 + rank)
 
     def acts(rows, cols, frac, factor):
-        x = torch.randn(rows, cols, generator=g, device=dev)
-        cols_idx = torch.randperm(cols, generator=g, device=dev)[: max(1, int(round(frac * cols)))]
+        x = torch.randn(rows, cols, generator=gen, device=dev)
+        cols_idx = torch.randperm(cols, generator=gen, device=dev)[: max(1, int(round(frac * cols)))]
         x[:, cols_idx] *= factor
         return x.half()
 
     sets = []
     for _ in range(NSETS):
         x = acts(M, K, 0.01, 30.0)
-        w = (torch.randn(N, K, generator=g, device=dev) * 0.02).half()
+        w = (torch.randn(N, K, generator=gen, device=dev) * 0.02).half()
         qw = spinq.quant_weight(w, None)                       # offline, not timed
         del w
-        q = torch.randn(B_KV, S_KV, HQ, D, generator=g, device=dev).half()
-        k = torch.randn(B_KV, S_KV, HKV, D, generator=g, device=dev).half()
-        v = torch.randn(B_KV, S_KV, HKV, D, generator=g, device=dev).half()
+        q = torch.randn(B_KV, S_KV, HQ, D, generator=gen, device=dev).half()
+        k = torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half()
+        v = torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half()
         sets.append((x, qw, q, k, v))
     qa_out = [spinq.ActCodes(torch.empty(M, K // 2, dtype=torch.uint8, device=dev),
                              torch.empty(M, dtype=torch.float32, device=dev),
@@ -175,8 +191,9 @@ def run_ours(args, rank, world, local_rank):
             fn(i % NSETS)
     torch.cuda.synchronize()
 
-    # one CUDA graph per (input set, kernel): replays keep the GPU fed without
-    # host launch gaps between the per-kernel timing events
+    # One CUDA graph per (input set, kernel).  Replays keep the GPU fed with no
+    # host launch gaps; the per-kernel events sit between replays, so each
+    # per-kernel duration includes its graph launch (a few microseconds).
     graphs = []
     for j in range(NSETS):
         row = []
@@ -187,14 +204,11 @@ def run_ours(args, rank, world, local_rank):
             row.append(g)
         graphs.append(row)
     torch.cuda.synchronize()
-
-    n_ev = args.steps
     ev = {k2: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(n_ev)] for k2 in names}
+               for _ in range(args.steps)] for k2 in names}
 
     def step(i, record=None):
-        j = i % NSETS
-        for name, g in zip(names, graphs[j]):
+        for name, g in zip(names, graphs[i % NSETS]):
             if record is not None:
                 ev[name][record][0].record(stream)
             g.replay()
@@ -291,6 +305,40 @@ def run_ours(args, rank, world, local_rank):
     h2d = (M * K + B_KV * S_KV * (HQ + 2 * HKV) * D) * 2
     d2h = M * N * 2 + B_KV * S_KV * HQ * D * 2 + 2 * B_KV * S_KV * HKV * D // 2 + B_KV * S_KV * HKV * 16
 
+    # ---- isolated timing of the two memory-bound kernels: 16 back-to-back
+    # launches in one graph over 16 input sets (footprint > L2), so the graph
+    # launch is amortised and every launch reads cold data
+    iso = {}
+    if rank == 0:
+        xs = [acts(M, K, 0.01, 30.0) for _ in range(16)]
+        qo = [spinq.ActCodes(torch.empty(M, K // 2, dtype=torch.uint8, device=dev),
+                             torch.empty(M, dtype=torch.float32, device=dev),
+                             torch.empty(M, dtype=torch.float32, device=dev)) for _ in range(16)]
+        kvs = [(torch.randn(B_KV, S_KV, HQ, D, generator=gen, device=dev).half(),
+                torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half(),
+                torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half()) for _ in range(16)]
+        kvo = [spinq.rotate_quant_kv(*t) for t in kvs]
+        for name, fn in (("act_quant", lambda i: spinq.rotate_quant_act(xs[i], None, False, 1.0, out=qo[i])),
+                         ("kv_quant", lambda i: spinq.rotate_quant_kv(*kvs[i], out=kvo[i]))):
+            for i in range(16):
+                fn(i)
+            torch.cuda.synchronize()
+            gi = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gi):
+                for i in range(16):
+                    fn(i)
+            gi.replay()
+            torch.cuda.synchronize()
+            e0i = torch.cuda.Event(enable_timing=True)
+            e1i = torch.cuda.Event(enable_timing=True)
+            e0i.record(stream)
+            for _ in range(3):
+                gi.replay()
+            e1i.record(stream)
+            torch.cuda.synchronize()
+            iso[name] = e0i.elapsed_time(e1i) / 48 / 1e3
+        del xs, qo, kvs, kvo
+
     st, _ = spinq.spinq_device_status()
     if st != spinq.SPINQ_OK:
         raise RuntimeError(f"device status after bench: {spinq.spinq_status_string(st)}")
@@ -324,19 +372,24 @@ def run_ours(args, rank, world, local_rank):
         "roofline": {
             "bound": "tensor", "kernel": "w4a4_gemm_kernel",
             "achieved": round(gemm_tops, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
-            "frac": round(gemm_tops / fp8_peak, 4), "traffic": None,
+            "frac": round(gemm_tops / fp8_peak, 4), "traffic": gemm_traffic_from_profile(),
             "peak_note": f"e4m3 dense = 2 x {peak_kind} bf16 ({bf16_peak} TFLOP/s); "
                          "int4 codes carried as e4m3 on tcgen05 kind::f8f6f4",
         },
         "rotate_quant_roofline": {
-            "bound": "hbm", "kernel": "rotate_quant_rows_kernel (act, K=4096)",
+            "bound": "hbm", "kernel": "rq_norot_kernel (act quant, 2048 x 4096, asym)",
             "achieved": round(rq_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
             "frac": round(rq_gbs / hbm_peak, 4), "us": round(t_rq * 1e6, 2),
+            "isolated_us": round(iso["act_quant"] * 1e6, 2),
+            "isolated_frac": round(step_bytes_rq() / iso["act_quant"] / 1e9 / hbm_peak, 4),
+            "note": "in-step time includes the graph launch; isolated = 16 launches per graph, cold inputs",
         },
         "kv_roofline": {
-            "bound": "hbm", "kernel": "rotate_quant_kv_kernel",
+            "bound": "hbm", "kernel": "rotate_quant_kv_kernel (2048 tokens)",
             "achieved": round(kv_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
             "frac": round(kv_gbs / hbm_peak, 4), "us": round(t_kv * 1e6, 2),
+            "isolated_us": round(iso["kv_quant"] * 1e6, 2),
+            "isolated_frac": round(step_bytes_kv() / iso["kv_quant"] / 1e9 / hbm_peak, 4),
         },
         "kernel_us": {"gemm": round(t_gemm * 1e6, 2), "act_quant": round(t_rq * 1e6, 2),
                       "kv_quant": round(t_kv * 1e6, 2)},
