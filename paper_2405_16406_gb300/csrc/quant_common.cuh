@@ -21,6 +21,15 @@ struct Range {
       lo = fminf(lo, v);
     }
   }
+  // two values at once with the 3-input min/max of sm_100+
+  __device__ __forceinline__ void add2(float a, float b) {
+    if (SYM) {
+      asm("max.f32 %0, %0, %1, %2;" : "+f"(hi) : "f"(fabsf(a)), "f"(fabsf(b)));
+    } else {
+      asm("max.f32 %0, %0, %1, %2;" : "+f"(hi) : "f"(a), "f"(b));
+      asm("min.f32 %0, %0, %1, %2;" : "+f"(lo) : "f"(a), "f"(b));
+    }
+  }
   __device__ __forceinline__ void warp_reduce() {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -72,6 +81,7 @@ struct QParams {
   }
   template <bool CLAMP>
   __device__ __forceinline__ uint32_t code_bits(float v) const {
+    if (SYM && !CLAMP) return __float_as_uint(fmaf(v, inv, kRoundMagic));  // one rounding: rint(v/alpha)
     float t = fmaf(v, inv, off);
     if (CLAMP) t = SYM ? fminf(fmaxf(t, -8.f), 7.f) : fminf(fmaxf(t, 0.f), 15.f);
     return round_bits(t);

@@ -89,22 +89,25 @@ struct Pow2Shape {
   static constexpr int GL = 1 << L;         // consecutive elements per group
 };
 
-// fp32 word index of element p in the swizzled row buffer
-template <int LW>
-__device__ __forceinline__ uint32_t swz_word(uint32_t p) {
-  const uint32_t q = p >> 2;
-  const uint32_t x = ((q >> 3) ^ (q >> (6 + LW))) & 1u;
-  return ((q ^ x) << 2) | (p & 3u);
-}
-
 constexpr uint64_t kRowWaitLimitNs = 2000000000ull;
+
+// fp32 transpose buffer: two planes, element p -> plane (p >> 2) & 1,
+// word 4 (p >> 3) + (p & 3); plane 1 starts 16 words (64 B) after the end of
+// plane 0 so that the two planes map to opposite halves of the bank space.
+// Phase 1 stores each chunk as one float4 per plane (8 lanes = 128 contiguous
+// bytes); phase 2 reads 2 or 4 consecutive elements whose word offsets are a
+// per-thread base plus compile-time constants.
+template <int P>
+__device__ __forceinline__ uint32_t plane_word(uint32_t p) {
+  return ((p >> 2) & 1u) * (P / 2 + 16) + ((p >> 3) << 2) + (p & 3u);
+}
 
 template <int LW, int L>
 struct Pow2Smem {
   using S = Pow2Shape<LW, L>;
   static constexpr int NST = S::P >= 4096 ? 1 : 2;     // fp16 rows staged ahead
-  static constexpr int OFF_F32 = 0;                     // P floats (transpose)
-  static constexpr int OFF_STAGE = S::P * 4;
+  static constexpr int OFF_F32 = 0;                     // two planes
+  static constexpr int OFF_STAGE = (S::P + 32) * 4;
   static constexpr int OFF_BAR = OFF_STAGE + NST * S::P * 2;
   static constexpr int OFF_MISC = OFF_BAR + NST * 8;   // abort flag + range scratch
   static constexpr int BYTES = OFF_MISC + 16 + 2 * S::W * 4;
@@ -114,6 +117,7 @@ template <int LW, int L, bool SYM, bool CLAMP>
 __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
   using S = Pow2Shape<LW, L>;
   using SM = Pow2Smem<LW, L>;
+  static_assert(L == 1 || L == 2, "phase-2 group of 2 or 4 elements");
   extern __shared__ __align__(128) uint8_t smem[];
   float* sm = reinterpret_cast<float*>(smem + SM::OFF_F32);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + SM::OFF_MISC);
@@ -134,11 +138,13 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
   __syncthreads();
   rs.prologue();
 
-  // phase-2 fixed element bits of this thread
+  // phase-2 fixed element bits of this thread: {L..2}, {3, 4}, v bits
   const uint32_t t_lo = (uint32_t)tid & ((1u << (3 - L)) - 1u);
   const uint32_t t_c = ((uint32_t)tid >> (3 - L)) & 3u;
   const uint32_t t_v = (uint32_t)tid >> (5 - L);
   const uint32_t fixed = (t_lo << L) | (t_c << 3) | (t_v << (8 + LW));
+  const float* zbase = sm + plane_word<S::P>(fixed);   // group m adds 4 * (m << 2) words
+  uint8_t* const codes0 = a.codes + (fixed >> 1);
 
   int it = 0;
   for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x, ++it) {
@@ -172,28 +178,22 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
         }
 #pragma unroll
     for (int v = 0; v < S::V; ++v) {
-      const uint32_t p = 8u * (uint32_t)(lane + 32 * (w + S::W * v));
-      *reinterpret_cast<float4*>(sm + swz_word<LW>(p)) = make_float4(y[v][0], y[v][1], y[v][2], y[v][3]);
-      *reinterpret_cast<float4*>(sm + swz_word<LW>(p + 4)) = make_float4(y[v][4], y[v][5], y[v][6], y[v][7]);
+      const uint32_t ch = (uint32_t)(lane + 32 * (w + S::W * v));
+      *reinterpret_cast<float4*>(sm + 4 * ch) = make_float4(y[v][0], y[v][1], y[v][2], y[v][3]);
+      *reinterpret_cast<float4*>(sm + S::P / 2 + 16 + 4 * ch) = make_float4(y[v][4], y[v][5], y[v][6], y[v][7]);
     }
     __syncthreads();
     rs.release(it);  // the staged row is consumed: the next copy overlaps phase 2
 
-    // ---------------- phase 2
+    // ---------------- phase 2: groups m cover element bits 5.. (g, then w)
     float z[S::NG][S::GL];
 #pragma unroll
     for (int m = 0; m < S::NG; ++m) {
-      const uint32_t p = fixed | ((uint32_t)(m & 7) << 5) | ((uint32_t)(m >> 3) << 8);
-      if constexpr (S::GL == 8) {
-        const float4 u0 = *reinterpret_cast<const float4*>(sm + swz_word<LW>(p));
-        const float4 u1 = *reinterpret_cast<const float4*>(sm + swz_word<LW>(p + 4));
-        z[m][0] = u0.x; z[m][1] = u0.y; z[m][2] = u0.z; z[m][3] = u0.w;
-        z[m][4 % S::GL] = u1.x; z[m][5 % S::GL] = u1.y; z[m][6 % S::GL] = u1.z; z[m][7 % S::GL] = u1.w;
-      } else if constexpr (S::GL == 4) {
-        const float4 u0 = *reinterpret_cast<const float4*>(sm + swz_word<LW>(p));
+      if constexpr (S::GL == 4) {
+        const float4 u0 = *reinterpret_cast<const float4*>(zbase + 16 * m);
         z[m][0] = u0.x; z[m][1 % S::GL] = u0.y; z[m][2 % S::GL] = u0.z; z[m][3 % S::GL] = u0.w;
       } else {
-        const float2 u0 = *reinterpret_cast<const float2*>(sm + swz_word<LW>(p));
+        const float2 u0 = *reinterpret_cast<const float2*>(zbase + 16 * m);
         z[m][0] = u0.x; z[m][1 % S::GL] = u0.y;
       }
     }
@@ -213,21 +213,21 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
 #pragma unroll
     for (int m = 0; m < S::NG; ++m)
 #pragma unroll
-      for (int j = 0; j < S::GL; ++j) r.add(z[m][j]);
+      for (int j = 0; j < S::GL; j += 2) r.add2(z[m][j], z[m][j + 1]);
     block_range<SYM, S::W>(r, red);
     const QParams<SYM> qp(r, a.clip);
 
-    uint8_t* out = a.codes + row * (a.K / 2);
+    uint8_t* out = codes0 + row * (a.K / 2);
 #pragma unroll
     for (int m = 0; m < S::NG; ++m) {
-      const uint32_t p = fixed | ((uint32_t)(m & 7) << 5) | ((uint32_t)(m >> 3) << 8);
-      uint32_t rb[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) rb[j] = j < S::GL ? qp.template code_bits<CLAMP>(z[m][j % S::GL]) : 0u;
-      const uint32_t word = pack8_nibbles(rb);
-      if constexpr (S::GL == 8) *reinterpret_cast<uint32_t*>(out + p / 2) = word;
-      else if constexpr (S::GL == 4) *reinterpret_cast<uint16_t*>(out + p / 2) = (uint16_t)word;
-      else out[p / 2] = (uint8_t)word;
+      // element offset of group m is 32 m (bits 5..), i.e. 16 m bytes of codes
+      if constexpr (S::GL == 4) {
+        const uint32_t wv = pack4_nibbles(qp.template code_bits<CLAMP>(z[m][0]), qp.template code_bits<CLAMP>(z[m][1 % S::GL]),
+                                          qp.template code_bits<CLAMP>(z[m][2 % S::GL]), qp.template code_bits<CLAMP>(z[m][3 % S::GL]));
+        *reinterpret_cast<uint16_t*>(out + 16 * m) = (uint16_t)wv;
+      } else {
+        out[16 * m] = (uint8_t)pack2_nibbles(qp.template code_bits<CLAMP>(z[m][0]), qp.template code_bits<CLAMP>(z[m][1 % S::GL]));
+      }
     }
     if (tid == 0) {
       a.scale[row] = qp.alpha * a.norm;

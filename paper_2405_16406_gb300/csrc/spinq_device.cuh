@@ -74,6 +74,15 @@ __device__ __forceinline__ uint32_t pack8_nibbles(const uint32_t r[8]) {
   return (ev & 0x0F0F0F0Fu) | ((od << 4) & 0xF0F0F0F0u);
 }
 
+// Two / four round_bits() words -> one byte / 16 bits of nibbles (first
+// element in the low nibble).
+__device__ __forceinline__ uint32_t pack2_nibbles(uint32_t r0, uint32_t r1) {
+  return (r0 & 0x0Fu) | ((r1 << 4) & 0xF0u);
+}
+__device__ __forceinline__ uint32_t pack4_nibbles(uint32_t r0, uint32_t r1, uint32_t r2, uint32_t r3) {
+  return __byte_perm(pack2_nibbles(r0, r1), pack2_nibbles(r2, r3), 0x0040);
+}
+
 // ---------------------------------------------------------------------------
 // mbarrier (shared::cta) with bounded waits
 // ---------------------------------------------------------------------------
