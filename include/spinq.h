@@ -131,6 +131,35 @@ spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const
                              void* y_f16, int32_t* acc_out, void* stream);
 
 /*
+ * spinq_w4a4_gemm_workspace_bytes -- device workspace, in bytes, that
+ * spinq_w4a4_gemm_splitk needs for an M x N output: M*N*4 + 4*ceil(N/128)
+ * for M <= 256, and 0 for larger M (those calls need no workspace).
+ */
+int64_t spinq_w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K);
+
+/*
+ * spinq_w4a4_gemm_splitk -- the same operation and outputs as
+ * spinq_w4a4_gemm, for small M (decode, M <= 256), where the GEMM is bound by
+ * streaming the weights from HBM.  Each CTA owns 128 output channels and a
+ * slice of K, so every SM streams a disjoint part of the weights; the slices'
+ * exact integer partial accumulators are summed in `workspace` and the last
+ * slice of each 128-channel tile applies the epilogue.  For M > 256 the call
+ * runs the same kernel as spinq_w4a4_gemm and does not touch `workspace`.
+ *   workspace       device buffer of spinq_w4a4_gemm_workspace_bytes(M, N, K)
+ *                   bytes, 16-byte aligned, all zero before the first call;
+ *                   each completed call leaves it zero again.  Calls that may
+ *                   overlap on the GPU need distinct workspaces.  After a call
+ *                   that recorded SPINQ_ETIMEOUT, clear it again.
+ *   workspace_bytes its size (SPINQ_EINVAL if smaller than required).
+ * Other arguments and requirements as spinq_w4a4_gemm.
+ */
+spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
+                                    const uint8_t* w_codes, const float* w_scale,
+                                    const int32_t* w_rowsum, int64_t M, int64_t N, int64_t K,
+                                    void* y_f16, int32_t* acc_out, void* workspace,
+                                    int64_t workspace_bytes, void* stream);
+
+/*
  * spinq_rotate_quant_kv -- R3 on Q and K over head_dim, then the 4-bit
  * KV-cache quantizer (Sec. 3.1: R3 is an online Hadamard inserted for low-bit
  * KV-cache quantization; appendix "Quantization choice": asymmetric).

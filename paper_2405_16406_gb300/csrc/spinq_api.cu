@@ -141,6 +141,31 @@ spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const
   return from_cuda(launch_w4a4_gemm(g, static_cast<cudaStream_t>(stream)));
 }
 
+int64_t spinq_w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K) {
+  (void)K;
+  return w4a4_gemm_workspace_bytes(M, N);
+}
+
+spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
+                                    const uint8_t* w_codes, const float* w_scale,
+                                    const int32_t* w_rowsum, int64_t M, int64_t N, int64_t K,
+                                    void* y_f16, int32_t* acc_out, void* workspace,
+                                    int64_t workspace_bytes, void* stream) {
+  if (M < 0 || N < 0 || K <= 0) return SPINQ_EINVAL;
+  if (M > 0 && N > 0 && (!a_codes || !a_scale || !w_codes || !w_scale || !w_rowsum || !y_f16))
+    return SPINQ_EINVAL;
+  if (K % 128 != 0 || N % 16 != 0) return SPINQ_EINVAL;
+  if (!aligned16(a_codes) || !aligned16(w_codes) || !aligned16(y_f16) || !aligned16(w_scale) ||
+      !aligned16(w_rowsum) || (acc_out && !aligned16(acc_out)))
+    return SPINQ_EINVAL;
+  const int64_t need = w4a4_gemm_workspace_bytes(M, N);
+  if (need > 0 && (!workspace || !aligned16(workspace) || workspace_bytes < need)) return SPINQ_EINVAL;
+  if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
+  if (M == 0 || N == 0) return SPINQ_OK;
+  GemmArgs g{a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y_f16, acc_out};
+  return from_cuda(launch_w4a4_gemm_splitk(g, workspace, static_cast<cudaStream_t>(stream)));
+}
+
 spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_in,
                                    const void* v_in, int64_t B, int64_t S, int64_t Hq,
                                    int64_t Hkv, int64_t D, const spinq_had_cfg* had,

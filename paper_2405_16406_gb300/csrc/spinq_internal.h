@@ -81,6 +81,17 @@ struct GemmArgs {
 // Returns cudaErrorNotSupported when the TMA descriptor cannot be encoded.
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
 
+// Largest M served by the split-K decode kernel.
+constexpr int64_t kDecodeMaxM = 256;
+
+// Workspace bytes of launch_w4a4_gemm_splitk for (M, N); 0 when M > kDecodeMaxM.
+int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N);
+
+// Split-K decode GEMM for M <= kDecodeMaxM (falls back to launch_w4a4_gemm
+// above).  `workspace` holds w4a4_gemm_workspace_bytes(M, N) bytes that are
+// zero before the call and zero again after it.
+cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, cudaStream_t stream);
+
 // Device status word written by bounded waits that gave up.
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail);
 

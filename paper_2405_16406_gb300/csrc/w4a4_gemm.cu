@@ -429,6 +429,278 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Decode / skinny GEMM (M <= 256): the weight tile is the MMA's M side
+// (128 output channels per CTA), the tokens its N side (MN = M rounded up to
+// 16), and K is split across CTAs so that every SM streams a disjoint slice of
+// the weights.  Each split adds its exact integer partial
+//   sum_k (u_a - 8)(u_w - 8) = S - 8 sum u_a - 8 sum u_w + 64 K_split
+// into an fp32 workspace [M][N] (integer values below 2^24: the sums are exact
+// and independent of the order of the adds); the last split of an output tile
+// (per-tile counter) converts the tile to fp16 with the epilogue formula and
+// clears its workspace rows and counter for the next call.
+// ---------------------------------------------------------------------------
+constexpr int kDecUnpackWarps = 4;
+constexpr int kDecThreads = (6 + kDecUnpackWarps) * 32;   // TMA, MMA, 4 epilogue, 4 unpack warps
+constexpr int kDecUnpackThreads = kDecUnpackWarps * 32;
+
+template <int MN>
+struct DecCfg {
+  static constexpr int NP = MN <= 64 ? 4 : 3;
+  static constexpr int NU = MN <= 64 ? 3 : 2;
+  static constexpr int TW = 128 * 4 / kDecUnpackThreads;                        // W chunks per unpack thread
+  static constexpr int TA = (MN * 4 + kDecUnpackThreads - 1) / kDecUnpackThreads;  // A chunks (last may idle)
+  static constexpr uint32_t uW = 0;
+  static constexpr uint32_t uA = uW + NU * 128 * 128;
+  static constexpr uint32_t pW = uA + NU * MN * 128;
+  static constexpr uint32_t pA = pW + NP * 128 * 64;
+  static constexpr uint32_t bars = (pA + NP * MN * 64 + 7) & ~7u;
+  // full_p[NP] empty_p[NP] full_u[NU] empty_u[NU] acc_full rs_full drain
+  static constexpr int nbars = 2 * NP + 2 * NU + 3;
+  static constexpr uint32_t misc = bars + nbars * 8;   // tmem slot, abort flag, last flag
+  static constexpr uint32_t rsw = (misc + 16 + 15) & ~15u;   // [128] weight row sums of this split
+  static constexpr uint32_t rsa = rsw + 128 * 4;               // [MN] token sums of this split
+  static constexpr uint32_t total = rsa + MN * 4;
+  static constexpr size_t dyn_bytes = total + 1024;
+  static constexpr uint32_t tmem_cols = MN <= 32 ? 32 : MN <= 64 ? 64 : MN <= 128 ? 128 : 256;
+};
+
+template <int MN, bool ASYM, bool ACC_OUT>
+__global__ void __launch_bounds__(kDecThreads, 2)
+    w4a4_decode_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmA,
+                       GemmArgs args, float* ws_acc, int* ws_cnt, int ksteps, int nsplit) {
+  using L = DecCfg<MN>;
+  constexpr int NP = L::NP, NU = L::NU;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + L::bars);
+  uint64_t* full_p = bars;
+  uint64_t* empty_p = full_p + NP;
+  uint64_t* full_u = empty_p + NP;
+  uint64_t* empty_u = full_u + NU;
+  uint64_t* acc_full = empty_u + NU;
+  uint64_t* rs_full = acc_full + 1;
+  uint64_t* drain = rs_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + L::misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + L::misc + 4);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(base + L::misc + 8);
+  int* rsw = reinterpret_cast<int*>(base + L::rsw);
+  int* rsa = reinterpret_cast<int*>(base + L::rsa);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int split = blockIdx.x, ntile = blockIdx.y;
+  const int n0 = ntile * 128;
+  const int k_begin = (int)((int64_t)split * ksteps / nsplit);
+  const int k_end = (int)((int64_t)(split + 1) * ksteps / nsplit);
+  const int nk = k_end - k_begin;
+
+  if (tid == 0) {
+    for (int i = 0; i < NP; ++i) {
+      mbar_init(&full_p[i], 1);
+      mbar_init(&empty_p[i], kDecUnpackWarps);
+    }
+    for (int i = 0; i < NU; ++i) {
+      mbar_init(&full_u[i], kDecUnpackWarps);
+      mbar_init(&empty_u[i], 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(rs_full, kDecUnpackWarps);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    *last_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmW);
+    prefetch_tmap(&tmA);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, L::tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int issued = 0;
+      for (int it = 0; it < nk; ++it) {
+        const int s = it % NP;
+        if (!wait_or_abort(&empty_p[s], ((it / NP) & 1) ^ 1, abort_flag, 11)) break;
+        mbar_arrive_expect_tx(&full_p[s], (128 + MN) * 64);
+        tma_load_2d(base + L::pW + s * 128 * 64, &tmW, &full_p[s], (k_begin + it) * 64, n0);
+        tma_load_2d(base + L::pA + s * MN * 64, &tmA, &full_p[s], (k_begin + it) * 64, 0);
+        issued = it + 1;
+      }
+      if (*abort_flag) {
+        for (int j = issued - NP < 0 ? 0 : issued - NP; j < issued; ++j) {
+          const uint64_t t0 = globaltimer_ns();
+          while (!mbar_try_wait(&full_p[j % NP], (j / NP) & 1) && globaltimer_ns() - t0 < kWaitLimitNs) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = umma_idesc_e4m3_f32(128, MN);
+      for (int it = 0; it < nk; ++it) {
+        const int su = it % NU;
+        if (!wait_or_abort(&full_u[su], (it / NU) & 1, abort_flag, 12)) break;
+        tc_fence_after();
+        const uint32_t w0 = smem_u32(base + L::uW + su * 128 * 128);
+        const uint32_t a0 = smem_u32(base + L::uA + su * MN * 128);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_f8f6f4(tmem, umma_desc_sw128(w0 + kk * 32), umma_desc_sw128(a0 + kk * 32), idesc, (it | kk) != 0);
+        tc_commit(&empty_u[su]);
+      }
+      tc_commit(acc_full);
+      tc_commit(drain);
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(drain, 0) && globaltimer_ns() - t0 < kWaitLimitNs) {
+      }
+    }
+  } else if (warp >= kFirstUnpackWarp) {
+    const int u = tid - kFirstUnpackWarp * 32;   // 0..127
+    const uint32_t xa = ASYM ? 0u : 0x88888888u;
+    const uint32_t sbase = smem_u32(base);
+    int sw[L::TW], sa[L::TA];
+#pragma unroll
+    for (int j = 0; j < L::TW; ++j) sw[j] = 0;
+#pragma unroll
+    for (int j = 0; j < L::TA; ++j) sa[j] = 0;
+    for (int it = 0; it < nk; ++it) {
+      const int s = it % NP, su = it % NU;
+      if (!wait_or_abort(&full_p[s], (it / NP) & 1, abort_flag, 13) ||
+          !wait_or_abort(&empty_u[su], ((it / NU) & 1) ^ 1, abort_flag, 14))
+        break;
+      const uint32_t PW = sbase + L::pW + s * 128 * 64, PA = sbase + L::pA + s * MN * 64;
+      const uint32_t UW = sbase + L::uW + su * 128 * 128, UA = sbase + L::uA + su * MN * 128;
+      uint4 ww[L::TW], wa[L::TA];
+#pragma unroll
+      for (int j = 0; j < L::TW; ++j) {
+        const int i = u + kDecUnpackThreads * j;
+        ww[j] = lds128(PW + (i >> 2) * 64 + (i & 3) * 16);
+      }
+#pragma unroll
+      for (int j = 0; j < L::TA; ++j) {
+        const int i = u + kDecUnpackThreads * j;
+        wa[j] = i < MN * 4 ? lds128(PA + (i >> 2) * 64 + (i & 3) * 16) : make_uint4(0, 0, 0, 0);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_p[s]);
+#pragma unroll
+      for (int j = 0; j < L::TW; ++j) {
+        const int i = u + kDecUnpackThreads * j, r = i >> 2, ch = i & 3;
+        uint4 lo, hi;
+        unpack16(ww[j], 0x88888888u, lo, hi);
+        sw[j] = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u, (unsigned)sw[j]);
+        sts128(UW + swz_off(r, 2 * ch), lo);
+        sts128(UW + swz_off(r, 2 * ch + 1), hi);
+      }
+#pragma unroll
+      for (int j = 0; j < L::TA; ++j) {
+        const int i = u + kDecUnpackThreads * j, r = i >> 2, ch = i & 3;
+        if (i < MN * 4) {
+          uint4 lo, hi;
+          unpack16(wa[j], xa, lo, hi);
+          sa[j] = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u, (unsigned)sa[j]);
+          sts128(UA + swz_off(r, 2 * ch), lo);
+          sts128(UA + swz_off(r, 2 * ch + 1), hi);
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&full_u[su]);
+    }
+    // row sums over this split: 4 lanes share a row
+#pragma unroll
+    for (int j = 0; j < L::TW; ++j) {
+      sw[j] += __shfl_xor_sync(0xffffffffu, sw[j], 1);
+      sw[j] += __shfl_xor_sync(0xffffffffu, sw[j], 2);
+      if ((u & 3) == 0) rsw[(u >> 2) + (kDecUnpackThreads / 4) * j] = sw[j];
+    }
+#pragma unroll
+    for (int j = 0; j < L::TA; ++j) {
+      sa[j] += __shfl_xor_sync(0xffffffffu, sa[j], 1);
+      sa[j] += __shfl_xor_sync(0xffffffffu, sa[j], 2);
+      const int r = (u >> 2) + (kDecUnpackThreads / 4) * j;
+      if ((u & 3) == 0 && r < MN) rsa[r] = sa[j];
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(rs_full);
+  } else if (warp >= kFirstEpiWarp && warp < kFirstEpiWarp + kEpiWarps) {
+    const int q = warp & 3;
+    const int nl = q * 32 + lane;                 // weight row of this lane (TMEM lane)
+    const int64_t n = n0 + nl;
+    const int et = tid - kFirstEpiWarp * 32;    // 0..127
+    bool ok = wait_or_abort(acc_full, 0, abort_flag, 15);
+    ok = ok && wait_or_abort(rs_full, 0, abort_flag, 16);
+    __syncwarp();
+    tc_fence_after();
+    const float kfix = 64.f * 128.f * (float)nk;
+    const float wfix = kfix - 8.f * (float)(ok ? rsw[nl] : 0);
+    const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+    for (int c0 = 0; c0 < MN; c0 += 16) {
+      uint32_t r[16];
+      tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
+      tmem_ld_wait();
+      if (!ok || n >= args.N) continue;
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const int m = c0 + e;
+        if (m < args.M) {
+          const float part = fmaf(__uint_as_float(r[e]), 262144.0f, wfix - 8.f * (float)rsa[m]);
+          atomicAdd(ws_acc + (int64_t)m * args.N + n, part);
+        }
+      }
+    }
+    tc_fence_before();
+    // the last split of this output tile finishes it
+    __threadfence();
+    named_bar_sync(1, kEpiWarps * 32);
+    if (et == 0) *last_flag = ok ? (atomicAdd(ws_cnt + ntile, 1) == nsplit - 1) : 0;
+    named_bar_sync(1, kEpiWarps * 32);
+    if (*last_flag) {
+      __threadfence();
+      // thread et owns channel n0 + et for every token; 8 tokens per batch of
+      // independent loads
+      const int64_t nn = n0 + et;
+      if (nn < args.N) {
+        const float sn = args.w_scale[nn];
+        const float rwf = (float)args.w_rowsum[nn];
+        for (int64_t mb = 0; mb < args.M; mb += 8) {
+          float accf[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            accf[e] = mb + e < args.M ? __ldcg(ws_acc + (mb + e) * args.N + nn) : 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int64_t m = mb + e;
+            if (m < args.M) {
+              ws_acc[m * args.N + nn] = 0.f;
+              const float alpha = __ldg(args.a_scale + m);
+              const float bp = ASYM ? __ldg(args.a_zero + m) + 8.f * alpha : 0.f;
+              reinterpret_cast<__half*>(args.y)[m * args.N + nn] = __float2half_rn(sn * fmaf(alpha, accf[e], bp * rwf));
+              if (ACC_OUT) args.acc_out[m * args.N + nn] = __float2int_rn(accf[e]);
+            }
+          }
+        }
+      }
+      if (et == 0) ws_cnt[ntile] = 0;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, L::tmem_cols);
+  }
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -490,6 +762,35 @@ cudaError_t launch_mt(const GemmArgs& a, cudaStream_t stream) {
   return acc ? launch_t<MT, false, true>(a, stream) : launch_t<MT, false, false>(a, stream);
 }
 
+template <int MN, bool ASYM, bool ACC_OUT>
+cudaError_t launch_dec_t(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStream_t stream) {
+  using L = DecCfg<MN>;
+  CUtensorMap tmW, tmA;
+  if (!encode_packed_map(&tmW, a.w_codes, a.N, a.K, 128)) return cudaErrorNotSupported;
+  if (!encode_packed_map(&tmA, a.a_codes, a.M, a.K, MN)) return cudaErrorNotSupported;
+  auto kern = w4a4_decode_kernel<MN, ASYM, ACC_OUT>;
+  int per_sm = 0;
+  cudaError_t e = prepare_launch(kern, kDecThreads, L::dyn_bytes, &per_sm);
+  if (e != cudaSuccess) return e;
+  const int ksteps = (int)(a.K / 128);
+  const int ntiles = (int)((a.N + 127) / 128);
+  int nsplit = (device_sm_count() * per_sm) / ntiles;
+  if (nsplit < 1) nsplit = 1;
+  if (nsplit > ksteps) nsplit = ksteps;
+  dim3 grid((unsigned)nsplit, (unsigned)ntiles);
+  kern<<<grid, kDecThreads, L::dyn_bytes, stream>>>(tmW, tmA, a, ws_acc, ws_cnt, ksteps, nsplit);
+  return cudaGetLastError();
+}
+
+template <int MN>
+cudaError_t launch_dec_mn(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStream_t stream) {
+  const bool asym = a.a_zero != nullptr, acc = a.acc_out != nullptr;
+  if (asym) return acc ? launch_dec_t<MN, true, true>(a, ws_acc, ws_cnt, stream)
+                       : launch_dec_t<MN, true, false>(a, ws_acc, ws_cnt, stream);
+  return acc ? launch_dec_t<MN, false, true>(a, ws_acc, ws_cnt, stream)
+             : launch_dec_t<MN, false, false>(a, ws_acc, ws_cnt, stream);
+}
+
 }  // namespace
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
@@ -498,6 +799,23 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   const int64_t tiles256 = ((a.M + 255) / 256) * ((a.N + BN - 1) / BN);
   if (a.K >= 3072 && tiles256 >= 2 * (int64_t)device_sm_count()) return launch_mt<2>(a, stream);
   return launch_mt<1>(a, stream);
+}
+
+int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N) {
+  if (M <= 0 || N <= 0 || M > kDecodeMaxM) return 0;
+  return M * N * 4 + ((N + 127) / 128) * 4;
+}
+
+cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, cudaStream_t stream) {
+  if (a.M == 0 || a.N == 0) return cudaSuccess;
+  if (a.M > kDecodeMaxM) return launch_w4a4_gemm(a, stream);
+  float* ws_acc = static_cast<float*>(workspace);
+  int* ws_cnt = reinterpret_cast<int*>(static_cast<char*>(workspace) + a.M * a.N * 4);
+  if (a.M <= 16) return launch_dec_mn<16>(a, ws_acc, ws_cnt, stream);
+  if (a.M <= 32) return launch_dec_mn<32>(a, ws_acc, ws_cnt, stream);
+  if (a.M <= 64) return launch_dec_mn<64>(a, ws_acc, ws_cnt, stream);
+  if (a.M <= 128) return launch_dec_mn<128>(a, ws_acc, ws_cnt, stream);
+  return launch_dec_mn<256>(a, ws_acc, ws_cnt, stream);
 }
 
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail) {

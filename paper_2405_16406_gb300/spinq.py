@@ -33,7 +33,8 @@ SPINQ_PER_TOKEN, SPINQ_PER_CHANNEL, SPINQ_PER_GROUP = range(3)
 
 EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",
-    "spinq_status_string", "spinq_device_status", "spinq_version",
+    "spinq_status_string", "spinq_device_status", "spinq_version", "spinq_w4a4_gemm_workspace_bytes",
+    "spinq_w4a4_gemm_splitk",
 )
 
 
@@ -69,6 +70,10 @@ _lib.spinq_quant_weight.argtypes = [_P, _I64, _I64, ctypes.POINTER(HadCfg), ctyp
                                     _P, _P, _P, _P]
 _lib.spinq_w4a4_gemm.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
+_lib.spinq_w4a4_gemm_workspace_bytes.restype = ctypes.c_int64
+_lib.spinq_w4a4_gemm_workspace_bytes.argtypes = [_I64, _I64, _I64]
+_lib.spinq_w4a4_gemm_splitk.restype = ctypes.c_int
+_lib.spinq_w4a4_gemm_splitk.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P, _I64, _P]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
 _lib.spinq_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
                                        ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
@@ -92,6 +97,16 @@ def spinq_quant_weight(w, N, K, had, q, codes, scale, rowsum, stream) -> int:
 def spinq_w4a4_gemm(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc, stream) -> int:
     return _lib.spinq_w4a4_gemm(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc,
                                 stream)
+
+
+def spinq_w4a4_gemm_workspace_bytes(M, N, K) -> int:
+    return int(_lib.spinq_w4a4_gemm_workspace_bytes(M, N, K))
+
+
+def spinq_w4a4_gemm_splitk(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc, ws,
+                           ws_bytes, stream) -> int:
+    return _lib.spinq_w4a4_gemm_splitk(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc,
+                                       ws, ws_bytes, stream)
 
 
 def spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k_codes, k_scale,
@@ -187,6 +202,33 @@ def w4a4_gemm(a: ActCodes, w: WeightCodes, want_acc: bool = False, y: Optional[t
     _check(_lib.spinq_w4a4_gemm(_ptr(a.codes), _ptr(a.scale), _ptr(a.zero), _ptr(w.codes), _ptr(w.scale),
                                 _ptr(w.rowsum), M, N, K, _ptr(y), _ptr(acc), _stream(stream)),
            "spinq_w4a4_gemm")
+    return (y, acc) if want_acc else y
+
+
+def gemm_workspace(M: int, N: int, K: int, device=None) -> Optional[torch.Tensor]:
+    """Zeroed workspace for w4a4_gemm_splitk (None when the shape needs none)."""
+    nbytes = spinq_w4a4_gemm_workspace_bytes(M, N, K)
+    if nbytes == 0:
+        return None
+    return torch.zeros((nbytes + 15) // 16 * 16, dtype=torch.uint8, device=device or "cuda")
+
+
+def w4a4_gemm_splitk(a: ActCodes, w: WeightCodes, workspace: Optional[torch.Tensor] = None,
+                     want_acc: bool = False, y: Optional[torch.Tensor] = None,
+                     stream: Optional[torch.cuda.Stream] = None):
+    M = a.codes.shape[0]
+    N, Kh = w.codes.shape
+    K = Kh * 2
+    if workspace is None:
+        workspace = gemm_workspace(M, N, K, a.codes.device)
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float16, device=a.codes.device)
+    acc = torch.empty((M, N), dtype=torch.int32, device=a.codes.device) if want_acc else None
+    ws_bytes = 0 if workspace is None else workspace.numel()
+    _check(_lib.spinq_w4a4_gemm_splitk(_ptr(a.codes), _ptr(a.scale), _ptr(a.zero), _ptr(w.codes), _ptr(w.scale),
+                                       _ptr(w.rowsum), M, N, K, _ptr(y), _ptr(acc), _ptr(workspace), ws_bytes,
+                                       _stream(stream)),
+           "spinq_w4a4_gemm_splitk")
     return (y, acc) if want_acc else y
 
 

@@ -192,3 +192,59 @@ def test_rotation_reduces_quantization_error(S):
     y = S.w4a4_gemm(S.rotate_quant_act(x, c.had, True), S.quant_weight(w, c.had))
     y0 = S.w4a4_gemm(S.rotate_quant_act(x, None, True), S.quant_weight(w, None))
     assert pu.rel_frob(y.cpu().numpy(), ref) < pu.rel_frob(y0.cpu().numpy(), ref)
+
+
+# ------------------------------------------------------------------ split-K decode path
+def run_splitk(S, ac, al, be, wc, ws_, workspace=None):
+    a = to_gpu_act(S, ac, al, be)
+    w = to_gpu_w(S, wc, ws_)
+    y, acc = S.w4a4_gemm_splitk(a, w, workspace=workspace, want_acc=True)
+    torch.cuda.synchronize()
+    return y.cpu().numpy(), acc.cpu().numpy()
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 16, 128), (3, 48, 256), (16, 512, 1024), (17, 272, 384), (33, 1024, 512),
+                                   (64, 256, 128), (100, 384, 640), (128, 3072, 1024), (200, 256, 256),
+                                   (256, 512, 512), (300, 256, 256)])
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_splitk_random_codes_exact(S, M, N, K, symmetric):
+    rng = np.random.default_rng(M * 13 + N + K + symmetric)
+    ac, al, be, wc, ws_ = random_codes(rng, M, N, K, symmetric)
+    y, acc = run_splitk(S, ac, al, be, wc, ws_)
+    ref = oracle_full(ac, al, be, wc, ws_)
+    assert np.array_equal(acc, ref.acc)
+    assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
+    assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
+
+
+def test_splitk_workspace_reused_and_left_zero(S):
+    rng = np.random.default_rng(21)
+    M, N, K = 16, 1024, 2048
+    ws = S.gemm_workspace(M, N, K)
+    for rep in range(3):
+        ac, al, be, wc, ws_ = random_codes(rng, M, N, K, rep % 2 == 0)
+        y, acc = run_splitk(S, ac, al, be, wc, ws_, workspace=ws)
+        assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc)
+        assert int(torch.count_nonzero(ws)) == 0
+
+
+def test_splitk_extreme_codes_long_k(S):
+    M, N, K = 16, 256, 65536
+    for aval, wval in ((7, 7), (-8, -8), (7, -8)):
+        ac = np.full((M, K), aval, dtype=np.int32)
+        wc = np.full((N, K), wval, dtype=np.int32)
+        al, ws_ = np.full(M, 0.5), np.full(N, 0.25)
+        y, acc = run_splitk(S, ac, al, None, wc, ws_)
+        assert np.array_equal(acc, oracle_full(ac, al, None, wc, ws_).acc)
+
+
+@pytest.mark.parametrize("name,M,K,N,symmetric", [("l32_up_M1", 1, 3072, 8192, False),
+                                                  ("l32_up_M16", 16, 3072, 8192, False),
+                                                  ("l32_down_M128", 128, 8192, 3072, False)])
+def test_splitk_decode_configs_full(S, name, M, K, N, symmetric):
+    rng = np.random.default_rng(len(name) + M)
+    ac, al, be, wc, ws_ = random_codes(rng, M, N, K, symmetric)
+    y, acc = run_splitk(S, ac, al, be, wc, ws_)
+    ref = oracle_full(ac, al, be, wc, ws_)
+    assert np.array_equal(acc, ref.acc)
+    assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
