@@ -160,6 +160,34 @@ spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale
                                     int64_t workspace_bytes, void* stream);
 
 /*
+ * spinq_w4a4_gemm_noalloc -- spinq_w4a4_gemm_splitk for callers that cannot
+ * allocate device memory where they run the layer (a serving runtime that
+ * reserves its whole memory budget at start-up, a thread that must not call
+ * an allocator while other streams are being captured, an embedder with no
+ * allocator of its own).  The paper has no counterpart: this is an interface
+ * convenience, not part of the method.
+ *   Same arguments, outputs and requirements as spinq_w4a4_gemm; no workspace
+ *   argument.  The workspace lives in a fixed 8 MiB device array owned by the
+ *   library, which every GPU that loads the library holds until the process
+ *   exits; requests whose workspace (spinq_w4a4_gemm_workspace_bytes) exceeds
+ *   8 MiB return SPINQ_EUNSUPPORTED before any launch (M > 256 needs none and
+ *   is always accepted).
+ *   The call itself allocates nothing: no cudaMalloc/cudaFree and no
+ *   allocating library routine.  It clears the part of the array it uses
+ *   (cudaMemsetAsync on `stream`) before the kernel, since the array keeps
+ *   the previous call's contents.
+ *   The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   outside any stream capture.
+ *   Every call shares the one array per device: calls that may overlap on the
+ *   GPU (different streams without ordering between them) race on it.
+ */
+spinq_status spinq_w4a4_gemm_noalloc(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
+                                     const uint8_t* w_codes, const float* w_scale,
+                                     const int32_t* w_rowsum, int64_t M, int64_t N, int64_t K,
+                                     void* y_f16, int32_t* acc_out, void* stream);
+
+/*
  * spinq_rotate_quant_kv -- R3 on Q and K over head_dim, then the 4-bit
  * KV-cache quantizer (Sec. 3.1: R3 is an online Hadamard inserted for low-bit
  * KV-cache quantization; appendix "Quantization choice": asymmetric).

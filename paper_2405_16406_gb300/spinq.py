@@ -34,7 +34,7 @@ SPINQ_PER_TOKEN, SPINQ_PER_CHANNEL, SPINQ_PER_GROUP = range(3)
 EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",
     "spinq_status_string", "spinq_device_status", "spinq_version", "spinq_w4a4_gemm_workspace_bytes",
-    "spinq_w4a4_gemm_splitk",
+    "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc",
 )
 
 
@@ -74,6 +74,8 @@ _lib.spinq_w4a4_gemm_workspace_bytes.restype = ctypes.c_int64
 _lib.spinq_w4a4_gemm_workspace_bytes.argtypes = [_I64, _I64, _I64]
 _lib.spinq_w4a4_gemm_splitk.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_splitk.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P, _I64, _P]
+_lib.spinq_w4a4_gemm_noalloc.restype = ctypes.c_int
+_lib.spinq_w4a4_gemm_noalloc.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
 _lib.spinq_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
                                        ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
@@ -107,6 +109,12 @@ def spinq_w4a4_gemm_splitk(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum,
                            ws_bytes, stream) -> int:
     return _lib.spinq_w4a4_gemm_splitk(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc,
                                        ws, ws_bytes, stream)
+
+
+def spinq_w4a4_gemm_noalloc(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc,
+                            stream) -> int:
+    return _lib.spinq_w4a4_gemm_noalloc(a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y,
+                                        acc, stream)
 
 
 def spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k_codes, k_scale,
