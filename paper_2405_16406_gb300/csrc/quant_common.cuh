@@ -30,6 +30,11 @@ struct Range {
       asm("min.f32 %0, %0, %1, %2;" : "+f"(lo) : "f"(a), "f"(b));
     }
   }
+  __device__ __forceinline__ void add_pair(F2 v) {
+    float a, b;
+    f2_split(v, a, b);
+    add2(a, b);
+  }
   __device__ __forceinline__ void warp_reduce() {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -64,6 +69,7 @@ __device__ __forceinline__ void block_range(Range<SYM>& r, float* red) {
 template <bool SYM>
 struct QParams {
   float inv, off, alpha, beta;
+  F2 inv2, bias2;  // (inv, inv); (magic, magic) for SYM, (off, off) otherwise
   __device__ __forceinline__ QParams(const Range<SYM>& r, float clip) {
     if (SYM) {
       const float m = clip * r.hi;
@@ -78,6 +84,8 @@ struct QParams {
       beta = l2;
       off = -l2 * inv;
     }
+    inv2 = f2_make(inv, inv);
+    bias2 = SYM ? f2_make(kRoundMagic, kRoundMagic) : f2_make(off, off);
   }
   template <bool CLAMP>
   __device__ __forceinline__ uint32_t code_bits(float v) const {
@@ -86,13 +94,34 @@ struct QParams {
     if (CLAMP) t = SYM ? fminf(fmaxf(t, -8.f), 7.f) : fminf(fmaxf(t, 0.f), 15.f);
     return round_bits(t);
   }
+  // code_bits() of both lanes of a pair, on the packed fp32 pipe: the same
+  // operations in the same order, so the same bits
+  template <bool CLAMP>
+  __device__ __forceinline__ void code_bits2(F2 v, uint32_t& b0, uint32_t& b1) const {
+    float x0, x1;
+    if (CLAMP) {
+      f2_split(v, x0, x1);
+      b0 = code_bits<true>(x0);
+      b1 = code_bits<true>(x1);
+      return;
+    }
+    F2 t = f2_fma(v, inv2, bias2);
+    if (!SYM) t = f2_add(t, f2_make(kRoundMagic, kRoundMagic));
+    f2_split(t, x0, x1);
+    b0 = __float_as_uint(x0);
+    b1 = __float_as_uint(x1);
+  }
 };
 
 // ---------------------------------------------------------------------------
 // RowStream: rows of a row-major fp16 matrix streamed into shared memory with
 // TMA bulk copies, NST rows ahead, for a CTA that walks rows r0, r0 + G, ...
-// Thread 0 issues; every thread waits.  A stage is refilled (release) once
-// the CTA has read it.  Waits are bounded in time and set `*abort` on expiry.
+// A row is copied as `nseg` segments of `seg_bytes` (consecutive in global
+// memory, `seg_stride` bytes apart in shared memory, so that a kernel can pad
+// its segments).  Every thread waits; a stage is refilled once the CTA has
+// read it, by whichever warp reads it last (release_warp) or by thread 0
+// after a CTA barrier (release).  Waits are bounded in time and set `*abort`
+// on expiry.
 // ---------------------------------------------------------------------------
 template <int NST>
 struct RowStream {
@@ -101,26 +130,29 @@ struct RowStream {
   uint64_t* bars;       // NST mbarriers
   const uint8_t* src;   // matrix base
   int64_t row_bytes;    // pitch
-  uint32_t copy_bytes;  // bytes copied per row (multiple of 16)
+  uint32_t seg_bytes;   // bytes per segment (multiple of 16)
+  uint32_t nseg;        // segments per row
+  uint32_t seg_stride;  // shared-memory distance of consecutive segments
   int64_t rows, r0, G;
-  int issued;           // iterations issued so far (thread 0)
 
   __device__ __forceinline__ void init() {
     if (threadIdx.x == 0)
       for (int s = 0; s < NST; ++s) mbar_init(&bars[s], 1);
   }
+  __device__ __forceinline__ bool has(int iter) const { return r0 + (int64_t)iter * G < rows; }
   __device__ __forceinline__ void issue(int iter) {
+    if (!has(iter)) return;
     const int64_t row = r0 + (int64_t)iter * G;
-    if (row >= rows) return;
     const int s = iter % NST;
+    uint8_t* dst = stage0 + (size_t)s * stage_bytes;
+    const uint8_t* from = src + row * row_bytes;
     fence_proxy_async_smem();
-    mbar_arrive_expect_tx(&bars[s], copy_bytes);
-    bulk_load(stage0 + (size_t)s * stage_bytes, src + row * row_bytes, copy_bytes, &bars[s]);
-    issued = iter + 1;
+    mbar_arrive_expect_tx(&bars[s], seg_bytes * nseg);
+#pragma unroll 1
+    for (uint32_t i = 0; i < nseg; ++i) bulk_load(dst + i * seg_stride, from + (size_t)i * seg_bytes, seg_bytes, &bars[s]);
   }
   // thread 0, after init() and a CTA barrier
   __device__ __forceinline__ void prologue() {
-    issued = 0;
     if (threadIdx.x == 0)
       for (int i = 0; i < NST; ++i) issue(i);
   }
@@ -138,14 +170,30 @@ struct RowStream {
     }
     return true;
   }
-  // thread 0, after the CTA has finished reading stage(iter)
+  // thread 0, after a CTA barrier that follows the last read of stage(iter)
   __device__ __forceinline__ void release(int iter) {
     if (threadIdx.x == 0) issue(iter + NST);
   }
-  // thread 0: let copies in flight land before the CTA exits (abort path)
+  // every warp, once it has finished reading stage(iter) (its loads have
+  // returned); the last of `nwarps` warps to get here refills the stage.
+  // `count` is a shared-memory word that starts at 0 and is left at 0.
+  __device__ __forceinline__ void release_warp(int iter, int* count, int nwarps) {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) {
+      __threadfence_block();
+      if (atomicAdd(count, 1) == nwarps - 1) {
+        *count = 0;
+        issue(iter + NST);
+      }
+    }
+  }
+  // thread 0 on the abort path at iteration `iter` (every earlier stage was
+  // released, so the copies of iter .. iter + NST - 1 may be in flight): let
+  // them land before the CTA exits
   __device__ __forceinline__ void drain(int iter, uint64_t limit_ns) {
     if (threadIdx.x != 0) return;
-    for (int j = iter; j < issued; ++j) {
+    for (int j = iter; j < iter + NST; ++j) {
+      if (!has(j)) break;
       const uint64_t t0 = globaltimer_ns();
       while (!mbar_try_wait(&bars[j % NST], (j / NST) & 1) && globaltimer_ns() - t0 < limit_ns) {
       }

@@ -59,20 +59,12 @@ __device__ __forceinline__ void make_b16(uint32_t b[2][2], bool hadamard) {
   }
 }
 
-// One 16-byte chunk (8 fp16) through the tensor core: y[e] for e = 0..7.
-__device__ __forceinline__ void chunk_mma(const uint4 in, const uint32_t b[2][2], float y[8]) {
+// One 16-byte chunk (8 fp16) through the tensor core: the results y[e],
+// e = 0..7, come back as the pairs y2[q] = (y[2q], y[2q + 1]).
+__device__ __forceinline__ void chunk_mma(const uint4 in, const uint32_t b[2][2], F2 y2[4]) {
   const uint32_t A[4] = {in.x, in.z, in.y, in.w};
-  float d0[4], d1[4];
-  mma_16816_f16_f32(d0, A, b[0][0], b[0][1]);
-  mma_16816_f16_f32(d1, A, b[1][0], b[1][1]);
-  y[0] = d0[0];
-  y[1] = d0[1];
-  y[4] = d0[2];
-  y[5] = d0[3];
-  y[2] = d1[0];
-  y[3] = d1[1];
-  y[6] = d1[2];
-  y[7] = d1[3];
+  mma_16816_f16_f32_pairs(y2[0], y2[2], A, b[0][0], b[0][1]);
+  mma_16816_f16_f32_pairs(y2[1], y2[3], A, b[1][0], b[1][1]);
 }
 
 // ------------------------------------------------------------------------
@@ -126,13 +118,15 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
   uint32_t bh[2][2];
   make_b16(bh, true);
 
+  int* release_count = reinterpret_cast<int*>(smem + SM::OFF_MISC + 4);
   RowStream<SM::NST> rs{smem + SM::OFF_STAGE, (uint32_t)(S::P * 2),
                         reinterpret_cast<uint64_t*>(smem + SM::OFF_BAR),
-                        reinterpret_cast<const uint8_t*>(a.x), a.ldx * 2, (uint32_t)(S::P * 2),
-                        a.rows, (int64_t)blockIdx.x, (int64_t)gridDim.x, 0};
+                        reinterpret_cast<const uint8_t*>(a.x), a.ldx * 2, (uint32_t)(S::P * 2), 1u, 0u,
+                        a.rows, (int64_t)blockIdx.x, (int64_t)gridDim.x};
   rs.init();
   if (tid == 0) {
     *abort_flag = 0;
+    *release_count = 0;
     fence_mbar_init();
   }
   __syncthreads();
@@ -153,48 +147,42 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
     if (*abort_flag) break;
     // ---------------- phase 1
     const uint4* src = reinterpret_cast<const uint4*>(rs.stage(it));
-    float y[S::V][8];
+    F2 y[S::V][4];  // y[v][q] = elements (2q, 2q + 1) of chunk v
 #pragma unroll
     for (int v = 0; v < S::V; ++v) chunk_mma(src[lane + 32 * (w + S::W * v)], bh, y[v]);
+    rs.release_warp(it, release_count, S::W);  // the next copy into this stage overlaps the rest of the row
 #pragma unroll
-    for (int v = 0; v < S::V; ++v)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float p0 = y[v][e], p1 = y[v][e + 4];
-        y[v][e] = p0 + p1;
-        y[v][e + 4] = p0 - p1;
-      }
+    for (int v = 0; v < S::V; ++v) {  // e2
+      f2_bfly(y[v][0], y[v][2]);
+      f2_bfly(y[v][1], y[v][3]);
+    }
 #pragma unroll
     for (int bit = 1; bit < S::V; bit <<= 1)
 #pragma unroll
       for (int v = 0; v < S::V; ++v)
         if (!(v & bit)) {
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float p0 = y[v][e], p1 = y[v | bit][e];
-            y[v][e] = p0 + p1;
-            y[v | bit][e] = p0 - p1;
-          }
+          for (int q = 0; q < 4; ++q) f2_bfly(y[v][q], y[v | bit][q]);
         }
 #pragma unroll
     for (int v = 0; v < S::V; ++v) {
       const uint32_t ch = (uint32_t)(lane + 32 * (w + S::W * v));
-      *reinterpret_cast<float4*>(sm + 4 * ch) = make_float4(y[v][0], y[v][1], y[v][2], y[v][3]);
-      *reinterpret_cast<float4*>(sm + S::P / 2 + 16 + 4 * ch) = make_float4(y[v][4], y[v][5], y[v][6], y[v][7]);
+      *reinterpret_cast<ulonglong2*>(sm + 4 * ch) = make_ulonglong2(y[v][0].u, y[v][1].u);
+      *reinterpret_cast<ulonglong2*>(sm + S::P / 2 + 16 + 4 * ch) = make_ulonglong2(y[v][2].u, y[v][3].u);
     }
     __syncthreads();
-    rs.release(it);  // the staged row is consumed: the next copy overlaps phase 2
 
     // ---------------- phase 2: groups m cover element bits 5.. (g, then w)
-    float z[S::NG][S::GL];
+    constexpr int GP = S::GL / 2;  // pairs per group
+    F2 z[S::NG][GP];
 #pragma unroll
     for (int m = 0; m < S::NG; ++m) {
-      if constexpr (S::GL == 4) {
-        const float4 u0 = *reinterpret_cast<const float4*>(zbase + 16 * m);
-        z[m][0] = u0.x; z[m][1 % S::GL] = u0.y; z[m][2 % S::GL] = u0.z; z[m][3 % S::GL] = u0.w;
+      if constexpr (GP == 2) {
+        const ulonglong2 u = *reinterpret_cast<const ulonglong2*>(zbase + 16 * m);
+        z[m][0].u = u.x;
+        z[m][GP - 1].u = u.y;
       } else {
-        const float2 u0 = *reinterpret_cast<const float2*>(zbase + 16 * m);
-        z[m][0] = u0.x; z[m][1 % S::GL] = u0.y;
+        z[m][0].u = *reinterpret_cast<const unsigned long long*>(zbase + 16 * m);
       }
     }
 #pragma unroll
@@ -203,17 +191,13 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
       for (int m = 0; m < S::NG; ++m)
         if (!(m & bit)) {
 #pragma unroll
-          for (int j = 0; j < S::GL; ++j) {
-            const float p0 = z[m][j], p1 = z[m | bit][j];
-            z[m][j] = p0 + p1;
-            z[m | bit][j] = p0 - p1;
-          }
+          for (int q = 0; q < GP; ++q) f2_bfly(z[m][q], z[m | bit][q]);
         }
     Range<SYM> r;
 #pragma unroll
     for (int m = 0; m < S::NG; ++m)
 #pragma unroll
-      for (int j = 0; j < S::GL; j += 2) r.add2(z[m][j], z[m][j + 1]);
+      for (int q = 0; q < GP; ++q) r.add_pair(z[m][q]);
     block_range<SYM, S::W>(r, red);
     const QParams<SYM> qp(r, a.clip);
 
@@ -221,12 +205,13 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
 #pragma unroll
     for (int m = 0; m < S::NG; ++m) {
       // element offset of group m is 32 m (bits 5..), i.e. 16 m bytes of codes
-      if constexpr (S::GL == 4) {
-        const uint32_t wv = pack4_nibbles(qp.template code_bits<CLAMP>(z[m][0]), qp.template code_bits<CLAMP>(z[m][1 % S::GL]),
-                                          qp.template code_bits<CLAMP>(z[m][2 % S::GL]), qp.template code_bits<CLAMP>(z[m][3 % S::GL]));
-        *reinterpret_cast<uint16_t*>(out + 16 * m) = (uint16_t)wv;
+      uint32_t rb[4];
+      qp.template code_bits2<CLAMP>(z[m][0], rb[0], rb[1]);
+      if constexpr (GP == 2) {
+        qp.template code_bits2<CLAMP>(z[m][GP - 1], rb[2], rb[3]);
+        *reinterpret_cast<uint16_t*>(out + 16 * m) = (uint16_t)pack4_nibbles(rb[0], rb[1], rb[2], rb[3]);
       } else {
-        out[16 * m] = (uint8_t)pack2_nibbles(qp.template code_bits<CLAMP>(z[m][0]), qp.template code_bits<CLAMP>(z[m][1 % S::GL]));
+        out[16 * m] = (uint8_t)pack2_nibbles(rb[0], rb[1]);
       }
     }
     if (tid == 0) {
@@ -258,11 +243,13 @@ __global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
   make_b16(bi, false);
   const int nchunk = (int)(a.K / 8);
 
+  int* release_count = const_cast<int*>(abort_flag) + 1;
   RowStream<kNoRotStages> rs{smem, stage_bytes, bars, reinterpret_cast<const uint8_t*>(a.x), a.ldx * 2,
-                             row_bytes, a.rows, (int64_t)blockIdx.x, (int64_t)gridDim.x, 0};
+                             row_bytes, 1u, 0u, a.rows, (int64_t)blockIdx.x, (int64_t)gridDim.x};
   rs.init();
   if (tid == 0) {
     *abort_flag = 0;
+    *release_count = 0;
     fence_mbar_init();
   }
   __syncthreads();
@@ -274,20 +261,19 @@ __global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
     __syncthreads();
     if (*abort_flag) break;
     const uint4* src = reinterpret_cast<const uint4*>(rs.stage(it));
-    float y[kNoRotV][8];
+    F2 y[kNoRotV][4];
 #pragma unroll
     for (int v = 0; v < kNoRotV; ++v) {
       const int ch = lane + 32 * (w + W * v);
       chunk_mma(ch < nchunk ? src[ch] : make_uint4(0, 0, 0, 0), bi, y[v]);  // exact fp16 -> fp32
     }
-    __syncthreads();
-    rs.release(it);
+    rs.release_warp(it, release_count, W);
     Range<SYM> r;
 #pragma unroll
     for (int v = 0; v < kNoRotV; ++v)
       if (lane + 32 * (w + W * v) < nchunk)
 #pragma unroll
-        for (int e = 0; e < 8; ++e) r.add(y[v][e]);
+        for (int q = 0; q < 4; ++q) r.add_pair(y[v][q]);
     block_range<SYM, W>(r, red);
     const QParams<SYM> qp(r, a.clip);
     uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
@@ -296,7 +282,7 @@ __global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
       const int ch = lane + 32 * (w + W * v);
       uint32_t rb[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) rb[e] = qp.template code_bits<CLAMP>(y[v][e]);
+      for (int q = 0; q < 4; ++q) qp.template code_bits2<CLAMP>(y[v][q], rb[2 * q], rb[2 * q + 1]);
       if (ch < nchunk) out[ch] = pack8_nibbles(rb);
     }
     if (tid == 0) {

@@ -3,298 +3,413 @@
 // P in {128, 256, 512} (Sec. 3.1, R4 of non-power-of-two size), fused with the
 // per-token Eq. 1 quantizer.  Element k = i * P + j (i: Paley index).
 //
-// One CTA (W = P/64 warps) owns one row at a time; rows stream in through
-// shared memory with TMA bulk copies, NST rows ahead (one copy per Paley
-// segment i, each segment padded by 16 bytes so that ldmatrix is free of bank
-// conflicts).
+// A persistent CTA walks rows r0, r0 + G, ... with two warp roles that hand
+// work to each other through mbarriers (no CTA-wide barrier in the loop):
+//
+//  * phase-1 warps (W = P/64): the H_s factor on the tensor core plus the
+//    first butterflies, written to one of two fp32 transpose buffers;
+//  * phase-2 warps (W): the remaining butterflies, the row range, Eq. 1 and
+//    the packed codes.
+//
+// Rows arrive in a ring of NSTG shared-memory stages, one TMA tensor copy per
+// row; the last phase-1 warp to finish reading a stage issues the copy of the
+// row NSTG iterations ahead into it.  The tensor map views a row as
+// (j_lo = j % 64, i, j_hi = j / 64), so a stage holds 128-byte lines
+// l = i + n_s j_hi with the 128-byte swizzle: the 16-byte chunk c of line l
+// sits at chunk c ^ (l % 8), which keeps ldmatrix free of bank conflicts.
+// Phase 1 of row r + 1 runs while phase 2 of row r runs, and the copies of
+// the next rows are in flight meanwhile.
 //
 // Phase 1 (tensor core, raw fp16).  Y[i][j] = sum_i' X[i'][j] H_s[i'][i] is an
 // m16n8k16 MMA per 16 consecutive j: A[m = j][k = i'] comes straight from the
 // staged fp16 rows with ldmatrix.trans, B = H_s (+-1, zero-padded to 16/32).
-// Lane (g, c) of warp w receives j = 16 (w + W v) + 8 h + g for h in {0, 1},
-// v in 0..3 and i = 2c + {0, 1} + 8 nt.  Radix-2 butterflies inside the lane
-// cover the j bits of h and v.
+// Lane (g, c) of phase-1 warp w receives j = 16 (w + W v) + 8 h + g for h in
+// {0, 1}, v in 0..3 and i = 2c + {0, 1} + 8 nt.  Radix-2 butterflies inside
+// the lane cover the j bits of h and v, on packed fp32 pairs (i, i + 1).
 //
-// Transpose.  Y goes to a padded fp32 buffer (row stride P + 4: conflict-free
-// for both the scalar stores here and the 16-byte loads of phase 2).
+// Transpose.  Y goes to an fp32 buffer with row stride P + 4 in which j is
+// stored at j ^ (bit (4 + log2 W) of j) << 2 ^ (bit (5 + log2 W) of j) << 4:
+// the scalar stores here and the 16-byte loads of phase 2 are both free of
+// bank conflicts.
 //
 // Phase 2.  A thread owns, for one i, the 8 consecutive j of bits 0..2 for
-// each value of the warp bits (8 W values), finishes the butterflies over
-// those bits, joins the row-wide range reduction and stores 32-bit words of 8
-// packed codes.  Eq. 1 runs on the unnormalised row; alpha and beta carry
-// 1/sqrt(K).
+// each value of the phase-1 warp bits (8 W values), finishes the butterflies
+// over those bits on pairs of consecutive elements and joins the row-wide
+// range reduction (one named barrier over the phase-2 warps).  The 8 lanes of
+// a quarter warp share i, so a warp writes 4 whole segments of codes: lane
+// pairs swap packed words so that each lane stores 16 contiguous bytes.
+// Eq. 1 runs on the unnormalised row; alpha and beta carry 1/sqrt(K).
+//
+// Every wait is bounded in time.  A warp that gives up raises the CTA's abort
+// flag; the others see it in their own waits, the phase-2 warps agree on it
+// through a barrier reduction before any global store, and the phase-1 warps
+// let the copies in flight land before they exit.
 #include <cuda_fp16.h>
 
 #include "launch_util.h"
 #include "quant_common.cuh"
 #include "spinq_device.cuh"
 #include "spinq_internal.h"
+#include "tensor_map.h"
 
 namespace spinq {
 namespace {
 
-constexpr uint64_t kRowWaitLimitNs = 2000000000ull;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr int kSmemBudget = 232448;  // dynamic shared memory a CTA may opt into
+constexpr int kPhase2Bar = 1;        // named barrier of the phase-2 warps
+constexpr int kPhase1Bar = 2;        // named barrier of the phase-1 warps (exit only)
 
 template <int NS, int LP>
 struct PaleyShape {
   static constexpr int P = 1 << LP;
-  static constexpr int W = P / 64;                 // warps
-  static constexpr int T = 32 * W;
+  static constexpr int W = P / 64;                 // warps per compute role
+  static constexpr int T = 32 * W;                 // threads per compute role
+  static constexpr int THREADS = 2 * T;            // phase-1 warps, then phase-2 warps
   static constexpr int KS = (NS + 15) / 16;        // k16 steps over i'
   static constexpr int NT = (NS + 7) / 8;          // n8 tiles over i
   static constexpr int NSP = NS <= 16 ? 16 : 32;   // phase-2 row slots
-  static constexpr int NCOMBO = NSP * 8;          // phase-2 (i slot, j group) combos
+  static constexpr int NCOMBO = NSP * 8;           // phase-2 (i slot, j group) combos
   static constexpr int NCB = (NCOMBO + T - 1) / T; // combos per thread
   static constexpr int PS = P + 4;                 // fp32 row stride
-  static constexpr int SEGB = 2 * P + 16;          // staged fp16 segment stride (bytes)
-  static constexpr int ROWB = NS * SEGB;           // staged row (bytes)
-  // rows in flight: one staged row for the large shapes so that two CTAs fit
-  // on an SM; the next row is requested as soon as phase 1 has consumed the
-  // current one, so its copy overlaps phase 2
-  static constexpr int NST = NS * P >= 8192 ? 1 : 2;
-  // shared memory layout (bytes)
+  static constexpr int ROWB = NS * P * 2;          // staged row (bytes, a multiple of 1024)
+  static constexpr int F32B = NS * PS * 4;         // one transpose buffer (bytes)
+  static constexpr int MISC = 16 + 4 * 8 + 16 + 2 * 2 * W * 4;  // zero chunk, 4 barriers, flag, range scratch
+  static constexpr int NSTG_FIT = (kSmemBudget - 1024 - 2 * F32B - MISC) / (ROWB + 16);  // 16: barrier + counters
+  static constexpr int NSTG = NSTG_FIT < 4 ? NSTG_FIT : 4;   // staged rows
+  static_assert(NSTG >= 2, "two staged rows must fit");
+  static_assert(ROWB % 1024 == 0, "stages keep the 1024-byte alignment of the swizzle pattern");
+  // shared memory layout (bytes from the 1024-aligned base)
   static constexpr int OFF_STAGE = 0;
-  static constexpr int OFF_ZERO = NST * ROWB;
-  static constexpr int OFF_F32 = OFF_ZERO + 16;
-  static constexpr int OFF_BAR = OFF_F32 + NS * PS * 4;
-  static constexpr int OFF_RED = OFF_BAR + NST * 8;
-  static constexpr int BYTES = OFF_RED + 2 * W * 4 + 16;
+  static constexpr int OFF_F32 = NSTG * ROWB;
+  static constexpr int OFF_ZERO = OFF_F32 + 2 * F32B;
+  static constexpr int OFF_BAR = OFF_ZERO + 16;    // full[NSTG] bfull[2] bempty[2]
+  static constexpr int OFF_CNT = OFF_BAR + (NSTG + 4) * 8;   // int readers[NSTG], int issued[NSTG]
+  static constexpr int OFF_FLAG = OFF_CNT + NSTG * 8;
+  static constexpr int OFF_RED = OFF_FLAG + 16;    // [2 rows][hi W, lo W]
+  static constexpr int BYTES = OFF_RED + 2 * 2 * W * 4 + 1024;  // + alignment slack
+  static_assert(BYTES <= kSmemBudget, "shared memory");
 };
 
-template <int NS, int LP, bool SYM, bool CLAMP>
-__global__ void __launch_bounds__(32 * ((1 << LP) / 64), 16 / ((1 << LP) / 64)) rq_paley_kernel(RotQuantArgs a) {
-  using S = PaleyShape<NS, LP>;
-  constexpr int P = S::P, W = S::W;
-  extern __shared__ __align__(128) uint8_t smem[];
-  float* sf = reinterpret_cast<float*>(smem + S::OFF_F32);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
-  float* red = reinterpret_cast<float*>(smem + S::OFF_RED);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + S::OFF_RED + 2 * W * 4);
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, g = lane >> 2, c = lane & 3;
-  const uint8_t* __restrict__ x = reinterpret_cast<const uint8_t*>(a.x);
-  const int64_t row_bytes = a.ldx * 2;
+// Paley row slot of phase-2 combo cb: the 8 lanes of a quarter warp share
+// it (cb & 7 is the j group), so a warp covers 4 consecutive slots
+__device__ __forceinline__ int combo_i(int cb) {
+  return ((cb >> 5) << 2) | ((cb >> 3) & 3);
+}
 
-  // B fragments of H_s (k = i', n = i), zero outside NS
-  uint32_t bs[S::KS][S::NT][2];
-#pragma unroll
-  for (int ks = 0; ks < S::KS; ++ks)
-#pragma unroll
-    for (int nt = 0; nt < S::NT; ++nt) {
-      const int n = g + 8 * nt;
-#pragma unroll
-      for (int hb = 0; hb < 2; ++hb) {
-        const int k0 = 2 * c + 8 * hb + 16 * ks;
-        float v[2];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int k = k0 + e;
-          v[e] = (k < NS && n < NS) ? (((a.hs.neg[k] >> n) & 1u) ? -1.f : 1.f) : 0.f;
-        }
-        bs[ks][nt][hb] = pack_half2_bits(v[0], v[1]);
-      }
+// Bounded wait for the phase of `bar` with `parity`.  Returns false when the
+// abort flag is up or the limit expired (then it raises the flag).
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      *abort_flag = 1;
+      return false;
     }
+  }
+  return true;
+}
+
+// bar.sync over `nthreads` threads whose result is the OR of `pred` over them.
+__device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
+template <int NS, int LP, bool SYM, bool CLAMP>
+__global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
+    rq_paley_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
+  using S = PaleyShape<NS, LP>;
+  constexpr int P = S::P, W = S::W, T = S::T, NSTG = S::NSTG;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
+  uint64_t* bfull = full + NSTG;
+  uint64_t* bempty = bfull + 2;
+  int* readers = reinterpret_cast<int*>(smem + S::OFF_CNT);  // phase-1 warps done with a stage
+  int* issued = readers + NSTG;                              // last iteration copied into a stage
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + S::OFF_FLAG);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t r0 = blockIdx.x, G = gridDim.x;
+  const int niter = a.rows > r0 ? (int)((a.rows - r0 + G - 1) / G) : 0;
+  // copy of iteration `it` into its stage (one thread)
+  auto issue = [&](int it) {
+    const int s = it % NSTG;
+    fence_proxy_async_smem();
+    mbar_arrive_expect_tx(&full[s], (uint32_t)S::ROWB);
+    tma_load_4d(smem + S::OFF_STAGE + s * S::ROWB, &tmx, &full[s], 0, 0, 0, (int32_t)(r0 + (int64_t)it * G));
+    issued[s] = it;
+  };
 
   if (tid == 0) {
-    for (int s = 0; s < S::NST; ++s) mbar_init(&full[s], 1);
+    for (int s = 0; s < NSTG; ++s) {
+      mbar_init(&full[s], 1);
+      readers[s] = 0;
+      issued[s] = -1;
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bfull[b], T);
+      mbar_init(&bempty[b], T);
+    }
     *reinterpret_cast<uint4*>(smem + S::OFF_ZERO) = make_uint4(0, 0, 0, 0);
     *abort_flag = 0;
     fence_mbar_init();
+    prefetch_tmap(&tmx);
   }
-  __syncthreads();
+  __syncthreads();  // the last CTA-wide barrier: the roles part here
+  if (tid == 0)
+    for (int it = 0; it < NSTG && it < niter; ++it) issue(it);
 
-  const int64_t r0 = blockIdx.x, G = gridDim.x;
-  auto issue = [&](int64_t row, int stage) {
-    uint8_t* dst = smem + S::OFF_STAGE + stage * S::ROWB;
-    fence_proxy_async_smem();  // earlier ldmatrix reads of this stage precede the copy
-    mbar_arrive_expect_tx(&full[stage], (uint32_t)(NS * P * 2));
-    const uint8_t* src = x + row * row_bytes;
-#pragma unroll 1
-    for (int i = 0; i < NS; ++i) bulk_load(dst + i * S::SEGB, src + i * P * 2, P * 2, &full[stage]);
-  };
-  int issued = 0;  // iterations whose row copy has been issued (thread 0 only)
-  if (tid == 0) {
-    for (int s = 0; s < S::NST; ++s)
-      if (r0 + s * G < a.rows) {
-        issue(r0 + s * G, s);
-        issued = s + 1;
-      }
-  }
-
-  // phase-2 identity
-  const uint32_t zero_addr = smem_u32(smem + S::OFF_ZERO);
-  int it = 0;
-  for (int64_t row = r0; row < a.rows; row += G, ++it) {
-    const int st = it % S::NST;
-    // wait for this row (bounded)
-    {
-      bool ok = mbar_try_wait(&full[st], (it / S::NST) & 1);
-      if (!ok) {
-        const uint64_t t0 = globaltimer_ns();
-        while (!(ok = mbar_try_wait(&full[st], (it / S::NST) & 1))) {
-          if (*abort_flag || globaltimer_ns() - t0 > kRowWaitLimitNs) break;
-        }
-      }
-      if (!ok) *abort_flag = 1;
-    }
-    __syncthreads();
-    if (*abort_flag) break;
-    const uint32_t stage_addr = smem_u32(smem + S::OFF_STAGE + st * S::ROWB);
-
-    // ---------------- phase 1: H_s on the tensor core
-    float y[S::NT][2][2][4];  // [nt][hi][h][v]
+  if (warp < W) {
+    // ---------------- phase 1: H_s on the tensor core, first butterflies
+    const int w = warp, g = lane >> 2, c = lane & 3;
+    // B fragments of H_s (k = i', n = i), zero outside NS
+    uint32_t bs[S::KS][S::NT][2];
 #pragma unroll
-    for (int v = 0; v < 4; ++v) {
-      const int jb = 16 * (w + W * v);
-      float d[S::NT][4];
-#pragma unroll
-      for (int nt = 0; nt < S::NT; ++nt) d[nt][0] = d[nt][1] = d[nt][2] = d[nt][3] = 0.f;
-#pragma unroll
-      for (int ks = 0; ks < S::KS; ++ks) {
-        const int q = lane >> 3, r = lane & 7;
-        const int ip = r + 8 * (q >> 1) + 16 * ks;
-        const int js = jb + 8 * (q & 1);
-        const uint32_t addr = ip < NS ? stage_addr + (uint32_t)(ip * S::SEGB + js * 2) : zero_addr;
-        uint32_t af[4];
-        ldmatrix_x4_trans(af, addr);
-#pragma unroll
-        for (int nt = 0; nt < S::NT; ++nt) mma_16816_f16_f32_acc(d[nt], af, bs[ks][nt][0], bs[ks][nt][1]);
-      }
+    for (int ks = 0; ks < S::KS; ++ks)
 #pragma unroll
       for (int nt = 0; nt < S::NT; ++nt) {
-        y[nt][0][0][v] = d[nt][0];
-        y[nt][1][0][v] = d[nt][1];
-        y[nt][0][1][v] = d[nt][2];
-        y[nt][1][1][v] = d[nt][3];
-      }
-    }
-    // butterflies over h (j bit 3) and v (the two highest j bits)
+        const int n = g + 8 * nt;
 #pragma unroll
-    for (int nt = 0; nt < S::NT; ++nt)
+        for (int hb = 0; hb < 2; ++hb) {
+          const int k0 = 2 * c + 8 * hb + 16 * ks;
+          float v[2];
 #pragma unroll
-      for (int hi = 0; hi < 2; ++hi) {
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          const float p0 = y[nt][hi][0][v], p1 = y[nt][hi][1][v];
-          y[nt][hi][0][v] = p0 + p1;
-          y[nt][hi][1][v] = p0 - p1;
+          for (int e = 0; e < 2; ++e) {
+            const int k = k0 + e;
+            v[e] = (k < NS && n < NS) ? (((a.hs.neg[k] >> n) & 1u) ? -1.f : 1.f) : 0.f;
+          }
+          bs[ks][nt][hb] = pack_half2_bits(v[0], v[1]);
         }
+      }
+    const uint32_t zero_addr = smem_u32(smem + S::OFF_ZERO);
+    // transpose-buffer position of j = 16 (w + W v) + 8 h + g, minus 8 h: bit 2
+    // of j flips with v & 1, bit 4 (the low bit of w) with v >> 1
+    int pos[4];
+#pragma unroll
+    for (int v = 0; v < 4; ++v) pos[v] = 16 * ((w ^ (v >> 1)) + W * v) + (g ^ ((v & 1) << 2));
+    for (int it = 0; it < niter; ++it) {
+      const int s = it % NSTG;
+      // warp-uniform decision: the MMAs below need every lane
+      if (!__all_sync(0xffffffffu, wait_or_abort(&full[s], (uint32_t)(it / NSTG) & 1u, abort_flag))) break;
+      const uint32_t stage_addr = smem_u32(smem + S::OFF_STAGE + s * S::ROWB);
+      // y[nt][h][v] = the pair of outputs i = 2c + 8 nt + {0, 1} at
+      // j = 16 (w + W v) + 8 h + g
+      F2 y[S::NT][2][4];
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const int jb = 16 * (w + W * v);
+#pragma unroll
+        for (int ks = 0; ks < S::KS; ++ks) {
+          const int q = lane >> 3, r = lane & 7;
+          const int ip = r + 8 * (q >> 1) + 16 * ks;
+          const int js = jb + 8 * (q & 1);
+          const int line = ip + NS * (js >> 6);
+          const uint32_t addr =
+              ip < NS ? stage_addr + (uint32_t)(line * 128 + ((((js & 63) >> 3) ^ (line & 7)) << 4)) : zero_addr;
+          uint32_t af[4];
+          ldmatrix_x4_trans(af, addr);
+#pragma unroll
+          for (int nt = 0; nt < S::NT; ++nt) {
+            if (ks == 0)
+              mma_16816_f16_f32_pairs(y[nt][0][v], y[nt][1][v], af, bs[ks][nt][0], bs[ks][nt][1]);
+            else
+              mma_16816_f16_f32_pairs_acc(y[nt][0][v], y[nt][1][v], af, bs[ks][nt][0], bs[ks][nt][1]);
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) {
+        // this warp no longer reads the stage; the last one refills it
+        __threadfence_block();
+        if (atomicAdd(&readers[s], 1) == W - 1) {
+          readers[s] = 0;
+          if (it + NSTG < niter) issue(it + NSTG);
+        }
+      }
+      // butterflies over h (j bit 3) and v (the two highest j bits)
+#pragma unroll
+      for (int nt = 0; nt < S::NT; ++nt) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) f2_bfly(y[nt][0][v], y[nt][1][v]);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
           for (int bit = 1; bit < 4; bit <<= 1)
 #pragma unroll
             for (int v = 0; v < 4; ++v)
-              if (!(v & bit)) {
-                const float p0 = y[nt][hi][h][v], p1 = y[nt][hi][h][v | bit];
-                y[nt][hi][h][v] = p0 + p1;
-                y[nt][hi][h][v | bit] = p0 - p1;
-              }
+              if (!(v & bit)) f2_bfly(y[nt][h][v], y[nt][h][v | bit]);
       }
-    // transpose through shared memory
+      const int b = it & 1;
+      if (it >= 2 &&
+          !__all_sync(0xffffffffu, wait_or_abort(&bempty[b], (uint32_t)((it >> 1) - 1) & 1u, abort_flag)))
+        break;
+      // transpose through shared memory (NS is even: both outputs of a pair
+      // are real or both are padding)
+      float* sf = reinterpret_cast<float*>(smem + S::OFF_F32 + b * S::F32B);
 #pragma unroll
-    for (int nt = 0; nt < S::NT; ++nt)
-#pragma unroll
-      for (int hi = 0; hi < 2; ++hi) {
-        const int i = 2 * c + 8 * nt + hi;
+      for (int nt = 0; nt < S::NT; ++nt) {
+        const int i = 2 * c + 8 * nt;
         if (i < NS) {
 #pragma unroll
           for (int h = 0; h < 2; ++h)
 #pragma unroll
-            for (int v = 0; v < 4; ++v) sf[i * S::PS + 16 * (w + W * v) + 8 * h + g] = y[nt][hi][h][v];
+            for (int v = 0; v < 4; ++v) {
+              float lo, hi;
+              f2_split(y[nt][h][v], lo, hi);
+              float* dst = sf + i * S::PS + pos[v] + 8 * h;
+              dst[0] = lo;
+              dst[S::PS] = hi;
+            }
         }
       }
-    __syncthreads();
-    // the staged row is consumed: request the row NST iterations ahead into it
-    if (tid == 0) {
-      const int64_t nxt = row + (int64_t)S::NST * G;
-      if (nxt < a.rows) {
-        issue(nxt, st);
-        issued = it + S::NST + 1;
-      }
+      mbar_arrive(&bfull[b]);
     }
+    // every phase-1 warp has stopped issuing; after an abort, let the copies
+    // still in flight land before the CTA can exit
+    named_bar_sync(kPhase1Bar, T);
+    if (*abort_flag && tid == 0)
+      for (int s = 0; s < NSTG; ++s)
+        if (issued[s] >= 0) mbar_wait_bounded(&full[s], (uint32_t)(issued[s] / NSTG) & 1u, kWaitLimitNs);
+    return;
+  }
 
-    // ---------------- phase 2
-    float z[S::NCB][W][8];
-    Range<SYM> rg;
+  // ---------------- phase 2: remaining butterflies, range, Eq. 1, codes
+  const int t2 = tid - T, w2 = warp - W;
+  float* red = reinterpret_cast<float*>(smem + S::OFF_RED);
+  for (int it = 0; it < niter; ++it) {
+    const int64_t row = r0 + (int64_t)it * G;
+    const int b = it & 1;
+    // on a failed wait the buffer is read anyway (in bounds, discarded below)
+    const bool ok = wait_or_abort(&bfull[b], (uint32_t)(it >> 1) & 1u, abort_flag);
+    const float* sf = reinterpret_cast<const float*>(smem + S::OFF_F32 + b * S::F32B);
+    // z[k][wv][q] = elements e = 2q, 2q + 1 of the 8 consecutive j at
+    // jf + 16 wv of combo k
+    F2 z[S::NCB][W][4];
 #pragma unroll
     for (int k = 0; k < S::NCB; ++k) {
-      const int cb = tid + S::T * k;
-      const int i2 = cb % S::NSP, jc = cb / S::NSP;
+      const int cb = t2 + T * k;
+      const int i2 = combo_i(cb), jc = cb & 7;
       const int jf = 8 * (jc & 1) + 16 * W * (jc >> 1);
-      const bool act = cb < S::NCOMBO && i2 < NS;
-      if (act) {
+      // position of j = jf + 16 wv + 4 u in the transpose buffer: bits 2 and 4
+      // of j flip with the two high bits of jc
+      const int xr = (((jc >> 1) & 1) << 2) | ((jc >> 2) << 4);
+      if (cb < S::NCOMBO && i2 < NS) {
 #pragma unroll
         for (int wv = 0; wv < W; ++wv) {
-          const float4 u0 = *reinterpret_cast<const float4*>(sf + i2 * S::PS + jf + 16 * wv);
-          const float4 u1 = *reinterpret_cast<const float4*>(sf + i2 * S::PS + jf + 16 * wv + 4);
-          z[k][wv][0] = u0.x; z[k][wv][1] = u0.y; z[k][wv][2] = u0.z; z[k][wv][3] = u0.w;
-          z[k][wv][4] = u1.x; z[k][wv][5] = u1.y; z[k][wv][6] = u1.z; z[k][wv][7] = u1.w;
+          const float* rowp = sf + i2 * S::PS + jf;
+          const ulonglong2 u0 = *reinterpret_cast<const ulonglong2*>(rowp + ((16 * wv) ^ xr));
+          const ulonglong2 u1 = *reinterpret_cast<const ulonglong2*>(rowp + ((16 * wv + 4) ^ xr));
+          z[k][wv][0].u = u0.x;
+          z[k][wv][1].u = u0.y;
+          z[k][wv][2].u = u1.x;
+          z[k][wv][3].u = u1.y;
         }
       } else {
 #pragma unroll
         for (int wv = 0; wv < W; ++wv)
 #pragma unroll
-          for (int e = 0; e < 8; ++e) z[k][wv][e] = 0.f;
+          for (int q = 0; q < 4; ++q) z[k][wv][q].u = 0ull;
       }
+    }
+    mbar_arrive(&bempty[b]);  // the buffer is in registers: phase 1 may refill it
+    Range<SYM> rg;
 #pragma unroll
-      for (int bit = 1; bit < 8; bit <<= 1)
+    for (int k = 0; k < S::NCB; ++k) {
+      const int cb = t2 + T * k;
+      const bool act = cb < S::NCOMBO && combo_i(cb) < NS;
 #pragma unroll
-        for (int wv = 0; wv < W; ++wv)
+      for (int wv = 0; wv < W; ++wv) {
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
-            if (!(e & bit)) {
-              const float p0 = z[k][wv][e], p1 = z[k][wv][e | bit];
-              z[k][wv][e] = p0 + p1;
-              z[k][wv][e | bit] = p0 - p1;
-            }
+        for (int q = 0; q < 4; ++q) f2_bfly_inner(z[k][wv][q]);  // e bit 0
+#pragma unroll
+        for (int bit = 1; bit < 4; bit <<= 1)                     // e bits 1, 2
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (!(q & bit)) f2_bfly(z[k][wv][q], z[k][wv][q | bit]);
+      }
 #pragma unroll
       for (int bit = 1; bit < W; bit <<= 1)
 #pragma unroll
         for (int wv = 0; wv < W; ++wv)
           if (!(wv & bit)) {
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float p0 = z[k][wv][e], p1 = z[k][wv | bit][e];
-              z[k][wv][e] = p0 + p1;
-              z[k][wv | bit][e] = p0 - p1;
-            }
+            for (int q = 0; q < 4; ++q) f2_bfly(z[k][wv][q], z[k][wv | bit][q]);
           }
       if (act)
 #pragma unroll
         for (int wv = 0; wv < W; ++wv)
 #pragma unroll
-          for (int e = 0; e < 8; ++e) rg.add(z[k][wv][e]);
+          for (int q = 0; q < 4; ++q) rg.add_pair(z[k][wv][q]);
     }
-    block_range<SYM, W>(rg, red);
+    // row range over the phase-2 warps (scratch alternates between rows, so
+    // one barrier per row suffices); the same barrier settles the abort
+    // decision for every phase-2 thread before any global store
+    rg.warp_reduce();
+    float* rd = red + (it & 1) * 2 * W;
+    if (lane == 0) {
+      rd[w2] = rg.hi;
+      rd[W + w2] = rg.lo;
+    }
+    if (named_bar_or(kPhase2Bar, T, !ok || *abort_flag)) break;
+    rg.hi = rd[0];
+    rg.lo = rd[W];
+#pragma unroll
+    for (int i = 1; i < W; ++i) {
+      rg.hi = fmaxf(rg.hi, rd[i]);
+      if (!SYM) rg.lo = fminf(rg.lo, rd[W + i]);
+    }
     const QParams<SYM> qp(rg, a.clip);
     uint8_t* out = a.codes + row * (a.K / 2);
 #pragma unroll
     for (int k = 0; k < S::NCB; ++k) {
-      const int cb = tid + S::T * k;
-      const int i2 = cb % S::NSP, jc = cb / S::NSP;
-      const int jf = 8 * (jc & 1) + 16 * W * (jc >> 1);
-      if (cb < S::NCOMBO && i2 < NS) {
+      const int cb = t2 + T * k;
+      const int i2 = combo_i(cb), jc = cb & 7;
+      const bool act = cb < S::NCOMBO && i2 < NS;
+      // wd[wv] = codes of j = jf + 16 wv .. + 7: word (jc & 1) + 2 W (jc >> 1) + 2 wv of segment i2
+      uint32_t wd[W];
 #pragma unroll
-        for (int wv = 0; wv < W; ++wv) {
-          uint32_t rb[8];
+      for (int wv = 0; wv < W; ++wv) {
+        uint32_t rb[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) rb[e] = qp.template code_bits<CLAMP>(z[k][wv][e]);
-          *reinterpret_cast<uint32_t*>(out + (i2 * P + jf + 16 * wv) / 2) = pack8_nibbles(rb);
+        for (int q = 0; q < 4; ++q) qp.template code_bits2<CLAMP>(z[k][wv][q], rb[2 * q], rb[2 * q + 1]);
+        wd[wv] = pack8_nibbles(rb);
+      }
+      // The pair (jc, jc ^ 1) (lanes l, l ^ 1) holds 2 W consecutive words,
+      // interleaved.  Cut them into chunks of CW words; the even lane stores
+      // the even chunks, the odd lane the odd ones, after swapping halves.
+      constexpr int CW = W >= 4 ? 4 : 2, NCH = 2 * W / CW, HV = CW / 2;
+      const bool odd = jc & 1;
+      uint32_t* seg = reinterpret_cast<uint32_t*>(out + i2 * (P / 2)) + 2 * W * (jc >> 1);
+#pragma unroll
+      for (int kk = 0; kk < NCH / 2; ++kk) {
+        uint32_t own[HV], oth[HV];
+#pragma unroll
+        for (int t = 0; t < HV; ++t) {
+          const uint32_t e = wd[(2 * kk) * HV + t], o = wd[(2 * kk + 1) * HV + t];
+          own[t] = odd ? o : e;
+          oth[t] = __shfl_xor_sync(0xffffffffu, odd ? e : o, 1);
+        }
+        uint32_t* dst = seg + (2 * kk + (odd ? 1 : 0)) * CW;
+        if (act) {
+          if constexpr (CW == 4)
+            *reinterpret_cast<uint4*>(dst) = odd ? make_uint4(oth[0], own[0], oth[HV - 1], own[HV - 1])
+                                                 : make_uint4(own[0], oth[0], own[HV - 1], oth[HV - 1]);
+          else
+            *reinterpret_cast<uint2*>(dst) = odd ? make_uint2(oth[0], own[0]) : make_uint2(own[0], oth[0]);
         }
       }
     }
-    if (tid == 0) {
+    if (t2 == 0) {
       a.scale[row] = qp.alpha * a.norm;
       if (!SYM) a.zero[row] = qp.beta * a.norm;
-    }
-    __syncthreads();  // stage, fp32 buffer and `red` are reused by the next row
-  }
-  if (*abort_flag && tid == 0) {
-    // let the copies still in flight (iterations it .. issued-1) land first
-    for (int j = it; j < issued; ++j) {
-      const uint64_t t0 = globaltimer_ns();
-      while (!mbar_try_wait(&full[j % S::NST], (j / S::NST) & 1) && globaltimer_ns() - t0 < kRowWaitLimitNs) {
-      }
     }
   }
 }
@@ -302,13 +417,25 @@ __global__ void __launch_bounds__(32 * ((1 << LP) / 64), 16 / ((1 << LP) / 64)) 
 template <int NS, int LP, bool SYM, bool CLAMP>
 cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
   using S = PaleyShape<NS, LP>;
+  // rows as (j_lo, i, j_hi, row): one copy lands a row as 128-byte swizzled lines i + NS j_hi
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return cudaErrorNotSupported;
+  CUtensorMap tmx;
+  const cuuint64_t gdim[4] = {64, (cuuint64_t)NS, (cuuint64_t)(S::P / 64), (cuuint64_t)a.rows};
+  const cuuint64_t gstride[3] = {(cuuint64_t)(S::P * 2), 128, (cuuint64_t)(a.ldx * 2)};
+  const cuuint32_t box[4] = {64, (cuuint32_t)NS, (cuuint32_t)(S::P / 64), 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  if (enc(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void*>(a.x), gdim, gstride, box, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorNotSupported;
   auto kern = rq_paley_kernel<NS, LP, SYM, CLAMP>;
   int per_sm = 0;
-  cudaError_t e = prepare_launch(kern, S::T, S::BYTES, &per_sm);
+  cudaError_t e = prepare_launch(kern, S::THREADS, S::BYTES, &per_sm);
   if (e != cudaSuccess) return e;
   const int64_t cap = (int64_t)device_sm_count() * per_sm;
   const int64_t grid = a.rows < cap ? a.rows : cap;
-  kern<<<(unsigned)grid, S::T, S::BYTES, stream>>>(a);
+  kern<<<(unsigned)grid, S::THREADS, S::BYTES, stream>>>(tmx, a);
   return cudaGetLastError();
 }
 

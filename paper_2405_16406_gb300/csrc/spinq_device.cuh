@@ -53,6 +53,79 @@ __device__ __forceinline__ uint32_t pack_half2_bits(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
+// ---------------------------------------------------------------------------
+// Packed fp32 pairs.  sm_100-family SMs execute add/sub/fma on two fp32 lanes
+// held in one 64-bit register pair (PTX add/sub/fma.rn.f32x2) as a single
+// instruction; each lane is rounded exactly like the scalar operation, so the
+// results are bit-identical to scalar FADD/FFMA code.  The Hadamard butterflies
+// and the quantizer's scale step run on these pairs.
+// ---------------------------------------------------------------------------
+struct F2 {
+  unsigned long long u;
+};
+
+__device__ __forceinline__ F2 f2_make(float lo, float hi) {
+  F2 r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r.u) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_split(F2 x, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(x.u));
+}
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
+  F2 r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r.u) : "l"(a.u), "l"(b.u));
+  return r;
+}
+__device__ __forceinline__ F2 f2_sub(F2 a, F2 b) {
+  F2 r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r.u) : "l"(a.u), "l"(b.u));
+  return r;
+}
+__device__ __forceinline__ F2 f2_fma(F2 a, F2 b, F2 c) {
+  F2 r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r.u) : "l"(a.u), "l"(b.u), "l"(c.u));
+  return r;
+}
+// radix-2 butterfly on two pairs: (a, b) <- (a + b, a - b), lane by lane
+__device__ __forceinline__ void f2_bfly(F2& a, F2& b) {
+  const F2 s = f2_add(a, b);
+  b = f2_sub(a, b);
+  a = s;
+}
+// butterfly between the two lanes of one pair: (lo, hi) <- (lo + hi, lo - hi)
+__device__ __forceinline__ void f2_bfly_inner(F2& a) {
+  float lo, hi;
+  f2_split(a, lo, hi);
+  a = f2_make(lo + hi, lo - hi);
+}
+
+// Accumulating form of mma_16816_f16_f32_pairs (C = D).
+__device__ __forceinline__ void mma_16816_f16_f32_pairs_acc(F2& d01, F2& d23, const uint32_t a[4], uint32_t b0,
+                                                            uint32_t b1) {
+  asm volatile(
+      "{\n\t.reg .f32 e0, e1, e2, e3;\n\t"
+      "mov.b64 {e0, e1}, %0;\n\tmov.b64 {e2, e3}, %1;\n\t"
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {e0,e1,e2,e3}, {%2,%3,%4,%5}, {%6,%7}, "
+      "{e0,e1,e2,e3};\n\t"
+      "mov.b64 %0, {e0, e1};\n\tmov.b64 %1, {e2, e3};\n\t}\n"
+      : "+l"(d01.u), "+l"(d23.u)
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// m16n8k16 MMA whose D fragment comes back as two pairs: d01 = (d[0], d[1])
+// (row g) and d23 = (d[2], d[3]) (row g + 8).
+__device__ __forceinline__ void mma_16816_f16_f32_pairs(F2& d01, F2& d23, const uint32_t a[4], uint32_t b0,
+                                                        uint32_t b1) {
+  asm volatile(
+      "{\n\t.reg .f32 e0, e1, e2, e3;\n\t"
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {e0,e1,e2,e3}, {%2,%3,%4,%5}, {%6,%7}, "
+      "{%8,%8,%8,%8};\n\t"
+      "mov.b64 %0, {e0, e1};\n\tmov.b64 %1, {e2, e3};\n\t}\n"
+      : "=l"(d01.u), "=l"(d23.u)
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
+}
+
 // 1.5 * 2^23: adding it to |v| < 2^22 leaves round-half-to-even(v) in the low
 // mantissa bits (the FADD rounds to nearest even), so the low nibble of the
 // sum's bit pattern is the two's complement 4-bit code of rint(v).
@@ -169,6 +242,15 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const void* tmap, ui
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
       "%3}], [%4];\n" ::"r"(smem_u32(smem_dst)),
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d(void* smem_dst, const void* tmap, uint64_t* bar, int32_t c0,
+                                            int32_t c1, int32_t c2, int32_t c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+      "%3, %4, %5}], [%6];\n" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar))
       : "memory");
 }
 
