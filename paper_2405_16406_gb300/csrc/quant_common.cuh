@@ -35,12 +35,11 @@ struct Range {
     f2_split(v, a, b);
     add2(a, b);
   }
+  // over the 32 lanes of a converged warp, with the float warp reductions of
+  // sm_100+ (max and min are exact, so this equals the shuffle tree)
   __device__ __forceinline__ void warp_reduce() {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-      if (!SYM) lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-    }
+    asm volatile("redux.sync.max.f32 %0, %0, 0xffffffff;" : "+f"(hi));
+    if (!SYM) asm volatile("redux.sync.min.f32 %0, %0, 0xffffffff;" : "+f"(lo));
   }
 };
 
@@ -71,15 +70,17 @@ struct QParams {
   float inv, off, alpha, beta;
   F2 inv2, bias2;  // (inv, inv); (magic, magic) for SYM, (off, off) otherwise
   __device__ __forceinline__ QParams(const Range<SYM>& r, float clip) {
+    // alpha is a scale factor (a product, no division needed); the codes use
+    // the correctly rounded reciprocal step inv
     if (SYM) {
       const float m = clip * r.hi;
-      alpha = m / 7.f;
+      alpha = m * (1.f / 7.f);
       inv = m > 0.f ? 7.f / m : 0.f;
       off = 0.f;
       beta = 0.f;
     } else {
       const float h2 = clip * r.hi, l2 = clip * r.lo;
-      alpha = (h2 - l2) / 15.f;
+      alpha = (h2 - l2) * (1.f / 15.f);
       inv = h2 > l2 ? 15.f / (h2 - l2) : 0.f;
       beta = l2;
       off = -l2 * inv;

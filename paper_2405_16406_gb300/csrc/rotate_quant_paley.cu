@@ -155,8 +155,8 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
       issued[s] = -1;
     }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&bfull[b], T);
-      mbar_init(&bempty[b], T);
+      mbar_init(&bfull[b], W);   // one arrival per warp, after __syncwarp
+      mbar_init(&bempty[b], W);
     }
     *reinterpret_cast<uint4*>(smem + S::OFF_ZERO) = make_uint4(0, 0, 0, 0);
     *abort_flag = 0;
@@ -229,7 +229,7 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
       if (lane == 0) {
         // this warp no longer reads the stage; the last one refills it
         __threadfence_block();
-        if (atomicAdd(&readers[s], 1) == W - 1) {
+        if (atom_add_shared(&readers[s], 1u) == (uint32_t)(W - 1)) {
           readers[s] = 0;
           if (it + NSTG < niter) issue(it + NSTG);
         }
@@ -270,7 +270,8 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
             }
         }
       }
-      mbar_arrive(&bfull[b]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bfull[b]);  // release: the warp's stores above are ordered before it
     }
     // every phase-1 warp has stopped issuing; after an abort, let the copies
     // still in flight land before the CTA can exit
@@ -319,7 +320,8 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
           for (int q = 0; q < 4; ++q) z[k][wv][q].u = 0ull;
       }
     }
-    mbar_arrive(&bempty[b]);  // the buffer is in registers: phase 1 may refill it
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&bempty[b]);  // the buffer is in registers: phase 1 may refill it
     Range<SYM> rg;
 #pragma unroll
     for (int k = 0; k < S::NCB; ++k) {
