@@ -160,16 +160,7 @@ struct RowStream {
   __device__ __forceinline__ uint8_t* stage(int iter) const { return stage0 + (size_t)(iter % NST) * stage_bytes; }
   // every thread; false on timeout or abort
   __device__ __forceinline__ bool wait(int iter, volatile int* abort, uint64_t limit_ns) {
-    const uint32_t par = (uint32_t)(iter / NST) & 1u;
-    if (mbar_try_wait(&bars[iter % NST], par)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    while (!mbar_try_wait(&bars[iter % NST], par)) {
-      if (*abort || globaltimer_ns() - t0 > limit_ns) {
-        *abort = 1;
-        return false;
-      }
-    }
-    return true;
+    return mbar_wait_backoff(&bars[iter % NST], (uint32_t)(iter / NST) & 1u, abort, limit_ns);
   }
   // thread 0, after a CTA barrier that follows the last read of stage(iter)
   __device__ __forceinline__ void release(int iter) {

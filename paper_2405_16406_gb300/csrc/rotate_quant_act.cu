@@ -10,10 +10,11 @@
 // Element index bits: e (0..2, inside a chunk), c = lane & 3 (3..4),
 // g = lane >> 2 (5..7), w (8 .. 8+LW-1), v (8+LW ..).
 // A tensor-core m16n8k16 with B = the 16-point Sylvester matrix contracts the
-// bits {e0, e1, c0, c1} of the RAW fp16 input (entries +-1: exact products,
+// bits {e0, e2, c0, c1} of the RAW fp16 input (entries +-1: exact products,
 // fp32 sums) and returns fp32 in the lane that supplied the data, at the same
-// element positions.  Radix-2 butterflies inside the lane then cover e2 and
-// the v bits.
+// element positions (the chunk's four 32-bit words are the A fragment as they
+// are: words 0/2 are rows g, words 1/3 rows g + 8, so e1 is the row bit).
+// Radix-2 butterflies inside the lane then cover e1 and the v bits.
 //
 // Transpose.  The rows go through shared memory once as fp32 (16-byte chunks
 // XOR-swizzled so that both the phase-1 stores and the phase-2 loads are free
@@ -60,11 +61,13 @@ __device__ __forceinline__ void make_b16(uint32_t b[2][2], bool hadamard) {
 }
 
 // One 16-byte chunk (8 fp16) through the tensor core: the results y[e],
-// e = 0..7, come back as the pairs y2[q] = (y[2q], y[2q + 1]).
+// e = 0..7, come back as the pairs y2[q] = (y[2q], y[2q + 1]).  The words of
+// the chunk are the A fragment in their own order (k = e0 + 2c + 8 e2, row
+// g + 8 e1), so no register moves are needed.
 __device__ __forceinline__ void chunk_mma(const uint4 in, const uint32_t b[2][2], F2 y2[4]) {
-  const uint32_t A[4] = {in.x, in.z, in.y, in.w};
-  mma_16816_f16_f32_pairs(y2[0], y2[2], A, b[0][0], b[0][1]);
-  mma_16816_f16_f32_pairs(y2[1], y2[3], A, b[1][0], b[1][1]);
+  const uint32_t A[4] = {in.x, in.y, in.z, in.w};
+  mma_16816_f16_f32_pairs(y2[0], y2[1], A, b[0][0], b[0][1]);
+  mma_16816_f16_f32_pairs(y2[2], y2[3], A, b[1][0], b[1][1]);
 }
 
 // ------------------------------------------------------------------------
@@ -152,9 +155,9 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
     for (int v = 0; v < S::V; ++v) chunk_mma(src[lane + 32 * (w + S::W * v)], bh, y[v]);
     rs.release_warp(it, release_count, S::W);  // the next copy into this stage overlaps the rest of the row
 #pragma unroll
-    for (int v = 0; v < S::V; ++v) {  // e2
-      f2_bfly(y[v][0], y[v][2]);
-      f2_bfly(y[v][1], y[v][3]);
+    for (int v = 0; v < S::V; ++v) {  // e1
+      f2_bfly(y[v][0], y[v][1]);
+      f2_bfly(y[v][2], y[v][3]);
     }
 #pragma unroll
     for (int bit = 1; bit < S::V; bit <<= 1)
@@ -167,8 +170,14 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
 #pragma unroll
     for (int v = 0; v < S::V; ++v) {
       const uint32_t ch = (uint32_t)(lane + 32 * (w + S::W * v));
-      *reinterpret_cast<ulonglong2*>(sm + 4 * ch) = make_ulonglong2(y[v][0].u, y[v][1].u);
-      *reinterpret_cast<ulonglong2*>(sm + S::P / 2 + 16 + 4 * ch) = make_ulonglong2(y[v][2].u, y[v][3].u);
+      // 8-byte stores of whole pairs: a 16-byte store would need the two
+      // pairs in four consecutive registers
+      unsigned long long* p0 = reinterpret_cast<unsigned long long*>(sm + 4 * ch);
+      unsigned long long* p1 = reinterpret_cast<unsigned long long*>(sm + S::P / 2 + 16 + 4 * ch);
+      p0[0] = y[v][0].u;
+      p0[1] = y[v][1].u;
+      p1[0] = y[v][2].u;
+      p1[1] = y[v][3].u;
     }
     __syncthreads();
 

@@ -10,11 +10,11 @@
 //
 // Stage 1 runs on the tensor core, on the raw fp16 input: one m16n8k16 MMA
 // per chunk with B = the 16-point Sylvester matrix contracts the 4 bits
-// {e0, e1, c0, c1} (k = 2c + e0 + 8 e1); the two A rows g and g+8 carry e2 = 0
-// and e2 = 1.  The outputs land in the lane that supplied the inputs, at the
+// {e0, e2, c0, c1} (k = 2c + e0 + 8 e2); the two A rows g and g+8 carry e1 = 0
+// and e1 = 1.  The outputs land in the lane that supplied the inputs, at the
 // same element positions, already in fp32 (entries are +-1, so the products
 // are exact and the sums are fp32 sums of 16 fp16 values).  The remaining
-// bits (e2 and v) are radix-2 butterflies inside the lane.  For V the same
+// bits (e1 and v) are radix-2 butterflies inside the lane.  For V the same
 // MMA with B = I16 only widens fp16 to fp32 (exactly).
 //
 // Eq. 1 on the unnormalised rotated row: the codes do not depend on the
@@ -89,7 +89,9 @@ __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) 
     float y[V][8];
 #pragma unroll
     for (int v = 0; v < V; ++v) {
-      const uint32_t A[4] = {in[v].x, in[v].z, in[v].y, in[v].w};
+      // the chunk's words are the A fragment as they are: k = e0 + 2c + 8 e2,
+      // row g + 8 e1 (no register moves), so the MMA contracts {e0, e2, c}
+      const uint32_t A[4] = {in[v].x, in[v].y, in[v].z, in[v].w};
       float d0[4], d1[4];
       if (kind == 2) {
         mma_16816_f16_f32(d0, A, bi[0][0], bi[0][1]);
@@ -98,25 +100,23 @@ __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) 
         mma_16816_f16_f32(d0, A, bh[0][0], bh[0][1]);
         mma_16816_f16_f32(d1, A, bh[1][0], bh[1][1]);
       }
-      y[v][0] = d0[0];
-      y[v][1] = d0[1];
-      y[v][4] = d0[2];
-      y[v][5] = d0[3];
-      y[v][2] = d1[0];
-      y[v][3] = d1[1];
-      y[v][6] = d1[2];
-      y[v][7] = d1[3];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        y[v][e] = d0[e];
+        y[v][e + 4] = d1[e];
+      }
     }
 
     if (kind != 2) {
 #pragma unroll
       for (int v = 0; v < V; ++v)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float u = y[v][e], w = y[v][e + 4];
-          y[v][e] = u + w;
-          y[v][e + 4] = u - w;
-        }
+        for (int e = 0; e < 8; ++e)
+          if (!(e & 2)) {  // e1, the bit the MMA leaves
+            const float u = y[v][e], w = y[v][e + 2];
+            y[v][e] = u + w;
+            y[v][e + 2] = u - w;
+          }
 #pragma unroll
       for (int bit = 1; bit < V; bit <<= 1)
 #pragma unroll

@@ -100,16 +100,7 @@ __device__ __forceinline__ int combo_i(int cb) {
 // Bounded wait for the phase of `bar` with `parity`.  Returns false when the
 // abort flag is up or the limit expired (then it raises the flag).
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (!mbar_try_wait(bar, parity)) {
-    if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
-      *abort_flag = 1;
-      return false;
-    }
-  }
-  return true;
+  return mbar_wait_backoff(bar, parity, abort_flag, kWaitLimitNs);
 }
 
 // bar.sync over `nthreads` threads whose result is the OR of `pred` over them.
@@ -129,7 +120,9 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
   using S = PaleyShape<NS, LP>;
   constexpr int P = S::P, W = S::W, T = S::T, NSTG = S::NSTG;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1024-aligned base, derived from the shared array itself so that every
+  // access below stays in the shared address space
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
   uint64_t* bfull = full + NSTG;
   uint64_t* bempty = bfull + 2;
