@@ -65,13 +65,18 @@ __device__ __forceinline__ void record_timeout(int site) {
   if (atomicCAS(&g_status_code, 0, (int)SPINQ_ETIMEOUT) == 0) atomicExch(&g_status_detail, site);
 }
 
-// Bounded wait that also gives up as soon as another role has aborted.
+// Bounded wait that also gives up as soon as another role has aborted.  The
+// abort flag and the clock are read once every 64 polls: between them the
+// loop touches only the barrier, which keeps polling warps from taking
+// shared-memory bandwidth from the unpack and MMA traffic.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                               int site) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
+#pragma unroll 1
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
     if (globaltimer_ns() - t0 > kWaitLimitNs) {
       record_timeout(site);
@@ -129,7 +134,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   using L = Cfg<MT>;
   constexpr int BMT = L::BMT, NP = L::NP, NU = L::NU, NACC = L::NACC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1024-aligned base derived from the shared array itself, so that the
+  // accesses through it stay shared-memory accesses
+  uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L::bars);
   uint64_t* full_p = bars;
   uint64_t* empty_p = full_p + NP;
@@ -472,7 +479,9 @@ __global__ void __launch_bounds__(kDecThreads, 2)
   using L = DecCfg<MN>;
   constexpr int NP = L::NP, NU = L::NU;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1024-aligned base derived from the shared array itself, so that the
+  // accesses through it stay shared-memory accesses
+  uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L::bars);
   uint64_t* full_p = bars;
   uint64_t* empty_p = full_p + NP;
