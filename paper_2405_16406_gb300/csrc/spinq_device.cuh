@@ -254,6 +254,23 @@ __device__ __forceinline__ uint32_t atom_add_shared(const void* p, uint32_t v) {
   return old;
 }
 
+// Returns only once the loads that produced w[] have completed.  The XOR of
+// one register of each vector cannot issue before those loads are done, and
+// it feeds a predicated store to a scratch word (which practically never
+// fires and is harmless when it does), so the assembler cannot drop it; the
+// store is ordered before the caller's __syncwarp and mbarrier arrive.  This
+// lets a warp release a shared-memory stage right after reading it without
+// the arrive overtaking the loads (an arrive issued right after the loads can
+// be seen before they have read shared memory, and a refill of the stage
+// would then race them).
+template <int N>
+__device__ __forceinline__ void wait_loaded(const uint4 (&w)[N], volatile uint32_t* scratch) {
+  uint32_t acc = 0x2545F491u;
+#pragma unroll
+  for (int j = 0; j < N; ++j) acc ^= w[j].x;
+  if (acc == 0x9E3779B9u) *scratch = acc;
+}
+
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(nthreads) : "memory");
 }
@@ -368,6 +385,19 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t r[16
 
 __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+}
+
+// tcgen05.ld writes its destination registers asynchronously: they hold the
+// data only after tcgen05.wait::ld.  Passing them through the wait as
+// read-write operands makes every later use depend on it, so the compiler
+// cannot schedule a use between the load and the wait.
+__device__ __forceinline__ void tmem_ld_wait(uint32_t r[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;\n"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15])
+               :
+               : "memory");
 }
 
 // Shared-memory matrix descriptor for a K-major operand tile stored with the

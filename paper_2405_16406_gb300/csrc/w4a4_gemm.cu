@@ -149,6 +149,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* drain = rs_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + L::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + L::misc + 4);
+  volatile uint32_t* scratch = reinterpret_cast<volatile uint32_t*>(base + L::misc + 8);   // see wait_loaded
   int* rs_a = reinterpret_cast<int*>(base + L::rs_a);   // [2][groups][BMT]
   float* col_s = reinterpret_cast<float*>(base + L::cols);   // [BN] w_scale of the tile's columns
   float* col_r = col_s + BN;                                  // [BN] w_rowsum as float
@@ -294,8 +295,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int j = 0; j < L::TA; ++j) wa[j] = lds128(PA + la[j]);
 #pragma unroll
         for (int j = 0; j < L::TB; ++j) wb[j] = lds128(PB + lb[j]);
+        // packed stage consumed, once every lane's loads have read it
+        wait_loaded(wa, scratch);
+        wait_loaded(wb, scratch);
         __syncwarp();
-        if (lane == 0) mbar_arrive(&empty_p[s]);   // packed stage consumed
+        if (lane == 0) mbar_arrive(&empty_p[s]);
 #pragma unroll
         for (int j = 0; j < L::TA; ++j) {
           uint4 lo, hi;
@@ -365,8 +369,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr int NCH = MT * (BN / 16);
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * MT * BN);
       uint32_t ra[16], rbuf[16];
-      auto step = [&](int ci, const uint32_t(&cur)[16], uint32_t(&nxt)[16]) {
-        tmem_ld_wait();
+      auto step = [&](int ci, uint32_t(&cur)[16], uint32_t(&nxt)[16]) {
+        tmem_ld_wait(cur);
         if (ci + 1 < NCH) {
           tmem_ld_32x32b_x16(tbase + (uint32_t)((ci + 1) * 16), nxt);
         } else {
@@ -493,6 +497,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + L::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + L::misc + 4);
   volatile int* last_flag = reinterpret_cast<volatile int*>(base + L::misc + 8);
+  volatile uint32_t* scratch = reinterpret_cast<volatile uint32_t*>(base + L::misc + 12);   // see wait_loaded
   int* rsw = reinterpret_cast<int*>(base + L::rsw);
   int* rsa = reinterpret_cast<int*>(base + L::rsa);
 
@@ -596,6 +601,9 @@ __global__ void __launch_bounds__(kDecThreads, 2)
         const int i = u + kDecUnpackThreads * j;
         wa[j] = i < MN * 4 ? lds128(PA + (i >> 2) * 64 + (i & 3) * 16) : make_uint4(0, 0, 0, 0);
       }
+      // packed stage consumed, once every lane's loads have read it
+      wait_loaded(ww, scratch);
+      wait_loaded(wa, scratch);
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty_p[s]);
 #pragma unroll
@@ -654,7 +662,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     for (int c0 = 0; c0 < MN; c0 += 16) {
       uint32_t r[16];
       tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
-      tmem_ld_wait();
+      tmem_ld_wait(r);
       if (!ok || n >= args.N) continue;
 #pragma unroll
       for (int e = 0; e < 16; ++e) {
