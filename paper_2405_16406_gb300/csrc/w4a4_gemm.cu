@@ -123,14 +123,20 @@ struct Cfg {
   static constexpr uint32_t misc = bars + nbars * 8;   // tmem slot, abort flag
   static constexpr uint32_t rs_a = (misc + 16 + 15) & ~15u;
   static constexpr uint32_t cols = rs_a + 2 * kUnpackGroups * BMT * 4;   // s_n and (float) rowsum_n
-  static constexpr uint32_t total = cols + 2 * BN * 4;
+  // 256-row tiles: the epilogue stages each warp's 32 x 32 block of y in
+  // shared memory (64-byte rows, 64-byte swizzle, two buffers per warp) and
+  // writes it with a TMA store
+  static constexpr bool TMA_Y = MT == 2;
+  static constexpr uint32_t ys = (cols + 2 * BN * 4 + 1023) & ~1023u;
+  static constexpr uint32_t total = TMA_Y ? ys + kEpiWarps * 2 * 2048 : cols + 2 * BN * 4;
   static constexpr size_t dyn_bytes = total + 1024;
 };
 
 template <int MT, bool ASYM, bool ACC_OUT>
 __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     GemmArgs args, int num_k, int m_tiles, int num_tiles) {
+                     const __grid_constant__ CUtensorMap tmY, GemmArgs args, int num_k, int m_tiles,
+                     int num_tiles) {
   using L = Cfg<MT>;
   constexpr int BMT = L::BMT, NP = L::NP, NU = L::NU, NACC = L::NACC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -340,6 +346,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ epilogue
     const int q = warp & 3;
     const int et = tid - kFirstEpiWarp * 32;   // 0..127
+    // y staging of this warp (256-row tiles): two 32 x 32 fp16 buffers
+    uint8_t* ystage = base + L::ys + (warp - kFirstEpiWarp) * 2 * 2048;
+    int ygroup = 0;   // 32-column groups stored so far (buffer = ygroup & 1)
+    if (L::TMA_Y && lane == 0) prefetch_tmap(&tmY);
     int lt = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
       const int b = lt % NACC, rb = lt & 1;
@@ -392,11 +402,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float cm = -8.f * alpha * (float)rsa[mt];
         const float dm = bp - 8.f * alpha;
         __half* yrow = reinterpret_cast<__half*>(args.y) + m * args.N;
+        uint8_t* ybuf = ystage + (ygroup & 1) * 2048;
+        if (L::TMA_Y && (ci & 1) == 0) {
+          // the store issued from this buffer two groups ago must have read it
+          if (lane == 0) bulk_wait_group_read<1>();
+          __syncwarp();
+        }
 #pragma unroll
         for (int g8 = 0; g8 < 2; ++g8) {
           const int j0 = cc * 16 + g8 * 8;
           const int64_t n = n0 + j0;
-          if (!mvalid || n >= args.N) continue;
+          if (!L::TMA_Y && (!mvalid || n >= args.N)) continue;
+          // (staged rows and columns outside y are dropped by the TMA store;
+          // their column constants and alpha are zero)
           const float4 s0 = *reinterpret_cast<const float4*>(col_s + j0);
           const float4 s1 = *reinterpret_cast<const float4*>(col_s + j0 + 4);
           const float4 q0 = *reinterpret_cast<const float4*>(col_r + j0);
@@ -407,10 +425,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int e = 0; e < 8; ++e)
             yv[e] = sc[e] * fmaf(alpha_s, __uint_as_float(cur[g8 * 8 + e]), fmaf(dm, rw[e], cm));
-          *reinterpret_cast<uint4*>(yrow + n) =
-              make_uint4(pack_half2_bits(yv[0], yv[1]), pack_half2_bits(yv[2], yv[3]),
-                         pack_half2_bits(yv[4], yv[5]), pack_half2_bits(yv[6], yv[7]));
-          if (ACC_OUT) {
+          const uint4 pk = make_uint4(pack_half2_bits(yv[0], yv[1]), pack_half2_bits(yv[2], yv[3]),
+                                      pack_half2_bits(yv[4], yv[5]), pack_half2_bits(yv[6], yv[7]));
+          if (L::TMA_Y) {
+            // row `lane`, 16-byte chunk c = 2 (ci & 1) + g8 of the 64-byte row, swizzled
+            const int c = 2 * (ci & 1) + g8;
+            sts128(smem_u32(ybuf + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)), pk);
+          } else {
+            *reinterpret_cast<uint4*>(yrow + n) = pk;
+          }
+          if (ACC_OUT && mvalid && n < args.N) {
             int accs[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e)
@@ -421,6 +445,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             ap[1] = make_int4(accs[4], accs[5], accs[6], accs[7]);
           }
         }
+        if (L::TMA_Y && (ci & 1) == 1) {
+          // the 32 x 32 block is complete: hand it to the TMA engine
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            const int64_t x = n0 + (cc - 1) * 16;   // a multiple of 32 elements: 16-byte aligned
+            const int64_t yrow0 = (int64_t)(tile % m_tiles) * BMT + mt * 128 + q * 32;
+            // a box that starts inside y is clipped to it by the TMA engine;
+            // one wholly outside is not issued
+            if (x < args.N && yrow0 < args.M) tma_store_2d(&tmY, ybuf, (int32_t)x, (int32_t)yrow0);
+            bulk_commit_group();
+          }
+          ++ygroup;
+        }
       };
       tmem_ld_32x32b_x16(tbase, ra);
 #pragma unroll 1
@@ -429,6 +467,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         step(ci + 1, rbuf, ra);
       }
     }
+    // the staged blocks must be read (and written) before the CTA exits
+    if (L::TMA_Y && lane == 0) bulk_wait_group<0>();
   }
 
   tc_fence_before();
@@ -734,12 +774,30 @@ bool encode_packed_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t 
   return r == CUDA_SUCCESS;
 }
 
+// y [M][N] fp16 for the epilogue's TMA stores: 32 x 32 boxes, 64-byte swizzle
+bool encode_y_map(CUtensorMap* map, void* y, int64_t M, int64_t N) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return false;
+  cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)M};
+  cuuint64_t gstride[1] = {(cuuint64_t)(N * 2)};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, y, gdim, gstride, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 template <int MT, bool ASYM, bool ACC_OUT>
 cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   using L = Cfg<MT>;
-  CUtensorMap tmA, tmB;
+  CUtensorMap tmA, tmB, tmY;
   if (!encode_packed_map(&tmA, a.a_codes, a.M, a.K, L::BMT)) return cudaErrorNotSupported;
   if (!encode_packed_map(&tmB, a.w_codes, a.N, a.K, BN)) return cudaErrorNotSupported;
+  if (L::TMA_Y) {
+    if (!encode_y_map(&tmY, a.y, a.M, a.N)) return cudaErrorNotSupported;
+  } else {
+    tmY = tmA;   // unused
+  }
   auto kern = w4a4_gemm_kernel<MT, ASYM, ACC_OUT>;
   const size_t smem = L::dyn_bytes;
   int per_sm = 0;
@@ -750,7 +808,7 @@ cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   const int n_tiles = (int)((a.N + BN - 1) / BN);
   const int tiles = m_tiles * n_tiles;
   const int grid = tiles < sms ? tiles : sms;
-  kern<<<grid, kThreads, smem, stream>>>(tmA, tmB, a, (int)(a.K / 128), m_tiles, tiles);
+  kern<<<grid, kThreads, smem, stream>>>(tmA, tmB, tmY, a, (int)(a.K / 128), m_tiles, tiles);
   return cudaGetLastError();
 }
 

@@ -112,8 +112,11 @@ FULL = [
     ("l32_up_M1", 1, 3072, 8192, False),
     ("l32_down_M16", 16, 8192, 3072, False),
     ("l32_up_M128", 128, 3072, 8192, False),
-    ("tile256_ragged_M2000", 2000, 1024, 10240, True),
-    ("tile256_ragged_M2001_asym", 2001, 512, 12288, False),
+    # 256-row tiles (K >= 3072, at least two tiles per SM) with ragged edges:
+    # M not a multiple of 32, N a multiple of 16 but not of 32 (clipped TMA stores)
+    ("tile256_ragged_M2000", 2000, 3072, 9744, True),
+    ("tile256_ragged_M2001_asym", 2001, 3072, 12304, False),
+    ("tile128_ragged_M2001_asym", 2001, 512, 12288, False),
 ]
 
 
