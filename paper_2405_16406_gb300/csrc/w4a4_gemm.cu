@@ -852,9 +852,18 @@ cudaError_t launch_dec_mn(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStr
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
-  // 256-row tiles when they still give every SM at least two tiles
+  // Tile height from a wave-quantised cost model: a CTA runs ceil(tiles / SMs)
+  // tiles back to back.  A 256-row tile costs about 0.66 us per 128-deep K
+  // step plus a 10 us epilogue that its single-buffered accumulator cannot
+  // overlap; a 128-row tile about 0.485 us per K step plus 3 us (its epilogue
+  // overlaps the next tile).  The constants were measured on GB300 for these
+  // kernels; only their ratios matter.
+  const int64_t sms = device_sm_count(), ks = a.K / 128;
   const int64_t tiles256 = ((a.M + 255) / 256) * ((a.N + BN - 1) / BN);
-  if (a.K >= 3072 && tiles256 >= 2 * (int64_t)device_sm_count()) return launch_mt<2>(a, stream);
+  const int64_t tiles128 = ((a.M + 127) / 128) * ((a.N + BN - 1) / BN);
+  const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 10.0);
+  const double est128 = (double)((tiles128 + sms - 1) / sms) * (0.485 * (double)ks + 3.0);
+  if (est256 < est128) return launch_mt<2>(a, stream);
   return launch_mt<1>(a, stream);
 }
 
