@@ -1,16 +1,20 @@
 """Benchmark of the rotated W4A4 hot path on GB300 (one JSON line on rank 0).
 
-A step is one pass of the hot path over one batch of 2048 tokens of a
+A step is one pass of the whole hot path over one batch of 2048 tokens of a
 LLaMA-3-8B layer (synthetic inputs):
   * R3 + KV4: spinq_rotate_quant_kv on Q/K/V of the 2048 tokens
     (32 query heads, 8 KV heads, head_dim 128);
   * act quant: spinq_rotate_quant_act on x [2048 x 4096] (gate/up input,
     R1 merged so no online rotation, asymmetric per-token int4);
-  * W4A4 GEMM: spinq_w4a4_gemm, 2048 x 4096 -> 14336 (gate/up projection).
+  * W4A4 GEMM: spinq_w4a4_gemm, 2048 x 4096 -> 14336 (gate/up projection);
+  * R4 + act quant: spinq_rotate_quant_act on h [2048 x 14336] (down_proj
+    input, online H28 (x) H512, symmetric per-token int4);
+  * W4A4 GEMM: spinq_w4a4_gemm, 2048 x 14336 -> 4096 (down_proj, R4 merged
+    into the weights).
 The weight quantization (spinq_quant_weight) is offline and runs once before
-timing.  `value` counts the GEMM's 2*M*N*K integer ops per step over the whole
-step time.  Inputs rotate over 4 independent sets (4 layers' weights and
-activations, ~284 MB, larger than the 129 MB L2), so every step reads cold
+timing.  `value` counts both GEMMs' 2*M*N*K integer ops per step over the
+whole step time.  Inputs rotate over 4 independent sets (4 layers' weights and
+activations, ~0.7 GB, larger than the 129 MB L2), so every step reads cold
 data.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
@@ -34,7 +38,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "W4A4 rotated-linear TOPS and rotate+quant HBM GB/s (% of GB300 peak)"
-M, K, N = 2048, 4096, 14336
+M, K, N = 2048, 4096, 14336          # gate/up projection
+K2, N2, HAD2 = 14336, 4096, (28, 512)   # down_proj with online R4 = H28 (x) H512
 B_KV, S_KV, HQ, HKV, D = 1, 2048, 32, 8, 128
 NSETS = 4
 # Measured GB300 peaks (generated MEASURED_PEAKS.json; fallbacks if absent)
@@ -54,6 +59,11 @@ def step_bytes_rq():
     return M * K * 2 + M * K // 2 + 8 * M
 
 
+def step_bytes_rq2():
+    # R4 + act quant (symmetric): read fp16 h, write packed codes + alpha
+    return M * K2 * 2 + M * K2 // 2 + 4 * M
+
+
 def step_bytes_kv():
     rq, rkv = B_KV * S_KV * HQ, B_KV * S_KV * HKV
     return rq * D * 4 + 2 * rkv * (D * 2 + D // 2 + 8)
@@ -61,6 +71,14 @@ def step_bytes_kv():
 
 def gemm_ops():
     return 2.0 * M * N * K
+
+
+def gemm2_ops():
+    return 2.0 * M * N2 * K2
+
+
+def step_ops():
+    return gemm_ops() + gemm2_ops()
 
 
 def gemm_traffic_from_profile():
@@ -156,26 +174,43 @@ def run_ours(args, rank, world, local_rank):
         x[:, cols_idx] *= factor
         return x.half()
 
+    def swiglu_acts(rows, cols, frac, factor):
+        # down_proj input: a * SiLU(b), a few channels scaled up
+        a = torch.randn(rows, cols, generator=gen, device=dev)
+        b = torch.randn(rows, cols, generator=gen, device=dev)
+        h = a * torch.nn.functional.silu(b)
+        del a, b
+        cols_idx = torch.randperm(cols, generator=gen, device=dev)[: max(1, int(round(frac * cols)))]
+        h[:, cols_idx] *= factor
+        return h.half()
+
     sets = []
     for _ in range(NSETS):
         x = acts(M, K, 0.01, 30.0)
         w = (torch.randn(N, K, generator=gen, device=dev) * 0.02).half()
         qw = spinq.quant_weight(w, None)                       # offline, not timed
         del w
+        h = swiglu_acts(M, K2, 0.005, 100.0)
+        w2 = (torch.randn(N2, K2, generator=gen, device=dev) * 0.02).half()
+        qw2 = spinq.quant_weight(w2, HAD2)                     # R4 merged, offline, not timed
+        del w2
         q = torch.randn(B_KV, S_KV, HQ, D, generator=gen, device=dev).half()
         k = torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half()
         v = torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half()
-        sets.append((x, qw, q, k, v))
+        sets.append((x, qw, q, k, v, h, qw2))
     qa_out = [spinq.ActCodes(torch.empty(M, K // 2, dtype=torch.uint8, device=dev),
                              torch.empty(M, dtype=torch.float32, device=dev),
                              torch.empty(M, dtype=torch.float32, device=dev)) for _ in range(NSETS)]
+    qa2_out = [spinq.ActCodes(torch.empty(M, K2 // 2, dtype=torch.uint8, device=dev),
+                              torch.empty(M, dtype=torch.float32, device=dev), None) for _ in range(NSETS)]
     ys = [torch.empty(M, N, dtype=torch.float16, device=dev) for _ in range(NSETS)]
+    y2s = [torch.empty(M, N2, dtype=torch.float16, device=dev) for _ in range(NSETS)]
     kv_out = [None] * NSETS
     torch.cuda.synchronize()
 
     # eager warm-up (also fills the library's launch-configuration caches)
     def kv_fn(j):
-        _, _, q, k, v = sets[j]
+        _, _, q, k, v = sets[j][:5]
         kv_out[j] = spinq.rotate_quant_kv(q, k, v, out=kv_out[j])
 
     def rq_fn(j):
@@ -184,8 +219,14 @@ def run_ours(args, rank, world, local_rank):
     def gemm_fn(j):
         spinq.w4a4_gemm(qa_out[j], sets[j][1], y=ys[j])
 
-    fns = (kv_fn, rq_fn, gemm_fn)
-    names = ("kv", "rq", "gemm")
+    def rq2_fn(j):
+        spinq.rotate_quant_act(sets[j][5], HAD2, True, 1.0, out=qa2_out[j])
+
+    def gemm2_fn(j):
+        spinq.w4a4_gemm(qa2_out[j], sets[j][6], y=y2s[j])
+
+    fns = (kv_fn, rq_fn, gemm_fn, rq2_fn, gemm2_fn)
+    names = ("kv", "rq", "gemm", "rq2", "gemm2")
     for i in range(max(args.warmup, 3)):
         for fn in fns:
             fn(i % NSETS)
@@ -253,18 +294,22 @@ def run_ours(args, rank, world, local_rank):
     def avg(key):
         return statistics.mean(a.elapsed_time(b) for a, b in ev[key]) / 1e3  # seconds
 
-    t_gemm, t_rq, t_kv = avg("gemm"), avg("rq"), avg("kv")
+    t_gemm, t_rq, t_kv, t_rq2, t_gemm2 = avg("gemm"), avg("rq"), avg("kv"), avg("rq2"), avg("gemm2")
     gemm_tops = gemm_ops() / t_gemm / 1e12
+    gemm2_tops = gemm2_ops() / t_gemm2 / 1e12
 
     # ---- end to end through the public API with host buffers
     x_h = [sets[j][0].cpu().pin_memory() for j in range(NSETS)]
-    qkv_h = [tuple(t.cpu().pin_memory() for t in sets[j][2:]) for j in range(NSETS)]
+    h_h = [sets[j][5].cpu().pin_memory() for j in range(NSETS)]
+    qkv_h = [tuple(t.cpu().pin_memory() for t in sets[j][2:5]) for j in range(NSETS)]
     y_h = torch.empty(M, N, dtype=torch.float16).pin_memory()
+    y2_h = torch.empty(M, N2, dtype=torch.float16).pin_memory()
     qo_h = torch.empty(B_KV, S_KV, HQ, D, dtype=torch.float16).pin_memory()
     kc_h = torch.empty(B_KV, S_KV, HKV, D // 2, dtype=torch.uint8).pin_memory()
     vc_h = torch.empty_like(kc_h).pin_memory()
     sc_h = [torch.empty(B_KV, S_KV, HKV, dtype=torch.float32).pin_memory() for _ in range(4)]
     x_d = torch.empty(M, K, dtype=torch.float16, device=dev)
+    h_d = torch.empty(M, K2, dtype=torch.float16, device=dev)
     q_d = torch.empty(B_KV, S_KV, HQ, D, dtype=torch.float16, device=dev)
     k_d = torch.empty(B_KV, S_KV, HKV, D, dtype=torch.float16, device=dev)
     v_d = torch.empty_like(k_d)
@@ -272,13 +317,17 @@ def run_ours(args, rank, world, local_rank):
     def e2e_step(i):
         j = i % NSETS
         x_d.copy_(x_h[j], non_blocking=True)
+        h_d.copy_(h_h[j], non_blocking=True)
         q_d.copy_(qkv_h[j][0], non_blocking=True)
         k_d.copy_(qkv_h[j][1], non_blocking=True)
         v_d.copy_(qkv_h[j][2], non_blocking=True)
         o = spinq.rotate_quant_kv(q_d, k_d, v_d, out=kv_out[j])
         spinq.rotate_quant_act(x_d, None, False, 1.0, out=qa_out[j])
         spinq.w4a4_gemm(qa_out[j], sets[j][1], y=ys[j])
+        spinq.rotate_quant_act(h_d, HAD2, True, 1.0, out=qa2_out[j])
+        spinq.w4a4_gemm(qa2_out[j], sets[j][6], y=y2s[j])
         y_h.copy_(ys[j], non_blocking=True)
+        y2_h.copy_(y2s[j], non_blocking=True)
         qo_h.copy_(o.q_out, non_blocking=True)
         kc_h.copy_(o.k_codes, non_blocking=True)
         vc_h.copy_(o.v_codes, non_blocking=True)
@@ -302,8 +351,8 @@ def run_ours(args, rank, world, local_rank):
         t = torch.tensor([ms_e2e], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms_e2e = float(t.item())
-    h2d = (M * K + B_KV * S_KV * (HQ + 2 * HKV) * D) * 2
-    d2h = M * N * 2 + B_KV * S_KV * HQ * D * 2 + 2 * B_KV * S_KV * HKV * D // 2 + B_KV * S_KV * HKV * 16
+    h2d = (M * K + M * K2 + B_KV * S_KV * (HQ + 2 * HKV) * D) * 2
+    d2h = (M * N + M * N2) * 2 + B_KV * S_KV * HQ * D * 2 + 2 * B_KV * S_KV * HKV * D // 2 + B_KV * S_KV * HKV * 16
 
     # ---- isolated timing of the two memory-bound kernels: 16 back-to-back
     # launches in one graph over 16 input sets (footprint > L2), so the graph
@@ -314,11 +363,15 @@ def run_ours(args, rank, world, local_rank):
         qo = [spinq.ActCodes(torch.empty(M, K // 2, dtype=torch.uint8, device=dev),
                              torch.empty(M, dtype=torch.float32, device=dev),
                              torch.empty(M, dtype=torch.float32, device=dev)) for _ in range(16)]
+        hs = [sets[i % NSETS][5] if i < NSETS else swiglu_acts(M, K2, 0.005, 100.0) for i in range(8)]
+        qo2 = [spinq.ActCodes(torch.empty(M, K2 // 2, dtype=torch.uint8, device=dev),
+                              torch.empty(M, dtype=torch.float32, device=dev), None) for _ in range(8)]
         kvs = [(torch.randn(B_KV, S_KV, HQ, D, generator=gen, device=dev).half(),
                 torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half(),
                 torch.randn(B_KV, S_KV, HKV, D, generator=gen, device=dev).half()) for _ in range(16)]
         kvo = [spinq.rotate_quant_kv(*t) for t in kvs]
         for name, fn in (("act_quant", lambda i: spinq.rotate_quant_act(xs[i], None, False, 1.0, out=qo[i])),
+                         ("r4_quant", lambda i: spinq.rotate_quant_act(hs[i % 8], HAD2, True, 1.0, out=qo2[i % 8])),
                          ("kv_quant", lambda i: spinq.rotate_quant_kv(*kvs[i], out=kvo[i]))):
             for i in range(16):
                 fn(i)
@@ -337,7 +390,7 @@ def run_ours(args, rank, world, local_rank):
             e1i.record(stream)
             torch.cuda.synchronize()
             iso[name] = e0i.elapsed_time(e1i) / 48 / 1e3
-        del xs, qo, kvs, kvo
+        del xs, qo, kvs, kvo, hs, qo2
 
     st, _ = spinq.spinq_device_status()
     if st != spinq.SPINQ_OK:
@@ -345,8 +398,9 @@ def run_ours(args, rank, world, local_rank):
 
     if rank != 0:
         return None
-    value = world * gemm_ops() / (ms / 1e3) / 1e12
+    value = world * step_ops() / (ms / 1e3) / 1e12
     rq_gbs = step_bytes_rq() / t_rq / 1e9
+    rq2_gbs = step_bytes_rq2() / t_rq2 / 1e9
     kv_gbs = step_bytes_kv() / t_kv / 1e9
     out = {
         "metric": METRIC,
@@ -362,11 +416,14 @@ def run_ours(args, rank, world, local_rank):
         "dtype": "int4",
         "data": "synthetic",
         "config": {
-            "workload": "llama3_8b_gate_up_M2048_K4096_N14336 + R3/KV4 for the same 2048 tokens "
-                        "(32 q heads, 8 kv heads, head_dim 128)",
-            "M": M, "K": K, "N": N, "act_quant": "asymmetric per-token int4, no online rotation",
+            "workload": "llama3_8b MLP hot path for 2048 tokens: gate_up 4096->14336 (act quant, R1 merged) "
+                        "+ down_proj 14336->4096 (online R4 = H28 (x) H512, act quant) "
+                        "+ R3/KV4 (32 q heads, 8 kv heads, head_dim 128)",
+            "M": M, "gate_up": {"K": K, "N": N, "act_quant": "asymmetric per-token int4, no online rotation"},
+            "down_proj": {"K": K2, "N": N2, "online_rotation": "H28 (Paley, GF(27)) (x) H512",
+                          "act_quant": "symmetric per-token int4"},
             "weights": "symmetric per-channel int4 (quantized once, not timed)",
-            "l2": f"{NSETS} rotating input sets (~284 MB) > 129 MB L2",
+            "l2": f"{NSETS} rotating input sets (~0.7 GB) > 129 MB L2",
             "parallelism": f"replicas{world}",
         },
         "roofline": {
@@ -376,13 +433,25 @@ def run_ours(args, rank, world, local_rank):
             "peak_note": f"e4m3 dense = 2 x {peak_kind} bf16 ({bf16_peak} TFLOP/s); "
                          "int4 codes carried as e4m3 on tcgen05 kind::f8f6f4",
         },
+        "roofline_down_proj": {
+            "bound": "tensor", "kernel": "w4a4_gemm_kernel (down_proj 2048 x 14336 -> 4096)",
+            "achieved": round(gemm2_tops, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
+            "frac": round(gemm2_tops / fp8_peak, 4),
+        },
         "rotate_quant_roofline": {
+            "bound": "hbm", "kernel": "rq_paley_kernel (R4 = H28 (x) H512 + act quant, 2048 x 14336, sym)",
+            "achieved": round(rq2_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+            "frac": round(rq2_gbs / hbm_peak, 4), "us": round(t_rq2 * 1e6, 2),
+            "isolated_us": round(iso["r4_quant"] * 1e6, 2),
+            "isolated_frac": round(step_bytes_rq2() / iso["r4_quant"] / 1e9 / hbm_peak, 4),
+            "note": "in-step time includes the graph launch; isolated = 16 launches per graph, cold inputs",
+        },
+        "act_quant_roofline": {
             "bound": "hbm", "kernel": "rq_norot_kernel (act quant, 2048 x 4096, asym)",
             "achieved": round(rq_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
             "frac": round(rq_gbs / hbm_peak, 4), "us": round(t_rq * 1e6, 2),
             "isolated_us": round(iso["act_quant"] * 1e6, 2),
             "isolated_frac": round(step_bytes_rq() / iso["act_quant"] / 1e9 / hbm_peak, 4),
-            "note": "in-step time includes the graph launch; isolated = 16 launches per graph, cold inputs",
         },
         "kv_roofline": {
             "bound": "hbm", "kernel": "rotate_quant_kv_kernel (2048 tokens)",
@@ -391,11 +460,12 @@ def run_ours(args, rank, world, local_rank):
             "isolated_us": round(iso["kv_quant"] * 1e6, 2),
             "isolated_frac": round(step_bytes_kv() / iso["kv_quant"] / 1e9 / hbm_peak, 4),
         },
-        "kernel_us": {"gemm": round(t_gemm * 1e6, 2), "act_quant": round(t_rq * 1e6, 2),
+        "kernel_us": {"gemm_gate_up": round(t_gemm * 1e6, 2), "act_quant": round(t_rq * 1e6, 2),
+                      "r4_act_quant": round(t_rq2 * 1e6, 2), "gemm_down_proj": round(t_gemm2 * 1e6, 2),
                       "kv_quant": round(t_kv * 1e6, 2)},
-        "e2e": {"value": round(world * gemm_ops() / (ms_e2e / 1e3) / 1e12, 2), "unit": "TOPS",
+        "e2e": {"value": round(world * step_ops() / (ms_e2e / 1e3) / 1e12, 2), "unit": "TOPS",
                 "ms_per_step": round(ms_e2e, 4), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": len(names) * args.steps,
         "clocks": clocks,
     }
     if not args.no_cpu_baseline:
@@ -416,16 +486,21 @@ def cpu_baseline(sample_rows=1024, threads=0):
     x = synth.activations(rng, sample_rows, K, outlier_frac=0.01, factor=30.0)
     w = synth.weights(rng, N, K)
     qw = oracle.quant_weight(w, None)       # offline, not timed
+    h = synth.activations(rng, sample_rows, K2, outlier_frac=0.005, factor=100.0, swiglu=True)
+    w2 = synth.weights(rng, N2, K2)
+    qw2 = oracle.quant_weight(w2, HAD2)     # offline, not timed
     kv = synth.kv_case(seed=1, B=1, S=sample_rows, Hq=HQ, Hkv=HKV, D=D)
     t0 = time.perf_counter()
     oracle.rotate_quant_kv(kv.q, kv.k, kv.v, kv.had)
     qa = oracle.rotate_quant_act(x, None, 4, False, 1.0)
     oracle.w4a4_linear(qa, qw)
+    qa2 = oracle.rotate_quant_act(h, HAD2, 4, True, 1.0)
+    oracle.w4a4_linear(qa2, qw2)
     dt = time.perf_counter() - t0
-    ops = 2.0 * sample_rows * N * K
+    ops = 2.0 * sample_rows * (N * K + N2 * K2)
     return {"value": round(ops / dt / 1e12, 6), "unit": "TOPS", "cores": cores, "kind": "oracle",
-            "sample": f"{sample_rows} of {M} tokens (KV rows for the same tokens, act quant, "
-                      f"GEMM {sample_rows}x{K}->{N}); {dt:.2f} s"}
+            "sample": f"{sample_rows} of {M} tokens (KV rows for the same tokens, act quant + GEMM "
+                      f"{sample_rows}x{K}->{N}, R4 + act quant + GEMM {sample_rows}x{K2}->{N2}); {dt:.2f} s"}
 
 
 def run_reference(args, rank, world):
@@ -436,7 +511,7 @@ def run_reference(args, rank, world):
         cpu_baseline(sample_rows=max(1, rows // 4))
     vals = [cpu_baseline(sample_rows=rows) for _ in range(args.steps)]
     v = statistics.mean(x["value"] for x in vals)
-    ms_per_step = 2.0 * M * N * K / (v * 1e12) * 1e3
+    ms_per_step = step_ops() / (v * 1e12) * 1e3
     cb = dict(vals[-1])
     cb["value"] = round(v, 6)
     return {
@@ -444,8 +519,9 @@ def run_reference(args, rank, world):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "impl": "reference",
-        "config": {"workload": "llama3_8b_gate_up_M2048_K4096_N14336 + R3/KV4 for the same 2048 tokens",
-                   "M": M, "K": K, "N": N, "note": "CPU oracle on a bounded token sample per step"},
+        "config": {"workload": "llama3_8b MLP hot path for 2048 tokens: gate_up 4096->14336 "
+                               "+ down_proj 14336->4096 (online R4 = H28 (x) H512) + R3/KV4",
+                   "M": M, "note": "CPU oracle on a bounded token sample per step"},
         "cpu_baseline": cb,
         "e2e": {"value": round(v, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -458,7 +534,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-rows", type=int, default=1024)
-    ap.add_argument("--ref-rows", type=int, default=128, help="tokens per --impl reference step")
+    ap.add_argument("--ref-rows", type=int, default=64, help="tokens per --impl reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
 
