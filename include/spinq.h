@@ -208,6 +208,27 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
                                    float* k_zero, uint8_t* v_codes, float* v_scale,
                                    float* v_zero, void* stream);
 
+/*
+ * spinq_gemm_select_kernel -- which prefill kernel spinq_w4a4_gemm (and
+ * spinq_w4a4_gemm_splitk / _noalloc for M > 256) runs, process-wide:
+ *   SPINQ_GEMM_AUTO     the built-in cost model picks (the default);
+ *   SPINQ_GEMM_TILE128  one CTA per 128 x 256 output tile;
+ *   SPINQ_GEMM_TILE256  one CTA per 256 x 256 output tile;
+ *   SPINQ_GEMM_PAIR     two CTAs (an SM pair) per 256 x 256 tile; calls it
+ *                       cannot serve (M <= 128, no pair resident) use AUTO.
+ * All kernels compute bit-identical outputs; this is a tuning and testing
+ * control.  Returns the previous selection, or -1 (and changes nothing) for
+ * an unknown value.  Not synchronized with GEMM calls in other threads.
+ */
+typedef enum {
+  SPINQ_GEMM_AUTO = 0,
+  SPINQ_GEMM_TILE128 = 1,
+  SPINQ_GEMM_TILE256 = 2,
+  SPINQ_GEMM_PAIR = 3
+} spinq_gemm_kernel;
+
+int spinq_gemm_select_kernel(int kernel);
+
 /* Human-readable name of a status code (static storage). */
 const char* spinq_status_string(spinq_status s);
 

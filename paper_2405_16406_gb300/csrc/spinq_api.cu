@@ -190,6 +190,8 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
   return from_cuda(launch_rotate_quant_kv(a, static_cast<cudaStream_t>(stream)));
 }
 
+int spinq_gemm_select_kernel(int kernel) { return w4a4_gemm_select(kernel); }
+
 spinq_status spinq_device_status(int32_t* detail) {
   int32_t code = 0, d = 0;
   if (read_and_clear_device_status(&code, &d) != cudaSuccess) return SPINQ_ECUDA;

@@ -94,5 +94,15 @@ cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, cudaStre
 
 // Device status word written by bounded waits that gave up.
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail);
+// Its device address (two ints: code, wait site), for kernels in other
+// translation units; null if it cannot be resolved.
+int* device_status_word();
+// Prefill GEMM on SM pairs (tcgen05 cta_group::2, 256 x 256 tiles).  Sets
+// *handled = false when the shape or device cannot take it.
+cudaError_t launch_w4a4_gemm_pair(const GemmArgs& a, cudaStream_t stream, bool* handled);
+// SM pairs the pair kernel can keep resident at once (0 if none).
+int w4a4_gemm_pair_clusters();
+// Prefill kernel selection (spinq_gemm_kernel values); returns the previous one.
+int w4a4_gemm_select(int kernel);
 
 }  // namespace spinq

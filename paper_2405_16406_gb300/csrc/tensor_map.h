@@ -5,6 +5,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <stdint.h>
+
 #include <mutex>
 
 namespace spinq {
@@ -28,5 +30,10 @@ inline EncodeTiledFn get_encode_fn() {
   });
   return fn;
 }
+
+// Packed 4-bit code matrix [rows][K/2] bytes, boxes of 64 bytes x box_rows.
+bool encode_packed_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t K, int box_rows);
+// y [M][N] fp16 for the GEMM epilogues' TMA stores: 32 x 32 boxes, 64-byte swizzle.
+bool encode_y_map(CUtensorMap* map, void* y, int64_t M, int64_t N);
 
 }  // namespace spinq

@@ -37,6 +37,7 @@
 #include <cuda.h>
 #include <cuda_fp16.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "../../include/spinq.h"
@@ -47,8 +48,8 @@
 
 namespace spinq {
 
-__device__ int g_status_code = 0;
-__device__ int g_status_detail = 0;
+// device status word: [0] = code (SPINQ_ETIMEOUT), [1] = the wait site that gave up
+__device__ int g_status[2] = {0, 0};
 
 namespace {
 
@@ -62,7 +63,7 @@ constexpr int kFirstEpiWarp = 2;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 __device__ __forceinline__ void record_timeout(int site) {
-  if (atomicCAS(&g_status_code, 0, (int)SPINQ_ETIMEOUT) == 0) atomicExch(&g_status_detail, site);
+  if (atomicCAS(&g_status[0], 0, (int)SPINQ_ETIMEOUT) == 0) atomicExch(&g_status[1], site);
 }
 
 // Bounded wait that also gives up as soon as another role has aborted.  The
@@ -761,6 +762,8 @@ __global__ void __launch_bounds__(kDecThreads, 2)
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+}  // namespace
+
 bool encode_packed_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t K, int box_rows) {
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return false;
@@ -786,6 +789,8 @@ bool encode_y_map(CUtensorMap* map, void* y, int64_t M, int64_t N) {
                    CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
+
+namespace {
 
 template <int MT, bool ASYM, bool ACC_OUT>
 cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
@@ -850,19 +855,47 @@ cudaError_t launch_dec_mn(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStr
 
 }  // namespace
 
+std::atomic<int> g_gemm_kernel{SPINQ_GEMM_AUTO};
+
+int w4a4_gemm_select(int kernel) {
+  if (kernel < SPINQ_GEMM_AUTO || kernel > SPINQ_GEMM_PAIR) return -1;
+  return g_gemm_kernel.exchange(kernel);
+}
+
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
-  // Tile height from a wave-quantised cost model: a CTA runs ceil(tiles / SMs)
-  // tiles back to back.  A 256-row tile costs about 0.66 us per 128-deep K
-  // step plus a 10 us epilogue that its single-buffered accumulator cannot
-  // overlap; a 128-row tile about 0.485 us per K step plus 3 us (its epilogue
-  // overlaps the next tile).  The constants were measured on GB300 for these
-  // kernels; only their ratios matter.
+  const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
+  if (forced == SPINQ_GEMM_TILE128) return launch_mt<1>(a, stream);
+  if (forced == SPINQ_GEMM_TILE256) return launch_mt<2>(a, stream);
+  if (forced == SPINQ_GEMM_PAIR && a.M > 128) {
+    bool handled = false;
+    const cudaError_t e = launch_w4a4_gemm_pair(a, stream, &handled);
+    if (e != cudaSuccess || handled) return e;
+  }
+  // Kernel and tile height from a wave-quantised cost model (microseconds,
+  // constants measured on GB300 for these kernels; only their ratios
+  // matter).  A persistent CTA (or SM pair) runs ceil(tiles / CTAs) tiles
+  // back to back:
+  //   128 x 256 tiles, one CTA:  0.485 us per 128-deep K step + 3 us (the
+  //     epilogue overlaps the next tile);
+  //   256 x 256 tiles, one CTA:  0.66 us per K step + 10 us (the single
+  //     accumulator buffer serialises the epilogue);
+  //   256 x 256 tiles, SM pair:  0.45 us per K step, epilogue overlapped,
+  //     + 3 us for the last tile's epilogue.
   const int64_t sms = device_sm_count(), ks = a.K / 128;
   const int64_t tiles256 = ((a.M + 255) / 256) * ((a.N + BN - 1) / BN);
   const int64_t tiles128 = ((a.M + 127) / 128) * ((a.N + BN - 1) / BN);
   const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 10.0);
   const double est128 = (double)((tiles128 + sms - 1) / sms) * (0.485 * (double)ks + 3.0);
+  const int64_t pairs = a.M > 128 ? w4a4_gemm_pair_clusters() : 0;
+  if (pairs > 0) {
+    const double est_pair = (double)((tiles256 + pairs - 1) / pairs) * 0.45 * (double)ks + 3.0;
+    if (est_pair < est256 && est_pair < est128) {
+      bool handled = false;
+      const cudaError_t e = launch_w4a4_gemm_pair(a, stream, &handled);
+      if (e != cudaSuccess || handled) return e;
+    }
+  }
   if (est256 < est128) return launch_mt<2>(a, stream);
   return launch_mt<1>(a, stream);
 }
@@ -884,20 +917,22 @@ cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, cudaStre
   return launch_dec_mn<256>(a, ws_acc, ws_cnt, stream);
 }
 
+int* device_status_word() {
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+  return static_cast<int*>(p);
+}
+
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail) {
-  int c = 0, d = 0;
+  int st[2] = {0, 0};
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return e;
-  e = cudaMemcpyFromSymbol(&c, g_status_code, sizeof(int));
+  e = cudaMemcpyFromSymbol(st, g_status, sizeof(st));
   if (e != cudaSuccess) return e;
-  e = cudaMemcpyFromSymbol(&d, g_status_detail, sizeof(int));
-  if (e != cudaSuccess) return e;
-  const int zero = 0;
-  e = cudaMemcpyToSymbol(g_status_code, &zero, sizeof(int));
-  if (e != cudaSuccess) return e;
-  e = cudaMemcpyToSymbol(g_status_detail, &zero, sizeof(int));
-  *code = c;
-  *detail = d;
+  const int zero[2] = {0, 0};
+  e = cudaMemcpyToSymbol(g_status, zero, sizeof(zero));
+  *code = st[0];
+  *detail = st[1];
   return e;
 }
 

@@ -30,11 +30,12 @@ _lib = ctypes.CDLL(LIB_PATH)
 
 SPINQ_OK, SPINQ_EINVAL, SPINQ_EUNSUPPORTED, SPINQ_ECUDA, SPINQ_ETIMEOUT = range(5)
 SPINQ_PER_TOKEN, SPINQ_PER_CHANNEL, SPINQ_PER_GROUP = range(3)
+SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR = range(4)
 
 EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",
     "spinq_status_string", "spinq_device_status", "spinq_version", "spinq_w4a4_gemm_workspace_bytes",
-    "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc",
+    "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel",
 )
 
 
@@ -76,6 +77,8 @@ _lib.spinq_w4a4_gemm_splitk.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_splitk.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P, _I64, _P]
 _lib.spinq_w4a4_gemm_noalloc.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_noalloc.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
+_lib.spinq_gemm_select_kernel.restype = ctypes.c_int
+_lib.spinq_gemm_select_kernel.argtypes = [ctypes.c_int]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
 _lib.spinq_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
                                        ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
@@ -121,6 +124,10 @@ def spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k
                           k_zero, v_codes, v_scale, v_zero, stream) -> int:
     return _lib.spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k_codes,
                                       k_scale, k_zero, v_codes, v_scale, v_zero, stream)
+
+
+def spinq_gemm_select_kernel(kernel: int) -> int:
+    return int(_lib.spinq_gemm_select_kernel(kernel))
 
 
 def spinq_status_string(st: int) -> str:

@@ -76,6 +76,58 @@ def test_gemm_random_codes_exact(S, M, N, K, symmetric):
     assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
 
 
+@pytest.fixture
+def gemm_kernel(S, request):
+    """Forces one prefill GEMM kernel for the test and restores the default."""
+    prev = S.spinq_gemm_select_kernel(request.param)
+    assert prev >= 0
+    yield request.param
+    S.spinq_gemm_select_kernel(prev)
+
+
+KERNELS = [1, 2, 3]   # 128 x 256 tiles, 256 x 256 tiles, 256 x 256 tiles on SM pairs
+
+
+@pytest.mark.parametrize("gemm_kernel", KERNELS, indirect=True, ids=["tile128", "tile256", "pair"])
+@pytest.mark.parametrize("M,N,K", [(129, 256, 128), (300, 528, 384), (1000, 1040, 1024), (2001, 784, 512),
+                                   (513, 4096, 2048)])
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_gemm_each_kernel_exact(S, gemm_kernel, M, N, K, symmetric):
+    """Every prefill kernel, forced, on ragged M and N (partial tiles and SM
+    pairs whose second CTA lies partly or wholly below M)."""
+    rng = np.random.default_rng(M * 5 + N * 3 + K + symmetric)
+    ac, al, be, wc, ws = random_codes(rng, M, N, K, symmetric)
+    y, acc = run(S, ac, al, be, wc, ws)
+    ref = oracle_full(ac, al, be, wc, ws)
+    assert np.array_equal(acc, ref.acc)
+    assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
+    assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
+    st, _ = S.spinq_device_status()
+    assert st == S.SPINQ_OK
+
+
+@pytest.mark.parametrize("gemm_kernel", KERNELS, indirect=True, ids=["tile128", "tile256", "pair"])
+def test_gemm_each_kernel_same_bits(S, gemm_kernel):
+    """The kernels agree bit for bit (y and acc) with the automatic choice."""
+    rng = np.random.default_rng(11)
+    M, N, K = 777, 1296, 1536
+    ac, al, be, wc, ws = random_codes(rng, M, N, K, False)
+    y, acc = run(S, ac, al, be, wc, ws)
+    prev = S.spinq_gemm_select_kernel(0)
+    try:
+        y0, acc0 = run(S, ac, al, be, wc, ws)
+    finally:
+        S.spinq_gemm_select_kernel(prev)
+    assert np.array_equal(acc, acc0)
+    assert np.array_equal(y.view(np.uint16), y0.view(np.uint16))
+
+
+def test_gemm_select_kernel_rejects_unknown(S):
+    assert S.spinq_gemm_select_kernel(7) == -1
+    assert S.spinq_gemm_select_kernel(-1) == -1
+    assert S.spinq_gemm_select_kernel(0) == 0
+
+
 @pytest.mark.parametrize("symmetric", [True, False])
 def test_gemm_extreme_codes_long_k(S, symmetric):
     # largest accumulator magnitudes: every product at its extreme, K = 65536
@@ -112,13 +164,14 @@ FULL = [
     ("l32_up_M1", 1, 3072, 8192, False),
     ("l32_down_M16", 16, 8192, 3072, False),
     ("l32_up_M128", 128, 3072, 8192, False),
-    # 256-row tiles (K >= 3072, at least two tiles per SM) with ragged edges:
-    # M not a multiple of 32, N a multiple of 16 but not of 32 (clipped TMA stores)
-    ("tile256_ragged_M2000", 2000, 3072, 14352, True),
-    ("tile256_ragged_M2001_asym", 2001, 3072, 12304, False),
-    ("tile128_ragged_M2001_asym", 2001, 512, 12288, False),
+    # ragged edges, each prefill kernel forced: M not a multiple of 32, N a
+    # multiple of 16 but not of 32 (clipped TMA stores of y)
+    ("ragged_M2000_pair", 2000, 3072, 14352, True, 3),
+    ("ragged_M2000_tile256", 2000, 3072, 14352, True, 2),
+    ("ragged_M2001_asym_pair", 2001, 3072, 12304, False, 3),
+    ("ragged_M2001_asym_tile256", 2001, 3072, 12304, False, 2),
+    ("ragged_M2001_asym_tile128", 2001, 512, 12288, False, 1),
 ]
-
 
 @pytest.mark.parametrize("name,M,K,N,symmetric", [FULL[0], FULL[1]], ids=[FULL[0][0], FULL[1][0]])
 def test_gemm_repeat_bit_identical(S, name, M, K, N, symmetric):
@@ -139,11 +192,17 @@ def test_gemm_repeat_bit_identical(S, name, M, K, N, symmetric):
     assert np.array_equal(acc0.cpu().numpy()[ms, ns], racc)
 
 
-@pytest.mark.parametrize("name,M,K,N,symmetric", FULL, ids=[f[0] for f in FULL])
-def test_gemm_full_size_sampled(S, name, M, K, N, symmetric):
+@pytest.mark.parametrize("case", FULL, ids=[f[0] for f in FULL])
+def test_gemm_full_size_sampled(S, case):
+    name, M, K, N, symmetric = case[:5]
+    kernel = case[5] if len(case) > 5 else 0
     rng = np.random.default_rng(len(name))
     ac, al, be, wc, ws = random_codes(rng, M, N, K, symmetric)
-    y, acc = run(S, ac, al, be, wc, ws)
+    prev = S.spinq_gemm_select_kernel(kernel)
+    try:
+        y, acc = run(S, ac, al, be, wc, ws)
+    finally:
+        S.spinq_gemm_select_kernel(prev)
     # sampled outputs (random + corners + tile edges)
     ms = np.concatenate([rng.integers(0, M, 3000), [0, M - 1, min(127, M - 1), min(128, M - 1)]])
     ns = np.concatenate([rng.integers(0, N, 3000), [N - 1, 0, min(255, N - 1), min(256, N - 1)]])
