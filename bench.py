@@ -81,15 +81,20 @@ def step_ops():
     return gemm_ops() + gemm2_ops()
 
 
-def gemm_traffic_from_profile():
-    """DRAM bytes per GEMM launch from the committed ncu summary, or None when
+GEMM_KERNELS = {1: ("w4a4_gemm_kernel (128 x 256 tiles)", "w4a4_gemm.cu"),
+                2: ("w4a4_gemm_kernel (256 x 256 tiles)", "w4a4_gemm.cu"),
+                3: ("w4a4_gemm_pair_kernel (SM pairs, 256 x 256 tiles)", "w4a4_gemm_pair.cu")}
+
+
+def gemm_traffic_from_profile(profile, source):
+    """DRAM bytes per GEMM launch from a committed ncu summary, or None when
     the kernel source changed since the counters were taken."""
     import hashlib
     import re
     try:
-        src = os.path.join(ROOT, "paper_2405_16406_gb300", "csrc", "w4a4_gemm.cu")
+        src = os.path.join(ROOT, "paper_2405_16406_gb300", "csrc", source)
         h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        txt = open(os.path.join(ROOT, "profiles", "w4a4_gemm_gate_up_M2048_K4096_N14336.md")).read()
+        txt = open(os.path.join(ROOT, "profiles", profile)).read()
         if re.search(r"sha256 \(first 16 hex\): ([0-9a-f]{16})", txt).group(1) != h:
             return None
         return int(re.search(r"traffic_bytes_per_launch: (\d+)", txt).group(1))
@@ -232,23 +237,47 @@ def run_ours(args, rank, world, local_rank):
             fn(i % NSETS)
     torch.cuda.synchronize()
 
-    # One CUDA graph per (input set, kernel).  Replays keep the GPU fed with no
-    # host launch gaps; the per-kernel events sit between replays, so each
-    # per-kernel duration includes its graph launch (a few microseconds).
-    graphs = []
+    # One CUDA graph per input set holding the whole step (the five kernels
+    # back to back, no host launch between them), with timing-event nodes
+    # between the kernels: each replay re-records them, so after the timed
+    # loop they hold the per-kernel durations of each set's last timed step.
+    # (Where this PyTorch cannot put events into a graph, one graph per
+    # (set, kernel) is replayed instead, with events between the replays.)
+    def timing_event():
+        try:
+            return torch.cuda.Event(enable_timing=True, external=True)
+        except TypeError:
+            return None
+
+    in_graph = timing_event() is not None
+    graphs, gev = [], []
     for j in range(NSETS):
-        row = []
-        for fn in fns:
+        if in_graph:
+            evs = [timing_event() for _ in range(len(fns) + 1)]
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
-                fn(j)
-            row.append(g)
-        graphs.append(row)
+                evs[0].record()
+                for f_i, fn in enumerate(fns):
+                    fn(j)
+                    evs[f_i + 1].record()
+            graphs.append(g)
+            gev.append(evs)
+        else:
+            row = []
+            for fn in fns:
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    fn(j)
+                row.append(g)
+            graphs.append(row)
     torch.cuda.synchronize()
     ev = {k2: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                for _ in range(args.steps)] for k2 in names}
 
     def step(i, record=None):
+        if in_graph:
+            graphs[i % NSETS].replay()
+            return
         for name, g in zip(names, graphs[i % NSETS]):
             if record is not None:
                 ev[name][record][0].record(stream)
@@ -292,11 +321,16 @@ def run_ours(args, rank, world, local_rank):
         ms = float(t.item())
 
     def avg(key):
+        if in_graph:
+            k_i = names.index(key)
+            last = min(args.steps, NSETS)   # sets whose last replay was a timed step
+            return statistics.mean(gev[j][k_i].elapsed_time(gev[j][k_i + 1]) for j in range(last)) / 1e3
         return statistics.mean(a.elapsed_time(b) for a, b in ev[key]) / 1e3  # seconds
 
     t_gemm, t_rq, t_kv, t_rq2, t_gemm2 = avg("gemm"), avg("rq"), avg("kv"), avg("rq2"), avg("gemm2")
     gemm_tops = gemm_ops() / t_gemm / 1e12
     gemm2_tops = gemm2_ops() / t_gemm2 / 1e12
+    kind1, kind2 = spinq.spinq_w4a4_gemm_plan(M, N, K), spinq.spinq_w4a4_gemm_plan(M, N2, K2)
 
     # ---- end to end through the public API with host buffers
     x_h = [sets[j][0].cpu().pin_memory() for j in range(NSETS)]
@@ -427,16 +461,18 @@ def run_ours(args, rank, world, local_rank):
             "parallelism": f"replicas{world}",
         },
         "roofline": {
-            "bound": "tensor", "kernel": "w4a4_gemm_kernel",
+            "bound": "tensor", "kernel": GEMM_KERNELS[kind1][0],
             "achieved": round(gemm_tops, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
-            "frac": round(gemm_tops / fp8_peak, 4), "traffic": gemm_traffic_from_profile(),
+            "frac": round(gemm_tops / fp8_peak, 4),
+            "traffic": gemm_traffic_from_profile(f"w4a4_gemm_gate_up_M{M}_K{K}_N{N}.md", GEMM_KERNELS[kind1][1]),
             "peak_note": f"e4m3 dense = 2 x {peak_kind} bf16 ({bf16_peak} TFLOP/s); "
                          "int4 codes carried as e4m3 on tcgen05 kind::f8f6f4",
         },
         "roofline_down_proj": {
-            "bound": "tensor", "kernel": "w4a4_gemm_kernel (down_proj 2048 x 14336 -> 4096)",
+            "bound": "tensor", "kernel": GEMM_KERNELS[kind2][0] + f" (down_proj {M} x {K2} -> {N2})",
             "achieved": round(gemm2_tops, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
             "frac": round(gemm2_tops / fp8_peak, 4),
+            "traffic": gemm_traffic_from_profile(f"w4a4_gemm_down_proj_M{M}_K{K2}_N{N2}.md", GEMM_KERNELS[kind2][1]),
         },
         "rotate_quant_roofline": {
             "bound": "hbm", "kernel": "rq_paley_kernel (R4 = H28 (x) H512 + act quant, 2048 x 14336, sym)",
@@ -444,7 +480,9 @@ def run_ours(args, rank, world, local_rank):
             "frac": round(rq2_gbs / hbm_peak, 4), "us": round(t_rq2 * 1e6, 2),
             "isolated_us": round(iso["r4_quant"] * 1e6, 2),
             "isolated_frac": round(step_bytes_rq2() / iso["r4_quant"] / 1e9 / hbm_peak, 4),
-            "note": "in-step time includes the graph launch; isolated = 16 launches per graph, cold inputs",
+            "note": ("in-step time between the timing nodes around the kernel in the whole-step graph"
+                     if in_graph else "in-step time includes the graph launch")
+                    + "; isolated = 16 launches per graph, cold inputs",
         },
         "act_quant_roofline": {
             "bound": "hbm", "kernel": "rq_norot_kernel (act quant, 2048 x 4096, asym)",

@@ -229,6 +229,14 @@ typedef enum {
 
 int spinq_gemm_select_kernel(int kernel);
 
+/*
+ * spinq_w4a4_gemm_plan -- the prefill kernel (SPINQ_GEMM_TILE128, _TILE256
+ * or _PAIR) that spinq_w4a4_gemm runs for an M x N x K call on the current
+ * CUDA device under the current selection; -1 for shapes the call rejects.
+ * Launches nothing.
+ */
+int spinq_w4a4_gemm_plan(int64_t M, int64_t N, int64_t K);
+
 /* Human-readable name of a status code (static storage). */
 const char* spinq_status_string(spinq_status s);
 

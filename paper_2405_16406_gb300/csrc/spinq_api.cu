@@ -192,6 +192,11 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
 
 int spinq_gemm_select_kernel(int kernel) { return w4a4_gemm_select(kernel); }
 
+int spinq_w4a4_gemm_plan(int64_t M, int64_t N, int64_t K) {
+  if (M <= 0 || N <= 0 || K <= 0 || K % 128 != 0 || N % 16 != 0) return -1;
+  return plan_w4a4_gemm(M, N, K);
+}
+
 spinq_status spinq_device_status(int32_t* detail) {
   int32_t code = 0, d = 0;
   if (read_and_clear_device_status(&code, &d) != cudaSuccess) return SPINQ_ECUDA;

@@ -104,5 +104,8 @@ cudaError_t launch_w4a4_gemm_pair(const GemmArgs& a, cudaStream_t stream, bool* 
 int w4a4_gemm_pair_clusters();
 // Prefill kernel selection (spinq_gemm_kernel values); returns the previous one.
 int w4a4_gemm_select(int kernel);
+// The prefill kernel (SPINQ_GEMM_TILE128 / TILE256 / PAIR) launch_w4a4_gemm
+// runs for this shape on the current device.
+int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K);
 
 }  // namespace spinq

@@ -862,16 +862,11 @@ int w4a4_gemm_select(int kernel) {
   return g_gemm_kernel.exchange(kernel);
 }
 
-cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
-  if (a.M == 0 || a.N == 0) return cudaSuccess;
+int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K) {
   const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
-  if (forced == SPINQ_GEMM_TILE128) return launch_mt<1>(a, stream);
-  if (forced == SPINQ_GEMM_TILE256) return launch_mt<2>(a, stream);
-  if (forced == SPINQ_GEMM_PAIR && a.M > 128) {
-    bool handled = false;
-    const cudaError_t e = launch_w4a4_gemm_pair(a, stream, &handled);
-    if (e != cudaSuccess || handled) return e;
-  }
+  if (forced == SPINQ_GEMM_TILE128 || forced == SPINQ_GEMM_TILE256) return forced;
+  const int64_t pairs = M > 128 ? w4a4_gemm_pair_clusters() : 0;
+  if (forced == SPINQ_GEMM_PAIR && pairs > 0) return SPINQ_GEMM_PAIR;
   // Kernel and tile height from a wave-quantised cost model (microseconds,
   // constants measured on GB300 for these kernels; only their ratios
   // matter).  A persistent CTA (or SM pair) runs ceil(tiles / CTAs) tiles
@@ -882,21 +877,28 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   //     accumulator buffer serialises the epilogue);
   //   256 x 256 tiles, SM pair:  0.45 us per K step, epilogue overlapped,
   //     + 3 us for the last tile's epilogue.
-  const int64_t sms = device_sm_count(), ks = a.K / 128;
-  const int64_t tiles256 = ((a.M + 255) / 256) * ((a.N + BN - 1) / BN);
-  const int64_t tiles128 = ((a.M + 127) / 128) * ((a.N + BN - 1) / BN);
+  const int64_t sms = device_sm_count(), ks = K / 128;
+  const int64_t tiles256 = ((M + 255) / 256) * ((N + BN - 1) / BN);
+  const int64_t tiles128 = ((M + 127) / 128) * ((N + BN - 1) / BN);
   const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 10.0);
   const double est128 = (double)((tiles128 + sms - 1) / sms) * (0.485 * (double)ks + 3.0);
-  const int64_t pairs = a.M > 128 ? w4a4_gemm_pair_clusters() : 0;
   if (pairs > 0) {
     const double est_pair = (double)((tiles256 + pairs - 1) / pairs) * 0.45 * (double)ks + 3.0;
-    if (est_pair < est256 && est_pair < est128) {
-      bool handled = false;
-      const cudaError_t e = launch_w4a4_gemm_pair(a, stream, &handled);
-      if (e != cudaSuccess || handled) return e;
-    }
+    if (est_pair < est256 && est_pair < est128) return SPINQ_GEMM_PAIR;
   }
-  if (est256 < est128) return launch_mt<2>(a, stream);
+  return est256 < est128 ? SPINQ_GEMM_TILE256 : SPINQ_GEMM_TILE128;
+}
+
+cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
+  if (a.M == 0 || a.N == 0) return cudaSuccess;
+  const int kind = plan_w4a4_gemm(a.M, a.N, a.K);
+  if (kind == SPINQ_GEMM_PAIR) {
+    bool handled = false;
+    const cudaError_t e = launch_w4a4_gemm_pair(a, stream, &handled);
+    if (e != cudaSuccess || handled) return e;
+    return launch_mt<2>(a, stream);
+  }
+  if (kind == SPINQ_GEMM_TILE256) return launch_mt<2>(a, stream);
   return launch_mt<1>(a, stream);
 }
 

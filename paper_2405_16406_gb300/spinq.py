@@ -35,7 +35,7 @@ SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR = range
 EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",
     "spinq_status_string", "spinq_device_status", "spinq_version", "spinq_w4a4_gemm_workspace_bytes",
-    "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel",
+    "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel", "spinq_w4a4_gemm_plan",
 )
 
 
@@ -79,6 +79,8 @@ _lib.spinq_w4a4_gemm_noalloc.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_noalloc.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
 _lib.spinq_gemm_select_kernel.restype = ctypes.c_int
 _lib.spinq_gemm_select_kernel.argtypes = [ctypes.c_int]
+_lib.spinq_w4a4_gemm_plan.restype = ctypes.c_int
+_lib.spinq_w4a4_gemm_plan.argtypes = [_I64, _I64, _I64]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
 _lib.spinq_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
                                        ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
@@ -128,6 +130,10 @@ def spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k
 
 def spinq_gemm_select_kernel(kernel: int) -> int:
     return int(_lib.spinq_gemm_select_kernel(kernel))
+
+
+def spinq_w4a4_gemm_plan(M: int, N: int, K: int) -> int:
+    return int(_lib.spinq_w4a4_gemm_plan(M, N, K))
 
 
 def spinq_status_string(st: int) -> str:

@@ -128,6 +128,22 @@ def test_gemm_select_kernel_rejects_unknown(S):
     assert S.spinq_gemm_select_kernel(0) == 0
 
 
+def test_gemm_plan_follows_selection(S):
+    assert S.spinq_w4a4_gemm_plan(2048, 4100, 4096) == -1   # N not a multiple of 16
+    assert S.spinq_w4a4_gemm_plan(2048, 14336, 4000) == -1  # K not a multiple of 128
+    for kind in (1, 2, 3):
+        prev = S.spinq_gemm_select_kernel(kind)
+        try:
+            assert S.spinq_w4a4_gemm_plan(2048, 14336, 4096) == kind
+            small = S.spinq_w4a4_gemm_plan(128, 14336, 4096)
+            # SM pairs need more than 128 rows: the cost model decides there
+            assert small == kind if kind != 3 else small in (1, 2)
+        finally:
+            S.spinq_gemm_select_kernel(prev)
+    assert S.spinq_w4a4_gemm_plan(128, 14336, 4096) in (1, 2)
+    assert S.spinq_w4a4_gemm_plan(2048, 14336, 4096) in (1, 2, 3)
+
+
 @pytest.mark.parametrize("symmetric", [True, False])
 def test_gemm_extreme_codes_long_k(S, symmetric):
     # largest accumulator magnitudes: every product at its extreme, K = 65536
