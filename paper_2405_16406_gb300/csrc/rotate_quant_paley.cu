@@ -97,6 +97,12 @@ __device__ __forceinline__ int combo_i(int cb) {
   return ((cb >> 5) << 2) | ((cb >> 3) & 3);
 }
 
+// True when every slot of the warp holding combo cb is padding (>= ns): the
+// warp then skips the arithmetic of that combo altogether (warp-uniform).
+__device__ __forceinline__ bool combo_warp_idle(int cb, int ns) {
+  return ((cb >> 5) << 2) >= ns;
+}
+
 // Bounded wait for the phase of `bar` with `parity`.  Returns false when the
 // abort flag is up or the limit expired (then it raises the flag).
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
@@ -320,6 +326,7 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
     for (int k = 0; k < S::NCB; ++k) {
       const int cb = t2 + T * k;
       const bool act = cb < S::NCOMBO && combo_i(cb) < NS;
+      if (cb >= S::NCOMBO || combo_warp_idle(cb, NS)) continue;
 #pragma unroll
       for (int wv = 0; wv < W; ++wv) {
 #pragma unroll
@@ -368,6 +375,7 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
       const int cb = t2 + T * k;
       const int i2 = combo_i(cb), jc = cb & 7;
       const bool act = cb < S::NCOMBO && i2 < NS;
+      if (cb >= S::NCOMBO || combo_warp_idle(cb, NS)) continue;
       // wd[wv] = codes of j = jf + 16 wv .. + 7: word (jc & 1) + 2 W (jc >> 1) + 2 wv of segment i2
       uint32_t wd[W];
 #pragma unroll
