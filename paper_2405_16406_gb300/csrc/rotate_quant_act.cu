@@ -133,6 +133,8 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
     fence_mbar_init();
   }
   __syncthreads();
+  pdl_wait();
+  pdl_trigger();
   rs.prologue();
 
   // phase-2 fixed element bits of this thread: {L..2}, {3, 4}, v bits
@@ -262,6 +264,8 @@ __global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
     fence_mbar_init();
   }
   __syncthreads();
+  pdl_wait();
+  pdl_trigger();
   rs.prologue();
 
   int it = 0;
@@ -310,7 +314,8 @@ cudaError_t launch_rows(Kern kern, int threads, size_t smem, const RotQuantArgs&
   if (e != cudaSuccess) return e;
   const int64_t cap = (int64_t)device_sm_count() * per_sm;
   const int64_t grid = a.rows < cap ? a.rows : cap;
-  kern<<<(unsigned)grid, threads, smem, stream>>>(a);
+  e = launch_pdl(kern, dim3((unsigned)grid), dim3(threads), smem, stream, 1, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -60,6 +60,8 @@ __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) 
     bi[nt][1] = h16_pair(2 * c + 8, 2 * c + 9, n, false);
   }
 
+  pdl_wait();
+  pdl_trigger();
   const int64_t gq = (a.rows_q + 7) / 8, gk = (a.rows_kv + 7) / 8;
   const int64_t total = gq + 2 * gk;
   const int64_t stride = (int64_t)gridDim.x * kWarps;
@@ -200,7 +202,9 @@ cudaError_t launch_t(const KVArgs& a, cudaStream_t stream) {
   const int64_t cap = (int64_t)sms * 16;  // persistent-style cap: 16 blocks of 8 warps per SM
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  rotate_quant_kv_kernel<D, CLAMP><<<(unsigned)blocks, kWarps * 32, 0, stream>>>(a);
+  const cudaError_t e = launch_pdl(rotate_quant_kv_kernel<D, CLAMP>, dim3((unsigned)blocks), dim3(kWarps * 32), 0,
+                                   stream, 1, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

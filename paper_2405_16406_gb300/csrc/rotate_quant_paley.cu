@@ -163,6 +163,8 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
     prefetch_tmap(&tmx);
   }
   __syncthreads();  // the last CTA-wide barrier: the roles part here
+  pdl_wait();
+  pdl_trigger();
   if (tid == 0)
     for (int it = 0; it < NSTG && it < niter; ++it) issue(it);
 
@@ -438,7 +440,8 @@ cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const int64_t cap = (int64_t)device_sm_count() * per_sm;
   const int64_t grid = a.rows < cap ? a.rows : cap;
-  kern<<<(unsigned)grid, S::THREADS, S::BYTES, stream>>>(tmx, a);
+  e = launch_pdl(kern, dim3((unsigned)grid), dim3(S::THREADS), S::BYTES, stream, 1, tmx, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

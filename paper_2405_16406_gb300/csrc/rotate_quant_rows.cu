@@ -48,6 +48,8 @@ __global__ void __launch_bounds__(kThreads) rotate_quant_rows_kernel(RotQuantArg
   const int P = a.n_pow2;
   const int log2P = a.n_small ? 31 - __clz(P) : 0;
   const __half* __restrict__ x = reinterpret_cast<const __half*>(a.x);
+  pdl_wait();
+  pdl_trigger();
 
   for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x) {
     const __half* xr = x + row * a.ldx;
@@ -173,7 +175,8 @@ cudaError_t launch_t(const RotQuantArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const int64_t cap = (int64_t)device_sm_count() * per_sm * 4;
   const int64_t grid = a.rows < cap ? a.rows : cap;
-  kern<<<(unsigned)grid, kThreads, smem, stream>>>(a);
+  e = launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), smem, stream, 1, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -282,6 +282,17 @@ __device__ __forceinline__ void wait_loaded(const uint4 (&w)[N], volatile uint32
   if (acc == 0x9E3779B9u) *scratch = acc;
 }
 
+// Programmatic dependent launch.  Every kernel of the library is launched so
+// that it may start while the kernel before it in the stream is finishing;
+// each thread runs pdl_wait() after its shared-memory prologue and before its
+// first global-memory access (read or write): it returns once the preceding
+// grid has completed and its writes are visible (at once when there is no
+// such grid).  pdl_trigger() lets the next kernel be scheduled once every CTA
+// of this grid has reached it (grids are sized to be resident at once, so
+// the next kernel's CTAs only take SM resources this grid leaves free).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(nthreads) : "memory");
 }

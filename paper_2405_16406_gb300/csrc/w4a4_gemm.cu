@@ -194,6 +194,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer
@@ -575,6 +577,8 @@ __global__ void __launch_bounds__(kDecThreads, 2)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -813,7 +817,9 @@ cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   const int n_tiles = (int)((a.N + BN - 1) / BN);
   const int tiles = m_tiles * n_tiles;
   const int grid = tiles < sms ? tiles : sms;
-  kern<<<grid, kThreads, smem, stream>>>(tmA, tmB, tmY, a, (int)(a.K / 128), m_tiles, tiles);
+  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, 1, tmA, tmB, tmY, a, (int)(a.K / 128), m_tiles,
+                 tiles);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -840,7 +846,8 @@ cudaError_t launch_dec_t(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStre
   if (nsplit < 1) nsplit = 1;
   if (nsplit > ksteps) nsplit = ksteps;
   dim3 grid((unsigned)nsplit, (unsigned)ntiles);
-  kern<<<grid, kDecThreads, L::dyn_bytes, stream>>>(tmW, tmA, a, ws_acc, ws_cnt, ksteps, nsplit);
+  e = launch_pdl(kern, grid, dim3(kDecThreads), L::dyn_bytes, stream, 1, tmW, tmA, a, ws_acc, ws_cnt, ksteps, nsplit);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -226,6 +226,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer (this CTA's halves)
@@ -561,20 +563,9 @@ cudaError_t launch_pair_t(const GemmArgs& a, cudaStream_t stream, bool* handled)
   const int n_tiles = (int)((a.N + BN - 1) / BN);
   const int tiles = m_tiles * n_tiles;
   const int clusters = tiles < ncl ? tiles : ncl;
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.gridDim = dim3(2 * (unsigned)clusters, 1, 1);
-  cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = L::dyn_bytes;
-  cfg.stream = stream;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
   *handled = true;
-  e = cudaLaunchKernelEx(&cfg, kern, tmA, tmB, tmY, a, device_status_word(), (int)(a.K / 128), m_tiles, tiles);
+  e = launch_pdl(kern, dim3(2 * (unsigned)clusters), dim3(kThreads), L::dyn_bytes, stream, 2, tmA, tmB, tmY, a,
+                 device_status_word(), (int)(a.K / 128), m_tiles, tiles);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
