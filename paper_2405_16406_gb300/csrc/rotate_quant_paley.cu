@@ -457,8 +457,36 @@ cudaError_t launch_ns(const RotQuantArgs& a, cudaStream_t stream, bool* handled)
   return cudaSuccess;
 }
 
+// H_s (x) H_P with P = 2 Q equals (H_s (x) H_2) (x) H_Q on the same element
+// order (k = i P + j = (2 i + j_top) Q + j_low, and the Sylvester H_P is H_2
+// on the top bit of j times H_Q on the rest), so a factor of 2 can move from
+// the butterflies to the tensor core.  H_12 (x) H_256 runs as H_24 (x) H_128:
+// the 24 rows of H_24 fill the MMA's three n8 tiles exactly, where the 12
+// rows of H_12 leave a quarter of two tiles empty.
+SmallHadamard kron_h2(const SmallHadamard& h) {
+  SmallHadamard r;
+  r.n = 2 * h.n;
+  for (int p = 0; p < h.n; ++p)
+    for (int a2 = 0; a2 < 2; ++a2) {
+      uint32_t bits = 0;
+      for (int q = 0; q < h.n; ++q)
+        for (int b2 = 0; b2 < 2; ++b2)
+          if ((((h.neg[p] >> q) & 1u) ^ (uint32_t)(a2 & b2)) != 0) bits |= 1u << (2 * q + b2);
+      r.neg[2 * p + a2] = bits;
+    }
+  return r;
+}
+
 template <bool SYM, bool CLAMP>
 cudaError_t launch_sc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  if (a.n_small == 12 && a.n_pow2 == 256) {
+    RotQuantArgs b = a;
+    b.hs = kron_h2(a.hs);
+    b.n_small = 24;
+    b.n_pow2 = 128;
+    *handled = true;
+    return launch_paley<24, 7, SYM, CLAMP>(b, stream);
+  }
   switch (a.n_small) {
     case 12: return launch_ns<12, SYM, CLAMP>(a, stream, handled);
     case 20: return launch_ns<20, SYM, CLAMP>(a, stream, handled);
