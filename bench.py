@@ -160,9 +160,8 @@ class ClockSampler:
 # --------------------------------------------------------------------------- ours
 def run_ours(args, rank, world, local_rank):
     import torch
-    import torch.distributed as dist
 
-    from paper_2405_16406_gb300 import spinq
+    from paper_2405_16406_gb300 import replicas, spinq
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
@@ -171,7 +170,7 @@ def run_ours(args, rank, world, local_rank):
     fp8_peak = 2.0 * bf16_peak  # nominal e4m3 : bf16 dense ratio on GB300 is 2
 
     gen = torch.Generator(device=dev)
-    gen.manual_seed(1000 + rank)
+    gen.manual_seed(replicas.input_seed(1000, rank))
 
     def acts(rows, cols, frac, factor):
         x = torch.randn(rows, cols, generator=gen, device=dev)
@@ -313,8 +312,7 @@ def run_ours(args, rank, world, local_rank):
             i += 1
         torch.cuda.synchronize()
 
-    if world > 1:
-        dist.barrier()
+    replicas.barrier(world)
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
@@ -323,18 +321,13 @@ def run_ours(args, rank, world, local_rank):
         step(s_i)
     t1.record(stream)
     torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
+    replicas.barrier(world)
     # per-kernel timed loop (same steps, with the timing nodes)
     for s_i in range(args.steps):
         step_timed(s_i)
     torch.cuda.synchronize()
     clocks = sampler.stop() if sampler else None
-    ms = t0.elapsed_time(t1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = replicas.max_over_ranks(t0.elapsed_time(t1) / args.steps, world, device=dev)
 
     def avg(key):
         if in_graph:
@@ -436,8 +429,7 @@ def run_ours(args, rank, world, local_rank):
 
     run_e2e(4)
     torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
+    replicas.barrier(world)
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -446,11 +438,7 @@ def run_ours(args, rank, world, local_rank):
     stream.wait_stream(s_down)
     e1.record(stream)
     torch.cuda.synchronize()
-    ms_e2e = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms_e2e], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_e2e = float(t.item())
+    ms_e2e = replicas.max_over_ranks(e0.elapsed_time(e1) / args.steps, world, device=dev)
     h2d = (M * K + M * K2 + B_KV * S_KV * (HQ + 2 * HKV) * D) * 2
     d2h = (M * N + M * N2) * 2 + B_KV * S_KV * HQ * D * 2 + 2 * B_KV * S_KV * HKV * D // 2 + B_KV * S_KV * HKV * 16
 
@@ -498,7 +486,7 @@ def run_ours(args, rank, world, local_rank):
 
     if rank != 0:
         return None
-    value = world * step_ops() / (ms / 1e3) / 1e12
+    value = replicas.whole_job_rate(step_ops(), ms / 1e3, world) / 1e12
     rq_gbs = step_bytes_rq() / t_rq / 1e9
     rq2_gbs = step_bytes_rq2() / t_rq2 / 1e9
     kv_gbs = step_bytes_kv() / t_kv / 1e9
@@ -567,7 +555,7 @@ def run_ours(args, rank, world, local_rank):
         "kernel_us": {"gemm_gate_up": round(t_gemm * 1e6, 2), "act_quant": round(t_rq * 1e6, 2),
                       "r4_act_quant": round(t_rq2 * 1e6, 2), "gemm_down_proj": round(t_gemm2 * 1e6, 2),
                       "kv_quant": round(t_kv * 1e6, 2)},
-        "e2e": {"value": round(world * step_ops() / (ms_e2e / 1e3) / 1e12, 2), "unit": "TOPS",
+        "e2e": {"value": round(replicas.whole_job_rate(step_ops(), ms_e2e / 1e3, world) / 1e12, 2), "unit": "TOPS",
                 "pipeline": "uploads, kernels and read-backs on three streams, overlapped across steps",
                 "ms_per_step": round(ms_e2e, 4), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": len(names) * args.steps,
