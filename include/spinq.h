@@ -132,19 +132,24 @@ spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const
 
 /*
  * spinq_w4a4_gemm_workspace_bytes -- device workspace, in bytes, that
- * spinq_w4a4_gemm_splitk needs for an M x N output: M*N*4 + 4*ceil(N/128)
- * for M <= 256, and 0 for larger M (those calls need no workspace).
+ * spinq_w4a4_gemm_splitk needs for an M x N x K call: M*N*4 + 4*ceil(N/128)
+ * for the calls the split-K kernel serves (M <= 256 and not served by the
+ * GEMV kernel: M <= 4 with M * K <= 160 KiB), and 0 otherwise (those calls
+ * need no workspace and may pass NULL).
  */
 int64_t spinq_w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K);
 
 /*
  * spinq_w4a4_gemm_splitk -- the same operation and outputs as
  * spinq_w4a4_gemm, for small M (decode, M <= 256), where the GEMM is bound by
- * streaming the weights from HBM.  Each CTA owns 128 output channels and a
- * slice of K, so every SM streams a disjoint part of the weights; the slices'
- * exact integer partial accumulators are summed in `workspace` and the last
- * slice of each 128-channel tile applies the epilogue.  For M > 256 the call
- * runs the same kernel as spinq_w4a4_gemm and does not touch `workspace`.
+ * streaming the weights from HBM.  Up to 4 tokens (M * K <= 160 KiB) it runs
+ * the GEMV kernel: each warp owns whole output channels, streams their packed
+ * weights from global memory and takes exact integer dot products (no
+ * workspace).  Otherwise each CTA owns 128 output channels and a slice of K,
+ * so every SM streams a disjoint part of the weights; the slices' exact
+ * integer partial accumulators are summed in `workspace` and the last slice
+ * of each 128-channel tile applies the epilogue.  For M > 256 the call runs
+ * the same kernel as spinq_w4a4_gemm and does not touch `workspace`.
  *   workspace       device buffer of spinq_w4a4_gemm_workspace_bytes(M, N, K)
  *                   bytes, 16-byte aligned, all zero before the first call;
  *                   each completed call leaves it zero again.  Calls that may
@@ -209,13 +214,17 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
                                    float* v_zero, void* stream);
 
 /*
- * spinq_gemm_select_kernel -- which prefill kernel spinq_w4a4_gemm (and
+ * spinq_gemm_select_kernel -- which kernel spinq_w4a4_gemm (and
  * spinq_w4a4_gemm_splitk / _noalloc for M > 256) runs, process-wide:
  *   SPINQ_GEMM_AUTO     the built-in cost model picks (the default);
  *   SPINQ_GEMM_TILE128  one CTA per 128 x 256 output tile;
  *   SPINQ_GEMM_TILE256  one CTA per 256 x 256 output tile;
  *   SPINQ_GEMM_PAIR     two CTAs (an SM pair) per 256 x 256 tile; calls it
- *                       cannot serve (M <= 128, no pair resident) use AUTO.
+ *                       cannot serve (M <= 128, no pair resident) use AUTO;
+ *   SPINQ_GEMM_GEMV     (M <= 4 with M * K <= 160 KiB; AUTO picks it there,
+ *                       on the _splitk / _noalloc entry points too) each warp
+ *                       owns whole output channels and streams their packed
+ *                       weights; calls it cannot serve use AUTO.
  * All kernels compute bit-identical outputs; this is a tuning and testing
  * control.  Returns the previous selection, or -1 (and changes nothing) for
  * an unknown value.  Not synchronized with GEMM calls in other threads.
@@ -224,7 +233,8 @@ typedef enum {
   SPINQ_GEMM_AUTO = 0,
   SPINQ_GEMM_TILE128 = 1,
   SPINQ_GEMM_TILE256 = 2,
-  SPINQ_GEMM_PAIR = 3
+  SPINQ_GEMM_PAIR = 3,
+  SPINQ_GEMM_GEMV = 4
 } spinq_gemm_kernel;
 
 int spinq_gemm_select_kernel(int kernel);

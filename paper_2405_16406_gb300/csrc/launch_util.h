@@ -26,12 +26,16 @@ inline int device_sm_count() {
   return cache[dev];
 }
 
-// Raises the kernel's dynamic shared memory limit (once per size) and returns
-// the number of resident blocks per SM for this launch shape (at least 1).
+// Makes sure the kernel may use `smem` bytes of dynamic shared memory and
+// returns the number of resident blocks per SM for this launch shape (at
+// least 1).  The kernel's limit only ever grows (one kernel is launched with
+// several sizes: lowering it for a small launch would make a larger size that
+// is already cached fail to launch).
 template <typename Kern>
 cudaError_t prepare_launch(Kern kern, int threads, size_t smem, int* blocks_per_sm) {
   static std::mutex mu;
   static std::map<std::tuple<int, const void*, size_t, int>, int> occ;
+  static std::map<std::pair<int, const void*>, size_t> limit;   // per device and kernel
   int dev = 0;
   cudaGetDevice(&dev);
   const auto key = std::make_tuple(dev, reinterpret_cast<const void*>(kern), smem, threads);
@@ -41,9 +45,11 @@ cudaError_t prepare_launch(Kern kern, int threads, size_t smem, int* blocks_per_
     *blocks_per_sm = it->second;
     return cudaSuccess;
   }
-  if (smem > 48 * 1024) {
+  size_t& lim = limit[std::make_pair(dev, reinterpret_cast<const void*>(kern))];
+  if (smem > 48 * 1024 && smem > lim) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
+    lim = smem;
   }
   int per_sm = 0;
   cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);

@@ -142,8 +142,7 @@ spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const
 }
 
 int64_t spinq_w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K) {
-  (void)K;
-  return w4a4_gemm_workspace_bytes(M, N);
+  return w4a4_gemm_workspace_bytes(M, N, K);
 }
 
 spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
@@ -158,7 +157,7 @@ spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale
   if (!aligned16(a_codes) || !aligned16(w_codes) || !aligned16(y_f16) || !aligned16(w_scale) ||
       !aligned16(w_rowsum) || (acc_out && !aligned16(acc_out)))
     return SPINQ_EINVAL;
-  const int64_t need = w4a4_gemm_workspace_bytes(M, N);
+  const int64_t need = w4a4_gemm_workspace_bytes(M, N, K);
   if (need > 0 && (!workspace || !aligned16(workspace) || workspace_bytes < need)) return SPINQ_EINVAL;
   if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
   if (M == 0 || N == 0) return SPINQ_OK;

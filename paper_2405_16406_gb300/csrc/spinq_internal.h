@@ -84,8 +84,22 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
 // Largest M served by the split-K decode kernel.
 constexpr int64_t kDecodeMaxM = 256;
 
-// Workspace bytes of launch_w4a4_gemm_splitk for (M, N); 0 when M > kDecodeMaxM.
-int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N);
+// Workspace bytes of launch_w4a4_gemm_splitk for (M, N, K); 0 when the GEMV
+// kernel serves the call or M > kDecodeMaxM.
+int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K);
+// GEMV kernel for M <= kGemvMaxM tokens (decode; beyond 4 tokens its integer
+// dot products cost more than the split-K kernel's latency, measured on
+// GB300): each warp owns whole output
+// channels and streams their packed weights from global memory.  Sets
+// *handled = false when M or the expanded tokens (M K bytes of shared
+// memory) are out of its range.
+constexpr int64_t kGemvMaxM = 4;
+constexpr int64_t kGemvMaxSmem = 160 * 1024;
+int64_t w4a4_gemv_smem_bytes(int64_t M, int64_t K);
+inline bool w4a4_gemv_fits(int64_t M, int64_t K) {
+  return M >= 1 && M <= kGemvMaxM && w4a4_gemv_smem_bytes(M, K) <= kGemvMaxSmem;
+}
+cudaError_t launch_w4a4_gemv(const GemmArgs& a, cudaStream_t stream, bool* handled);
 
 // Split-K decode GEMM for M <= kDecodeMaxM (falls back to launch_w4a4_gemm
 // above).  `workspace` holds w4a4_gemm_workspace_bytes(M, N) bytes that are

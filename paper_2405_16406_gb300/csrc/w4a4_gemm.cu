@@ -865,13 +865,16 @@ cudaError_t launch_dec_mn(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStr
 std::atomic<int> g_gemm_kernel{SPINQ_GEMM_AUTO};
 
 int w4a4_gemm_select(int kernel) {
-  if (kernel < SPINQ_GEMM_AUTO || kernel > SPINQ_GEMM_PAIR) return -1;
+  if (kernel < SPINQ_GEMM_AUTO || kernel > SPINQ_GEMM_GEMV) return -1;
   return g_gemm_kernel.exchange(kernel);
 }
 
 int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K) {
   const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
+  // a handful of tokens: the product streams the weights, no tile kernel fits
+  if ((forced == SPINQ_GEMM_AUTO || forced == SPINQ_GEMM_GEMV) && w4a4_gemv_fits(M, K)) return SPINQ_GEMM_GEMV;
   if (forced == SPINQ_GEMM_TILE128 || forced == SPINQ_GEMM_TILE256) return forced;
+  // (a forced GEMV that does not fit falls through to the cost model)
   const int64_t pairs = M > 128 ? w4a4_gemm_pair_clusters() : 0;
   if (forced == SPINQ_GEMM_PAIR && pairs > 0) return SPINQ_GEMM_PAIR;
   // Kernel and tile height from a wave-quantised cost model (microseconds,
@@ -899,6 +902,12 @@ int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K) {
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
   const int kind = plan_w4a4_gemm(a.M, a.N, a.K);
+  if (kind == SPINQ_GEMM_GEMV) {
+    bool handled = false;
+    const cudaError_t e = launch_w4a4_gemv(a, stream, &handled);
+    if (e != cudaSuccess || handled) return e;
+    return launch_mt<1>(a, stream);
+  }
   if (kind == SPINQ_GEMM_PAIR) {
     bool handled = false;
     const cudaError_t e = launch_w4a4_gemm_pair(a, stream, &handled);
@@ -909,14 +918,17 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   return launch_mt<1>(a, stream);
 }
 
-int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N) {
-  if (M <= 0 || N <= 0 || M > kDecodeMaxM) return 0;
+int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K) {
+  if (M <= 0 || N <= 0 || M > kDecodeMaxM || w4a4_gemv_fits(M, K)) return 0;
   return M * N * 4 + ((N + 127) / 128) * 4;
 }
 
 cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
   if (a.M > kDecodeMaxM) return launch_w4a4_gemm(a, stream);
+  bool handled = false;
+  const cudaError_t eg = launch_w4a4_gemv(a, stream, &handled);
+  if (eg != cudaSuccess || handled) return eg;
   float* ws_acc = static_cast<float*>(workspace);
   int* ws_cnt = reinterpret_cast<int*>(static_cast<char*>(workspace) + a.M * a.N * 4);
   if (a.M <= 16) return launch_dec_mn<16>(a, ws_acc, ws_cnt, stream);

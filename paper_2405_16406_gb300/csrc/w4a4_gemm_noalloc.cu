@@ -64,7 +64,7 @@ extern "C" spinq_status spinq_w4a4_gemm_noalloc(const uint8_t* a_codes, const fl
       !is_aligned16(w_rowsum) || (acc_out && !is_aligned16(acc_out)))
     return SPINQ_EINVAL;
   if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
-  const int64_t need = spinq::w4a4_gemm_workspace_bytes(M, N);
+  const int64_t need = spinq::w4a4_gemm_workspace_bytes(M, N, K);
   if (need > kNoAllocScratchBytes) return SPINQ_EUNSUPPORTED;   // scratch too small for M x N
   if (M == 0 || N == 0) return SPINQ_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

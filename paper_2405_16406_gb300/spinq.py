@@ -30,7 +30,7 @@ _lib = ctypes.CDLL(LIB_PATH)
 
 SPINQ_OK, SPINQ_EINVAL, SPINQ_EUNSUPPORTED, SPINQ_ECUDA, SPINQ_ETIMEOUT = range(5)
 SPINQ_PER_TOKEN, SPINQ_PER_CHANNEL, SPINQ_PER_GROUP = range(3)
-SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR = range(4)
+SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR, SPINQ_GEMM_GEMV = range(5)
 
 EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",

@@ -142,6 +142,9 @@ def test_gemm_plan_follows_selection(S):
             S.spinq_gemm_select_kernel(prev)
     assert S.spinq_w4a4_gemm_plan(128, 14336, 4096) in (1, 2)
     assert S.spinq_w4a4_gemm_plan(2048, 14336, 4096) in (1, 2, 3)
+    assert S.spinq_w4a4_gemm_plan(4, 14336, 4096) == 4      # a handful of tokens: GEMV
+    assert S.spinq_w4a4_gemm_plan(5, 14336, 4096) != 4
+    assert S.spinq_gemm_select_kernel(6) == -1
 
 
 @pytest.mark.parametrize("symmetric", [True, False])
@@ -314,9 +317,57 @@ def test_splitk_random_codes_exact(S, M, N, K, symmetric):
     assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
 
 
+def test_splitk_no_workspace_for_the_gemv_path(S):
+    for M in (1, 3, 4):
+        assert S.spinq_w4a4_gemm_workspace_bytes(M, 8192, 3072) == 0
+        assert S.gemm_workspace(M, 8192, 3072) is None
+    assert S.spinq_w4a4_gemm_workspace_bytes(5, 8192, 3072) > 0
+    # the tokens no longer fit in shared memory: split-K with a workspace
+    assert S.spinq_w4a4_gemm_workspace_bytes(4, 8192, 65536) > 0
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 16, 128), (2, 48, 256), (3, 272, 384), (4, 512, 1024), (1, 1040, 4096),
+                                   (4, 8192, 8192), (3, 100 * 16, 14336), (1, 8192, 40960)])
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_gemv_random_codes_exact(S, M, N, K, symmetric):
+    """The GEMV kernel (M <= 4) through both entry points."""
+    rng = np.random.default_rng(M * 31 + N + K + symmetric)
+    ac, al, be, wc, ws_ = random_codes(rng, M, N, K, symmetric)
+    ref = oracle_full(ac, al, be, wc, ws_)
+    for entry in ("splitk", "gemm"):
+        if entry == "splitk":
+            y, acc = run_splitk(S, ac, al, be, wc, ws_)
+        else:
+            y, acc = run(S, ac, al, be, wc, ws_)
+        assert np.array_equal(acc, ref.acc), entry
+        assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
+        assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
+    assert S.spinq_w4a4_gemm_plan(M, N, K) == 4
+
+
+def test_gemv_shared_memory_sizes_in_any_order(S):
+    """One kernel launched with a large, a smaller and again the large shared
+    memory size (the per-kernel limit must not shrink)."""
+    rng = np.random.default_rng(5)
+    for (M, N, K) in [(4, 256, 32768), (3, 256, 14336), (4, 256, 32768), (2, 256, 1024), (4, 256, 32768)]:
+        ac, al, be, wc, ws_ = random_codes(rng, M, N, K, False)
+        y, acc = run_splitk(S, ac, al, be, wc, ws_)
+        assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc)
+
+
+def test_gemv_extreme_codes_long_k(S):
+    M, N, K = 3, 64, 65536 // 8   # M * K within the kernel's shared memory
+    for aval, wval in ((7, 7), (-8, -8), (7, -8)):
+        ac = np.full((M, K), aval, dtype=np.int32)
+        wc = np.full((N, K), wval, dtype=np.int32)
+        al, ws_ = np.full(M, 0.5), np.full(N, 0.25)
+        y, acc = run_splitk(S, ac, al, None, wc, ws_)
+        assert np.array_equal(acc, oracle_full(ac, al, None, wc, ws_).acc)
+
+
 def test_splitk_workspace_reused_and_left_zero(S):
     rng = np.random.default_rng(21)
-    M, N, K = 16, 1024, 2048
+    M, N, K = 100, 1024, 2048
     ws = S.gemm_workspace(M, N, K)
     for rep in range(3):
         ac, al, be, wc, ws_ = random_codes(rng, M, N, K, rep % 2 == 0)
