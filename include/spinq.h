@@ -132,10 +132,10 @@ spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const
 
 /*
  * spinq_w4a4_gemm_workspace_bytes -- device workspace, in bytes, that
- * spinq_w4a4_gemm_splitk needs for an M x N x K call: M*N*4 + 4*ceil(N/128)
- * for the calls the split-K kernel serves (M <= 256 and not served by the
- * GEMV kernel: M <= 4 with M * K <= 160 KiB), and 0 otherwise (those calls
- * need no workspace and may pass NULL).
+ * spinq_w4a4_gemm_splitk needs for an M x N x K call on the current CUDA
+ * device: M*N*4 + 4*ceil(N/128) for the calls whose K range it splits across
+ * CTAs (spinq_w4a4_gemm_splitk_plan), and 0 otherwise (those calls need no
+ * workspace and may pass NULL).
  */
 int64_t spinq_w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K);
 
@@ -145,10 +145,13 @@ int64_t spinq_w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K);
  * streaming the weights from HBM.  Up to 4 tokens (M * K <= 160 KiB) it runs
  * the GEMV kernel: each warp owns whole output channels, streams their packed
  * weights from global memory and takes exact integer dot products (no
- * workspace).  Otherwise each CTA owns 128 output channels and a slice of K,
- * so every SM streams a disjoint part of the weights; the slices' exact
- * integer partial accumulators are summed in `workspace` and the last slice
- * of each 128-channel tile applies the epilogue.  For M > 256 the call runs
+ * workspace).  Otherwise a cost model fitted on GB300 picks between the
+ * split-K kernel and the kernels of spinq_w4a4_gemm.  In the split-K kernel
+ * each CTA owns 128 output channels and a slice of K, so every SM streams a
+ * disjoint part of the weights; the slices' exact integer partial
+ * accumulators are summed in `workspace` and the last slice of each
+ * 128-channel tile applies the epilogue (with a single slice the CTA writes
+ * the outputs itself and no workspace is used).  For M > 256 the call runs
  * the same kernel as spinq_w4a4_gemm and does not touch `workspace`.
  *   workspace       device buffer of spinq_w4a4_gemm_workspace_bytes(M, N, K)
  *                   bytes, 16-byte aligned, all zero before the first call;
@@ -174,9 +177,9 @@ spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale
  *   Same arguments, outputs and requirements as spinq_w4a4_gemm; no workspace
  *   argument.  The workspace lives in a fixed 8 MiB device array owned by the
  *   library, which every GPU that loads the library holds until the process
- *   exits; requests whose workspace (spinq_w4a4_gemm_workspace_bytes) exceeds
- *   8 MiB return SPINQ_EUNSUPPORTED before any launch (M > 256 needs none and
- *   is always accepted).
+ *   exits; a call whose split-K workspace (spinq_w4a4_gemm_workspace_bytes)
+ *   exceeds 8 MiB does not split K (each 128-channel tile keeps its whole K
+ *   range) and needs none of it.
  *   The call itself allocates nothing: no cudaMalloc/cudaFree and no
  *   allocating library routine.  It clears the part of the array it uses
  *   (cudaMemsetAsync on `stream`) before the kernel, since the array keeps
@@ -224,7 +227,10 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
  *   SPINQ_GEMM_GEMV     (M <= 4 with M * K <= 160 KiB; AUTO picks it there,
  *                       on the _splitk / _noalloc entry points too) each warp
  *                       owns whole output channels and streams their packed
- *                       weights; calls it cannot serve use AUTO.
+ *                       weights; calls it cannot serve use AUTO;
+ *   SPINQ_GEMM_SPLITK   the split-K kernel on the _splitk / _noalloc entry
+ *                       points for every M <= 256 (GEMV and prefill kernels
+ *                       excluded); spinq_w4a4_gemm treats it as AUTO.
  * All kernels compute bit-identical outputs; this is a tuning and testing
  * control.  Returns the previous selection, or -1 (and changes nothing) for
  * an unknown value.  Not synchronized with GEMM calls in other threads.
@@ -234,18 +240,39 @@ typedef enum {
   SPINQ_GEMM_TILE128 = 1,
   SPINQ_GEMM_TILE256 = 2,
   SPINQ_GEMM_PAIR = 3,
-  SPINQ_GEMM_GEMV = 4
+  SPINQ_GEMM_GEMV = 4,
+  SPINQ_GEMM_SPLITK = 5
 } spinq_gemm_kernel;
 
 int spinq_gemm_select_kernel(int kernel);
 
 /*
- * spinq_w4a4_gemm_plan -- the prefill kernel (SPINQ_GEMM_TILE128, _TILE256
- * or _PAIR) that spinq_w4a4_gemm runs for an M x N x K call on the current
- * CUDA device under the current selection; -1 for shapes the call rejects.
+ * spinq_gemm_split_k -- process-wide number of K slices per 128-channel tile
+ * of the split-K kernel: 1..64 fixes it (at most K / 128), 0 lets the cost
+ * model pick (the default).  A tuning and testing control like
+ * spinq_gemm_select_kernel; spinq_w4a4_gemm_workspace_bytes and
+ * spinq_w4a4_gemm_splitk_plan follow it.  Returns the previous value, or -1
+ * (and changes nothing) for a value out of range.
+ */
+int spinq_gemm_split_k(int n);
+
+/*
+ * spinq_w4a4_gemm_plan -- the kernel (SPINQ_GEMM_TILE128, _TILE256, _PAIR or
+ * _GEMV) that spinq_w4a4_gemm runs for an M x N x K call on the current CUDA
+ * device under the current selection; -1 for shapes the call rejects.
  * Launches nothing.
  */
 int spinq_w4a4_gemm_plan(int64_t M, int64_t N, int64_t K);
+
+/*
+ * spinq_w4a4_gemm_splitk_plan -- the kernel that spinq_w4a4_gemm_splitk runs
+ * for an M x N x K call given a workspace of spinq_w4a4_gemm_workspace_bytes
+ * bytes: SPINQ_GEMM_SPLITK, with *nsplit (may be NULL) set to its number of K
+ * slices per 128-channel tile (1: no slicing, no workspace), or the kernel
+ * spinq_w4a4_gemm would run (*nsplit = 0).  -1 for shapes the call rejects.
+ * Launches nothing.
+ */
+int spinq_w4a4_gemm_splitk_plan(int64_t M, int64_t N, int64_t K, int* nsplit);
 
 /* Human-readable name of a status code (static storage). */
 const char* spinq_status_string(spinq_status s);

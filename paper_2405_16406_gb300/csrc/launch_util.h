@@ -6,6 +6,7 @@
 
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <map>
 #include <mutex>
 #include <tuple>
@@ -57,6 +58,36 @@ cudaError_t prepare_launch(Kern kern, int threads, size_t smem, int* blocks_per_
   if (per_sm < 1) per_sm = 1;
   occ[key] = per_sm;
   *blocks_per_sm = per_sm;
+  return cudaSuccess;
+}
+
+// prepare_launch for a kernel that allocates `tmem_cols` columns of tensor
+// memory per block.  The occupancy query answers one block per SM for every
+// kernel that allocates tensor memory (measured on GB300), so the resident
+// blocks come from the per-SM limits instead: shared memory (with the
+// per-block reservation), registers (whole warps, 256-register granules),
+// threads, and the SM's 512 tensor-memory columns.
+template <typename Kern>
+cudaError_t prepare_launch_tmem(Kern kern, int threads, size_t smem, int tmem_cols, int* blocks_per_sm) {
+  int q = 0;
+  cudaError_t e = prepare_launch(kern, threads, smem, &q);
+  if (e != cudaSuccess) return e;
+  int dev = 0, smem_sm = 0, smem_rsv = 0, regs_sm = 0, thr_sm = 0;
+  cudaGetDevice(&dev);
+  cudaFuncAttributes fa;
+  if ((e = cudaFuncGetAttributes(&fa, kern)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess ||
+      (e = cudaDeviceGetAttribute(&smem_rsv, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess ||
+      (e = cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev)) != cudaSuccess ||
+      (e = cudaDeviceGetAttribute(&thr_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev)) != cudaSuccess)
+    return e;
+  const int warps = (threads + 31) / 32;
+  const int regs_warp = (fa.numRegs * 32 + 255) / 256 * 256;
+  int n = (int)((size_t)smem_sm / (smem + fa.sharedSizeBytes + (size_t)smem_rsv));
+  if (regs_warp > 0) n = std::min(n, regs_sm / (warps * regs_warp));
+  n = std::min(n, thr_sm / (warps * 32));
+  if (tmem_cols > 0) n = std::min(n, 512 / tmem_cols);
+  *blocks_per_sm = std::max(1, std::min(n, 32));
   return cudaSuccess;
 }
 

@@ -162,7 +162,7 @@ spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale
   if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
   if (M == 0 || N == 0) return SPINQ_OK;
   GemmArgs g{a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y_f16, acc_out};
-  return from_cuda(launch_w4a4_gemm_splitk(g, workspace, static_cast<cudaStream_t>(stream)));
+  return from_cuda(launch_w4a4_gemm_splitk(g, workspace, workspace_bytes, static_cast<cudaStream_t>(stream)));
 }
 
 spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_in,
@@ -191,9 +191,20 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
 
 int spinq_gemm_select_kernel(int kernel) { return w4a4_gemm_select(kernel); }
 
+int spinq_gemm_split_k(int n) { return w4a4_gemm_split_k(n); }
+
 int spinq_w4a4_gemm_plan(int64_t M, int64_t N, int64_t K) {
   if (M <= 0 || N <= 0 || K <= 0 || K % 128 != 0 || N % 16 != 0) return -1;
   return plan_w4a4_gemm(M, N, K);
+}
+
+int spinq_w4a4_gemm_splitk_plan(int64_t M, int64_t N, int64_t K, int* nsplit) {
+  if (nsplit) *nsplit = 0;
+  if (M <= 0 || N <= 0 || K <= 0 || K % 128 != 0 || N % 16 != 0 || K > 65536) return -1;
+  int ns = 0;
+  const int kind = plan_w4a4_gemm_splitk(M, N, K, &ns);
+  if (nsplit) *nsplit = ns;
+  return kind;
 }
 
 spinq_status spinq_device_status(int32_t* detail) {

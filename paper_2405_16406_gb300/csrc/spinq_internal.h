@@ -84,8 +84,9 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
 // Largest M served by the split-K decode kernel.
 constexpr int64_t kDecodeMaxM = 256;
 
-// Workspace bytes of launch_w4a4_gemm_splitk for (M, N, K); 0 when the GEMV
-// kernel serves the call or M > kDecodeMaxM.
+// Workspace bytes of launch_w4a4_gemm_splitk for (M, N, K); 0 unless its
+// plan splits K (the GEMV kernel, the prefill kernels and unsplit tiles
+// write y directly).
 int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K);
 // GEMV kernel for M <= kGemvMaxM tokens (decode; beyond 4 tokens its integer
 // dot products cost more than the split-K kernel's latency, measured on
@@ -101,10 +102,14 @@ inline bool w4a4_gemv_fits(int64_t M, int64_t K) {
 }
 cudaError_t launch_w4a4_gemv(const GemmArgs& a, cudaStream_t stream, bool* handled);
 
-// Split-K decode GEMM for M <= kDecodeMaxM (falls back to launch_w4a4_gemm
-// above).  `workspace` holds w4a4_gemm_workspace_bytes(M, N) bytes that are
-// zero before the call and zero again after it.
-cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, cudaStream_t stream);
+// Decode GEMM for M <= kDecodeMaxM (launch_w4a4_gemm above): the GEMV kernel,
+// the split-K kernel or the prefill kernels, as a fitted cost model predicts
+// fastest.  `workspace` holds `workspace_bytes` bytes that are zero before
+// the call and zero again after it; K is split only when they hold the
+// partial sums (M N 4 + 4 ceil(N / 128) bytes), else each tile keeps its
+// whole K range.
+cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, int64_t workspace_bytes,
+                                    cudaStream_t stream);
 
 // Device status word written by bounded waits that gave up.
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail);
@@ -118,8 +123,15 @@ cudaError_t launch_w4a4_gemm_pair(const GemmArgs& a, cudaStream_t stream, bool* 
 int w4a4_gemm_pair_clusters();
 // Prefill kernel selection (spinq_gemm_kernel values); returns the previous one.
 int w4a4_gemm_select(int kernel);
+// Process-wide fixed count of the split-K kernel's K slices (0: the cost
+// model picks).
+int w4a4_gemm_split_k(int n);
 // The prefill kernel (SPINQ_GEMM_TILE128 / TILE256 / PAIR) launch_w4a4_gemm
 // runs for this shape on the current device.
 int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K);
+// The kernel launch_w4a4_gemm_splitk runs with a full workspace:
+// SPINQ_GEMM_SPLITK with its K slices in *nsplit, or another SPINQ_GEMM_*
+// kernel (*nsplit = 0).
+int plan_w4a4_gemm_splitk(int64_t M, int64_t N, int64_t K, int* nsplit);
 
 }  // namespace spinq

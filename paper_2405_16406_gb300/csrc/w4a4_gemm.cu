@@ -37,7 +37,9 @@
 #include <cuda.h>
 #include <cuda_fp16.h>
 
+#include <algorithm>
 #include <atomic>
+#include <cmath>
 #include <mutex>
 
 #include "../../include/spinq.h"
@@ -514,7 +516,9 @@ struct DecCfg {
   static constexpr uint32_t misc = bars + nbars * 8;   // tmem slot, abort flag, last flag
   static constexpr uint32_t rsw = (misc + 16 + 15) & ~15u;   // [128] weight row sums of this split
   static constexpr uint32_t rsa = rsw + 128 * 4;               // [MN] token sums of this split
-  static constexpr uint32_t total = rsa + MN * 4;
+  static constexpr uint32_t tal = rsa + MN * 4;                // [MN] token scales alpha_m
+  static constexpr uint32_t tbp = tal + MN * 4;                // [MN] beta'_m (asymmetric tokens)
+  static constexpr uint32_t total = tbp + MN * 4;
   static constexpr size_t dyn_bytes = total + 1024;
   static constexpr uint32_t tmem_cols = MN <= 32 ? 32 : MN <= 64 ? 64 : MN <= 128 ? 128 : 256;
 };
@@ -543,6 +547,8 @@ __global__ void __launch_bounds__(kDecThreads, 2)
   volatile uint32_t* scratch = reinterpret_cast<volatile uint32_t*>(base + L::misc + 12);   // see wait_loaded
   int* rsw = reinterpret_cast<int*>(base + L::rsw);
   int* rsa = reinterpret_cast<int*>(base + L::rsa);
+  float* tal = reinterpret_cast<float*>(base + L::tal);
+  float* tbp = reinterpret_cast<float*>(base + L::tbp);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int split = blockIdx.x, ntile = blockIdx.y;
@@ -696,6 +702,13 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     const int nl = q * 32 + lane;                 // weight row of this lane (TMEM lane)
     const int64_t n = n0 + nl;
     const int et = tid - kFirstEpiWarp * 32;    // 0..127
+    // the tokens' scales, staged while the main loop runs
+    for (int m = et; m < MN; m += kEpiWarps * 32) {
+      const float alpha = m < args.M ? __ldg(args.a_scale + m) : 0.f;
+      tal[m] = alpha;
+      tbp[m] = ASYM && m < args.M ? __ldg(args.a_zero + m) + 8.f * alpha : 0.f;
+    }
+    named_bar_sync(1, kEpiWarps * 32);
     bool ok = wait_or_abort(acc_full, 0, abort_flag, 15);
     ok = ok && wait_or_abort(rs_full, 0, abort_flag, 16);
     __syncwarp();
@@ -709,6 +722,22 @@ __global__ void __launch_bounds__(kDecThreads, 2)
       tmem_ld_32x32b_x16(taddr + (uint32_t)c0, r);
       tmem_ld_wait(r);
       if (!ok || n >= args.N) continue;
+      if (nsplit == 1) {
+        // the whole K range: this is the final sum, no workspace
+        const float sn = __ldg(args.w_scale + n);
+        const float rwf = (float)__ldg(args.w_rowsum + n);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const int m = c0 + e;
+          if (m < args.M) {
+            const float accf = fmaf(__uint_as_float(r[e]), 262144.0f, wfix - 8.f * (float)rsa[m]);
+            reinterpret_cast<__half*>(args.y)[(int64_t)m * args.N + n] =
+                __float2half_rn(sn * fmaf(tal[m], accf, tbp[m] * rwf));
+            if (ACC_OUT) args.acc_out[(int64_t)m * args.N + n] = __float2int_rn(accf);
+          }
+        }
+        continue;
+      }
 #pragma unroll
       for (int e = 0; e < 16; ++e) {
         const int m = c0 + e;
@@ -719,6 +748,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
       }
     }
     tc_fence_before();
+    if (nsplit > 1) {
     // the last split of this output tile finishes it
     __threadfence();
     named_bar_sync(1, kEpiWarps * 32);
@@ -726,31 +756,31 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     named_bar_sync(1, kEpiWarps * 32);
     if (*last_flag) {
       __threadfence();
-      // thread et owns channel n0 + et for every token; 8 tokens per batch of
-      // independent loads
+      // thread et owns channel n0 + et for every token; a batch of 32
+      // independent loads per round trip to L2
       const int64_t nn = n0 + et;
       if (nn < args.N) {
         const float sn = args.w_scale[nn];
         const float rwf = (float)args.w_rowsum[nn];
-        for (int64_t mb = 0; mb < args.M; mb += 8) {
-          float accf[8];
+        for (int mb = 0; mb < MN && mb < args.M; mb += 32) {
+          float accf[32];
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
-            accf[e] = mb + e < args.M ? __ldcg(ws_acc + (mb + e) * args.N + nn) : 0.f;
+          for (int e = 0; e < 32; ++e)
+            accf[e] = mb + e < args.M ? __ldcg(ws_acc + (int64_t)(mb + e) * args.N + nn) : 0.f;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int64_t m = mb + e;
+          for (int e = 0; e < 32; ++e) {
+            const int m = mb + e;
             if (m < args.M) {
-              ws_acc[m * args.N + nn] = 0.f;
-              const float alpha = __ldg(args.a_scale + m);
-              const float bp = ASYM ? __ldg(args.a_zero + m) + 8.f * alpha : 0.f;
-              reinterpret_cast<__half*>(args.y)[m * args.N + nn] = __float2half_rn(sn * fmaf(alpha, accf[e], bp * rwf));
-              if (ACC_OUT) args.acc_out[m * args.N + nn] = __float2int_rn(accf[e]);
+              ws_acc[(int64_t)m * args.N + nn] = 0.f;
+              reinterpret_cast<__half*>(args.y)[(int64_t)m * args.N + nn] =
+                  __float2half_rn(sn * fmaf(tal[m], accf[e], tbp[m] * rwf));
+              if (ACC_OUT) args.acc_out[(int64_t)m * args.N + nn] = __float2int_rn(accf[e]);
             }
           }
         }
       }
       if (et == 0) ws_cnt[ntile] = 0;
+    }
     }
   }
 
@@ -831,7 +861,7 @@ cudaError_t launch_mt(const GemmArgs& a, cudaStream_t stream) {
 }
 
 template <int MN, bool ASYM, bool ACC_OUT>
-cudaError_t launch_dec_t(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStream_t stream) {
+cudaError_t launch_dec_t(const GemmArgs& a, float* ws_acc, int* ws_cnt, int nsplit, cudaStream_t stream) {
   using L = DecCfg<MN>;
   CUtensorMap tmW, tmA;
   if (!encode_packed_map(&tmW, a.w_codes, a.N, a.K, 128)) return cudaErrorNotSupported;
@@ -842,9 +872,9 @@ cudaError_t launch_dec_t(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStre
   if (e != cudaSuccess) return e;
   const int ksteps = (int)(a.K / 128);
   const int ntiles = (int)((a.N + 127) / 128);
-  int nsplit = (device_sm_count() * per_sm) / ntiles;
-  if (nsplit < 1) nsplit = 1;
-  if (nsplit > ksteps) nsplit = ksteps;
+  // every slice owns at least one K step; slices need the workspace
+  if (nsplit < 1 || nsplit > ksteps || (nsplit > 1 && (ws_acc == nullptr || ws_cnt == nullptr)))
+    return cudaErrorInvalidValue;
   dim3 grid((unsigned)nsplit, (unsigned)ntiles);
   e = launch_pdl(kern, grid, dim3(kDecThreads), L::dyn_bytes, stream, 1, tmW, tmA, a, ws_acc, ws_cnt, ksteps, nsplit);
   if (e != cudaSuccess) return e;
@@ -852,12 +882,30 @@ cudaError_t launch_dec_t(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStre
 }
 
 template <int MN>
-cudaError_t launch_dec_mn(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStream_t stream) {
+cudaError_t launch_dec_mn(const GemmArgs& a, float* ws_acc, int* ws_cnt, int nsplit, cudaStream_t stream) {
   const bool asym = a.a_zero != nullptr, acc = a.acc_out != nullptr;
-  if (asym) return acc ? launch_dec_t<MN, true, true>(a, ws_acc, ws_cnt, stream)
-                       : launch_dec_t<MN, true, false>(a, ws_acc, ws_cnt, stream);
-  return acc ? launch_dec_t<MN, false, true>(a, ws_acc, ws_cnt, stream)
-             : launch_dec_t<MN, false, false>(a, ws_acc, ws_cnt, stream);
+  if (asym) return acc ? launch_dec_t<MN, true, true>(a, ws_acc, ws_cnt, nsplit, stream)
+                       : launch_dec_t<MN, true, false>(a, ws_acc, ws_cnt, nsplit, stream);
+  return acc ? launch_dec_t<MN, false, true>(a, ws_acc, ws_cnt, nsplit, stream)
+             : launch_dec_t<MN, false, false>(a, ws_acc, ws_cnt, nsplit, stream);
+}
+
+// Resident CTAs per SM of the split-K kernel for M tokens (the variants of one
+// token bucket share their shared memory size).
+template <int MN>
+int dec_per_sm() {
+  int p = 1;
+  if (prepare_launch_tmem(w4a4_decode_kernel<MN, false, false>, kDecThreads, DecCfg<MN>::dyn_bytes,
+                         (int)DecCfg<MN>::tmem_cols, &p) != cudaSuccess)
+    return 1;
+  return p;
+}
+int dec_per_sm_for(int64_t M, int* mn) {
+  if (M <= 16) return *mn = 16, dec_per_sm<16>();
+  if (M <= 32) return *mn = 32, dec_per_sm<32>();
+  if (M <= 64) return *mn = 64, dec_per_sm<64>();
+  if (M <= 128) return *mn = 128, dec_per_sm<128>();
+  return *mn = 256, dec_per_sm<256>();
 }
 
 }  // namespace
@@ -865,38 +913,61 @@ cudaError_t launch_dec_mn(const GemmArgs& a, float* ws_acc, int* ws_cnt, cudaStr
 std::atomic<int> g_gemm_kernel{SPINQ_GEMM_AUTO};
 
 int w4a4_gemm_select(int kernel) {
-  if (kernel < SPINQ_GEMM_AUTO || kernel > SPINQ_GEMM_GEMV) return -1;
+  if (kernel < SPINQ_GEMM_AUTO || kernel > SPINQ_GEMM_SPLITK) return -1;
   return g_gemm_kernel.exchange(kernel);
 }
 
-int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K) {
-  const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
-  // a handful of tokens: the product streams the weights, no tile kernel fits
-  if ((forced == SPINQ_GEMM_AUTO || forced == SPINQ_GEMM_GEMV) && w4a4_gemv_fits(M, K)) return SPINQ_GEMM_GEMV;
-  if (forced == SPINQ_GEMM_TILE128 || forced == SPINQ_GEMM_TILE256) return forced;
-  // (a forced GEMV that does not fit falls through to the cost model)
-  const int64_t pairs = M > 128 ? w4a4_gemm_pair_clusters() : 0;
-  if (forced == SPINQ_GEMM_PAIR && pairs > 0) return SPINQ_GEMM_PAIR;
-  // Kernel and tile height from a wave-quantised cost model (microseconds,
-  // constants measured on GB300 for these kernels; only their ratios
-  // matter).  A persistent CTA (or SM pair) runs ceil(tiles / CTAs) tiles
-  // back to back:
-  //   128 x 256 tiles, one CTA:  0.485 us per 128-deep K step + 3 us (the
-  //     epilogue overlaps the next tile);
-  //   256 x 256 tiles, one CTA:  0.66 us per K step + 10 us (the single
-  //     accumulator buffer serialises the epilogue);
-  //   256 x 256 tiles, SM pair:  0.45 us per K step, epilogue overlapped,
-  //     + 3 us for the last tile's epilogue.
+std::atomic<int> g_split_k{0};
+
+int w4a4_gemm_split_k(int n) {
+  if (n < 0 || n > 64) return -1;
+  return g_split_k.exchange(n);
+}
+
+namespace {
+
+// Kernel and tile height from a wave-quantised cost model (microseconds,
+// constants measured on GB300 for these kernels; only their ratios matter).
+// A persistent CTA (or SM pair) runs ceil(tiles / CTAs) tiles back to back:
+//   128 x 256 tiles, one CTA:  0.485 us per 128-deep K step + 3 us (the
+//     epilogue overlaps the next tile);
+//   256 x 256 tiles, one CTA:  0.66 us per K step + 10 us (the single
+//     accumulator buffer serialises the epilogue);
+//   256 x 256 tiles, SM pair:  0.45 us per K step, epilogue overlapped,
+//     + 3 us for the last tile's epilogue.
+struct PrefillChoice {
+  int kind;
+  double us;
+};
+
+PrefillChoice choose_prefill(int64_t M, int64_t N, int64_t K, bool allow_pair) {
+  const int64_t pairs = allow_pair && M > 128 ? w4a4_gemm_pair_clusters() : 0;
   const int64_t sms = device_sm_count(), ks = K / 128;
   const int64_t tiles256 = ((M + 255) / 256) * ((N + BN - 1) / BN);
   const int64_t tiles128 = ((M + 127) / 128) * ((N + BN - 1) / BN);
   const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 10.0);
   const double est128 = (double)((tiles128 + sms - 1) / sms) * (0.485 * (double)ks + 3.0);
+  PrefillChoice c = est256 < est128 ? PrefillChoice{SPINQ_GEMM_TILE256, est256} : PrefillChoice{SPINQ_GEMM_TILE128, est128};
   if (pairs > 0) {
     const double est_pair = (double)((tiles256 + pairs - 1) / pairs) * 0.45 * (double)ks + 3.0;
-    if (est_pair < est256 && est_pair < est128) return SPINQ_GEMM_PAIR;
+    if (est_pair < c.us) c = {SPINQ_GEMM_PAIR, est_pair};
   }
-  return est256 < est128 ? SPINQ_GEMM_TILE256 : SPINQ_GEMM_TILE128;
+  return c;
+}
+
+}  // namespace
+
+int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K) {
+  const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
+  // a handful of tokens: the product streams the weights, no tile kernel fits
+  // (the split-K selection concerns the other entry point only)
+  if ((forced == SPINQ_GEMM_AUTO || forced == SPINQ_GEMM_GEMV || forced == SPINQ_GEMM_SPLITK) &&
+      w4a4_gemv_fits(M, K))
+    return SPINQ_GEMM_GEMV;
+  if (forced == SPINQ_GEMM_TILE128 || forced == SPINQ_GEMM_TILE256) return forced;
+  // (a forced GEMV that does not fit falls through to the cost model)
+  if (forced == SPINQ_GEMM_PAIR && M > 128 && w4a4_gemm_pair_clusters() > 0) return SPINQ_GEMM_PAIR;
+  return choose_prefill(M, N, K, true).kind;
 }
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
@@ -918,24 +989,111 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   return launch_mt<1>(a, stream);
 }
 
-int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K) {
-  if (M <= 0 || N <= 0 || M > kDecodeMaxM || w4a4_gemv_fits(M, K)) return 0;
-  return M * N * 4 + ((N + 127) / 128) * 4;
+// How spinq_w4a4_gemm_splitk serves 5..256 tokens, from a cost model fitted
+// on GB300 over K x N in {3072 x 8192, 8192 x 3072, 4096 x 14336,
+// 14336 x 4096}, 8..256 tokens and 1..32 slices (microseconds, within 5% on
+// average): the split-K kernel with `nsplit` K slices per 128-channel tile,
+// or the prefill kernels.  One CTA (a tile's K slice) takes
+//   ceil(ks / nsplit) (0.322 + 0.0018 MN)    its 128-deep K steps (MN = tokens
+//                                            rounded up to 16 .. 256: the
+//                                            unpack and MMA of the tokens' tile)
+//   + 3.92 + 0.0375 M                        start-up, epilogue
+//   + (nsplit > 1) (1.83 + 0.089 M)          the partial sums' atomics, the
+//                                            tile counter and the last
+//                                            slice's pass over the workspace
+// and the grid runs in ceil(tiles nsplit / resident CTAs) waves.  The
+// prefill kernels take their own model + 3 (its constants were fitted on
+// large shapes).
+// The K slices range over [ns_lo, ns_hi] (both 1 when the caller has no room
+// for the partial sums); `allow_prefill` false keeps the split-K kernel.
+namespace {
+
+struct DecodePlan {
+  bool prefill;
+  int nsplit;
+};
+
+DecodePlan plan_decode(int64_t M, int64_t N, int64_t K, int ns_lo, int ns_hi, bool allow_prefill) {
+  int mn = 16;
+  const int per_sm = dec_per_sm_for(M, &mn);
+  const double slots = (double)device_sm_count() * per_sm;
+  const int ks = (int)(K / 128), ntiles = (int)((N + 127) / 128);
+  const double tk = 0.322 + 0.0018 * mn;
+  double best = 1e30;
+  int best_ns = 1;
+  for (int ns = ns_lo; ns <= ns_hi; ++ns) {
+    const double waves = std::ceil((double)ntiles * ns / slots);
+    const double cta = std::ceil((double)ks / ns) * tk + 3.92 + 0.0375 * (double)M +
+                       (ns > 1 ? 1.83 + 0.089 * (double)M : 0.0);
+    const double t = waves * cta;
+    if (t < best) {
+      best = t;
+      best_ns = ns;
+    }
+  }
+  if (allow_prefill && choose_prefill(M, N, K, true).us + 3.0 < best) return {true, 0};
+  return {false, best_ns};
 }
 
-cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, cudaStream_t stream) {
+constexpr int kMaxSplit = 64;
+
+int64_t split_workspace_bytes(int64_t M, int64_t N) { return M * N * 4 + ((N + 127) / 128) * 4; }
+
+// The plan of the split-K entry point for 1 <= M <= kDecodeMaxM under the
+// current selection; `room`: the caller's workspace holds the partial sums.
+DecodePlan plan_splitk_entry(int64_t M, int64_t N, int64_t K, bool room) {
+  const int ks = (int)(K / 128);
+  const int fixed = g_split_k.load(std::memory_order_relaxed);
+  int lo = 1, hi = std::min(ks, kMaxSplit);
+  if (fixed > 0) lo = hi = std::min(fixed, ks);
+  if (!room) lo = hi = 1;
+  // a forced split-K kernel runs whatever the model predicts for the others
+  return plan_decode(M, N, K, lo, hi, g_gemm_kernel.load(std::memory_order_relaxed) != SPINQ_GEMM_SPLITK);
+}
+
+bool gemv_serves(int64_t M, int64_t K) {
+  return g_gemm_kernel.load(std::memory_order_relaxed) != SPINQ_GEMM_SPLITK && w4a4_gemv_fits(M, K);
+}
+
+}  // namespace
+
+int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K) {
+  // only split K slices sum through the workspace
+  if (M <= 0 || N <= 0 || M > kDecodeMaxM || gemv_serves(M, K)) return 0;
+  const DecodePlan p = plan_splitk_entry(M, N, K, true);
+  if (p.prefill || p.nsplit <= 1) return 0;
+  return split_workspace_bytes(M, N);
+}
+
+int plan_w4a4_gemm_splitk(int64_t M, int64_t N, int64_t K, int* nsplit) {
+  *nsplit = 0;
+  if (M > kDecodeMaxM) return plan_w4a4_gemm(M, N, K);
+  if (gemv_serves(M, K)) return SPINQ_GEMM_GEMV;
+  const DecodePlan p = plan_splitk_entry(M, N, K, true);
+  if (p.prefill) return plan_w4a4_gemm(M, N, K);
+  *nsplit = p.nsplit;
+  return SPINQ_GEMM_SPLITK;
+}
+
+cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, int64_t workspace_bytes,
+                                    cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
   if (a.M > kDecodeMaxM) return launch_w4a4_gemm(a, stream);
-  bool handled = false;
-  const cudaError_t eg = launch_w4a4_gemv(a, stream, &handled);
-  if (eg != cudaSuccess || handled) return eg;
-  float* ws_acc = static_cast<float*>(workspace);
-  int* ws_cnt = reinterpret_cast<int*>(static_cast<char*>(workspace) + a.M * a.N * 4);
-  if (a.M <= 16) return launch_dec_mn<16>(a, ws_acc, ws_cnt, stream);
-  if (a.M <= 32) return launch_dec_mn<32>(a, ws_acc, ws_cnt, stream);
-  if (a.M <= 64) return launch_dec_mn<64>(a, ws_acc, ws_cnt, stream);
-  if (a.M <= 128) return launch_dec_mn<128>(a, ws_acc, ws_cnt, stream);
-  return launch_dec_mn<256>(a, ws_acc, ws_cnt, stream);
+  if (gemv_serves(a.M, a.K)) {
+    bool handled = false;
+    const cudaError_t eg = launch_w4a4_gemv(a, stream, &handled);
+    if (eg != cudaSuccess || handled) return eg;
+  }
+  const bool room = workspace != nullptr && workspace_bytes >= split_workspace_bytes(a.M, a.N);
+  const DecodePlan p = plan_splitk_entry(a.M, a.N, a.K, room);
+  if (p.prefill) return launch_w4a4_gemm(a, stream);
+  float* ws_acc = p.nsplit > 1 ? static_cast<float*>(workspace) : nullptr;
+  int* ws_cnt = ws_acc == nullptr ? nullptr : reinterpret_cast<int*>(static_cast<char*>(workspace) + a.M * a.N * 4);
+  if (a.M <= 16) return launch_dec_mn<16>(a, ws_acc, ws_cnt, p.nsplit, stream);
+  if (a.M <= 32) return launch_dec_mn<32>(a, ws_acc, ws_cnt, p.nsplit, stream);
+  if (a.M <= 64) return launch_dec_mn<64>(a, ws_acc, ws_cnt, p.nsplit, stream);
+  if (a.M <= 128) return launch_dec_mn<128>(a, ws_acc, ws_cnt, p.nsplit, stream);
+  return launch_dec_mn<256>(a, ws_acc, ws_cnt, p.nsplit, stream);
 }
 
 int* device_status_word() {

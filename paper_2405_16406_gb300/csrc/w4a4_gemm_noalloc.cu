@@ -64,9 +64,11 @@ extern "C" spinq_status spinq_w4a4_gemm_noalloc(const uint8_t* a_codes, const fl
       !is_aligned16(w_rowsum) || (acc_out && !is_aligned16(acc_out)))
     return SPINQ_EINVAL;
   if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
-  const int64_t need = spinq::w4a4_gemm_workspace_bytes(M, N, K);
-  if (need > kNoAllocScratchBytes) return SPINQ_EUNSUPPORTED;   // scratch too small for M x N
   if (M == 0 || N == 0) return SPINQ_OK;
+  // a split whose partial sums do not fit the scratch is not taken: the
+  // tiles then keep their whole K range
+  int64_t need = spinq::w4a4_gemm_workspace_bytes(M, N, K);
+  if (need > kNoAllocScratchBytes) need = 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void* ws = nullptr;
   if (need > 0) {
@@ -76,7 +78,7 @@ extern "C" spinq_status spinq_w4a4_gemm_noalloc(const uint8_t* a_codes, const fl
     if (cudaMemsetAsync(ws, 0, (size_t)need, s) != cudaSuccess) return SPINQ_ECUDA;
   }
   const spinq::GemmArgs g{a_codes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y_f16, acc_out};
-  const cudaError_t e = spinq::launch_w4a4_gemm_splitk(g, ws, s);
+  const cudaError_t e = spinq::launch_w4a4_gemm_splitk(g, ws, need, s);
   if (e == cudaSuccess) return SPINQ_OK;
   return e == cudaErrorNotSupported ? SPINQ_EUNSUPPORTED : SPINQ_ECUDA;
 }

@@ -30,12 +30,13 @@ _lib = ctypes.CDLL(LIB_PATH)
 
 SPINQ_OK, SPINQ_EINVAL, SPINQ_EUNSUPPORTED, SPINQ_ECUDA, SPINQ_ETIMEOUT = range(5)
 SPINQ_PER_TOKEN, SPINQ_PER_CHANNEL, SPINQ_PER_GROUP = range(3)
-SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR, SPINQ_GEMM_GEMV = range(5)
+SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR, SPINQ_GEMM_GEMV, SPINQ_GEMM_SPLITK = range(6)
 
 EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",
     "spinq_status_string", "spinq_device_status", "spinq_version", "spinq_w4a4_gemm_workspace_bytes",
-    "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel", "spinq_w4a4_gemm_plan",
+    "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel", "spinq_gemm_split_k",
+    "spinq_w4a4_gemm_plan", "spinq_w4a4_gemm_splitk_plan",
 )
 
 
@@ -79,8 +80,12 @@ _lib.spinq_w4a4_gemm_noalloc.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_noalloc.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
 _lib.spinq_gemm_select_kernel.restype = ctypes.c_int
 _lib.spinq_gemm_select_kernel.argtypes = [ctypes.c_int]
+_lib.spinq_gemm_split_k.restype = ctypes.c_int
+_lib.spinq_gemm_split_k.argtypes = [ctypes.c_int]
 _lib.spinq_w4a4_gemm_plan.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_plan.argtypes = [_I64, _I64, _I64]
+_lib.spinq_w4a4_gemm_splitk_plan.restype = ctypes.c_int
+_lib.spinq_w4a4_gemm_splitk_plan.argtypes = [_I64, _I64, _I64, ctypes.POINTER(ctypes.c_int)]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
 _lib.spinq_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
                                        ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
@@ -132,8 +137,19 @@ def spinq_gemm_select_kernel(kernel: int) -> int:
     return int(_lib.spinq_gemm_select_kernel(kernel))
 
 
+def spinq_gemm_split_k(n: int) -> int:
+    return int(_lib.spinq_gemm_split_k(n))
+
+
 def spinq_w4a4_gemm_plan(M: int, N: int, K: int) -> int:
     return int(_lib.spinq_w4a4_gemm_plan(M, N, K))
+
+
+def spinq_w4a4_gemm_splitk_plan(M: int, N: int, K: int) -> tuple:
+    """(kernel, K slices) of spinq_w4a4_gemm_splitk for an M x N x K call."""
+    ns = ctypes.c_int(0)
+    kind = int(_lib.spinq_w4a4_gemm_splitk_plan(M, N, K, ctypes.byref(ns)))
+    return kind, int(ns.value)
 
 
 def spinq_status_string(st: int) -> str:

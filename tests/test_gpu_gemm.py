@@ -303,13 +303,35 @@ def run_splitk(S, ac, al, be, wc, ws_, workspace=None):
     return y.cpu().numpy(), acc.cpu().numpy()
 
 
-@pytest.mark.parametrize("M,N,K", [(1, 16, 128), (3, 48, 256), (16, 512, 1024), (17, 272, 384), (33, 1024, 512),
-                                   (64, 256, 128), (100, 384, 640), (128, 3072, 1024), (200, 256, 256),
-                                   (256, 512, 512), (300, 256, 256)])
+@pytest.fixture
+def splitk_route(S, request):
+    """Routes of the split-K entry point: the cost model's choice ("auto"),
+    the split-K kernel with the slices the model picks ("sliced"), and the
+    split-K kernel with the whole K range per tile ("whole_k")."""
+    route = request.param
+    prev_kind = S.spinq_gemm_select_kernel(0 if route == "auto" else S.SPINQ_GEMM_SPLITK)
+    prev_cap = S.spinq_gemm_split_k(1 if route == "whole_k" else 0)
+    assert prev_kind >= 0 and prev_cap >= 0
+    yield route
+    S.spinq_gemm_select_kernel(prev_kind)
+    S.spinq_gemm_split_k(prev_cap)
+
+
+SPLITK_SHAPES = [(1, 16, 128), (3, 48, 256), (16, 512, 1024), (17, 272, 384), (33, 1024, 512),
+                 (64, 256, 128), (100, 384, 640), (128, 3072, 1024), (200, 256, 256),
+                 (256, 512, 512), (300, 256, 256)]
+
+
+@pytest.mark.parametrize("splitk_route", ["auto", "sliced", "whole_k"], indirect=True)
+@pytest.mark.parametrize("M,N,K", SPLITK_SHAPES)
 @pytest.mark.parametrize("symmetric", [True, False])
-def test_splitk_random_codes_exact(S, M, N, K, symmetric):
+def test_splitk_random_codes_exact(S, splitk_route, M, N, K, symmetric):
     rng = np.random.default_rng(M * 13 + N + K + symmetric)
     ac, al, be, wc, ws_ = random_codes(rng, M, N, K, symmetric)
+    kind, nsplit = S.spinq_w4a4_gemm_splitk_plan(M, N, K)
+    if splitk_route != "auto" and M <= 256:
+        assert kind == S.SPINQ_GEMM_SPLITK
+        assert nsplit == 1 if splitk_route == "whole_k" else 1 <= nsplit <= min(64, K // 128)
     y, acc = run_splitk(S, ac, al, be, wc, ws_)
     ref = oracle_full(ac, al, be, wc, ws_)
     assert np.array_equal(acc, ref.acc)
@@ -317,13 +339,55 @@ def test_splitk_random_codes_exact(S, M, N, K, symmetric):
     assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
 
 
-def test_splitk_no_workspace_for_the_gemv_path(S):
+def test_splitk_plan_covers_every_route(S):
+    """Under the default selection the split-K entry point's shapes above,
+    with the decode configurations, reach the GEMV kernel, the split-K kernel
+    with and without K slices, and the prefill kernels."""
+    shapes = SPLITK_SHAPES + [(1, 8192, 3072), (16, 8192, 3072), (64, 8192, 3072), (128, 8192, 3072),
+                              (128, 3072, 8192), (256, 8192, 3072)]
+    routes = set()
+    for M, N, K in shapes:
+        kind, nsplit = S.spinq_w4a4_gemm_splitk_plan(M, N, K)
+        assert kind in (1, 2, 3, 4, 5)
+        assert (nsplit >= 1) == (kind == S.SPINQ_GEMM_SPLITK)
+        routes.add("sliced" if nsplit > 1 else "whole_k" if nsplit == 1 else kind)
+        # the workspace exists exactly for K slices
+        assert (S.spinq_w4a4_gemm_workspace_bytes(M, N, K) > 0) == (nsplit > 1)
+    assert {"sliced", "whole_k", 4}.issubset(routes)
+    assert routes & {1, 2, 3}
+    assert S.spinq_w4a4_gemm_splitk_plan(16, 100, 1024)[0] == -1    # N not a multiple of 16
+    assert S.spinq_w4a4_gemm_splitk_plan(16, 128, 1000)[0] == -1    # K not a multiple of 128
+
+
+def test_splitk_workspace_follows_the_plan(S):
     for M in (1, 3, 4):
         assert S.spinq_w4a4_gemm_workspace_bytes(M, 8192, 3072) == 0
         assert S.gemm_workspace(M, 8192, 3072) is None
-    assert S.spinq_w4a4_gemm_workspace_bytes(5, 8192, 3072) > 0
-    # the tokens no longer fit in shared memory: split-K with a workspace
-    assert S.spinq_w4a4_gemm_workspace_bytes(4, 8192, 65536) > 0
+        assert S.spinq_w4a4_gemm_splitk_plan(M, 8192, 3072) == (S.SPINQ_GEMM_GEMV, 0)
+    # few tokens, narrow outputs, long K: every SM streams a slice of the weights
+    kind, nsplit = S.spinq_w4a4_gemm_splitk_plan(16, 3072, 8192)
+    assert kind == S.SPINQ_GEMM_SPLITK and nsplit > 1
+    assert S.spinq_w4a4_gemm_workspace_bytes(16, 3072, 8192) == 16 * 3072 * 4 + 24 * 4
+    # the tokens no longer fit in the GEMV kernel's shared memory
+    assert S.spinq_w4a4_gemm_splitk_plan(4, 8192, 65536)[0] == S.SPINQ_GEMM_SPLITK
+    # no slices, no workspace
+    prev = S.spinq_gemm_split_k(1)
+    try:
+        assert S.spinq_w4a4_gemm_workspace_bytes(16, 3072, 8192) == 0
+        assert S.spinq_w4a4_gemm_splitk_plan(16, 3072, 8192) == (S.SPINQ_GEMM_SPLITK, 1)
+    finally:
+        S.spinq_gemm_split_k(prev)
+    assert S.spinq_gemm_split_k(65) == -1 and S.spinq_gemm_split_k(-1) == -1
+    # a fixed count, at most one slice per 128-deep K step
+    prev = S.spinq_gemm_split_k(7)
+    prev_kind = S.spinq_gemm_select_kernel(S.SPINQ_GEMM_SPLITK)
+    try:
+        assert S.spinq_w4a4_gemm_splitk_plan(16, 3072, 8192) == (S.SPINQ_GEMM_SPLITK, 7)
+        assert S.spinq_w4a4_gemm_splitk_plan(16, 3072, 512) == (S.SPINQ_GEMM_SPLITK, 4)
+        assert S.spinq_w4a4_gemm_splitk_plan(2, 3072, 512) == (S.SPINQ_GEMM_SPLITK, 4)
+    finally:
+        S.spinq_gemm_split_k(prev)
+        S.spinq_gemm_select_kernel(prev_kind)
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 16, 128), (2, 48, 256), (3, 272, 384), (4, 512, 1024), (1, 1040, 4096),
@@ -367,8 +431,9 @@ def test_gemv_extreme_codes_long_k(S):
 
 def test_splitk_workspace_reused_and_left_zero(S):
     rng = np.random.default_rng(21)
-    M, N, K = 100, 1024, 2048
+    M, N, K = 16, 1024, 2048
     ws = S.gemm_workspace(M, N, K)
+    assert ws is not None   # the plan slices K here
     for rep in range(3):
         ac, al, be, wc, ws_ = random_codes(rng, M, N, K, rep % 2 == 0)
         y, acc = run_splitk(S, ac, al, be, wc, ws_, workspace=ws)
@@ -376,19 +441,28 @@ def test_splitk_workspace_reused_and_left_zero(S):
         assert int(torch.count_nonzero(ws)) == 0
 
 
-def test_splitk_extreme_codes_long_k(S):
-    M, N, K = 16, 256, 65536
+@pytest.mark.parametrize("splitk_route", ["sliced", "whole_k"], indirect=True)
+@pytest.mark.parametrize("M", [16, 256])
+def test_splitk_extreme_codes_long_k(S, splitk_route, M):
+    """|acc| up to 64 K = 2^22 stays exact through the fp32 accumulator, the
+    slices' partial sums and the unsliced epilogue."""
+    N, K = 256, 65536
     for aval, wval in ((7, 7), (-8, -8), (7, -8)):
         ac = np.full((M, K), aval, dtype=np.int32)
         wc = np.full((N, K), wval, dtype=np.int32)
         al, ws_ = np.full(M, 0.5), np.full(N, 0.25)
         y, acc = run_splitk(S, ac, al, None, wc, ws_)
-        assert np.array_equal(acc, oracle_full(ac, al, None, wc, ws_).acc)
+        # constant codes: every output's sum is K a w
+        assert np.array_equal(acc, np.full((M, N), K * aval * wval, dtype=np.int32))
+        if M <= 16:
+            assert np.array_equal(acc, oracle_full(ac, al, None, wc, ws_).acc)
 
 
 @pytest.mark.parametrize("name,M,K,N,symmetric", [("l32_up_M1", 1, 3072, 8192, False),
                                                   ("l32_up_M16", 16, 3072, 8192, False),
-                                                  ("l32_down_M128", 128, 8192, 3072, False)])
+                                                  ("l32_up_M64", 64, 3072, 8192, False),
+                                                  ("l32_down_M128", 128, 8192, 3072, False),
+                                                  ("l32_down_M256", 256, 8192, 3072, False)])
 def test_splitk_decode_configs_full(S, name, M, K, N, symmetric):
     rng = np.random.default_rng(len(name) + M)
     ac, al, be, wc, ws_ = random_codes(rng, M, N, K, symmetric)

@@ -4,8 +4,8 @@ It serves callers that cannot allocate device memory where they run the
 layer: its split-K workspace is a fixed array inside the library instead of a
 buffer the caller passes in.  This file checks, through the C ABI, that two
 calls in a row give the same result as spinq_w4a4_gemm on the same inputs
-(integer accumulator exact, fp16 output within the tests' tolerance), and
-that a request larger than the fixed array is refused.  It runs last and does
+(integer accumulator exact, fp16 output within the tests' tolerance), also
+for a request whose K slices would not fit the fixed array.  It runs last and does
 not depend on any other test.
 """
 import ctypes
@@ -62,12 +62,27 @@ def test_noalloc_matches_gemm_on_two_calls_in_a_row():
     assert S.spinq_device_status()[0] == S.SPINQ_OK
 
 
-def test_noalloc_refuses_requests_beyond_its_scratch():
+def test_noalloc_serves_requests_beyond_its_scratch_unsliced():
+    """A call whose K slices would need more partial sums than the 8 MiB
+    scratch holds keeps the whole K range per tile and matches
+    spinq_w4a4_gemm (the split-K kernel and two K slices are forced, so that
+    the plan needs the workspace for this shape)."""
     from paper_2405_16406_gb300 import spinq as S
     gen = torch.Generator(device="cuda")
     gen.manual_seed(1)
-    M, N, K = 256, 16384, 128          # workspace 16 MiB + counters > 8 MiB
-    assert S.spinq_w4a4_gemm_workspace_bytes(M, N, K) > 8 << 20
+    M, N, K = 256, 9728, 8192          # partial sums of 9.5 MiB
     args = _inputs(gen, M, N, K, True)
-    st, _, _ = _call(S.spinq_w4a4_gemm_noalloc, args, M, N, K)
-    assert st == S.SPINQ_EUNSUPPORTED
+    st_ref, y_ref, acc_ref = _call(S.spinq_w4a4_gemm, args, M, N, K)
+    prev = S.spinq_gemm_select_kernel(S.SPINQ_GEMM_SPLITK)
+    prev_split = S.spinq_gemm_split_k(2)
+    try:
+        assert S.spinq_w4a4_gemm_workspace_bytes(M, N, K) > 8 << 20
+        st, y, acc = _call(S.spinq_w4a4_gemm_noalloc, args, M, N, K)
+    finally:
+        S.spinq_gemm_select_kernel(prev)
+        S.spinq_gemm_split_k(prev_split)
+    torch.cuda.synchronize()
+    assert st_ref == S.SPINQ_OK and st == S.SPINQ_OK
+    assert torch.equal(acc, acc_ref)
+    assert (y.float() - y_ref.float()).norm() <= 1e-2 * y_ref.float().norm()
+    assert S.spinq_device_status()[0] == S.SPINQ_OK
