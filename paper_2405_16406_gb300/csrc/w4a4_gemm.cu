@@ -27,7 +27,11 @@
 //                per stage into the accumulator buffer of the current tile.
 //   warps 2..5   epilogue, one TMEM lane quadrant each (warp % 4): tcgen05.ld
 //                of a finished accumulator, integer recovery, scales, fp16
-//                stores; runs while the MMA fills the other buffer.
+//                stores.  128-row tiles: runs while the MMA fills the other
+//                accumulator buffer.  256-row tiles (one accumulator): the
+//                unpack warps share it (five warps per quadrant) and stage
+//                y in the then idle operand ring, so that every store
+//                instruction writes whole 128-byte row pieces.
 //   warps 6..21  unpack the packed tiles into the 128-byte-swizzled K-major
 //                E4M3 operand tiles (ring of NU stages) and count sum_k u_a;
 //                two groups of 8 warps take alternate K stages so that one
@@ -89,6 +93,18 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   }
 }
 
+// bar.sync of the four epilogue warps (named barrier 1) whose result is the
+// OR of `pred` over them: a decision every epilogue warp takes alike.
+__device__ __forceinline__ bool epi_bar_or(bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, %2, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(kEpiWarps * 32)
+      : "memory");
+  return r != 0;
+}
+
 __device__ __forceinline__ uint32_t swz_off(int r, int chunk) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4));
 }
@@ -121,25 +137,189 @@ struct Cfg {
   static constexpr uint32_t pB = pA + NP * BMT * 64;
   static constexpr uint32_t bars = pB + NP * BN * 64;
   // full_p[NP] empty_p[NP] full_u[NU] empty_u[NU] acc_full[NACC] acc_empty[NACC]
-  // rs_full[2] rs_empty[2] drain
-  static constexpr int nbars = 2 * NP + 2 * NU + 2 * NACC + 5;
+  // rs_full[2] rs_empty[2] drain cols_full[2] stg_free
+  static constexpr int nbars = 2 * NP + 2 * NU + 2 * NACC + 8;
   static constexpr uint32_t misc = bars + nbars * 8;   // tmem slot, abort flag
   static constexpr uint32_t rs_a = (misc + 16 + 15) & ~15u;
-  static constexpr uint32_t cols = rs_a + 2 * kUnpackGroups * BMT * 4;   // s_n and (float) rowsum_n
-  // 256-row tiles: the epilogue stages each warp's 32 x 32 block of y in
-  // shared memory (64-byte rows, 64-byte swizzle, two buffers per warp) and
-  // writes it with a TMA store
-  static constexpr bool TMA_Y = MT == 2;
-  static constexpr uint32_t ys = (cols + 2 * BN * 4 + 1023) & ~1023u;
-  static constexpr uint32_t total = TMA_Y ? ys + kEpiWarps * 2 * 2048 : cols + 2 * BN * 4;
+  // [tile parity][s_n, (float) rowsum_n][BN]: the column constants of a tile
+  static constexpr uint32_t cols = rs_a + 2 * kUnpackGroups * BMT * 4;
+  static constexpr uint32_t total = cols + 2 * 2 * BN * 4;
   static constexpr size_t dyn_bytes = total + 1024;
+  // warps that share the epilogue of a 256-row tile per TMEM lane quadrant:
+  // its epilogue warp and the four unpack warps of that quadrant.  The unpack
+  // warps take their share before they unpack the next tile, so the operand
+  // stages are free meanwhile and hold the warps' y staging blocks
+  // (EPI_STAGE bytes each).
+  static constexpr int EPI_PARTS = MT == 2 ? 1 + kUnpackGroups * kUnpackWarps / 4 : 1;
+  static constexpr uint32_t EPI_STAGE = 32 * 128;
+  static_assert(MT == 1 || kEpiWarps * EPI_PARTS * EPI_STAGE <= 2 * NU * BMT * 128, "staging fits the operand ring");
 };
+
+// One warp's share of the epilogue of a 256 x 256 tile.  The tile's rows
+// q * 32 + lane (accumulator 0) and 128 + q * 32 + lane (accumulator 1) of
+// TMEM lane quadrant q form 8 blocks of 32 rows x 64 columns; this warp takes
+// blocks g = part, part + nparts, ...  A block is read from tensor memory in
+// four 16-column loads (a lane holds its row), turned into y with the
+// epilogue formula on packed fp32 pairs and written as fp16 to the warp's
+// 4 KB staging block in shared memory (row r at r * 128 bytes, 16-byte chunk
+// c at (c ^ (r % 8)) * 16: conflict-free both ways); it is then read back
+// with 8 lanes per row and stored with 16-byte stores, so that each store
+// instruction writes 4 rows x 128 contiguous bytes of y instead of 32
+// separate 16-byte pieces.  The accumulator is released (acc_empty) after
+// the warp's last tensor-memory load, the staging block (stg_free) after its
+// last read.
+//   y = s_n (alpha (S - 8 rs_a - 8 rw_n) + beta' rw_n), S = acc * 2^18,
+//   evaluated as y = s_n * fma(alpha * 2^18, acc, c + d * rw_n) with
+//   c = -8 alpha rs_a and d = beta' - 8 alpha (the roundings of the other
+//   kernels, so that every kernel gives the same bits).
+template <bool ASYM, bool ACC_OUT>
+__device__ __forceinline__ void epi256_share(const GemmArgs& args, uint32_t tq, int q, int lane, int part,
+                                             int nparts, int64_t m_tile0, int64_t n0, const float* col_s,
+                                             const float* col_r, int rsa0, int rsa1, uint32_t stage,
+                                             uint64_t* acc_empty, uint64_t* stg_free) {
+  constexpr int NBLK = 2 * (BN / 64);
+  // per-row constants of the two accumulators, kept in scalars: the block
+  // loop selects them with a runtime accumulator index
+  F2 as2_0, cm2_0, dm2_0, as2_1, cm2_1, dm2_1;
+  const int64_t m_0 = m_tile0 + q * 32 + lane, m_1 = m_0 + 128;
+#pragma unroll
+  for (int mt = 0; mt < 2; ++mt) {
+    const int64_t m = mt ? m_1 : m_0;
+    float alpha = 0.f, bp = 0.f;
+    if (m < args.M) {
+      alpha = __ldg(args.a_scale + m);
+      if (ASYM) bp = __ldg(args.a_zero + m) + 8.f * alpha;
+    }
+    const float as = alpha * 262144.0f, cm = -8.f * alpha * (float)(mt ? rsa1 : rsa0), dm = bp - 8.f * alpha;
+    (mt ? as2_1 : as2_0) = f2_make(as, as);
+    (mt ? cm2_1 : cm2_0) = f2_make(cm, cm);
+    (mt ? dm2_1 : dm2_0) = f2_make(dm, dm);
+  }
+  const uint32_t srow = stage + (uint32_t)lane * 128;
+#pragma unroll 1
+  for (int g = part; g < NBLK; g += nparts) {
+    const int mt = g / (BN / 64), cb = g % (BN / 64);
+    const int64_t m = mt ? m_1 : m_0;
+    const F2 as2 = mt ? as2_1 : as2_0, cm2 = mt ? cm2_1 : cm2_0, dm2 = mt ? dm2_1 : dm2_0;
+    const int rsam = mt ? rsa1 : rsa0;
+#pragma unroll 1
+    for (int c2 = 0; c2 < 2; ++c2) {
+      // two 16-column loads in flight per wait
+      uint32_t cur[32];
+      tmem_ld_32x32b_x16(tq + (uint32_t)(mt * BN + cb * 64 + c2 * 32), cur);
+      tmem_ld_32x32b_x16(tq + (uint32_t)(mt * BN + cb * 64 + c2 * 32 + 16), cur + 16);
+      // (one wait covers both loads; each call ties its registers to the wait)
+      tmem_ld_wait(cur);
+      tmem_ld_wait(cur + 16);
+#pragma unroll
+      for (int g8 = 0; g8 < 4; ++g8) {
+        const int j0 = cb * 64 + c2 * 32 + g8 * 8;
+        const ulonglong2 S0 = *reinterpret_cast<const ulonglong2*>(col_s + j0);
+        const ulonglong2 S1 = *reinterpret_cast<const ulonglong2*>(col_s + j0 + 4);
+        const ulonglong2 R0 = *reinterpret_cast<const ulonglong2*>(col_r + j0);
+        const ulonglong2 R1 = *reinterpret_cast<const ulonglong2*>(col_r + j0 + 4);
+        uint32_t pw[4];
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          F2 sc2, rw2;
+          sc2.u = p == 0 ? S0.x : p == 1 ? S0.y : p == 2 ? S1.x : S1.y;
+          rw2.u = p == 0 ? R0.x : p == 1 ? R0.y : p == 2 ? R1.x : R1.y;
+          const F2 acc2 = f2_from_bits(cur[g8 * 8 + 2 * p], cur[g8 * 8 + 2 * p + 1]);
+          const F2 y2 = f2_mul(sc2, f2_fma(as2, acc2, f2_fma(dm2, rw2, cm2)));
+          float lo, hi;
+          f2_split(y2, lo, hi);
+          pw[p] = pack_half2_bits(lo, hi);
+        }
+        const int c = c2 * 4 + g8;
+        sts128(srow + (uint32_t)((c ^ (lane & 7)) << 4), make_uint4(pw[0], pw[1], pw[2], pw[3]));
+        if (ACC_OUT) {
+          // the integer accumulator (a debugging output): straight from the lane's row
+          const int64_t n = n0 + j0;
+          if (m < args.M && n < args.N) {
+            int accs[8];
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+              const unsigned long long r2 = p == 0 ? R0.x : p == 1 ? R0.y : p == 2 ? R1.x : R1.y;
+#pragma unroll
+              for (int h = 0; h < 2; ++h) {
+                const float rwf = __uint_as_float((uint32_t)(r2 >> (32 * h)));
+                accs[2 * p + h] =
+                    __float2int_rn(__uint_as_float(cur[g8 * 8 + 2 * p + h]) * 262144.0f) - 8 * rsam - 8 * (int)rwf;
+              }
+            }
+            int4* ap = reinterpret_cast<int4*>(args.acc_out + m * args.N + n);
+            ap[0] = make_int4(accs[0], accs[1], accs[2], accs[3]);
+            ap[1] = make_int4(accs[4], accs[5], accs[6], accs[7]);
+          }
+        }
+      }
+    }
+    if (g + nparts >= NBLK) {
+      // the warp's last tensor-memory load has completed
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty);
+    }
+    __syncwarp();   // the block's rows are in shared memory
+    // lane l stores 16-byte chunk l % 8 of rows 4 i + l / 8 (N is a multiple
+    // of 16: a chunk of 8 columns is wholly inside y or outside it)
+    const int c = lane & 7;
+    const int64_t n = n0 + cb * 64 + c * 8;
+    const int64_t mrow0 = m_tile0 + mt * 128 + q * 32;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int r = 4 * i + (lane >> 3);
+      const uint4 v = lds128(stage + (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)));
+      if (mrow0 + r < args.M && n < args.N)
+        *reinterpret_cast<uint4*>(reinterpret_cast<__half*>(args.y) + (mrow0 + r) * args.N + n) = v;
+    }
+    __syncwarp();   // every lane has read the block before it is overwritten
+  }
+  if (part >= NBLK) {
+    // (no block for this warp: nothing to wait for)
+    __syncwarp();
+    if (lane == 0) mbar_arrive(acc_empty);
+  }
+  __syncwarp();
+  if (lane == 0) mbar_arrive(stg_free);   // release: orders the block reads above before it
+}
+
+// An unpack warp's share of the epilogue of 256-row tile `plt` (local index;
+// global tile index `ptile`): waits for the accumulator, the activation row
+// sums and the column constants of that tile, then runs its share.  False
+// when a wait gave up (the share is skipped; the accumulator and staging
+// barriers are then left to the bounded waits of the other roles).
+template <bool ASYM, bool ACC_OUT>
+__device__ __forceinline__ bool unpack_epi_share(const GemmArgs& args, uint32_t tmem, int warp, int lane, int plt,
+                                                 int ptile, int m_tiles, uint64_t* acc_full, uint64_t* acc_empty,
+                                                 uint64_t* rs_full, uint64_t* cols_full, uint64_t* stg_free,
+                                                 const int* rs_a, const float* cols, uint32_t stage_base,
+                                                 volatile int* abort_flag) {
+  constexpr int BMT = 256;
+  const int rb = plt & 1;
+  bool ok = wait_or_abort(&acc_full[0], plt & 1, abort_flag, 10);
+  ok = ok && wait_or_abort(&rs_full[rb], (plt >> 1) & 1, abort_flag, 10);
+  ok = ok && wait_or_abort(&cols_full[rb], (plt >> 1) & 1, abort_flag, 10);
+  // warp-uniform: the tensor-memory loads are warp-collective
+  if (!__all_sync(0xffffffffu, ok)) return false;
+  tc_fence_after();
+  const int q = warp & 3, part = 1 + (warp - kFirstUnpackWarp) / 4;
+  const int r0 = q * 32 + lane, r1 = 128 + q * 32 + lane;
+  const int rsa0 = rs_a[(rb * kUnpackGroups) * BMT + r0] + rs_a[(rb * kUnpackGroups + 1) * BMT + r0];
+  const int rsa1 = rs_a[(rb * kUnpackGroups) * BMT + r1] + rs_a[(rb * kUnpackGroups + 1) * BMT + r1];
+  const float* col_s = cols + rb * 2 * BN;
+  constexpr int NPARTS = Cfg<2>::EPI_PARTS;
+  epi256_share<ASYM, ACC_OUT>(args, tmem + ((uint32_t)(q * 32) << 16), q, lane, part, NPARTS,
+                              (int64_t)(ptile % m_tiles) * BMT, (int64_t)(ptile / m_tiles) * BN, col_s, col_s + BN,
+                              rsa0, rsa1, stage_base + (uint32_t)((q * NPARTS + part) * Cfg<2>::EPI_STAGE),
+                              &acc_empty[0], stg_free);
+  return true;
+}
 
 template <int MT, bool ASYM, bool ACC_OUT>
 __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const __grid_constant__ CUtensorMap tmY, GemmArgs args, int num_k, int m_tiles,
-                     int num_tiles) {
+                     GemmArgs args, int num_k, int m_tiles, int num_tiles) {
   using L = Cfg<MT>;
   constexpr int BMT = L::BMT, NP = L::NP, NU = L::NU, NACC = L::NACC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -156,12 +336,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* rs_full = acc_empty + NACC;
   uint64_t* rs_empty = rs_full + 2;
   uint64_t* drain = rs_empty + 2;
+  uint64_t* cols_full = drain + 1;   // [tile parity]: the tile's column constants are staged
+  uint64_t* stg_free = cols_full + 2;   // 256-row tiles: the epilogue's staging blocks are read out
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + L::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + L::misc + 4);
   volatile uint32_t* scratch = reinterpret_cast<volatile uint32_t*>(base + L::misc + 8);   // see wait_loaded
   int* rs_a = reinterpret_cast<int*>(base + L::rs_a);   // [2][groups][BMT]
-  float* col_s = reinterpret_cast<float*>(base + L::cols);   // [BN] w_scale of the tile's columns
-  float* col_r = col_s + BN;                                  // [BN] w_rowsum as float
+  // column constants of tile lt at parity lt & 1: w_scale, then w_rowsum as float
+  float* cols = reinterpret_cast<float*>(base + L::cols);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -176,13 +358,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < NACC; ++i) {
       mbar_init(&acc_full[i], 1);
-      mbar_init(&acc_empty[i], kEpiWarps);
+      mbar_init(&acc_empty[i], kEpiWarps * L::EPI_PARTS);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&rs_full[i], kUnpackGroups * kUnpackWarps);
       mbar_init(&rs_empty[i], kEpiWarps);
+      mbar_init(&cols_full[i], kEpiWarps);
     }
     mbar_init(drain, 1);
+    mbar_init(stg_free, kEpiWarps * L::EPI_PARTS);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmA);
@@ -269,28 +453,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int grp = (warp - kFirstUnpackWarp) / kUnpackWarps;
     const int u = tid - (kFirstUnpackWarp + grp * kUnpackWarps) * 32;   // 0..255
     const uint32_t xa = ASYM ? 0u : 0x88888888u;
-    uint32_t la[L::TA], sa[L::TA], ha[L::TA], lb[L::TB], sb[L::TB], hb[L::TB];
-#pragma unroll
-    for (int j = 0; j < L::TA; ++j) {
-      const int i = u + 256 * j, r = i >> 2, ch = i & 3;
-      la[j] = r * 64 + ch * 16;
-      sa[j] = swz_off(r, 2 * ch);
-      ha[j] = swz_off(r, 2 * ch + 1);
-    }
-#pragma unroll
-    for (int j = 0; j < L::TB; ++j) {
-      const int i = u + 256 * j, r = i >> 2, ch = i & 3;
-      lb[j] = r * 64 + ch * 16;
-      sb[j] = swz_off(r, 2 * ch);
-      hb[j] = swz_off(r, 2 * ch + 1);
-    }
+    // chunk j of this thread: packed row r = u / 4 + 64 j, 16-byte chunk u % 4;
+    // its two unpacked 16-byte chunks 2 (u % 4) and 2 (u % 4) + 1 of that row
+    // (swizzled: they differ in address bit 4).  Rows 64 j further down are
+    // 4096 bytes further in the packed tile and 8192 in the unpacked one,
+    // for the activation and the weight tile alike.
+    const uint32_t l0 = (uint32_t)((u >> 2) * 64 + (u & 3) * 16);
+    const uint32_t s0 = swz_off(u >> 2, 2 * (u & 3));
     const uint32_t sbase = smem_u32(base);
+    // 256-row tiles: after unpacking a tile, the warp takes its share of that
+    // tile's epilogue, staging y in the operand stages; before unpacking the
+    // next tile it waits until every warp has read its staging block out.
     int it = 0, lt = 0;
     bool stop = false;
     for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x, ++lt) {
       int rsum[L::TA];
 #pragma unroll
       for (int j = 0; j < L::TA; ++j) rsum[j] = 0;
+      if (MT == 2 && lt > 0 && !wait_or_abort(stg_free, (lt - 1) & 1, abort_flag, 11)) break;
       for (int kt = 0; kt < num_k; ++kt, ++it) {
         if ((it & 1) != grp) continue;
         const int s = it % NP, su = it % NU;
@@ -303,9 +483,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t UA = sbase + L::uA + su * BMT * 128, UB = sbase + L::uB + su * BN * 128;
         uint4 wa[L::TA], wb[L::TB];
 #pragma unroll
-        for (int j = 0; j < L::TA; ++j) wa[j] = lds128(PA + la[j]);
+        for (int j = 0; j < L::TA; ++j) wa[j] = lds128(PA + l0 + 4096 * j);
 #pragma unroll
-        for (int j = 0; j < L::TB; ++j) wb[j] = lds128(PB + lb[j]);
+        for (int j = 0; j < L::TB; ++j) wb[j] = lds128(PB + l0 + 4096 * j);
         // packed stage consumed, once every lane's loads have read it
         wait_loaded(wa, scratch);
         wait_loaded(wb, scratch);
@@ -317,15 +497,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           unpack16(wa[j], xa, lo, hi);
           rsum[j] = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u,
                                 (unsigned)rsum[j]);
-          sts128(UA + sa[j], lo);
-          sts128(UA + ha[j], hi);
+          sts128(UA + s0 + 8192 * j, lo);
+          sts128(UA + (s0 ^ 16u) + 8192 * j, hi);
         }
 #pragma unroll
         for (int j = 0; j < L::TB; ++j) {
           uint4 lo, hi;
           unpack16(wb[j], 0x88888888u, lo, hi);
-          sts128(UB + sb[j], lo);
-          sts128(UB + hb[j], hi);
+          sts128(UB + s0 + 8192 * j, lo);
+          sts128(UB + (s0 ^ 16u) + 8192 * j, hi);
         }
         fence_proxy_async_smem();
         __syncwarp();
@@ -346,31 +526,41 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&rs_full[b]);
+      if (MT == 2 && !unpack_epi_share<ASYM, ACC_OUT>(args, tmem, warp, lane, lt, tile, m_tiles, acc_full, acc_empty,
+                                                      rs_full, cols_full, stg_free, rs_a, cols, sbase + L::uA,
+                                                      abort_flag))
+        break;
     }
   } else if (warp >= kFirstEpiWarp && warp < kFirstEpiWarp + kEpiWarps) {
     // ------------------------------------------------ epilogue
     const int q = warp & 3;
     const int et = tid - kFirstEpiWarp * 32;   // 0..127
-    // y staging of this warp (256-row tiles): two 32 x 32 fp16 buffers
-    uint8_t* ystage = base + L::ys + (warp - kFirstEpiWarp) * 2 * 2048;
-    int ygroup = 0;   // 32-column groups stored so far (buffer = ygroup & 1)
-    if (L::TMA_Y && lane == 0) prefetch_tmap(&tmY);
     int lt = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
       const int b = lt % NACC, rb = lt & 1;
       const int64_t n0 = (int64_t)(tile / m_tiles) * BN;
-      // column constants of this tile, staged once (the previous tile's epilogue is done)
-      named_bar_sync(1, kEpiWarps * 32);
+      const int64_t m_tile0 = (int64_t)(tile % m_tiles) * BMT;
+      // column constants of this tile into the buffer of its parity.  Its
+      // last readers worked on tile lt - 2: with 256-row tiles they all
+      // finished before the accumulator of lt - 1 was released; with the
+      // double-buffered 128-row accumulators a warp may run a tile ahead of
+      // the others, so the four warps meet first
+      if constexpr (MT == 1) named_bar_sync(1, kEpiWarps * 32);
+      float* col_s = cols + rb * 2 * BN;
+      float* col_r = col_s + BN;
       for (int j = et; j < BN; j += kEpiWarps * 32) {
         const int64_t n = n0 + j;
         col_s[j] = n < args.N ? __ldg(args.w_scale + n) : 0.f;
         col_r[j] = n < args.N ? (float)__ldg(args.w_rowsum + n) : 0.f;
       }
-      named_bar_sync(1, kEpiWarps * 32);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&cols_full[rb]);   // release: the warp's stores are ordered before it
       bool ok = wait_or_abort(&acc_full[b], (lt / NACC) & 1, abort_flag, 7);
       ok = ok && wait_or_abort(&rs_full[rb], (lt >> 1) & 1, abort_flag, 8);
-      __syncwarp();
-      if (!ok) break;
+      ok = ok && wait_or_abort(&cols_full[rb], (lt >> 1) & 1, abort_flag, 9);
+      // the tensor-memory loads below are warp-collective; with 128-row tiles
+      // the four warps also meet at a barrier each tile, so they decide alike
+      if (MT == 1 ? epi_bar_or(!ok) : !__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
       int rsa[MT];
 #pragma unroll
@@ -380,21 +570,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&rs_empty[rb]);
-      // chunks of 16 accumulator columns, loads double-buffered across chunks
+      const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * MT * BN);
+      if constexpr (MT == 2) {
+        epi256_share<ASYM, ACC_OUT>(args, tq, q, lane, 0, L::EPI_PARTS, m_tile0, n0, col_s, col_r, rsa[0],
+                                    rsa[MT - 1], smem_u32(base + L::uA) + (uint32_t)(q * L::EPI_PARTS * L::EPI_STAGE),
+                                    &acc_empty[b], stg_free);
+        continue;
+      }
+      // 128-row tiles: chunks of 16 accumulator columns, loads double-buffered
+      // across chunks; the other accumulator buffer is meanwhile being filled
       constexpr int NCH = MT * (BN / 16);
-      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * MT * BN);
       uint32_t ra[16], rbuf[16];
       auto step = [&](int ci, uint32_t(&cur)[16], uint32_t(&nxt)[16]) {
         tmem_ld_wait(cur);
         if (ci + 1 < NCH) {
-          tmem_ld_32x32b_x16(tbase + (uint32_t)((ci + 1) * 16), nxt);
+          tmem_ld_32x32b_x16(tq + (uint32_t)((ci + 1) * 16), nxt);
         } else {
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&acc_empty[b]);   // accumulator buffer free again
         }
         const int mt = ci / (BN / 16), cc = ci % (BN / 16);
-        const int64_t m = (int64_t)(tile % m_tiles) * BMT + mt * 128 + q * 32 + lane;
+        const int64_t m = m_tile0 + mt * 128 + q * 32 + lane;
         const bool mvalid = m < args.M;
         // y = s_n (alpha (S - 8 rs_a - 8 rw_n) + beta' rw_n), S = acc * 2^18, evaluated as
         // y = s_n * fma(alpha * 2^18, acc, c + d * rw_n), c = -8 alpha rs_a, d = beta' - 8 alpha
@@ -407,19 +604,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float cm = -8.f * alpha * (float)rsa[mt];
         const float dm = bp - 8.f * alpha;
         __half* yrow = reinterpret_cast<__half*>(args.y) + m * args.N;
-        uint8_t* ybuf = ystage + (ygroup & 1) * 2048;
-        if (L::TMA_Y && (ci & 1) == 0) {
-          // the store issued from this buffer two groups ago must have read it
-          if (lane == 0) bulk_wait_group_read<1>();
-          __syncwarp();
-        }
 #pragma unroll
         for (int g8 = 0; g8 < 2; ++g8) {
           const int j0 = cc * 16 + g8 * 8;
           const int64_t n = n0 + j0;
-          if (!L::TMA_Y && (!mvalid || n >= args.N)) continue;
-          // (staged rows and columns outside y are dropped by the TMA store;
-          // their column constants and alpha are zero)
+          if (!mvalid || n >= args.N) continue;
           const float4 s0 = *reinterpret_cast<const float4*>(col_s + j0);
           const float4 s1 = *reinterpret_cast<const float4*>(col_s + j0 + 4);
           const float4 q0 = *reinterpret_cast<const float4*>(col_r + j0);
@@ -430,16 +619,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int e = 0; e < 8; ++e)
             yv[e] = sc[e] * fmaf(alpha_s, __uint_as_float(cur[g8 * 8 + e]), fmaf(dm, rw[e], cm));
-          const uint4 pk = make_uint4(pack_half2_bits(yv[0], yv[1]), pack_half2_bits(yv[2], yv[3]),
-                                      pack_half2_bits(yv[4], yv[5]), pack_half2_bits(yv[6], yv[7]));
-          if (L::TMA_Y) {
-            // row `lane`, 16-byte chunk c = 2 (ci & 1) + g8 of the 64-byte row, swizzled
-            const int c = 2 * (ci & 1) + g8;
-            sts128(smem_u32(ybuf + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)), pk);
-          } else {
-            *reinterpret_cast<uint4*>(yrow + n) = pk;
-          }
-          if (ACC_OUT && mvalid && n < args.N) {
+          *reinterpret_cast<uint4*>(yrow + n) =
+              make_uint4(pack_half2_bits(yv[0], yv[1]), pack_half2_bits(yv[2], yv[3]),
+                         pack_half2_bits(yv[4], yv[5]), pack_half2_bits(yv[6], yv[7]));
+          if (ACC_OUT) {
             int accs[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e)
@@ -450,30 +633,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             ap[1] = make_int4(accs[4], accs[5], accs[6], accs[7]);
           }
         }
-        if (L::TMA_Y && (ci & 1) == 1) {
-          // the 32 x 32 block is complete: hand it to the TMA engine
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            const int64_t x = n0 + (cc - 1) * 16;   // a multiple of 32 elements: 16-byte aligned
-            const int64_t yrow0 = (int64_t)(tile % m_tiles) * BMT + mt * 128 + q * 32;
-            // a box that starts inside y is clipped to it by the TMA engine;
-            // one wholly outside is not issued
-            if (x < args.N && yrow0 < args.M) tma_store_2d(&tmY, ybuf, (int32_t)x, (int32_t)yrow0);
-            bulk_commit_group();
-          }
-          ++ygroup;
-        }
       };
-      tmem_ld_32x32b_x16(tbase, ra);
+      tmem_ld_32x32b_x16(tq, ra);
 #pragma unroll 1
       for (int ci = 0; ci < NCH; ci += 2) {
         step(ci, ra, rbuf);
         step(ci + 1, rbuf, ra);
       }
     }
-    // the staged blocks must be read (and written) before the CTA exits
-    if (L::TMA_Y && lane == 0) bulk_wait_group<0>();
   }
 
   tc_fence_before();
@@ -829,14 +996,9 @@ namespace {
 template <int MT, bool ASYM, bool ACC_OUT>
 cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   using L = Cfg<MT>;
-  CUtensorMap tmA, tmB, tmY;
+  CUtensorMap tmA, tmB;
   if (!encode_packed_map(&tmA, a.a_codes, a.M, a.K, L::BMT)) return cudaErrorNotSupported;
   if (!encode_packed_map(&tmB, a.w_codes, a.N, a.K, BN)) return cudaErrorNotSupported;
-  if (L::TMA_Y) {
-    if (!encode_y_map(&tmY, a.y, a.M, a.N)) return cudaErrorNotSupported;
-  } else {
-    tmY = tmA;   // unused
-  }
   auto kern = w4a4_gemm_kernel<MT, ASYM, ACC_OUT>;
   const size_t smem = L::dyn_bytes;
   int per_sm = 0;
@@ -847,7 +1009,7 @@ cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   const int n_tiles = (int)((a.N + BN - 1) / BN);
   const int tiles = m_tiles * n_tiles;
   const int grid = tiles < sms ? tiles : sms;
-  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, 1, tmA, tmB, tmY, a, (int)(a.K / 128), m_tiles,
+  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, 1, tmA, tmB, a, (int)(a.K / 128), m_tiles,
                  tiles);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
@@ -931,8 +1093,9 @@ namespace {
 // A persistent CTA (or SM pair) runs ceil(tiles / CTAs) tiles back to back:
 //   128 x 256 tiles, one CTA:  0.485 us per 128-deep K step + 3 us (the
 //     epilogue overlaps the next tile);
-//   256 x 256 tiles, one CTA:  0.66 us per K step + 10 us (the single
-//     accumulator buffer serialises the epilogue);
+//   256 x 256 tiles, one CTA:  0.66 us per K step + 5.6 us per tile (the
+//     single accumulator buffer serialises the epilogue, which all unpack
+//     warps share) + 5.4 us once;
 //   256 x 256 tiles, SM pair:  0.45 us per K step, epilogue overlapped,
 //     + 3 us for the last tile's epilogue.
 struct PrefillChoice {
@@ -945,7 +1108,7 @@ PrefillChoice choose_prefill(int64_t M, int64_t N, int64_t K, bool allow_pair) {
   const int64_t sms = device_sm_count(), ks = K / 128;
   const int64_t tiles256 = ((M + 255) / 256) * ((N + BN - 1) / BN);
   const int64_t tiles128 = ((M + 127) / 128) * ((N + BN - 1) / BN);
-  const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 10.0);
+  const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 5.6) + 5.4;
   const double est128 = (double)((tiles128 + sms - 1) / sms) * (0.485 * (double)ks + 3.0);
   PrefillChoice c = est256 < est128 ? PrefillChoice{SPINQ_GEMM_TILE256, est256} : PrefillChoice{SPINQ_GEMM_TILE128, est128};
   if (pairs > 0) {
