@@ -143,16 +143,21 @@ struct Cfg {
   static constexpr uint32_t rs_a = (misc + 16 + 15) & ~15u;
   // [tile parity][s_n, (float) rowsum_n][BN]: the column constants of a tile
   static constexpr uint32_t cols = rs_a + 2 * kUnpackGroups * BMT * 4;
-  static constexpr uint32_t total = cols + 2 * 2 * BN * 4;
-  static constexpr size_t dyn_bytes = total + 1024;
   // warps that share the epilogue of a 256-row tile per TMEM lane quadrant:
-  // its epilogue warp and the four unpack warps of that quadrant.  The unpack
-  // warps take their share before they unpack the next tile, so the operand
-  // stages are free meanwhile and hold the warps' y staging blocks
-  // (EPI_STAGE bytes each).
+  // its epilogue warp and the four unpack warps of that quadrant.  Each
+  // stages y in blocks of EPI_STAGE bytes: the epilogue warps in a region of
+  // their own (estage), the unpack warps in the operand stage that the next
+  // tile's first K step does not use (with two stages and two unpack groups,
+  // group g always fills stage g: the group that owns the next tile's first
+  // step unpacks it before its share, so that its MMA overlaps the stores).
   static constexpr int EPI_PARTS = MT == 2 ? 1 + kUnpackGroups * kUnpackWarps / 4 : 1;
   static constexpr uint32_t EPI_STAGE = 32 * 128;
-  static_assert(MT == 1 || kEpiWarps * EPI_PARTS * EPI_STAGE <= 2 * NU * BMT * 128, "staging fits the operand ring");
+  static constexpr uint32_t estage = (cols + 2 * 2 * BN * 4 + 1023) & ~1023u;
+  static constexpr uint32_t total = MT == 2 ? estage + kEpiWarps * EPI_STAGE : cols + 2 * 2 * BN * 4;
+  static constexpr size_t dyn_bytes = total + 1024;
+  static_assert(MT == 1 || (NU == 2 && kUnpackGroups == 2 &&
+                            kUnpackGroups * kUnpackWarps * EPI_STAGE == BMT * 128 + BN * 128),
+                "the unpack warps' staging fills one operand stage");
 };
 
 // One warp's share of the epilogue of a 256 x 256 tile.  The tile's rows
@@ -166,8 +171,8 @@ struct Cfg {
 // with 8 lanes per row and stored with 16-byte stores, so that each store
 // instruction writes 4 rows x 128 contiguous bytes of y instead of 32
 // separate 16-byte pieces.  The accumulator is released (acc_empty) after
-// the warp's last tensor-memory load, the staging block (stg_free) after its
-// last read.
+// the warp's last tensor-memory load, the staging block (stg_free, unless
+// null) after its last read.
 //   y = s_n (alpha (S - 8 rs_a - 8 rw_n) + beta' rw_n), S = acc * 2^18,
 //   evaluated as y = s_n * fma(alpha * 2^18, acc, c + d * rw_n) with
 //   c = -8 alpha rs_a and d = beta' - 8 alpha (the roundings of the other
@@ -281,7 +286,7 @@ __device__ __forceinline__ void epi256_share(const GemmArgs& args, uint32_t tq, 
     if (lane == 0) mbar_arrive(acc_empty);
   }
   __syncwarp();
-  if (lane == 0) mbar_arrive(stg_free);   // release: orders the block reads above before it
+  if (stg_free != nullptr && lane == 0) mbar_arrive(stg_free);   // release: orders the block reads above before it
 }
 
 // An unpack warp's share of the epilogue of 256-row tile `plt` (local index;
@@ -293,7 +298,7 @@ template <bool ASYM, bool ACC_OUT>
 __device__ __forceinline__ bool unpack_epi_share(const GemmArgs& args, uint32_t tmem, int warp, int lane, int plt,
                                                  int ptile, int m_tiles, uint64_t* acc_full, uint64_t* acc_empty,
                                                  uint64_t* rs_full, uint64_t* cols_full, uint64_t* stg_free,
-                                                 const int* rs_a, const float* cols, uint32_t stage_base,
+                                                 const int* rs_a, const float* cols, uint32_t stage,
                                                  volatile int* abort_flag) {
   constexpr int BMT = 256;
   const int rb = plt & 1;
@@ -311,8 +316,7 @@ __device__ __forceinline__ bool unpack_epi_share(const GemmArgs& args, uint32_t 
   constexpr int NPARTS = Cfg<2>::EPI_PARTS;
   epi256_share<ASYM, ACC_OUT>(args, tmem + ((uint32_t)(q * 32) << 16), q, lane, part, NPARTS,
                               (int64_t)(ptile % m_tiles) * BMT, (int64_t)(ptile / m_tiles) * BN, col_s, col_s + BN,
-                              rsa0, rsa1, stage_base + (uint32_t)((q * NPARTS + part) * Cfg<2>::EPI_STAGE),
-                              &acc_empty[0], stg_free);
+                              rsa0, rsa1, stage, &acc_empty[0], stg_free);
   return true;
 }
 
@@ -366,7 +370,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&cols_full[i], kEpiWarps);
     }
     mbar_init(drain, 1);
-    mbar_init(stg_free, kEpiWarps * L::EPI_PARTS);
+    mbar_init(stg_free, kUnpackGroups * kUnpackWarps);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmA);
@@ -461,55 +465,78 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t l0 = (uint32_t)((u >> 2) * 64 + (u & 3) * 16);
     const uint32_t s0 = swz_off(u >> 2, 2 * (u & 3));
     const uint32_t sbase = smem_u32(base);
-    // 256-row tiles: after unpacking a tile, the warp takes its share of that
-    // tile's epilogue, staging y in the operand stages; before unpacking the
-    // next tile it waits until every warp has read its staging block out.
+    // One K step `it` into operand stage it % NU; false when a wait gave up.
+    // The activation row sums of the step are added to rs[].
+    auto unpack_step = [&](int it, int (&rs)[L::TA]) -> bool {
+      const int s = it % NP, su = it % NU;
+      if (!wait_or_abort(&full_p[s], (it / NP) & 1, abort_flag, 4) ||
+          !wait_or_abort(&empty_u[su], ((it / NU) & 1) ^ 1, abort_flag, 5))
+        return false;
+      const uint32_t PA = sbase + L::pA + s * BMT * 64, PB = sbase + L::pB + s * BN * 64;
+      const uint32_t UA = sbase + L::uA + su * BMT * 128, UB = sbase + L::uB + su * BN * 128;
+      uint4 wa[L::TA], wb[L::TB];
+#pragma unroll
+      for (int j = 0; j < L::TA; ++j) wa[j] = lds128(PA + l0 + 4096 * j);
+#pragma unroll
+      for (int j = 0; j < L::TB; ++j) wb[j] = lds128(PB + l0 + 4096 * j);
+      // packed stage consumed, once every lane's loads have read it
+      wait_loaded(wa, scratch);
+      wait_loaded(wb, scratch);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_p[s]);
+#pragma unroll
+      for (int j = 0; j < L::TA; ++j) {
+        uint4 lo, hi;
+        unpack16(wa[j], xa, lo, hi);
+        rs[j] = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u, (unsigned)rs[j]);
+        sts128(UA + s0 + 8192 * j, lo);
+        sts128(UA + (s0 ^ 16u) + 8192 * j, hi);
+      }
+#pragma unroll
+      for (int j = 0; j < L::TB; ++j) {
+        uint4 lo, hi;
+        unpack16(wb[j], 0x88888888u, lo, hi);
+        sts128(UB + s0 + 8192 * j, lo);
+        sts128(UB + (s0 ^ 16u) + 8192 * j, hi);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&full_u[su]);
+      return true;
+    };
+    // 256-row tiles: after unpacking a tile the warp takes its share of the
+    // tile's epilogue, staging y in the operand stage that the next tile's
+    // first K step does not use; the group that owns that first step unpacks
+    // it before its share (`early`, its row sums in `carry`).  A group waits
+    // for the staging blocks in its stage to be read out (stg_free of tile
+    // `stg_due`) before it writes that stage again.
+    int early = -1, stg_due = -1;
+    int carry[L::TA];
+#pragma unroll
+    for (int j = 0; j < L::TA; ++j) carry[j] = 0;
     int it = 0, lt = 0;
     bool stop = false;
     for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x, ++lt) {
       int rsum[L::TA];
 #pragma unroll
-      for (int j = 0; j < L::TA; ++j) rsum[j] = 0;
-      if (MT == 2 && lt > 0 && !wait_or_abort(stg_free, (lt - 1) & 1, abort_flag, 11)) break;
+      for (int j = 0; j < L::TA; ++j) {
+        rsum[j] = carry[j];
+        carry[j] = 0;
+      }
       for (int kt = 0; kt < num_k; ++kt, ++it) {
         if ((it & 1) != grp) continue;
-        const int s = it % NP, su = it % NU;
-        if (!wait_or_abort(&full_p[s], (it / NP) & 1, abort_flag, 4) ||
-            !wait_or_abort(&empty_u[su], ((it / NU) & 1) ^ 1, abort_flag, 5)) {
+        if (it == early) continue;   // unpacked ahead, with the previous tile's epilogue
+        if (MT == 2 && stg_due >= 0) {
+          if (!wait_or_abort(stg_free, stg_due & 1, abort_flag, 11)) {
+            stop = true;
+            break;
+          }
+          stg_due = -1;
+        }
+        if (!unpack_step(it, rsum)) {
           stop = true;
           break;
         }
-        const uint32_t PA = sbase + L::pA + s * BMT * 64, PB = sbase + L::pB + s * BN * 64;
-        const uint32_t UA = sbase + L::uA + su * BMT * 128, UB = sbase + L::uB + su * BN * 128;
-        uint4 wa[L::TA], wb[L::TB];
-#pragma unroll
-        for (int j = 0; j < L::TA; ++j) wa[j] = lds128(PA + l0 + 4096 * j);
-#pragma unroll
-        for (int j = 0; j < L::TB; ++j) wb[j] = lds128(PB + l0 + 4096 * j);
-        // packed stage consumed, once every lane's loads have read it
-        wait_loaded(wa, scratch);
-        wait_loaded(wb, scratch);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty_p[s]);
-#pragma unroll
-        for (int j = 0; j < L::TA; ++j) {
-          uint4 lo, hi;
-          unpack16(wa[j], xa, lo, hi);
-          rsum[j] = (int)__dp4a(lo.x + lo.y + lo.z + lo.w + hi.x + hi.y + hi.z + hi.w, 0x01010101u,
-                                (unsigned)rsum[j]);
-          sts128(UA + s0 + 8192 * j, lo);
-          sts128(UA + (s0 ^ 16u) + 8192 * j, hi);
-        }
-#pragma unroll
-        for (int j = 0; j < L::TB; ++j) {
-          uint4 lo, hi;
-          unpack16(wb[j], 0x88888888u, lo, hi);
-          sts128(UB + s0 + 8192 * j, lo);
-          sts128(UB + (s0 ^ 16u) + 8192 * j, hi);
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&full_u[su]);
       }
       if (stop) break;
       // row sums of the unsigned activation codes: 4 lanes share a row
@@ -526,10 +553,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&rs_full[b]);
-      if (MT == 2 && !unpack_epi_share<ASYM, ACC_OUT>(args, tmem, warp, lane, lt, tile, m_tiles, acc_full, acc_empty,
-                                                      rs_full, cols_full, stg_free, rs_a, cols, sbase + L::uA,
-                                                      abort_flag))
-        break;
+      if constexpr (MT == 2) {
+        // `it` is now the next tile's first K step, in stage it & 1
+        const int first = it & 1;
+        if (tile + (int)gridDim.x < num_tiles && first == grp) {
+          if (stg_due >= 0) {
+            if (!wait_or_abort(stg_free, stg_due & 1, abort_flag, 11)) break;
+            stg_due = -1;
+          }
+          if (!unpack_step(it, carry)) break;
+          early = it;
+        }
+        const int h = warp - kFirstUnpackWarp;   // 0..15
+        const uint32_t stage = sbase + (h < 8 ? L::uA + (1 - first) * BMT * 128 : L::uB + (1 - first) * BN * 128) +
+                               (uint32_t)(h & 7) * L::EPI_STAGE;
+        if (!unpack_epi_share<ASYM, ACC_OUT>(args, tmem, warp, lane, lt, tile, m_tiles, acc_full, acc_empty, rs_full,
+                                             cols_full, stg_free, rs_a, cols, stage, abort_flag))
+          break;
+        if (1 - first == grp) stg_due = lt;
+      }
     }
   } else if (warp >= kFirstEpiWarp && warp < kFirstEpiWarp + kEpiWarps) {
     // ------------------------------------------------ epilogue
@@ -573,8 +615,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * MT * BN);
       if constexpr (MT == 2) {
         epi256_share<ASYM, ACC_OUT>(args, tq, q, lane, 0, L::EPI_PARTS, m_tile0, n0, col_s, col_r, rsa[0],
-                                    rsa[MT - 1], smem_u32(base + L::uA) + (uint32_t)(q * L::EPI_PARTS * L::EPI_STAGE),
-                                    &acc_empty[b], stg_free);
+                                    rsa[MT - 1], smem_u32(base + L::estage) + (uint32_t)(q * L::EPI_STAGE),
+                                    &acc_empty[b], nullptr);
         continue;
       }
       // 128-row tiles: chunks of 16 accumulator columns, loads double-buffered
@@ -1093,9 +1135,9 @@ namespace {
 // A persistent CTA (or SM pair) runs ceil(tiles / CTAs) tiles back to back:
 //   128 x 256 tiles, one CTA:  0.485 us per 128-deep K step + 3 us (the
 //     epilogue overlaps the next tile);
-//   256 x 256 tiles, one CTA:  0.66 us per K step + 5.6 us per tile (the
+//   256 x 256 tiles, one CTA:  0.66 us per K step + 5.0 us per tile (the
 //     single accumulator buffer serialises the epilogue, which all unpack
-//     warps share) + 5.4 us once;
+//     warps share) + 4.9 us once;
 //   256 x 256 tiles, SM pair:  0.45 us per K step, epilogue overlapped,
 //     + 3 us for the last tile's epilogue.
 struct PrefillChoice {
@@ -1108,7 +1150,7 @@ PrefillChoice choose_prefill(int64_t M, int64_t N, int64_t K, bool allow_pair) {
   const int64_t sms = device_sm_count(), ks = K / 128;
   const int64_t tiles256 = ((M + 255) / 256) * ((N + BN - 1) / BN);
   const int64_t tiles128 = ((M + 127) / 128) * ((N + BN - 1) / BN);
-  const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 5.6) + 5.4;
+  const double est256 = (double)((tiles256 + sms - 1) / sms) * (0.66 * (double)ks + 5.0) + 4.9;
   const double est128 = (double)((tiles128 + sms - 1) / sms) * (0.485 * (double)ks + 3.0);
   PrefillChoice c = est256 < est128 ? PrefillChoice{SPINQ_GEMM_TILE256, est256} : PrefillChoice{SPINQ_GEMM_TILE128, est128};
   if (pairs > 0) {
