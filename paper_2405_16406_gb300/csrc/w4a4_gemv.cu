@@ -40,6 +40,10 @@ __device__ __forceinline__ void expand16(const uint4 w, uint32_t x, uint32_t lo[
   }
 }
 
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ uint32_t dp4a_u(uint32_t a, uint32_t b, uint32_t c) {
   return __dp4a(a, b, c);
 }
@@ -59,6 +63,16 @@ __global__ void __launch_bounds__(kGemvThreads) w4a4_gemv_kernel(GemmArgs a) {
   const uint32_t xa = ASYM ? 0u : 0x88888888u;
 
   if (tid < MT) su[tid] = 0;
+  // The weight row of this warp's first channel into L2 while the previous
+  // kernel may still run: L2 is coherent with that kernel's stores, and
+  // nothing is read into registers before griddepcontrol.wait.
+  {
+    const int64_t n = (int64_t)blockIdx.x * kGemvWarps + warp;
+    if (n < a.N) {
+      const char* row = reinterpret_cast<const char*>(a.w_codes) + n * kh;
+      for (int64_t off = (int64_t)lane * 128; off < kh; off += 32 * 128) prefetch_l2(row + off);
+    }
+  }
   __syncthreads();
   pdl_wait();
   pdl_trigger();
