@@ -105,6 +105,17 @@ __device__ __forceinline__ bool epi_bar_or(bool pred) {
   return r != 0;
 }
 
+// L2 prefetch of the box at (x, y) of a tensor map.  Issued before
+// griddepcontrol.wait for the weights only: L2 is coherent with the previous
+// kernel's stores and nothing reaches registers or shared memory.
+__device__ __forceinline__ void tma_prefetch_2d(const void* tmap, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];\n" ::"l"(
+                   reinterpret_cast<uint64_t>(tmap)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+constexpr int kPrefetchSteps = 4;   // K steps of the first tile's weights prefetched into L2
+
 __device__ __forceinline__ uint32_t swz_off(int r, int chunk) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4));
 }
@@ -375,6 +386,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
+    if ((int)blockIdx.x < num_tiles)
+      for (int kt = 0; kt < kPrefetchSteps && kt < num_k; ++kt)
+        tma_prefetch_2d(&tmB, kt * 64, (int)(blockIdx.x / m_tiles) * BN);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, 512);
@@ -783,6 +797,8 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     fence_mbar_init();
     prefetch_tmap(&tmW);
     prefetch_tmap(&tmA);
+    // this CTA's slice of the weights (up to 16 K steps) into L2
+    for (int it = 0; it < nk && it < 16; ++it) tma_prefetch_2d(&tmW, (k_begin + it) * 64, n0);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, L::tmem_cols);
