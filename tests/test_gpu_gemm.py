@@ -211,6 +211,34 @@ def test_gemm_repeat_bit_identical(S, name, M, K, N, symmetric):
     assert np.array_equal(acc0.cpu().numpy()[ms, ns], racc)
 
 
+@pytest.mark.parametrize("M,N,K", [(2048, 16384, 128), (2048, 16384, 384), (1100, 16400, 640), (4096, 9728, 256)])
+def test_gemm_tile256_many_tiles_per_cta(S, M, N, K):
+    """256-row tiles, several per CTA, with an odd and an even number of K
+    steps per tile (one step included): the unpack group that owns the next
+    tile's first step alternates with the parity of the step count and
+    unpacks it ahead, during the epilogue of the current tile.  Checked bit
+    for bit against 128-row tiles and on sampled outputs against the oracle."""
+    rng = np.random.default_rng(M + N + K)
+    ac, al, be, wc, ws_ = random_codes(rng, M, N, K, False)
+    a = to_gpu_act(S, ac, al, be)
+    w = to_gpu_w(S, wc, ws_)
+    prev = S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TILE256)
+    try:
+        y, acc = S.w4a4_gemm(a, w, want_acc=True)
+        S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TILE128)
+        y1, acc1 = S.w4a4_gemm(a, w, want_acc=True)
+    finally:
+        S.spinq_gemm_select_kernel(prev)
+    torch.cuda.synchronize()
+    assert torch.equal(acc, acc1)
+    assert torch.equal(y.view(torch.int16), y1.view(torch.int16))
+    ms = np.concatenate([rng.integers(0, M, 2000), [0, M - 1, 255, 256]])
+    ns = np.concatenate([rng.integers(0, N, 2000), [N - 1, 0, 255, 256]])
+    racc, _ = oracle.w4a4_linear_sampled(ac, al, be, wc, ws_, ms, ns)
+    assert np.array_equal(acc.cpu().numpy()[ms, ns], racc)
+    assert S.spinq_device_status()[0] == S.SPINQ_OK
+
+
 @pytest.mark.parametrize("case", FULL, ids=[f[0] for f in FULL])
 def test_gemm_full_size_sampled(S, case):
     name, M, K, N, symmetric = case[:5]
