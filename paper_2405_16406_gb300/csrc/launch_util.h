@@ -67,13 +67,27 @@ cudaError_t prepare_launch(Kern kern, int threads, size_t smem, int* blocks_per_
 // blocks come from the per-SM limits instead: shared memory (with the
 // per-block reservation), registers (whole warps, 256-register granules),
 // threads, and the SM's 512 tensor-memory columns.
+// The answer is cached per device, kernel and launch shape (the cost models
+// ask on every call).
 template <typename Kern>
 cudaError_t prepare_launch_tmem(Kern kern, int threads, size_t smem, int tmem_cols, int* blocks_per_sm) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, const void*, size_t, int, int>, int> cache;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const auto key = std::make_tuple(dev, reinterpret_cast<const void*>(kern), smem, threads, tmem_cols);
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      *blocks_per_sm = it->second;
+      return cudaSuccess;
+    }
+  }
   int q = 0;
   cudaError_t e = prepare_launch(kern, threads, smem, &q);
   if (e != cudaSuccess) return e;
-  int dev = 0, smem_sm = 0, smem_rsv = 0, regs_sm = 0, thr_sm = 0;
-  cudaGetDevice(&dev);
+  int smem_sm = 0, smem_rsv = 0, regs_sm = 0, thr_sm = 0;
   cudaFuncAttributes fa;
   if ((e = cudaFuncGetAttributes(&fa, kern)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess ||
@@ -88,6 +102,8 @@ cudaError_t prepare_launch_tmem(Kern kern, int threads, size_t smem, int tmem_co
   n = std::min(n, thr_sm / (warps * 32));
   if (tmem_cols > 0) n = std::min(n, 512 / tmem_cols);
   *blocks_per_sm = std::max(1, std::min(n, 32));
+  std::lock_guard<std::mutex> lock(mu);
+  cache[key] = *blocks_per_sm;
   return cudaSuccess;
 }
 
