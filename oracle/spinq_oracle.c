@@ -25,7 +25,7 @@
  *   - Appendix "Quantization choice": clipping ratio of the min-max range;
  *     asymmetric quantization for activations and the KV cache.
  *
- * Readings where the paper is silent (each also listed in the design doc):
+ * Readings where the paper is silent:
  *   - Sylvester H_{2^k}[i][j] = (-1)^popcount(i & j) (natural order).
  *   - Paley I for a prime power q = 3 mod 4, order q + 1: H = I + S with
  *     S = [[0, 1^T], [-1, Q]], Q[i][j] = chi(a_i - a_j), chi the quadratic
