@@ -102,3 +102,28 @@ def test_empty_problems_are_ok_without_launch(lib):
     fake = ctypes.c_void_p(1 << 20)
     assert S.spinq_rotate_quant_act(fake, 0, 256, 256, None, ctypes.byref(q), fake, fake, None, None) == S.SPINQ_OK
     assert S.spinq_w4a4_gemm(fake, fake, None, fake, fake, fake, 0, 32, 128, fake, None, None) == S.SPINQ_OK
+
+
+def test_gemm_controls_validate_on_the_host(lib):
+    """The kernel selection, the K-slice control and the plan queries check
+    their arguments on the host; rejected values change nothing."""
+    from paper_2405_16406_gb300 import spinq as S
+    for bad in (-1, S.SPINQ_GEMM_SPLITK + 1, 99):
+        assert S.spinq_gemm_select_kernel(bad) == -1
+    prev = S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TILE256)
+    try:
+        assert S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TILE128) == S.SPINQ_GEMM_TILE256
+    finally:
+        S.spinq_gemm_select_kernel(prev)
+    for bad in (-1, 65, 1000):
+        assert S.spinq_gemm_split_k(bad) == -1
+    prev = S.spinq_gemm_split_k(7)
+    try:
+        assert S.spinq_gemm_split_k(0) == 7
+    finally:
+        S.spinq_gemm_split_k(prev)
+    # shapes every GEMM entry point rejects: no device query, -1
+    for M, N, K in ((0, 256, 128), (16, 100, 128), (16, 256, 100), (16, 256, 0), (-1, 256, 128)):
+        assert S.spinq_w4a4_gemm_plan(M, N, K) == -1
+        assert S.spinq_w4a4_gemm_splitk_plan(M, N, K) == (-1, 0)
+    assert S.spinq_w4a4_gemm_splitk_plan(16, 256, 65536 + 128) == (-1, 0)   # K above the exact-accumulator bound
