@@ -215,6 +215,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
+    // the first K steps of this CTA's half of the first tile's weights into
+    // L2 before the wait on the previous kernel (L2 is coherent with its
+    // stores; nothing reaches registers or shared memory before the wait)
+    if (cluster < num_tiles)
+      for (int kt = 0; kt < 4 && kt < num_k; ++kt)
+        asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];\n" ::"l"(
+                         reinterpret_cast<uint64_t>(&tmB)),
+                     "r"(kt * 64), "r"((cluster / m_tiles) * BN + BNH * (int)rank)
+                     : "memory");
   }
   if (warp == 1) {
     tmem_alloc_pair(tmem_slot, 512);
