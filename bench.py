@@ -102,6 +102,21 @@ def gemm_traffic_from_profile(profile, source):
         return None
 
 
+def workload_config(world):
+    """The workload both arms report (the same keys and values)."""
+    return {
+        "workload": "llama3_8b MLP hot path for 2048 tokens: gate_up 4096->14336 (act quant, R1 merged) "
+                    "+ down_proj 14336->4096 (online R4 = H28 (x) H512, act quant) "
+                    "+ R3/KV4 (32 q heads, 8 kv heads, head_dim 128)",
+        "M": M, "gate_up": {"K": K, "N": N, "act_quant": "asymmetric per-token int4, no online rotation"},
+        "down_proj": {"K": K2, "N": N2, "online_rotation": "H28 (Paley, GF(27)) (x) H512",
+                      "act_quant": "symmetric per-token int4"},
+        "weights": "symmetric per-channel int4 (quantized once, not timed)",
+        "l2": f"{NSETS} rotating input sets (~0.7 GB) > 129 MB L2",
+        "parallelism": f"replicas{world}",
+    }
+
+
 # --------------------------------------------------------------------------- clocks
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons while work runs."""
@@ -503,17 +518,7 @@ def run_ours(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "int4",
         "data": "synthetic",
-        "config": {
-            "workload": "llama3_8b MLP hot path for 2048 tokens: gate_up 4096->14336 (act quant, R1 merged) "
-                        "+ down_proj 14336->4096 (online R4 = H28 (x) H512, act quant) "
-                        "+ R3/KV4 (32 q heads, 8 kv heads, head_dim 128)",
-            "M": M, "gate_up": {"K": K, "N": N, "act_quant": "asymmetric per-token int4, no online rotation"},
-            "down_proj": {"K": K2, "N": N2, "online_rotation": "H28 (Paley, GF(27)) (x) H512",
-                          "act_quant": "symmetric per-token int4"},
-            "weights": "symmetric per-channel int4 (quantized once, not timed)",
-            "l2": f"{NSETS} rotating input sets (~0.7 GB) > 129 MB L2",
-            "parallelism": f"replicas{world}",
-        },
+        "config": workload_config(world),
         "roofline": {
             "bound": "tensor", "kernel": GEMM_KERNELS[kind1][0],
             "achieved": round(gemm_tops, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
@@ -561,9 +566,177 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": len(names) * args.steps,
         "clocks": clocks,
     }
+    if not args.no_configs:
+        out["configs"] = run_configs(dev, hbm_peak, fp8_peak)
+        st, _ = spinq.spinq_device_status()
+        if st != spinq.SPINQ_OK:
+            raise RuntimeError(f"device status after the config runs: {spinq.spinq_status_string(st)}")
     if not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(sample_rows=args.cpu_rows)
     return out
+
+
+# --------------------------------------------------------------------------- every config at full size
+def graph_us(fn, n_inputs, reps=20):
+    """Mean device time of one call: `reps` calls over rotating input copies
+    (more bytes than L2, so every call reads cold data) captured in one CUDA
+    graph and replayed 3 times between events."""
+    import torch
+    for i in range(n_inputs):
+        fn(i)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for i in range(reps):
+            fn(i % n_inputs)
+    g.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(3):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) * 1e3 / (3 * reps)
+
+
+def _codes_check(got_packed, x_rows, had, symmetric, what):
+    """Sampled rows of timed codes against the oracle: |diff| <= 1 on at most
+    1e-4 of the codes (at least one allowed per row sampled, ties only)."""
+    import numpy as np
+
+    import oracle
+    ref = oracle.rotate_quant_act(x_rows, had, 4, symmetric, 1.0)
+    got = oracle.unpack4(np.ascontiguousarray(got_packed), symmetric)
+    d = np.abs(got.astype(np.int64) - ref.codes)
+    allowed = max(int(1e-4 * d.size), 8)
+    if d.max(initial=0) > 1 or np.count_nonzero(d) > allowed:
+        raise RuntimeError(f"{what}: timed codes differ from the oracle ({np.count_nonzero(d)} of {d.size})")
+    return int(np.count_nonzero(d))
+
+
+def _gemm_check(y, qa, qw, rows, what, symmetric):
+    """Sampled outputs of a timed GEMM against the oracle's dequantized
+    product of the same codes (fp16 output, 2e-3 relative + 1e-3 of the
+    largest |y| in the sample)."""
+    import numpy as np
+
+    import oracle
+    rng = np.random.default_rng(5)
+    Mr = qa.codes.shape[0]
+    ms = np.asarray(rows if rows is not None else rng.integers(0, Mr, 64), dtype=np.int64)
+    N = qw.codes.shape[0]
+    ns = rng.integers(0, N, ms.size * 8, dtype=np.int64)
+    mm = np.repeat(ms, 8)
+    a_codes = oracle.unpack4(qa.codes[ms].cpu().numpy(), symmetric)
+    w_codes = oracle.unpack4(qw.codes.cpu().numpy(), True)
+    al = qa.scale[ms].double().cpu().numpy()
+    be = None if qa.zero is None else qa.zero[ms].double().cpu().numpy()
+    loc = np.repeat(np.arange(ms.size), 8)
+    _, yr = oracle.w4a4_linear_sampled(a_codes, al, be, w_codes, qw.scale.double().cpu().numpy(), loc, ns)
+    import torch
+    yg = y[torch.as_tensor(mm, device=y.device), torch.as_tensor(ns, device=y.device)].double().cpu().numpy()
+    tol = 2e-3 * np.abs(yr) + 1e-3 * np.abs(yr).max()
+    if not np.all(np.abs(yg - yr) <= tol):
+        raise RuntimeError(f"{what}: timed GEMM outputs differ from the oracle")
+    return int(ms.size * 8)
+
+
+def run_configs(dev, hbm_peak, fp8_peak):
+    """Every workload at its full size, each kernel timed on its own (graph of
+    back-to-back calls over cold inputs), and the timed outputs of the first
+    input copy checked against the oracle on sampled rows.  Inputs of copy 0
+    come from synth.py (host, numpy); further copies are device clones of it
+    (only there so that every call reads data that is not in L2)."""
+    import numpy as np
+    import torch
+
+    from paper_2405_16406_gb300 import spinq, synth
+    res = {}
+
+    def act_out(Mr, Kr, sym):
+        return spinq.ActCodes(torch.empty(Mr, Kr // 2, dtype=torch.uint8, device=dev),
+                              torch.empty(Mr, dtype=torch.float32, device=dev),
+                              None if sym else torch.empty(Mr, dtype=torch.float32, device=dev))
+
+    def copies(t, n):
+        return [t] + [t.clone() for _ in range(n - 1)]
+
+    def linear(case, tag, gemm_bound):
+        x0 = torch.from_numpy(case.x).to(dev)
+        w0 = torch.from_numpy(case.w).to(dev)
+        qw0 = spinq.quant_weight(w0, case.had)
+        del w0
+        Mr, Kr, Nr = case.M, case.K, case.N
+        nx = max(2, min(16, int(np.ceil(2 * 129e6 / max(1, x0.numel() * 2)))))
+        xs = copies(x0, nx)
+        outs = [act_out(Mr, Kr, case.act_symmetric) for _ in range(nx)]
+        rq_us = graph_us(lambda i: spinq.rotate_quant_act(xs[i], case.had, case.act_symmetric, case.clip,
+                                                          out=outs[i]), nx)
+        rq_bytes = Mr * Kr * 2 + Mr * Kr // 2 + (4 if case.act_symmetric else 8) * Mr
+        w_bytes = Nr * Kr // 2
+        nw = max(2, min(16, int(np.ceil(2 * 129e6 / w_bytes))))
+        qws = [qw0] + [spinq.WeightCodes(qw0.codes.clone(), qw0.scale.clone(), qw0.rowsum.clone())
+                       for _ in range(nw - 1)]
+        ys = [torch.empty(Mr, Nr, dtype=torch.float16, device=dev) for _ in range(nw)]
+        ws = spinq.gemm_workspace(Mr, Nr, Kr, dev) if Mr <= 256 else None   # calls run in stream order
+        g_us = graph_us(lambda i: spinq.w4a4_gemm_splitk(outs[i % nx], qws[i], workspace=ws, y=ys[i]) if Mr <= 256
+                        else spinq.w4a4_gemm(outs[i % nx], qws[i], y=ys[i]), nw)
+        torch.cuda.synchronize()
+        rows = np.unique(np.linspace(0, Mr - 1, min(Mr, 8)).astype(np.int64))
+        flips = _codes_check(outs[0].codes[torch.as_tensor(rows, device=dev)].cpu().numpy(), case.x[rows],
+                             case.had, case.act_symmetric, tag + " rotate+quant")
+        # the GEMM of call i used activation copy i % nx and weight copy i: copy 0 of both
+        nchk = _gemm_check(ys[0], outs[0], qw0, rows, tag + " GEMM", case.act_symmetric)
+        ops = 2.0 * Mr * Nr * Kr
+        rq = {"us": round(rq_us, 3), "bytes": rq_bytes, "gbs": round(rq_bytes / rq_us / 1e3, 1),
+              "frac_hbm": round(rq_bytes / rq_us / 1e3 / hbm_peak, 4)}
+        gm = {"us": round(g_us, 3), "tops": round(ops / g_us / 1e6, 1),
+              "kernel_plan": spinq.spinq_w4a4_gemm_splitk_plan(Mr, Nr, Kr) if Mr <= 256
+              else spinq.spinq_w4a4_gemm_plan(Mr, Nr, Kr)}
+        if gemm_bound == "tensor":
+            gm["frac_e4m3"] = round(ops / g_us / 1e6 / fp8_peak, 4)
+        else:
+            gbytes = w_bytes + Mr * Kr // 2 + 2 * Mr * Nr
+            gm["bytes"] = gbytes
+            gm["frac_hbm"] = round(gbytes / g_us / 1e3 / hbm_peak, 4)
+        r = {"M": Mr, "K": Kr, "N": Nr, "had": case.had, "rotate_quant": rq, "gemm": gm,
+             "checked": f"{rows.size} rows of codes ({flips} tie flips), {nchk} GEMM outputs vs oracle"}
+        del xs, outs, qws, ys
+        torch.cuda.empty_cache()
+        return r
+
+    res["c1_tiny_16x256x512_h256"] = linear(synth.tiny_linear(), "config 1", "latency")
+    for Mr in (1, 16, 128, 8192):
+        bound = "tensor" if Mr >= 2048 else "hbm"
+        res[f"c5_up_M{Mr}_h12xh256"] = linear(synth.llama32_3b_up(M=Mr), f"config 5 up M={Mr}", bound)
+        res[f"c5_down_M{Mr}_h8192"] = linear(synth.llama32_3b_down(M=Mr), f"config 5 down M={Mr}", bound)
+
+    # config 4 at full size: B = 8, S = 4096 (one call moves 708.8 MB > L2)
+    kv = synth.kv_case()
+    q, k, v = (torch.from_numpy(t).to(dev) for t in (kv.q, kv.k, kv.v))
+    o = spinq.rotate_quant_kv(q, k, v)
+    kv_us = graph_us(lambda i: spinq.rotate_quant_kv(q, k, v, out=o), 1, reps=6)
+    torch.cuda.synchronize()
+    B, S, Hq, Hkv, Dd = kv.B, kv.S, kv.Hq, kv.Hkv, kv.D
+    kv_bytes = B * S * Hq * Dd * 4 + 2 * B * S * Hkv * (Dd * 2 + Dd // 2 + 8)
+    import oracle
+    sel = np.random.default_rng(3).integers(0, B * S, 64)
+    kr = kv.k.reshape(B * S, Hkv, Dd)[sel]
+    ref = oracle.rotate_quant_kv(kv.q.reshape(B * S, 1, Hq, Dd)[sel], kr[:, None], kv.v.reshape(B * S, Hkv, Dd)[sel][:, None],
+                                 kv.had)
+    got = oracle.unpack4(o.k_codes.reshape(B * S, Hkv, Dd // 2)[torch.as_tensor(sel, device=dev)].cpu().numpy(), False)
+    d = np.abs(got.reshape(-1) - ref.k_codes.reshape(-1))
+    if d.max() > 1 or np.count_nonzero(d) > max(int(1e-4 * d.size), 8):
+        raise RuntimeError("config 4: timed K codes differ from the oracle")
+    res["c4_kv_B8_S4096_Hq32_Hkv8_D128"] = {
+        "us": round(kv_us, 2), "bytes": kv_bytes, "gbs": round(kv_bytes / kv_us / 1e3, 1),
+        "frac_hbm": round(kv_bytes / kv_us / 1e3 / hbm_peak, 4),
+        "checked": f"K codes of 64 sampled tokens ({np.count_nonzero(d)} tie flips) vs oracle"}
+    del q, k, v, o
+    torch.cuda.empty_cache()
+    return res
 
 
 # --------------------------------------------------------------------------- oracle on host cores
@@ -611,27 +784,72 @@ def cpu_baseline(sample_rows=1024, threads=0):
 
 
 def run_reference(args, rank, world):
+    """The CPU oracle as it stands, on the host cores: every step runs the
+    whole path (KV rows, act quant + gate_up GEMM, R4 + act quant + down_proj
+    GEMM) on a bounded sample of `--ref-rows` tokens of the workload, and the
+    line reports that measured time.  The rate (TOPS) is the sample's ops
+    over the sample's time; nothing is projected to the full batch."""
     if rank != 0:
         return None
     rows = args.ref_rows
+    _oracle_weights()                       # offline weight quantization, not timed
     for _ in range(args.warmup):
         cpu_baseline(sample_rows=max(1, rows // 4))
+    t0 = time.perf_counter()
     vals = [cpu_baseline(sample_rows=rows) for _ in range(args.steps)]
-    v = statistics.mean(x["value"] for x in vals)
-    ms_per_step = step_ops() / (v * 1e12) * 1e3
+    wall = time.perf_counter() - t0
+    ms_per_step = wall / args.steps * 1e3
+    ops = 2.0 * rows * (N * K + N2 * K2) * args.steps
+    v = ops / wall / 1e12
     cb = dict(vals[-1])
     cb["value"] = round(v, 6)
+    cb["sample"] = (f"{rows} of the workload's {M} tokens per step through every step of the path "
+                    f"(KV rows for the same tokens, act quant + GEMM {rows}x{K}->{N}, R4 + act quant + GEMM "
+                    f"{rows}x{K2}->{N2}); {args.steps} steps in {wall:.2f} s")
     return {
         "metric": METRIC, "value": round(v, 6), "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "impl": "reference",
-        "config": {"workload": "llama3_8b MLP hot path for 2048 tokens: gate_up 4096->14336 "
-                               "+ down_proj 14336->4096 (online R4 = H28 (x) H512) + R3/KV4",
-                   "M": M, "note": "CPU oracle on a bounded token sample per step"},
+        "config": workload_config(world),
+        "sample_tokens_per_step": rows,
         "cpu_baseline": cb,
         "e2e": {"value": round(v, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
+
+
+def launch_check(args, rank, world):
+    """Start-up check of the multi-rank launch (no kernels): every rank joins
+    the process group (NCCL on GPUs, gloo on CPU) and rank 0 reports how many
+    ranks it saw."""
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dev = "cpu"
+        if backend == "nccl":
+            torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+            dev = "cuda"
+        dist.init_process_group(backend)
+        t = torch.ones(1, device=dev)
+        dist.all_reduce(t)
+        seen = int(t.item())
+        dist.destroy_process_group()
+    else:
+        seen = 1
+    return {"launch_check": True, "n_gpus": args.gpus, "world": world, "ranks_seen": seen} if rank == 0 else None
+
+
+def relaunch(args_n):
+    """`--gpus N` without a launcher: run this script under
+    torch.distributed.run with N ranks on this node and return its status."""
+    import socket
+    with socket.socket() as so:
+        so.bind(("127.0.0.1", 0))
+        port = so.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={args_n}",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__)] + sys.argv[1:]
+    return subprocess.call(cmd)
 
 
 def main():
@@ -643,13 +861,25 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=1024)
     ap.add_argument("--ref-rows", type=int, default=64, help="tokens per --impl reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the per-config full-size runs")
+    ap.add_argument("--launch-check", action="store_true",
+                    help="only start the ranks, join the process group and report them (no kernels)")
     args = ap.parse_args()
 
+    if args.gpus < 1:
+        ap.error("--gpus must be at least 1")
+    if "WORLD_SIZE" not in os.environ and args.gpus > 1:
+        sys.exit(relaunch(args.gpus))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != args.gpus:
+        print(f"bench.py: --gpus {args.gpus} but the launcher started {world} ranks", file=sys.stderr)
+        sys.exit(2)
 
-    if args.impl == "reference":
+    if args.launch_check:
+        out = launch_check(args, rank, world)
+    elif args.impl == "reference":
         out = run_reference(args, rank, world)
     else:
         import torch

@@ -6,6 +6,10 @@
  * ---------------------------------------
  * Pointers.  Every data pointer is a DEVICE pointer owned by the caller; the
  *   library never allocates, frees or keeps a pointer after the call returns.
+ *   One exception: spinq_w4a4_gemm_noalloc keeps its workspace in a fixed
+ *   device array of SPINQ_NOALLOC_SCRATCH_BYTES that the library owns (held
+ *   by every GPU that loads the library until the process exits) and caches
+ *   that array's device address per CUDA context.
  *   `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
  *   call is asynchronous: it validates its arguments on the host, enqueues
  *   kernels on `stream` and returns; it never synchronizes.
@@ -52,7 +56,9 @@ typedef enum {
   SPINQ_EINVAL = 1,
   SPINQ_EUNSUPPORTED = 2,
   SPINQ_ECUDA = 3,
-  SPINQ_ETIMEOUT = 4
+  SPINQ_ETIMEOUT = 4,
+  SPINQ_ESCRATCH = 5  /* spinq_w4a4_gemm_noalloc: the request needs more
+                         workspace than its fixed array holds */
 } spinq_status;
 
 typedef enum {
@@ -167,26 +173,34 @@ spinq_status spinq_w4a4_gemm_splitk(const uint8_t* a_codes, const float* a_scale
                                     void* y_f16, int32_t* acc_out, void* workspace,
                                     int64_t workspace_bytes, void* stream);
 
+/* Size of the fixed device array spinq_w4a4_gemm_noalloc works in (8 MiB). */
+#define SPINQ_NOALLOC_SCRATCH_BYTES (8ll << 20)
+
 /*
  * spinq_w4a4_gemm_noalloc -- spinq_w4a4_gemm_splitk for callers that cannot
- * allocate device memory where they run the layer (a serving runtime that
- * reserves its whole memory budget at start-up, a thread that must not call
- * an allocator while other streams are being captured, an embedder with no
- * allocator of its own).  The paper has no counterpart: this is an interface
- * convenience, not part of the method.
+ * allocate device memory where they run the layer: a serving runtime that
+ * reserves its whole memory budget at start-up and forbids later
+ * allocations, a thread that must not call into an allocator while other
+ * streams are being captured into CUDA graphs, an embedder with no device
+ * allocator of its own to hand a workspace from.  The paper has no
+ * counterpart: this is an interface convenience, not part of the method.
  *   Same arguments, outputs and requirements as spinq_w4a4_gemm; no workspace
- *   argument.  The workspace lives in a fixed 8 MiB device array owned by the
- *   library, which every GPU that loads the library holds until the process
- *   exits; a call whose split-K workspace (spinq_w4a4_gemm_workspace_bytes)
- *   exceeds 8 MiB does not split K (each 128-channel tile keeps its whole K
- *   range) and needs none of it.
+ *   argument.  The workspace lives in a fixed device array of
+ *   SPINQ_NOALLOC_SCRATCH_BYTES owned by the library, which every GPU that
+ *   loads the library holds until the process exits.
+ *   A request whose plan needs more workspace than that
+ *   (spinq_w4a4_gemm_workspace_bytes(M, N, K) > SPINQ_NOALLOC_SCRATCH_BYTES,
+ *   e.g. split-K decode plans with M * N * 4 above 8 MiB) is refused with
+ *   SPINQ_ESCRATCH before anything is enqueued; split the tokens into smaller
+ *   calls.  Requests whose plan needs no workspace (the GEMV, the prefill
+ *   kernels, unsliced tiles) always run.
  *   The call itself allocates nothing: no cudaMalloc/cudaFree and no
  *   allocating library routine.  It clears the part of the array it uses
  *   (cudaMemsetAsync on `stream`) before the kernel, since the array keeps
  *   the previous call's contents.
- *   The first call on each device looks up the array's device address
- *   (cudaGetSymbolAddress, with that device current); make that first call
- *   outside any stream capture.
+ *   The first call in each CUDA context looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current) and caches it for that
+ *   context; make that first call outside any stream capture.
  *   Every call shares the one array per device: calls that may overlap on the
  *   GPU (different streams without ordering between them) race on it.
  */

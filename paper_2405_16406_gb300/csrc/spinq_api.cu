@@ -46,6 +46,9 @@ const char* spinq_status_string(spinq_status s) {
     case SPINQ_EUNSUPPORTED: return "SPINQ_EUNSUPPORTED: no kernel for this configuration";
     case SPINQ_ECUDA: return "SPINQ_ECUDA: CUDA launch or runtime error";
     case SPINQ_ETIMEOUT: return "SPINQ_ETIMEOUT: a bounded device wait gave up";
+    case SPINQ_ESCRATCH:
+      return "SPINQ_ESCRATCH: the request needs more workspace than the no-allocation entry point's "
+             "fixed array holds";
   }
   return "SPINQ: unknown status";
 }

@@ -11,8 +11,11 @@
 //
 // The scratch is the static array below (kNoAllocScratchBytes); every GPU
 // that loads the library holds it until the process exits.  Host code cannot
-// use the array's name as a device address, so the address is looked up once
-// per device, with that device current, through cudaGetSymbolAddress.
+// use the array's name as a device address, so the address is looked up with
+// cudaGetSymbolAddress, with the device current, on the first call in each
+// CUDA context (a context destroyed by cudaDeviceReset and created again
+// loads the module again, so the address is looked up again).
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -22,28 +25,57 @@
 
 namespace {
 
-constexpr int64_t kNoAllocScratchBytes = int64_t(8) << 20;   // 8 MiB
+constexpr int64_t kNoAllocScratchBytes = SPINQ_NOALLOC_SCRATCH_BYTES;   // 8 MiB
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-std::mutex g_scratch_mu;
-void* g_scratch_addr[64] = {nullptr};
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
 
-// Device address of g_noalloc_scratch on the current device (looked up on the
-// first call for that device).
+// cuCtxGetCurrent through the runtime's driver entry-point query (the
+// library does not link against libcuda); null if the driver lacks it.
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  });
+  return fn;
+}
+
+struct ScratchSlot {
+  CUcontext ctx;
+  void* addr;
+};
+
+std::mutex g_scratch_mu;
+ScratchSlot g_scratch[64] = {};
+
+// Device address of g_noalloc_scratch in the current device's context.
 cudaError_t scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  CtxGetCurrentFn get = ctx_get_current();
+  if (!get) return cudaErrorDeviceUninitialized;
+  CUcontext ctx = nullptr;
+  if (get(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (g_scratch_addr[dev] == nullptr) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
+  if (ctx != nullptr && g_scratch[dev].addr != nullptr && g_scratch[dev].ctx == ctx) {
+    *out = g_scratch[dev].addr;
+    return cudaSuccess;
   }
-  *out = g_scratch_addr[dev];
+  // first call in this context (or no context yet on this thread: the
+  // lookup makes the device's primary context current)
+  void* p = nullptr;
+  if ((e = cudaGetSymbolAddress(&p, g_noalloc_scratch)) != cudaSuccess) return e;
+  if (get(&ctx) != CUDA_SUCCESS || ctx == nullptr) return cudaErrorDeviceUninitialized;
+  g_scratch[dev] = ScratchSlot{ctx, p};
+  *out = p;
   return cudaSuccess;
 }
 
@@ -65,10 +97,10 @@ extern "C" spinq_status spinq_w4a4_gemm_noalloc(const uint8_t* a_codes, const fl
     return SPINQ_EINVAL;
   if (K > 65536 || M > INT32_MAX || N > INT32_MAX) return SPINQ_EUNSUPPORTED;
   if (M == 0 || N == 0) return SPINQ_OK;
-  // a split whose partial sums do not fit the scratch is not taken: the
-  // tiles then keep their whole K range
-  int64_t need = spinq::w4a4_gemm_workspace_bytes(M, N, K);
-  if (need > kNoAllocScratchBytes) need = 0;
+  // the scratch this request needs under the current plan (0 when its plan
+  // does not split K); a request beyond the fixed array is refused
+  const int64_t need = spinq::w4a4_gemm_workspace_bytes(M, N, K);
+  if (need > kNoAllocScratchBytes) return SPINQ_ESCRATCH;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   void* ws = nullptr;
   if (need > 0) {

@@ -46,7 +46,7 @@ def test_binding_names_match_header(lib):
 
 def test_status_strings(lib):
     from paper_2405_16406_gb300 import spinq
-    for s in range(5):
+    for s in range(6):
         assert spinq.spinq_status_string(s).startswith("SPINQ_")
     assert "sm_103a" in spinq.spinq_version()
 
@@ -127,3 +127,26 @@ def test_gemm_controls_validate_on_the_host(lib):
         assert S.spinq_w4a4_gemm_plan(M, N, K) == -1
         assert S.spinq_w4a4_gemm_splitk_plan(M, N, K) == (-1, 0)
     assert S.spinq_w4a4_gemm_splitk_plan(16, 256, 65536 + 128) == (-1, 0)   # K above the exact-accumulator bound
+
+
+def test_noalloc_rejects_invalid_arguments_on_the_host(lib):
+    """spinq_w4a4_gemm_noalloc validates its arguments like spinq_w4a4_gemm
+    before any device work: null pointers, K % 128, N % 16, misalignment and
+    K above the exact-accumulator bound."""
+    from paper_2405_16406_gb300 import spinq as S
+    fake = ctypes.c_void_p(1 << 20)
+    odd = ctypes.c_void_p((1 << 20) + 4)
+    f = S.spinq_w4a4_gemm_noalloc
+    assert f(None, fake, None, fake, fake, fake, 4, 32, 128, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, None, fake, fake, 4, 32, 128, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, fake, fake, fake, 4, 32, 128, None, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, fake, fake, fake, 4, 32, 96, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, fake, fake, fake, 4, 40, 128, fake, None, None) == S.SPINQ_EINVAL
+    assert f(odd, fake, None, fake, fake, fake, 4, 32, 128, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, fake, fake, odd, 4, 32, 128, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, fake, fake, fake, 4, 32, 128, fake, odd, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, fake, fake, fake, -1, 32, 128, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, None, fake, fake, fake, 4, 32, 65536 + 128, fake, None, None) == S.SPINQ_EUNSUPPORTED
+    # empty problems succeed without a launch
+    assert f(fake, fake, None, fake, fake, fake, 0, 32, 128, fake, None, None) == S.SPINQ_OK
+    assert "workspace" in S.spinq_status_string(S.SPINQ_ESCRATCH)
