@@ -235,76 +235,116 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
 }
 
 // ------------------------------------------------------------------------
-// quantizer only (no online rotation): W warps per row, up to 8 chunks a lane
+// quantizer only (no online rotation): one CTA of W warps per row.  Every
+// lane loads its (up to kNoRotCPT) 16-byte chunks straight into registers with
+// streaming loads issued back to back, so a whole row is in flight at once
+// and, with every CTA of the grid resident, so is the whole matrix.  The row
+// range is taken on the fp16 values themselves (max and min of fp16 numbers
+// are exact, and equal the range of their fp32 values); then the tensor core
+// widens each chunk to fp32 exactly (B = I16) for Eq. 1.
 // ------------------------------------------------------------------------
-constexpr int kNoRotV = 8;
+constexpr int kNoRotCPT = 8;   // chunks per lane
 
-constexpr int kNoRotStages = 2;
+__device__ __forceinline__ uint4 ld_stream_v4(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
 
-template <bool SYM, bool CLAMP, int W>
-__global__ void __launch_bounds__(32 * W) rq_norot_kernel(RotQuantArgs a) {
-  extern __shared__ __align__(128) uint8_t smem[];
-  const uint32_t row_bytes = (uint32_t)(a.K * 2);
-  const uint32_t stage_bytes = (row_bytes + 127u) & ~127u;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kNoRotStages * stage_bytes);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + kNoRotStages);
-  float* red = reinterpret_cast<float*>(smem + kNoRotStages * stage_bytes + kNoRotStages * 8 + 16);
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+__device__ __forceinline__ uint32_t h2_absmax(uint32_t m, uint32_t x) {
+  uint32_t r;
+  asm("{\n .reg .b32 t;\n abs.f16x2 t, %2;\n max.f16x2 %0, %1, t;\n}\n" : "=r"(r) : "r"(m), "r"(x));
+  return r;
+}
+__device__ __forceinline__ uint32_t h2_max(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ uint32_t h2_min(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("min.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ float h2_hi_lo_max(uint32_t v) {
+  const __half2 h = *reinterpret_cast<const __half2*>(&v);
+  return fmaxf(__low2float(h), __high2float(h));
+}
+__device__ __forceinline__ float h2_hi_lo_min(uint32_t v) {
+  const __half2 h = *reinterpret_cast<const __half2*>(&v);
+  return fminf(__low2float(h), __high2float(h));
+}
+
+template <bool SYM, bool CLAMP>
+__global__ void __launch_bounds__(512) rq_norot_kernel(RotQuantArgs a) {
+  __shared__ float red[2 * 16];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5, W = (int)(blockDim.x >> 5);
+  const int64_t row = blockIdx.x;
+  const int nchunk = (int)(a.K / 8);
   uint32_t bi[2][2];
   make_b16(bi, false);
-  const int nchunk = (int)(a.K / 8);
-
-  int* release_count = const_cast<int*>(abort_flag) + 1;
-  RowStream<kNoRotStages> rs{smem, stage_bytes, bars, reinterpret_cast<const uint8_t*>(a.x), a.ldx * 2,
-                             row_bytes, 1u, 0u, a.rows, (int64_t)blockIdx.x, (int64_t)gridDim.x};
-  rs.init();
-  if (tid == 0) {
-    *abort_flag = 0;
-    *release_count = 0;
-    fence_mbar_init();
-  }
-  __syncthreads();
   pdl_wait();
   pdl_trigger();
-  rs.prologue();
-
-  int it = 0;
-  for (int64_t row = blockIdx.x; row < a.rows; row += gridDim.x, ++it) {
-    rs.wait(it, abort_flag, kRowWaitLimitNs);
-    __syncthreads();
-    if (*abort_flag) break;
-    const uint4* src = reinterpret_cast<const uint4*>(rs.stage(it));
-    F2 y[kNoRotV][4];
+  const uint8_t* src = reinterpret_cast<const uint8_t*>(a.x) + row * a.ldx * 2;
+  uint4 c[kNoRotCPT];
 #pragma unroll
-    for (int v = 0; v < kNoRotV; ++v) {
-      const int ch = lane + 32 * (w + W * v);
-      chunk_mma(ch < nchunk ? src[ch] : make_uint4(0, 0, 0, 0), bi, y[v]);  // exact fp16 -> fp32
-    }
-    rs.release_warp(it, release_count, W);
-    Range<SYM> r;
-#pragma unroll
-    for (int v = 0; v < kNoRotV; ++v)
-      if (lane + 32 * (w + W * v) < nchunk)
-#pragma unroll
-        for (int q = 0; q < 4; ++q) r.add_pair(y[v][q]);
-    block_range<SYM, W>(r, red);
-    const QParams<SYM> qp(r, a.clip);
-    uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
-#pragma unroll
-    for (int v = 0; v < kNoRotV; ++v) {
-      const int ch = lane + 32 * (w + W * v);
-      uint32_t rb[8];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) qp.template code_bits2<CLAMP>(y[v][q], rb[2 * q], rb[2 * q + 1]);
-      if (ch < nchunk) out[ch] = pack8_nibbles(rb);
-    }
-    if (tid == 0) {
-      a.scale[row] = qp.alpha * a.norm;
-      if (!SYM) a.zero[row] = qp.beta * a.norm;
-    }
-    if (W > 1) __syncthreads();
+  for (int v = 0; v < kNoRotCPT; ++v) {
+    const int ch = lane + 32 * (w + W * v);
+    c[v] = ch < nchunk ? ld_stream_v4(src + (size_t)ch * 16) : make_uint4(0, 0, 0, 0);
   }
-  if (*abort_flag) rs.drain(it, kRowWaitLimitNs);
+  // row range on the fp16 values: +-inf start values for the asymmetric
+  // form, absolute values from 0 for the symmetric one
+  uint32_t hi2 = SYM ? 0u : 0xFC00FC00u, lo2 = 0x7C007C00u;
+#pragma unroll
+  for (int v = 0; v < kNoRotCPT; ++v) {
+    if (lane + 32 * (w + W * v) < nchunk) {
+      const uint32_t q[4] = {c[v].x, c[v].y, c[v].z, c[v].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (SYM) {
+          hi2 = h2_absmax(hi2, q[e]);
+        } else {
+          hi2 = h2_max(hi2, q[e]);
+          lo2 = h2_min(lo2, q[e]);
+        }
+      }
+    }
+  }
+  Range<SYM> r;
+  r.hi = h2_hi_lo_max(hi2);
+  if (!SYM) r.lo = h2_hi_lo_min(lo2);
+  r.warp_reduce();
+  if (W > 1) {
+    if (lane == 0) {
+      red[w] = r.hi;
+      red[16 + w] = r.lo;
+    }
+    __syncthreads();
+    r.hi = red[0];
+    r.lo = red[16];
+    for (int i = 1; i < W; ++i) {
+      r.hi = fmaxf(r.hi, red[i]);
+      if (!SYM) r.lo = fminf(r.lo, red[16 + i]);
+    }
+  }
+  const QParams<SYM> qp(r, a.clip);
+  uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
+#pragma unroll
+  for (int v = 0; v < kNoRotCPT; ++v) {
+    const int ch = lane + 32 * (w + W * v);
+    F2 y[4];
+    chunk_mma(c[v], bi, y);   // exact fp16 -> fp32 (all lanes take part)
+    uint32_t rb[8];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) qp.template code_bits2<CLAMP>(y[q], rb[2 * q], rb[2 * q + 1]);
+    if (ch < nchunk) out[ch] = pack8_nibbles(rb);
+  }
+  if (tid == 0) {
+    a.scale[row] = qp.alpha * a.norm;
+    if (!SYM) a.zero[row] = qp.beta * a.norm;
+  }
 }
 
 template <typename Kern>
@@ -343,16 +383,19 @@ cudaError_t launch_pow2_for(const RotQuantArgs& a, cudaStream_t stream, bool* ha
 template <bool SYM, bool CLAMP>
 cudaError_t launch_norot_for(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
   const int64_t nchunk = a.K / 8;
-  const int64_t warps = (nchunk + 32 * kNoRotV - 1) / (32 * kNoRotV);
-  const size_t smem = kNoRotStages * (((size_t)a.K * 2 + 127) & ~(size_t)127) + kNoRotStages * 8 + 16 + 2 * 16 * 4;
-  *handled = true;
-  if (warps <= 1) return launch_rows(rq_norot_kernel<SYM, CLAMP, 1>, 32, smem, a, stream);
-  if (warps <= 2) return launch_rows(rq_norot_kernel<SYM, CLAMP, 2>, 64, smem, a, stream);
-  if (warps <= 4) return launch_rows(rq_norot_kernel<SYM, CLAMP, 4>, 128, smem, a, stream);
-  if (warps <= 8) return launch_rows(rq_norot_kernel<SYM, CLAMP, 8>, 256, smem, a, stream);
-  if (warps <= 16) return launch_rows(rq_norot_kernel<SYM, CLAMP, 16>, 512, smem, a, stream);
-  *handled = false;
-  return cudaSuccess;
+  const int64_t warps = (nchunk + 32 * kNoRotCPT - 1) / (32 * kNoRotCPT);
+  *handled = warps <= 16;
+  if (!*handled) return cudaSuccess;
+  // one CTA per row, no persistence: every row's loads are in flight at once
+  // when the grid is resident (2048 rows of 4096 need 2048 CTAs of 64 threads)
+  auto kern = rq_norot_kernel<SYM, CLAMP>;
+  const int threads = (int)(32 * warps);
+  int per_sm = 0;
+  cudaError_t e = prepare_launch(kern, threads, 0, &per_sm);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(kern, dim3((unsigned)a.rows), dim3(threads), 0, stream, 1, a);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
 }
 
 }  // namespace
