@@ -81,6 +81,8 @@ def _load():
         "oracle_w4a4_gemm": (i32, [P, P, P, P, P, i64, i64, i64, P, P]),
         "oracle_w4a4_gemm_sampled": (i32, [P, P, P, P, P, i64, P, P, i64, P, P]),
         "oracle_rowsum": (None, [P, i64, i64, P]),
+        "oracle_cayley_y": (i32, [P, P, i64, P]),
+        "oracle_cayley_step": (i32, [P, P, i64, i64, dbl, i32, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -336,3 +338,48 @@ def rotate_quant_kv(q_f16: np.ndarray, k_f16: np.ndarray, v_f16: np.ndarray,
                    kc.reshape(B, S, Hkv, D), ka.reshape(sh), kb.reshape(sh),
                    vc.reshape(B, S, Hkv, D), va.reshape(sh), vb.reshape(sh),
                    kr.reshape(B, S, Hkv, D))
+
+
+# --------------------------------------------------------------------------
+# Cayley SGD step (Sec. 3.2)
+# --------------------------------------------------------------------------
+def cayley_y(R: np.ndarray, G: np.ndarray) -> np.ndarray:
+    """Y = G_hat - G_hat^T with G_hat = G R^T - 1/2 R R^T G R^T (Sec. 3.2)."""
+    R = _c(R, np.float64)
+    G = _c(G, np.float64)
+    n = R.shape[-1]
+    Y = np.empty((n, n), dtype=np.float64)
+    _check(_load().oracle_cayley_y(_ptr(R), _ptr(G), n, _ptr(Y)), "cayley_y")
+    return Y
+
+
+def cayley_step(R: np.ndarray, G: np.ndarray, alpha: float, iters: int = 2
+                ) -> Tuple[np.ndarray, np.ndarray]:
+    """One Cayley SGD update of each rotation in a batch [B, n, n] (or one
+    [n, n]) by the fixed-point iteration: R'_0 = R + a Y R, then
+    R'_{k+1} = R + (a/2) Y (R + R'_k), ``iters`` times.  ``G`` is the loss
+    gradient; Y is built from -G (the descent reading of the printed update:
+    the cited Cayley SGD forms G_hat from the negative gradient).  Returns
+    (R', Y)."""
+    R = _c(R, np.float64)
+    G = _c(G, np.float64)
+    single = R.ndim == 2
+    Rb = R[None] if single else R
+    Gb = G[None] if single else G
+    B, n = Rb.shape[0], Rb.shape[-1]
+    out = np.empty_like(Rb)
+    Y = np.empty_like(Rb)
+    _check(_load().oracle_cayley_step(_ptr(Rb), _ptr(Gb), B, n, float(alpha), int(iters), _ptr(out), _ptr(Y)),
+           "cayley_step")
+    return (out[0], Y[0]) if single else (out, Y)
+
+
+def cayley_exact(R: np.ndarray, G: np.ndarray, alpha: float) -> np.ndarray:
+    """The Cayley update by its definition, R' = (I - a/2 Y)^-1 (I + a/2 Y) R
+    with Y built from -G, through a library linear solve (the fixed point of
+    ``cayley_step``)."""
+    R = np.asarray(R, dtype=np.float64)
+    n = R.shape[-1]
+    Y = cayley_y(R, -np.asarray(G, dtype=np.float64))
+    eye = np.eye(n)
+    return np.linalg.solve(eye - 0.5 * alpha * Y, (eye + 0.5 * alpha * Y) @ R)

@@ -420,3 +420,89 @@ void oracle_rowsum(const int32_t* codes, int64_t rows, int64_t K, int32_t* rowsu
     rowsum[r] = (int32_t)s;
   }
 }
+
+/* ------------------------------------------------------------------ */
+/* Cayley SGD step (Sec. 3.2)                                          */
+/* ------------------------------------------------------------------ */
+/* C = op(A) op(B) for n x n row-major matrices, op = transpose when the
+ * flag is set; the plain triple loop in double. */
+static void mat_mul(const double* A, int ta, const double* B, int tb, int64_t n, double* C) {
+  for (int64_t i = 0; i < n; ++i)
+    for (int64_t j = 0; j < n; ++j) {
+      double s = 0.0;
+      for (int64_t k = 0; k < n; ++k) {
+        const double a = ta ? A[k * n + i] : A[i * n + k];
+        const double b = tb ? B[j * n + k] : B[k * n + j];
+        s += a * b;
+      }
+      C[i * n + j] = s;
+    }
+}
+
+/* Y of Sec. 3.2 for one rotation R and the loss gradient G:
+ *   G_hat = G R^T - 1/2 R R^T G R^T,   Y = G_hat - G_hat^T. */
+int oracle_cayley_y(const double* R, const double* G, int64_t n, double* Y) {
+  if (n <= 0) return OR_EINVAL;
+  double* GRt = (double*)malloc(sizeof(double) * n * n);
+  double* RtGRt = (double*)malloc(sizeof(double) * n * n);
+  double* RRtGRt = (double*)malloc(sizeof(double) * n * n);
+  double* Gh = (double*)malloc(sizeof(double) * n * n);
+  if (!GRt || !RtGRt || !RRtGRt || !Gh) {
+    free(GRt), free(RtGRt), free(RRtGRt), free(Gh);
+    return OR_EINVAL;
+  }
+  mat_mul(G, 0, R, 1, n, GRt);         /* G R^T           */
+  mat_mul(R, 1, GRt, 0, n, RtGRt);     /* R^T G R^T       */
+  mat_mul(R, 0, RtGRt, 0, n, RRtGRt);  /* R R^T G R^T     */
+  for (int64_t e = 0; e < n * n; ++e) Gh[e] = GRt[e] - 0.5 * RRtGRt[e];
+  for (int64_t i = 0; i < n; ++i)
+    for (int64_t j = 0; j < n; ++j) Y[i * n + j] = Gh[i * n + j] - Gh[j * n + i];
+  free(GRt), free(RtGRt), free(RRtGRt), free(Gh);
+  return OR_OK;
+}
+
+/* R' of Sec. 3.2, R' = (I - a/2 Y)^-1 (I + a/2 Y) R, by the fixed-point
+ * iteration the paper cites for it (Cayley SGD):
+ *   R'_0 = R + a Y R,   R'_{k+1} = R + (a/2) Y (R + R'_k),  k = 0 .. iters-1,
+ * whose fixed point solves (I - a/2 Y) R' = (I + a/2 Y) R.
+ * Reading of the sign: the objective is an argmin, and the cited Cayley SGD
+ * forms G_hat from the negative gradient (its momentum buffer accumulates
+ * -grad); with G = +grad the printed update would climb the loss.  So `grad`
+ * here is the loss gradient and Y is built from G = -grad.
+ * A batch of independent (R, grad) pairs; Y_out (may be NULL) receives each Y. */
+int oracle_cayley_step(const double* R, const double* grad, int64_t batch, int64_t n, double alpha, int iters,
+                       double* R_out, double* Y_out) {
+  if (n <= 0 || batch < 0 || iters < 0) return OR_EINVAL;
+  int err = 0;
+#pragma omp parallel for schedule(dynamic)
+  for (int64_t b = 0; b < batch; ++b) {
+    const double* Rb = R + b * n * n;
+    double* Y = (double*)malloc(sizeof(double) * n * n);
+    double* T = (double*)malloc(sizeof(double) * n * n);
+    double* P = (double*)malloc(sizeof(double) * n * n);
+    if (!Y || !T || !P) {
+#pragma omp atomic write
+      err = 1;
+      free(Y), free(T), free(P);
+      continue;
+    }
+    for (int64_t e = 0; e < n * n; ++e) T[e] = -grad[b * n * n + e]; /* G = -grad */
+    if (oracle_cayley_y(Rb, T, n, Y) != OR_OK) {
+#pragma omp atomic write
+      err = 1;
+      free(Y), free(T), free(P);
+      continue;
+    }
+    mat_mul(Y, 0, Rb, 0, n, T); /* Y R */
+    for (int64_t e = 0; e < n * n; ++e) P[e] = Rb[e] + alpha * T[e];
+    for (int k = 0; k < iters; ++k) {
+      for (int64_t e = 0; e < n * n; ++e) P[e] = Rb[e] + P[e]; /* R + R'_k */
+      mat_mul(Y, 0, P, 0, n, T);                               /* Y (R + R'_k) */
+      for (int64_t e = 0; e < n * n; ++e) P[e] = Rb[e] + 0.5 * alpha * T[e];
+    }
+    memcpy(R_out + b * n * n, P, sizeof(double) * n * n);
+    if (Y_out) memcpy(Y_out + b * n * n, Y, sizeof(double) * n * n);
+    free(Y), free(T), free(P);
+  }
+  return err ? OR_EINVAL : OR_OK;
+}
