@@ -736,7 +736,44 @@ def run_configs(dev, hbm_peak, fp8_peak):
         "checked": f"K codes of 64 sampled tokens ({np.count_nonzero(d)} tie flips) vs oracle"}
     del q, k, v, o
     torch.cuda.empty_cache()
+    res.update(cayley_records(dev))
     return res
+
+
+def cayley_records(dev):
+    """Cayley SGD step (Sec. 3.2) on batches of head_dim x head_dim rotations:
+    32 (one R2 per layer of a 32-layer model) and 152 (one per SM).  Bound by
+    fp32 FMA issue: (4 + iters) n x n products, 2 n^3 flops each, against
+    the fp32 peak 152 SMs x 128 FMA/clk x 2 flops x 2.07 GHz = 80.5 TFLOP/s."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2405_16406_gb300 import spinq
+    out = {}
+    n, iters = 128, 2
+    peak = 152 * 128 * 2 * 2.07e9 / 1e12
+    for batch in (32, 152):
+        rng = np.random.default_rng(batch)
+        R = np.stack([np.linalg.qr(rng.standard_normal((n, n)))[0] for _ in range(batch)]).astype(np.float32)
+        g = (0.5 * rng.standard_normal((batch, n, n))).astype(np.float32)
+        alpha = 0.01
+        Rt, gt = torch.from_numpy(R).to(dev), torch.from_numpy(g).to(dev)
+        outs = [torch.empty_like(Rt) for _ in range(2)]
+        us = graph_us(lambda i: spinq.cayley_step(Rt, gt, alpha, iters, out=outs[i]), 2)
+        torch.cuda.synchronize()
+        ref, _ = oracle.cayley_step(R[:2].astype(np.float64), g[:2].astype(np.float64), alpha, iters)
+        err = float(np.abs(outs[0][:2].cpu().numpy() - ref).max())
+        if err > 5e-5:
+            raise RuntimeError(f"Cayley step: timed output differs from the oracle by {err}")
+        flops = batch * (4 + iters) * 2.0 * n ** 3
+        tf = flops / us / 1e6
+        out[f"f4_cayley_step_{batch}x{n}x{n}_iters{iters}"] = {
+            "us": round(us, 2), "tflops": round(tf, 2), "bound": "alu (fp32 FMA)",
+            "peak_tflops": round(peak, 1), "frac": round(tf / peak, 4),
+            "frac_of_used_sms": round(tf / (peak * min(batch, 152) / 152), 4),
+            "checked": f"2 rotations vs oracle, max abs diff {err:.1e}"}
+    return out
 
 
 # --------------------------------------------------------------------------- oracle on host cores

@@ -288,6 +288,30 @@ int spinq_w4a4_gemm_plan(int64_t M, int64_t N, int64_t K);
  */
 int spinq_w4a4_gemm_splitk_plan(int64_t M, int64_t N, int64_t K, int* nsplit);
 
+/*
+ * spinq_cayley_step -- one Cayley SGD update of a batch of rotations
+ * (Sec. 3.2, the R' update and its Y / G_hat definitions), for learning R2
+ * (head_dim x head_dim, one per layer) with the weights frozen:
+ *   G_hat = G R^T - 1/2 R R^T G R^T,   Y = G_hat - G_hat^T,
+ *   R'    = (I - alpha/2 Y)^-1 (I + alpha/2 Y) R,
+ * computed, as the paper does, by the fixed-point iteration of Cayley SGD:
+ *   R'_0 = R + alpha Y R,   R'_{k+1} = R + (alpha/2) Y (R + R'_k),
+ *   k = 0 .. iters-1 (it converges to R' when |alpha Y / 2| < 1).
+ * G is the NEGATIVE of the loss gradient `grad` passed here: the objective
+ * is an argmin and the cited Cayley SGD forms G_hat from the negative
+ * gradient (with G = +grad the printed update would climb the loss).
+ *   R      [batch][n][n] fp32 row-major, each orthonormal (device).
+ *   grad   [batch][n][n] fp32, dL/dR (device).
+ *   alpha  learning rate (finite); iters in 0 .. 64.
+ *   R_out  [batch][n][n] fp32; may be R itself (in-place update), must not
+ *          overlap R or grad otherwise.
+ *   Y_out  [batch][n][n] fp32 or NULL: the skew-symmetric Y of each update.
+ *   Supported n: 16, 32, 64, 128.  Pointers 16-byte aligned.  Arithmetic in
+ *   fp32 (the oracle works in double).
+ */
+spinq_status spinq_cayley_step(const float* R, const float* grad, int64_t batch, int64_t n, float alpha,
+                               int32_t iters, float* R_out, float* Y_out, void* stream);
+
 /* Human-readable name of a status code (static storage). */
 const char* spinq_status_string(spinq_status s);
 

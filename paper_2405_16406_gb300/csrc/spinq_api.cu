@@ -192,6 +192,19 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
   return from_cuda(launch_rotate_quant_kv(a, static_cast<cudaStream_t>(stream)));
 }
 
+spinq_status spinq_cayley_step(const float* R, const float* grad, int64_t batch, int64_t n, float alpha,
+                               int32_t iters, float* R_out, float* Y_out, void* stream) {
+  if (batch < 0 || n <= 0 || iters < 0 || iters > 64 || !std::isfinite(alpha)) return SPINQ_EINVAL;
+  if (batch > 0 && (!R || !grad || !R_out)) return SPINQ_EINVAL;
+  for (const void* p : {(const void*)R, (const void*)grad, (const void*)R_out, (const void*)Y_out})
+    if (p && !aligned16(p)) return SPINQ_EINVAL;
+  if (n != 16 && n != 32 && n != 64 && n != 128) return SPINQ_EUNSUPPORTED;
+  if (batch > INT32_MAX) return SPINQ_EUNSUPPORTED;
+  if (batch == 0) return SPINQ_OK;
+  CayleyArgs a{R, grad, batch, (int)n, alpha, (int)iters, R_out, Y_out};
+  return from_cuda(launch_cayley_step(a, static_cast<cudaStream_t>(stream)));
+}
+
 int spinq_gemm_select_kernel(int kernel) { return w4a4_gemm_select(kernel); }
 
 int spinq_gemm_split_k(int n) { return w4a4_gemm_split_k(n); }

@@ -111,6 +111,21 @@ cudaError_t launch_w4a4_gemv(const GemmArgs& a, cudaStream_t stream, bool* handl
 cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, int64_t workspace_bytes,
                                     cudaStream_t stream);
 
+struct CayleyArgs {
+  const float* R;     // [batch][n][n]
+  const float* grad;  // [batch][n][n] loss gradient
+  int64_t batch;
+  int n;
+  float alpha;
+  int iters;
+  float* R_out;       // [batch][n][n]
+  float* Y_out;       // [batch][n][n] or nullptr
+};
+
+// One Cayley SGD step per rotation (n in {16, 32, 64, 128}); returns
+// cudaErrorNotSupported for other n.
+cudaError_t launch_cayley_step(const CayleyArgs& a, cudaStream_t stream);
+
 // Device status word written by bounded waits that gave up.
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail);
 // Its device address (two ints: code, wait site), for kernels in other

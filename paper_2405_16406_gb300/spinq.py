@@ -37,7 +37,7 @@ EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",
     "spinq_status_string", "spinq_device_status", "spinq_version", "spinq_w4a4_gemm_workspace_bytes",
     "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel", "spinq_gemm_split_k",
-    "spinq_w4a4_gemm_plan", "spinq_w4a4_gemm_splitk_plan",
+    "spinq_w4a4_gemm_plan", "spinq_w4a4_gemm_splitk_plan", "spinq_cayley_step",
 )
 
 
@@ -87,6 +87,8 @@ _lib.spinq_w4a4_gemm_plan.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_plan.argtypes = [_I64, _I64, _I64]
 _lib.spinq_w4a4_gemm_splitk_plan.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_splitk_plan.argtypes = [_I64, _I64, _I64, ctypes.POINTER(ctypes.c_int)]
+_lib.spinq_cayley_step.restype = ctypes.c_int
+_lib.spinq_cayley_step.argtypes = [_P, _P, _I64, _I64, ctypes.c_float, ctypes.c_int32, _P, _P, _P]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
 _lib.spinq_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
                                        ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
@@ -132,6 +134,10 @@ def spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k
                           k_zero, v_codes, v_scale, v_zero, stream) -> int:
     return _lib.spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k_codes,
                                       k_scale, k_zero, v_codes, v_scale, v_zero, stream)
+
+
+def spinq_cayley_step(R, grad, batch, n, alpha, iters, R_out, Y_out, stream) -> int:
+    return _lib.spinq_cayley_step(R, grad, batch, n, alpha, iters, R_out, Y_out, stream)
 
 
 def spinq_gemm_select_kernel(kernel: int) -> int:
@@ -303,3 +309,18 @@ def rotate_quant_kv(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, clip: flo
                                       _ptr(out.v_scale), _ptr(out.v_zero), _stream(stream)),
            "spinq_rotate_quant_kv")
     return out
+
+
+def cayley_step(R: torch.Tensor, grad: torch.Tensor, alpha: float, iters: int = 2, out: Optional[torch.Tensor] = None,
+                want_y: bool = False, stream: Optional[torch.cuda.Stream] = None):
+    """One Cayley SGD update of rotations R [B, n, n] (or [n, n]) with loss
+    gradient ``grad`` (fp32, device); returns R' (and Y when ``want_y``)."""
+    assert R.dtype == torch.float32 and grad.dtype == torch.float32 and R.is_contiguous() and grad.is_contiguous()
+    n = R.shape[-1]
+    batch = R.numel() // (n * n)
+    if out is None:
+        out = torch.empty_like(R)
+    y = torch.empty_like(R) if want_y else None
+    _check(_lib.spinq_cayley_step(_ptr(R), _ptr(grad), batch, n, float(alpha), int(iters), _ptr(out), _ptr(y),
+                                  _stream(stream)), "spinq_cayley_step")
+    return (out, y) if want_y else out

@@ -150,3 +150,17 @@ def test_noalloc_rejects_invalid_arguments_on_the_host(lib):
     # empty problems succeed without a launch
     assert f(fake, fake, None, fake, fake, fake, 0, 32, 128, fake, None, None) == S.SPINQ_OK
     assert "workspace" in S.spinq_status_string(S.SPINQ_ESCRATCH)
+
+
+def test_cayley_step_rejects_invalid_arguments_on_the_host(lib):
+    from paper_2405_16406_gb300 import spinq as S
+    fake = ctypes.c_void_p(1 << 20)
+    f = S.spinq_cayley_step
+    assert f(None, fake, 2, 128, 0.1, 2, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, 2, 128, 0.1, -1, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, 2, 128, 0.1, 65, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, 2, 128, float("nan"), 2, fake, None, None) == S.SPINQ_EINVAL
+    assert f(ctypes.c_void_p((1 << 20) + 4), fake, 2, 128, 0.1, 2, fake, None, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, 2, 96, 0.1, 2, fake, None, None) == S.SPINQ_EUNSUPPORTED
+    assert f(fake, fake, 2, 256, 0.1, 2, fake, None, None) == S.SPINQ_EUNSUPPORTED
+    assert f(fake, fake, 0, 128, 0.1, 2, fake, None, None) == S.SPINQ_OK
