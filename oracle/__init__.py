@@ -82,6 +82,12 @@ def _load():
         "oracle_w4a4_gemm_sampled": (i32, [P, P, P, P, P, i64, P, P, i64, P, P]),
         "oracle_rowsum": (None, [P, i64, i64, P]),
         "oracle_cayley_y": (i32, [P, P, i64, P]),
+        "oracle_e4m3_to_double": (dbl, [ctypes.c_uint8]),
+        "oracle_double_to_e4m3": (ctypes.c_uint8, [dbl]),
+        "oracle_e4m3_array_to_double": (None, [P, P, i64]),
+        "oracle_quantize_rows_e4m3": (i32, [P, i64, i64, dbl, P, P]),
+        "oracle_w4a8_gemm": (i32, [P, P, P, P, P, i64, i64, i64, P, P]),
+        "oracle_fp8_gemm": (i32, [P, P, P, P, i64, i64, i64, P]),
         "oracle_cayley_step": (i32, [P, P, i64, i64, dbl, i32, P, P]),
     }
     for name, (res, args) in sig.items():
@@ -383,3 +389,79 @@ def cayley_exact(R: np.ndarray, G: np.ndarray, alpha: float) -> np.ndarray:
     Y = cayley_y(R, -np.asarray(G, dtype=np.float64))
     eye = np.eye(n)
     return np.linalg.solve(eye - 0.5 * alpha * Y, (eye + 0.5 * alpha * Y) @ R)
+
+
+# --------------------------------------------------------------------------
+# 8-bit variants: W4A8 and W-fp8-A-fp8 (main results table, 4-8-x rows;
+# appendix "Latency measurement on GPU", FP8 GEMM setting)
+# --------------------------------------------------------------------------
+def e4m3_to_f64(b: np.ndarray) -> np.ndarray:
+    """Decode E4M3 bytes (finite-only FP8: bias 7, 3 mantissa bits, max 448)."""
+    b = _c(b, np.uint8)
+    out = np.empty(b.shape, dtype=np.float64)
+    _load().oracle_e4m3_array_to_double(_ptr(b), _ptr(out), b.size)
+    return out
+
+
+def f64_to_e4m3(x: np.ndarray) -> np.ndarray:
+    """Round to the nearest E4M3 value (ties to even), saturating at +-448."""
+    lib = _load()
+    x = np.asarray(x, dtype=np.float64)
+    return np.array([lib.oracle_double_to_e4m3(float(v)) for v in x.reshape(-1)], dtype=np.uint8).reshape(x.shape)
+
+
+@dataclass
+class QuantActFP8:
+    codes: np.ndarray    # uint8 E4M3 [M, K]
+    alpha: np.ndarray    # f64 [M]
+    rotated: np.ndarray  # f64 [M, K]
+
+
+def rotate_quant_act_fp8(x_f16: np.ndarray, had: Optional[Tuple[int, int]], clip: float = 1.0) -> QuantActFP8:
+    """Sec. 3.1 rotation (skipped when ``had`` is None), then per-token FP8:
+    alpha = clip max|x'| / 448, code = E4M3(x' / alpha)."""
+    x = f16_to_f64(x_f16)
+    xr = rotate(x, had[0], had[1]) if had is not None else x
+    xr = _c(xr, np.float64)
+    K = xr.shape[-1]
+    rows = xr.size // K
+    codes = np.empty(xr.shape, dtype=np.uint8)
+    alpha = np.empty(rows, dtype=np.float64)
+    _check(_load().oracle_quantize_rows_e4m3(_ptr(xr), rows, K, float(clip), _ptr(codes), _ptr(alpha)),
+           "quantize_rows_e4m3")
+    return QuantActFP8(codes, alpha, xr)
+
+
+def quant_weight_fp8(w_f16: np.ndarray, had: Optional[Tuple[int, int]], clip: float = 1.0) -> QuantActFP8:
+    """W' = W R (Sec. 3.1), then per-output-channel FP8 (same rule as the
+    activations, one scale per row of W')."""
+    return rotate_quant_act_fp8(w_f16, had, clip)
+
+
+def w4a8_linear(a: QuantAct, w: QuantWeight) -> Linear:
+    """Integer accumulator and dequantized product of 8-bit activation codes
+    (q, or u with the 128 offset) and 4-bit weight codes."""
+    M, K = a.codes.shape
+    N = w.codes.shape[0]
+    acc = np.empty((M, N), dtype=np.int32)
+    y = np.empty((M, N), dtype=np.float64)
+    ac = _c(a.codes, np.int32)
+    wc = _c(w.codes, np.int32)
+    al = _c(a.alpha, np.float64)
+    be = None if a.beta is None else _c(a.beta, np.float64)
+    sc = _c(w.scale, np.float64)
+    _check(_load().oracle_w4a8_gemm(_ptr(ac), _ptr(al), _ptr(be), _ptr(wc), _ptr(sc), M, N, K, _ptr(acc), _ptr(y)),
+           "w4a8_gemm")
+    return Linear(acc, y, f64_to_f16(y))
+
+
+def fp8_linear(a_codes: np.ndarray, a_alpha: np.ndarray, w_codes: np.ndarray, w_scale: np.ndarray) -> np.ndarray:
+    """y = sum_k (alpha_m a_mk)(s_n w_nk) over decoded E4M3 codes (double)."""
+    ac = _c(a_codes, np.uint8)
+    wc = _c(w_codes, np.uint8)
+    M, K = ac.shape
+    N = wc.shape[0]
+    y = np.empty((M, N), dtype=np.float64)
+    _check(_load().oracle_fp8_gemm(_ptr(ac), _ptr(_c(a_alpha, np.float64)), _ptr(wc), _ptr(_c(w_scale, np.float64)),
+                                   M, N, K, _ptr(y)), "fp8_gemm")
+    return y

@@ -506,3 +506,109 @@ int oracle_cayley_step(const double* R, const double* grad, int64_t batch, int64
   }
   return err ? OR_EINVAL : OR_OK;
 }
+
+/* ------------------------------------------------------------------ */
+/* 8-bit variants: W4A8 and W-fp8-A-fp8 (main results table, 4-8-x    */
+/* rows; appendix "Latency measurement on GPU", FP8 GEMM setting)      */
+/* ------------------------------------------------------------------ */
+/* E4M3 (the FP8 format of the FP8 setting, in its finite-only form):
+ * 1 sign, 4 exponent (bias 7) and 3 mantissa bits; exponent field 0 holds
+ * the subnormals m 2^-9; no infinities; 448 is the largest finite value and
+ * S.1111.111 is NaN. */
+double oracle_e4m3_to_double(uint8_t b) {
+  const int s = b >> 7, e = (b >> 3) & 15, m = b & 7;
+  if (e == 15 && m == 7) return NAN;
+  const double v = e == 0 ? ldexp((double)m, -9) : ldexp(1.0 + m / 8.0, e - 7);
+  return s ? -v : v;
+}
+
+/* Round to the nearest E4M3 value (ties to the even mantissa), saturating at
+ * +-448; the sign of a value that rounds to zero is kept. */
+uint8_t oracle_double_to_e4m3(double v) {
+  const uint8_t sign = (v < 0 || (v == 0 && signbit(v))) ? 0x80 : 0;
+  double a = fabs(v);
+  if (a >= 448.0) return sign | 0x7E;
+  int e2;
+  frexp(a, &e2);                 /* a = f 2^e2, f in [0.5, 1) */
+  int E = e2 - 1;                /* exponent of the leading bit */
+  if (E < -6) E = -6;            /* the subnormal quantum 2^-9 */
+  const double q = ldexp(1.0, E - 3);
+  double r = nearbyint(a / q) * q;
+  if (r > 448.0) r = 448.0;
+  if (r == 0.0) return sign;
+  if (r < ldexp(1.0, -6)) return sign | (uint8_t)(r / ldexp(1.0, -9));
+  int e3;
+  frexp(r, &e3);
+  const int Er = e3 - 1;
+  const int mant = (int)((r / ldexp(1.0, Er) - 1.0) * 8.0);
+  return sign | (uint8_t)(((Er + 7) << 3) | mant);
+}
+
+void oracle_e4m3_array_to_double(const uint8_t* b, double* d, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) d[i] = oracle_e4m3_to_double(b[i]);
+}
+
+/* Per-row FP8 quantization (the FP8 setting's per-token / per-channel
+ * scaling): alpha = clip * max|x| / 448, code = E4M3(x / alpha); a zero row
+ * stores alpha = 0 and zero codes. */
+int oracle_quantize_rows_e4m3(const double* x, int64_t rows, int64_t K, double clip, uint8_t* codes,
+                              double* alpha) {
+  if (rows < 0 || K <= 0 || !(clip > 0.0 && clip <= 1.0)) return OR_EINVAL;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < rows; ++r) {
+    const double* xr = x + r * K;
+    double mx = 0.0;
+    for (int64_t k = 0; k < K; ++k) mx = fmax(mx, fabs(xr[k]));
+    const double a = clip * mx / 448.0;
+    alpha[r] = a;
+    for (int64_t k = 0; k < K; ++k) codes[r * K + k] = a > 0.0 ? oracle_double_to_e4m3(xr[k] / a) : 0;
+  }
+  return OR_OK;
+}
+
+/* W4A8 linear: acc[m][n] = sum_k a_int * q_w with a_int = q (symmetric
+ * 8-bit codes) or u - 128 (asymmetric), exact in int64 and checked to fit
+ * int32; y = sum_k (alpha_m c_mk + beta_m)(s_n q_w,nk), the dequantized
+ * product of the two Eq. 1 operands. */
+int oracle_w4a8_gemm(const int32_t* a_codes, const double* a_scale, const double* a_zero,
+                     const int32_t* w_codes, const double* w_scale, int64_t M, int64_t N, int64_t K,
+                     int32_t* acc, double* y) {
+  const int sym = a_zero == NULL;
+  int err = 0;
+#pragma omp parallel for schedule(static) collapse(2)
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n) {
+      int64_t s = 0;
+      double yy = 0.0;
+      const int32_t* a = a_codes + m * K;
+      const int32_t* w = w_codes + n * K;
+      const double am = a_scale[m], bm = sym ? 0.0 : a_zero[m], sn = w_scale[n];
+      for (int64_t k = 0; k < K; ++k) {
+        s += (int64_t)(sym ? a[k] : a[k] - 128) * w[k];
+        yy += (am * (double)a[k] + bm) * (sn * (double)w[k]);
+      }
+      if (s > INT32_MAX || s < INT32_MIN) {
+#pragma omp atomic write
+        err = 1;
+      }
+      acc[m * N + n] = (int32_t)s;
+      y[m * N + n] = yy;
+    }
+  return err ? OR_EINVAL : OR_OK;
+}
+
+/* W-fp8-A-fp8 linear: y = sum_k (alpha_m a_mk)(s_n w_nk) with a, w the
+ * decoded E4M3 codes. */
+int oracle_fp8_gemm(const uint8_t* a_codes, const double* a_scale, const uint8_t* w_codes,
+                    const double* w_scale, int64_t M, int64_t N, int64_t K, double* y) {
+#pragma omp parallel for schedule(static) collapse(2)
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t n = 0; n < N; ++n) {
+      double s = 0.0;
+      for (int64_t k = 0; k < K; ++k)
+        s += (a_scale[m] * oracle_e4m3_to_double(a_codes[m * K + k])) *
+             (w_scale[n] * oracle_e4m3_to_double(w_codes[n * K + k]));
+      y[m * N + n] = s;
+    }
+  return OR_OK;
+}
