@@ -737,7 +737,74 @@ def run_configs(dev, hbm_peak, fp8_peak):
     del q, k, v, o
     torch.cuda.empty_cache()
     res.update(cayley_records(dev))
+    res.update(variant8_records(dev, hbm_peak, fp8_peak))
     return res
+
+
+def variant8_records(dev, hbm_peak, fp8_peak):
+    """W4A8 and W-fp8-A-fp8 at the LLaMA-3-8B MLP shapes (2048 tokens):
+    gate_up 4096 -> 14336 (no rotation) and down_proj 14336 -> 4096 (online
+    H28 (x) H512).  Quantizers against HBM (read 2K + write the codes and
+    scales), GEMMs against the e4m3 peak; W4A8 runs 2 M N K multiply-adds on
+    the tensor core (two code planes) for M N K useful ones."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2405_16406_gb300 import spinq, synth
+    out = {}
+    for tag, case in (("gate_up", synth.llama3_8b_gate_up()), ("down_proj", synth.llama3_8b_down_proj())):
+        Mr, Kr, Nr = case.M, case.K, case.N
+        xt, wt = torch.from_numpy(case.x).to(dev), torch.from_numpy(case.w).to(dev)
+        nx = 4
+        xs = [xt] + [xt.clone() for _ in range(nx - 1)]
+        for variant, afmt, wfmt in (("w4a8", spinq.SPINQ_FMT_INT8_PLANES, spinq.SPINQ_FMT_INT4_BYTES),
+                                    ("fp8", spinq.SPINQ_FMT_E4M3, spinq.SPINQ_FMT_E4M3)):
+            sym = case.act_symmetric or variant == "fp8"
+            outs = [spinq.rotate_quant_act8(xs[i], case.had, afmt, sym) for i in range(nx)]
+            rq_us = graph_us(lambda i: spinq.rotate_quant_act8(xs[i], case.had, afmt, sym, out=outs[i]), nx)
+            planes = 2 if variant == "w4a8" else 1
+            rq_bytes = Mr * Kr * 2 + planes * Mr * Kr + (4 if sym else 8) * Mr
+            wq = spinq.quant_weight8(wt, case.had, wfmt)
+            ys = [torch.empty(Mr, Nr, dtype=torch.float16, device=dev) for _ in range(2)]
+            if variant == "w4a8":
+                g_us = graph_us(lambda i: spinq.w4a8_gemm(outs[i % nx], wq, y=ys[i]), 2)
+            else:
+                g_us = graph_us(lambda i: spinq.fp8_gemm(outs[i % nx], wq, y=ys[i]), 2)
+            torch.cuda.synchronize()
+            # timed output of copy 0 against the oracle on 4 rows x 256 columns
+            rows = np.array([0, 700, 1400, 2047])
+            cols = np.arange(0, Nr, Nr // 256)
+            sel = torch.as_tensor(rows, device=dev)
+            a_rows = outs[0].codes[sel].cpu().numpy()
+            if variant == "w4a8":
+                c = (oracle.e4m3_to_f64(a_rows[:, :Kr]) + oracle.e4m3_to_f64(a_rows[:, Kr:])).astype(np.int32)
+                wc = oracle.e4m3_to_f64(wq.codes[torch.as_tensor(cols, device=dev)].cpu().numpy()).astype(np.int32)
+                zero = None if sym else outs[0].zero[sel].double().cpu().numpy()
+                qa = oracle.QuantAct(c if sym else c + 128, None, outs[0].scale[sel].double().cpu().numpy(), zero, None)
+                qw = oracle.QuantWeight(wc, None, wq.scale[torch.as_tensor(cols, device=dev)].double().cpu().numpy(),
+                                        wc.sum(1), None)
+                yr = oracle.w4a8_linear(qa, qw).y
+            else:
+                yr = oracle.fp8_linear(a_rows, outs[0].scale[sel].double().cpu().numpy(),
+                                       wq.codes[torch.as_tensor(cols, device=dev)].cpu().numpy(),
+                                       wq.scale[torch.as_tensor(cols, device=dev)].double().cpu().numpy())
+            yg = ys[0][sel][:, torch.as_tensor(cols, device=dev)].double().cpu().numpy()
+            if not np.allclose(yg, yr, rtol=2e-3, atol=1e-3 * np.abs(yr).max()):
+                raise RuntimeError(f"{variant} {tag}: timed GEMM outputs differ from the oracle")
+            ops = 2.0 * Mr * Nr * Kr
+            out[f"f3_{variant}_{tag}_{Mr}x{Kr}x{Nr}"] = {
+                "rotate_quant": {"us": round(rq_us, 2), "bytes": rq_bytes,
+                                 "frac_hbm": round(rq_bytes / rq_us / 1e3 / hbm_peak, 4),
+                                 "kernel": "rq8_rows_kernel (one CTA per row)"},
+                "gemm": {"us": round(g_us, 2), "tops": round(ops / g_us / 1e6, 1),
+                         "tensor_frac_e4m3": round(planes * ops / g_us / 1e6 / fp8_peak, 4),
+                         "kernel": "fp8_gemm_kernel" + (" (two activation planes, K' = 2K)" if planes == 2 else "")},
+                "checked": "4 rows x 256 columns of the timed output vs the oracle's product of the same codes"}
+            del outs, ys, wq
+            torch.cuda.empty_cache()
+        del xs, xt, wt
+    return out
 
 
 def cayley_records(dev):

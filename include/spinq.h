@@ -289,6 +289,85 @@ int spinq_w4a4_gemm_plan(int64_t M, int64_t N, int64_t K);
 int spinq_w4a4_gemm_splitk_plan(int64_t M, int64_t N, int64_t K, int* nsplit);
 
 /*
+ * 8-bit variants (main results table, W4A8 rows "4-8-x"; appendix "Latency
+ * measurement on GPU": W-fp8-A-fp8 with the dequantization fused into the
+ * GEMM epilogue).  They share the rotation convention above and run on the
+ * E4M3 tensor-core pipe without unpacking.
+ *
+ * Code formats:
+ *   SPINQ_FMT_INT8_PLANES  Eq. 1 with N = 8 per token: the code c = q
+ *       (symmetric, [-128, 127]) or u - 128 (asymmetric, u in [0, 255]) is
+ *       stored as two E4M3 planes, row [2K] bytes: byte k = E4M3(16 (c >> 4)),
+ *       byte K + k = E4M3(c & 15) (both exact), so c = dec(k) + dec(K + k).
+ *   SPINQ_FMT_E4M3         per-row FP8: alpha = clip max|x'| / 448, code =
+ *       E4M3(x' / alpha), round to nearest even, saturating at +-448
+ *       (E4M3: 1 sign, 4 exponent bits with bias 7, 3 mantissa bits, no
+ *       infinities), [K] bytes per row.
+ *   SPINQ_FMT_INT4_BYTES   (weights of the W4A8 linear) Eq. 1 with N = 4,
+ *       symmetric per output channel, each code q in [-8, 7] stored as the
+ *       E4M3 byte of q, [K] bytes per row, plus rowsum = sum_k q.
+ */
+typedef enum {
+  SPINQ_FMT_INT8_PLANES = 1,
+  SPINQ_FMT_E4M3 = 2,
+  SPINQ_FMT_INT4_BYTES = 3
+} spinq_code_format;
+
+/*
+ * spinq_rotate_quant_act8 -- online rotation (as spinq_rotate_quant_act)
+ * then the 8-bit per-token quantizer `format`:
+ *   SPINQ_FMT_INT8_PLANES  q: bits = 8, symmetric or asymmetric; codes
+ *                          [M][2K]; scale [M]; zero [M] (asymmetric) or NULL.
+ *   SPINQ_FMT_E4M3         q: bits = 8, symmetric = 1; codes [M][K]; scale [M].
+ *   q->granularity = SPINQ_PER_TOKEN.  K % 128 == 0, K <= 32768, x rows and
+ *   codes 16-byte aligned.  Other formats return SPINQ_EINVAL.
+ */
+spinq_status spinq_rotate_quant_act8(const void* x_f16, int64_t M, int64_t K, int64_t ldx,
+                                     const spinq_had_cfg* had, const spinq_quant_cfg* q, int32_t format,
+                                     uint8_t* codes, float* scale, float* zero, void* stream);
+
+/*
+ * spinq_quant_weight8 -- offline weight preparation of the 8-bit linears:
+ * W' = W R (when had != NULL), then per output channel
+ *   SPINQ_FMT_E4M3        q: bits = 8, symmetric; codes [N][K]; scale [N];
+ *                         rowsum unused (may be NULL);
+ *   SPINQ_FMT_INT4_BYTES  q: bits = 4, symmetric; codes [N][K]; scale [N];
+ *                         rowsum [N].
+ *   q->granularity = SPINQ_PER_CHANNEL; sizes as spinq_rotate_quant_act8.
+ */
+spinq_status spinq_quant_weight8(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
+                                 const spinq_quant_cfg* q, int32_t format, uint8_t* codes, float* scale,
+                                 int32_t* rowsum, void* stream);
+
+/*
+ * spinq_fp8_gemm -- W-fp8-A-fp8 linear:
+ *   y[m][n] = fp16(alpha_m s_n sum_k a_mk w_nk), a, w decoded E4M3 codes,
+ * products exact and summed in fp32 on the tensor core.
+ *   a_codes [M][K] (SPINQ_FMT_E4M3), a_scale [M]; w_codes [N][K], w_scale [N].
+ *   K % 128 == 0, K <= 65536, N % 16 == 0; code and output pointers 16-byte
+ *   aligned.
+ */
+spinq_status spinq_fp8_gemm(const uint8_t* a_codes, const float* a_scale, const uint8_t* w_codes,
+                            const float* w_scale, int64_t M, int64_t N, int64_t K, void* y_f16, void* stream);
+
+/*
+ * spinq_w4a8_gemm -- W4A8 linear on Eq. 1 codes, exact integer accumulator:
+ *   acc[m][n] = sum_k c_mk q_nk (c = q or u - 128, exact in fp32: every
+ *               partial sum is an integer of magnitude <= 1024 K <= 2^24);
+ *   y[m][n]   = fp16(s_n (alpha_m acc + beta'_m rowsum_n)),
+ *               beta'_m = beta_m + 128 alpha_m (asymmetric) or 0,
+ *   the dequantized product of the two Eq. 1 operands.
+ *   a_planes [M][2K] (SPINQ_FMT_INT8_PLANES), a_scale [M], a_zero [M] or NULL;
+ *   w_codes [N][K] (SPINQ_FMT_INT4_BYTES), w_scale [N], w_rowsum [N];
+ *   acc_out [M][N] int32 or NULL (debug).
+ *   K % 128 == 0, K <= 16384, N % 16 == 0; code and output pointers 16-byte
+ *   aligned.
+ */
+spinq_status spinq_w4a8_gemm(const uint8_t* a_planes, const float* a_scale, const float* a_zero,
+                             const uint8_t* w_codes, const float* w_scale, const int32_t* w_rowsum, int64_t M,
+                             int64_t N, int64_t K, void* y_f16, int32_t* acc_out, void* stream);
+
+/*
  * spinq_cayley_step -- one Cayley SGD update of a batch of rotations
  * (Sec. 3.2, the R' update and its Y / G_hat definitions), for learning R2
  * (head_dim x head_dim, one per layer) with the weights frozen:

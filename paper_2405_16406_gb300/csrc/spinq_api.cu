@@ -205,6 +205,90 @@ spinq_status spinq_cayley_step(const float* R, const float* grad, int64_t batch,
   return from_cuda(launch_cayley_step(a, static_cast<cudaStream_t>(stream)));
 }
 
+static spinq_status rq8(const void* x, int64_t rows, int64_t K, int64_t ldx, const spinq_had_cfg* had,
+                        const spinq_quant_cfg* q, int format, bool weights, uint8_t* codes, float* scale,
+                        float* zero, int32_t* rowsum, void* stream) {
+  if (!q || rows < 0 || K <= 0 || ldx < K) return SPINQ_EINVAL;
+  if (rows > 0 && (!x || !codes || !scale)) return SPINQ_EINVAL;
+  if (!clip_ok(q->clip_ratio)) return SPINQ_EINVAL;
+  if (q->symmetric != 0 && q->symmetric != 1) return SPINQ_EINVAL;
+  if (K % 128 != 0 || ldx % 8 != 0 || !aligned16(x) || !aligned16(codes)) return SPINQ_EINVAL;
+  const bool act = !weights;
+  if (act && format != SPINQ_FMT_INT8_PLANES && format != SPINQ_FMT_E4M3) return SPINQ_EINVAL;
+  if (weights && format != SPINQ_FMT_E4M3 && format != SPINQ_FMT_INT4_BYTES) return SPINQ_EINVAL;
+  if (act && !q->symmetric && format == SPINQ_FMT_INT8_PLANES && rows > 0 && !zero) return SPINQ_EINVAL;
+  if (weights && format == SPINQ_FMT_INT4_BYTES && rows > 0 && !rowsum) return SPINQ_EINVAL;
+  const int want_bits = format == SPINQ_FMT_INT4_BYTES ? 4 : 8;
+  const int want_gran = weights ? SPINQ_PER_CHANNEL : SPINQ_PER_TOKEN;
+  if (q->bits != want_bits || q->granularity != want_gran) return SPINQ_EUNSUPPORTED;
+  if (format != SPINQ_FMT_INT8_PLANES && !q->symmetric) return SPINQ_EUNSUPPORTED;
+  if (K > 32768) return SPINQ_EUNSUPPORTED;
+  Rq8Args a{};
+  if (had) {
+    spinq_status st = check_had(had, K, &a.hs);
+    if (st != SPINQ_OK) return st;
+    a.n_small = had->n_small;
+    a.n_pow2 = had->n_pow2;
+    a.norm = (float)(1.0 / std::sqrt((double)K));
+  } else {
+    a.n_small = 0;
+    a.n_pow2 = 1;
+    a.norm = 1.f;
+  }
+  if (rows == 0) return SPINQ_OK;
+  a.x = x;
+  a.rows = rows;
+  a.K = K;
+  a.ldx = ldx;
+  a.format = format;
+  a.symmetric = q->symmetric != 0;
+  a.clip = q->clip_ratio;
+  a.codes = codes;
+  a.scale = scale;
+  a.zero = a.symmetric ? nullptr : zero;
+  a.rowsum = rowsum;
+  return from_cuda(launch_rotate_quant_8bit(a, static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_rotate_quant_act8(const void* x_f16, int64_t M, int64_t K, int64_t ldx, const spinq_had_cfg* had,
+                                     const spinq_quant_cfg* q, int32_t format, uint8_t* codes, float* scale,
+                                     float* zero, void* stream) {
+  return rq8(x_f16, M, K, ldx, had, q, format, false, codes, scale, zero, nullptr, stream);
+}
+
+spinq_status spinq_quant_weight8(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
+                                 const spinq_quant_cfg* q, int32_t format, uint8_t* codes, float* scale,
+                                 int32_t* rowsum, void* stream) {
+  return rq8(w_f16, N, K, K, had, q, format, true, codes, scale, nullptr, rowsum, stream);
+}
+
+static spinq_status gemm8(bool w4a8, const uint8_t* a_codes, const float* a_scale, const float* a_zero,
+                          const uint8_t* w_codes, const float* w_scale, const int32_t* w_rowsum, int64_t M,
+                          int64_t N, int64_t K, void* y_f16, int32_t* acc_out, void* stream) {
+  if (M < 0 || N < 0 || K <= 0) return SPINQ_EINVAL;
+  if (M > 0 && N > 0 && (!a_codes || !a_scale || !w_codes || !w_scale || !y_f16 || (w4a8 && !w_rowsum)))
+    return SPINQ_EINVAL;
+  if (K % 128 != 0 || N % 16 != 0) return SPINQ_EINVAL;
+  for (const void* p : {(const void*)a_codes, (const void*)w_codes, (const void*)y_f16, (const void*)acc_out})
+    if (p && !aligned16(p)) return SPINQ_EINVAL;
+  if (M > INT32_MAX || N > INT32_MAX || K > (w4a8 ? 16384 : 65536)) return SPINQ_EUNSUPPORTED;
+  if (M == 0 || N == 0) return SPINQ_OK;
+  Fp8GemmArgs g{w4a8, a_codes, a_scale, w4a8 ? a_zero : nullptr, w_codes, w_scale, w4a8 ? w_rowsum : nullptr,
+                M, N, K, y_f16, w4a8 ? acc_out : nullptr};
+  return from_cuda(launch_fp8_gemm(g, static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_fp8_gemm(const uint8_t* a_codes, const float* a_scale, const uint8_t* w_codes,
+                            const float* w_scale, int64_t M, int64_t N, int64_t K, void* y_f16, void* stream) {
+  return gemm8(false, a_codes, a_scale, nullptr, w_codes, w_scale, nullptr, M, N, K, y_f16, nullptr, stream);
+}
+
+spinq_status spinq_w4a8_gemm(const uint8_t* a_planes, const float* a_scale, const float* a_zero,
+                             const uint8_t* w_codes, const float* w_scale, const int32_t* w_rowsum, int64_t M,
+                             int64_t N, int64_t K, void* y_f16, int32_t* acc_out, void* stream) {
+  return gemm8(true, a_planes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y_f16, acc_out, stream);
+}
+
 int spinq_gemm_select_kernel(int kernel) { return w4a4_gemm_select(kernel); }
 
 int spinq_gemm_split_k(int n) { return w4a4_gemm_split_k(n); }

@@ -126,6 +126,46 @@ struct CayleyArgs {
 // cudaErrorNotSupported for other n.
 cudaError_t launch_cayley_step(const CayleyArgs& a, cudaStream_t stream);
 
+// Code formats of the 8-bit quantizers (spinq_code_format in spinq.h).
+constexpr int kFmtInt8Planes = 1;
+constexpr int kFmtE4M3 = 2;
+constexpr int kFmtInt4Bytes = 3;
+
+struct Rq8Args {
+  const void* x;      // fp16 [rows][ldx]
+  int64_t rows, K, ldx;
+  int n_small;        // 0 = no rotation
+  int n_pow2;
+  SmallHadamard hs;
+  int format;         // kFmt*
+  bool symmetric;
+  float clip;
+  float norm;         // 1/sqrt(K) with a rotation, else 1
+  uint8_t* codes;     // [rows][2K] (int8 planes) or [rows][K]
+  float* scale;       // [rows]
+  float* zero;        // [rows] (asymmetric int8) or nullptr
+  int32_t* rowsum;    // [rows] (int4 bytes) or nullptr
+};
+
+cudaError_t launch_rotate_quant_8bit(const Rq8Args& a, cudaStream_t stream);
+
+struct Fp8GemmArgs {
+  bool w4a8;              // false: FP8 x FP8; true: W4A8 (activation planes [M][2K])
+  const uint8_t* a_codes; // E4M3 bytes [M][K] (FP8) or [M][2K] (W4A8 planes)
+  const float* a_scale;   // [M]
+  const float* a_zero;    // [M] (W4A8 asymmetric) or nullptr
+  const uint8_t* w_codes; // E4M3 bytes [N][K]
+  const float* w_scale;   // [N]
+  const int32_t* w_rowsum;// [N] (W4A8) or nullptr
+  int64_t M, N, K;
+  void* y;                // fp16 [M][N]
+  int32_t* acc_out;       // W4A8 only, optional
+};
+
+// 8-bit linears on the E4M3 pipe; cudaErrorNotSupported when a tensor map
+// cannot be encoded.
+cudaError_t launch_fp8_gemm(const Fp8GemmArgs& a, cudaStream_t stream);
+
 // Device status word written by bounded waits that gave up.
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail);
 // Its device address (two ints: code, wait site), for kernels in other

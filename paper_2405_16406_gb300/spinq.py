@@ -38,7 +38,9 @@ EXPORTED = (
     "spinq_status_string", "spinq_device_status", "spinq_version", "spinq_w4a4_gemm_workspace_bytes",
     "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel", "spinq_gemm_split_k",
     "spinq_w4a4_gemm_plan", "spinq_w4a4_gemm_splitk_plan", "spinq_cayley_step",
+    "spinq_rotate_quant_act8", "spinq_quant_weight8", "spinq_fp8_gemm", "spinq_w4a8_gemm",
 )
+SPINQ_FMT_INT8_PLANES, SPINQ_FMT_E4M3, SPINQ_FMT_INT4_BYTES = 1, 2, 3
 
 
 class QuantCfg(ctypes.Structure):
@@ -87,6 +89,16 @@ _lib.spinq_w4a4_gemm_plan.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_plan.argtypes = [_I64, _I64, _I64]
 _lib.spinq_w4a4_gemm_splitk_plan.restype = ctypes.c_int
 _lib.spinq_w4a4_gemm_splitk_plan.argtypes = [_I64, _I64, _I64, ctypes.POINTER(ctypes.c_int)]
+_lib.spinq_rotate_quant_act8.restype = ctypes.c_int
+_lib.spinq_rotate_quant_act8.argtypes = [_P, _I64, _I64, _I64, ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
+                                         ctypes.c_int32, _P, _P, _P, _P]
+_lib.spinq_quant_weight8.restype = ctypes.c_int
+_lib.spinq_quant_weight8.argtypes = [_P, _I64, _I64, ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg), ctypes.c_int32,
+                                     _P, _P, _P, _P]
+_lib.spinq_fp8_gemm.restype = ctypes.c_int
+_lib.spinq_fp8_gemm.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _P, _P]
+_lib.spinq_w4a8_gemm.restype = ctypes.c_int
+_lib.spinq_w4a8_gemm.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
 _lib.spinq_cayley_step.restype = ctypes.c_int
 _lib.spinq_cayley_step.argtypes = [_P, _P, _I64, _I64, ctypes.c_float, ctypes.c_int32, _P, _P, _P]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
@@ -134,6 +146,22 @@ def spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k
                           k_zero, v_codes, v_scale, v_zero, stream) -> int:
     return _lib.spinq_rotate_quant_kv(q_in, q_out, k_in, v_in, B, S, Hq, Hkv, D, had, kvq, k_codes,
                                       k_scale, k_zero, v_codes, v_scale, v_zero, stream)
+
+
+def spinq_rotate_quant_act8(x, M, K, ldx, had, q, fmt, codes, scale, zero, stream) -> int:
+    return _lib.spinq_rotate_quant_act8(x, M, K, ldx, had, q, fmt, codes, scale, zero, stream)
+
+
+def spinq_quant_weight8(w, N, K, had, q, fmt, codes, scale, rowsum, stream) -> int:
+    return _lib.spinq_quant_weight8(w, N, K, had, q, fmt, codes, scale, rowsum, stream)
+
+
+def spinq_fp8_gemm(a_codes, a_scale, w_codes, w_scale, M, N, K, y, stream) -> int:
+    return _lib.spinq_fp8_gemm(a_codes, a_scale, w_codes, w_scale, M, N, K, y, stream)
+
+
+def spinq_w4a8_gemm(a_planes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc, stream) -> int:
+    return _lib.spinq_w4a8_gemm(a_planes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc, stream)
 
 
 def spinq_cayley_step(R, grad, batch, n, alpha, iters, R_out, Y_out, stream) -> int:
@@ -324,3 +352,57 @@ def cayley_step(R: torch.Tensor, grad: torch.Tensor, alpha: float, iters: int = 
     _check(_lib.spinq_cayley_step(_ptr(R), _ptr(grad), batch, n, float(alpha), int(iters), _ptr(out), _ptr(y),
                                   _stream(stream)), "spinq_cayley_step")
     return (out, y) if want_y else out
+
+
+def rotate_quant_act8(x: torch.Tensor, had: Optional[Tuple[int, int]], fmt: int, symmetric: bool = True,
+                      clip: float = 1.0, out: Optional[ActCodes] = None,
+                      stream: Optional[torch.cuda.Stream] = None) -> ActCodes:
+    """8-bit activation codes: SPINQ_FMT_INT8_PLANES ([M, 2K]) or SPINQ_FMT_E4M3 ([M, K])."""
+    assert x.dtype == torch.float16 and x.dim() == 2 and x.stride(1) == 1
+    M, K = x.shape
+    width = 2 * K if fmt == SPINQ_FMT_INT8_PLANES else K
+    if out is None:
+        out = ActCodes(torch.empty((M, width), dtype=torch.uint8, device=x.device),
+                       torch.empty(M, dtype=torch.float32, device=x.device),
+                       None if symmetric else torch.empty(M, dtype=torch.float32, device=x.device))
+    q = quant_cfg(8, symmetric, SPINQ_PER_TOKEN, 0, clip)
+    _check(_lib.spinq_rotate_quant_act8(_ptr(x), M, K, x.stride(0), _had(had), ctypes.byref(q), fmt, _ptr(out.codes),
+                                        _ptr(out.scale), _ptr(out.zero), _stream(stream)), "spinq_rotate_quant_act8")
+    return out
+
+
+def quant_weight8(w: torch.Tensor, had: Optional[Tuple[int, int]], fmt: int, clip: float = 1.0,
+                  stream: Optional[torch.cuda.Stream] = None) -> WeightCodes:
+    """Weights of the 8-bit linears: SPINQ_FMT_E4M3 (FP8) or SPINQ_FMT_INT4_BYTES (W4A8)."""
+    assert w.dtype == torch.float16 and w.is_contiguous()
+    N, K = w.shape
+    out = WeightCodes(torch.empty((N, K), dtype=torch.uint8, device=w.device),
+                      torch.empty(N, dtype=torch.float32, device=w.device),
+                      torch.empty(N, dtype=torch.int32, device=w.device))
+    q = quant_cfg(4 if fmt == SPINQ_FMT_INT4_BYTES else 8, True, SPINQ_PER_CHANNEL, 0, clip)
+    _check(_lib.spinq_quant_weight8(_ptr(w), N, K, _had(had), ctypes.byref(q), fmt, _ptr(out.codes), _ptr(out.scale),
+                                    _ptr(out.rowsum), _stream(stream)), "spinq_quant_weight8")
+    return out
+
+
+def fp8_gemm(a: ActCodes, w: WeightCodes, y: Optional[torch.Tensor] = None,
+             stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    M, K = a.codes.shape
+    N = w.codes.shape[0]
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float16, device=a.codes.device)
+    _check(_lib.spinq_fp8_gemm(_ptr(a.codes), _ptr(a.scale), _ptr(w.codes), _ptr(w.scale), M, N, K, _ptr(y),
+                               _stream(stream)), "spinq_fp8_gemm")
+    return y
+
+
+def w4a8_gemm(a: ActCodes, w: WeightCodes, want_acc: bool = False, y: Optional[torch.Tensor] = None,
+              stream: Optional[torch.cuda.Stream] = None):
+    M = a.codes.shape[0]
+    N, K = w.codes.shape
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float16, device=a.codes.device)
+    acc = torch.empty((M, N), dtype=torch.int32, device=a.codes.device) if want_acc else None
+    _check(_lib.spinq_w4a8_gemm(_ptr(a.codes), _ptr(a.scale), _ptr(a.zero), _ptr(w.codes), _ptr(w.scale),
+                                _ptr(w.rowsum), M, N, K, _ptr(y), _ptr(acc), _stream(stream)), "spinq_w4a8_gemm")
+    return (y, acc) if want_acc else y

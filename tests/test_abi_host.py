@@ -164,3 +164,29 @@ def test_cayley_step_rejects_invalid_arguments_on_the_host(lib):
     assert f(fake, fake, 2, 96, 0.1, 2, fake, None, None) == S.SPINQ_EUNSUPPORTED
     assert f(fake, fake, 2, 256, 0.1, 2, fake, None, None) == S.SPINQ_EUNSUPPORTED
     assert f(fake, fake, 0, 128, 0.1, 2, fake, None, None) == S.SPINQ_OK
+
+
+def test_8bit_entry_points_reject_invalid_arguments_on_the_host(lib):
+    from paper_2405_16406_gb300 import spinq as S
+    fake = ctypes.c_void_p(1 << 20)
+    q8 = S.quant_cfg(8, True, S.SPINQ_PER_TOKEN, 0, 1.0)
+    q4 = S.quant_cfg(4, True, S.SPINQ_PER_TOKEN, 0, 1.0)
+    a8 = S.spinq_rotate_quant_act8
+    assert a8(fake, 4, 200, 256, None, ctypes.byref(q8), S.SPINQ_FMT_E4M3, fake, fake, None, None) == S.SPINQ_EINVAL
+    assert a8(fake, 4, 256, 256, None, ctypes.byref(q8), S.SPINQ_FMT_INT4_BYTES, fake, fake, None, None) == S.SPINQ_EINVAL
+    assert a8(fake, 4, 256, 256, None, ctypes.byref(q4), S.SPINQ_FMT_E4M3, fake, fake, None, None) == S.SPINQ_EUNSUPPORTED
+    qa = S.quant_cfg(8, False, S.SPINQ_PER_TOKEN, 0, 1.0)
+    assert a8(fake, 4, 256, 256, None, ctypes.byref(qa), S.SPINQ_FMT_INT8_PLANES, fake, fake, None, None) == S.SPINQ_EINVAL
+    assert a8(fake, 4, 256, 256, None, ctypes.byref(qa), S.SPINQ_FMT_E4M3, fake, fake, fake, None) == S.SPINQ_EUNSUPPORTED
+    assert a8(fake, 0, 256, 256, None, ctypes.byref(q8), S.SPINQ_FMT_E4M3, fake, fake, None, None) == S.SPINQ_OK
+    w8 = S.spinq_quant_weight8
+    qw = S.quant_cfg(4, True, S.SPINQ_PER_CHANNEL, 0, 1.0)
+    assert w8(fake, 8, 256, None, ctypes.byref(qw), S.SPINQ_FMT_INT4_BYTES, fake, fake, None, None) == S.SPINQ_EINVAL
+    assert w8(fake, 8, 256, None, ctypes.byref(qw), S.SPINQ_FMT_INT8_PLANES, fake, fake, fake, None) == S.SPINQ_EINVAL
+    g = S.spinq_w4a8_gemm
+    assert g(fake, fake, None, fake, fake, fake, 4, 32, 16384 + 128, fake, None, None) == S.SPINQ_EUNSUPPORTED
+    assert g(fake, fake, None, fake, fake, None, 4, 32, 256, fake, None, None) == S.SPINQ_EINVAL
+    assert g(fake, fake, None, fake, fake, fake, 4, 40, 256, fake, None, None) == S.SPINQ_EINVAL
+    f = S.spinq_fp8_gemm
+    assert f(fake, fake, fake, fake, 4, 32, 96, fake, None) == S.SPINQ_EINVAL
+    assert f(fake, fake, fake, fake, 0, 32, 128, fake, None) == S.SPINQ_OK
