@@ -82,6 +82,8 @@ def _load():
         "oracle_w4a4_gemm_sampled": (i32, [P, P, P, P, P, i64, P, P, i64, P, P]),
         "oracle_rowsum": (None, [P, i64, i64, P]),
         "oracle_cayley_y": (i32, [P, P, i64, P]),
+        "oracle_rope": (i32, [P, P, i64, i64, dbl, P]),
+        "oracle_decode_attention": (i32, [P, P, P, P, i64, i64, i64, i64, i64, dbl, P]),
         "oracle_e4m3_to_double": (dbl, [ctypes.c_uint8]),
         "oracle_double_to_e4m3": (ctypes.c_uint8, [dbl]),
         "oracle_e4m3_array_to_double": (None, [P, P, i64]),
@@ -465,3 +467,55 @@ def fp8_linear(a_codes: np.ndarray, a_alpha: np.ndarray, w_codes: np.ndarray, w_
     _check(_load().oracle_fp8_gemm(_ptr(ac), _ptr(_c(a_alpha, np.float64)), _ptr(wc), _ptr(_c(w_scale, np.float64)),
                                    M, N, K, _ptr(y)), "fp8_gemm")
     return y
+
+
+# --------------------------------------------------------------------------
+# RoPE in front of R3, and decode attention over the 4-bit KV cache
+# (Sec. 3.1 R3; appendix "Latency measurement on GPU")
+# --------------------------------------------------------------------------
+def rope(x: np.ndarray, pos: np.ndarray, base: float = 500000.0) -> np.ndarray:
+    """Rotary embedding (rotate-half form) of rows [..., D] at positions
+    ``pos`` (one per row of the flattened leading dimensions), in double."""
+    x = _c(x, np.float64)
+    D = x.shape[-1]
+    rows = x.size // D
+    p = _c(np.asarray(pos, dtype=np.int64).reshape(-1), np.int64)
+    assert p.size == rows, "one position per row"
+    y = np.empty_like(x)
+    _check(_load().oracle_rope(_ptr(x), _ptr(p), rows, D, float(base), _ptr(y)), "rope")
+    return y
+
+
+def rope_rotate_quant_kv(q_f16: np.ndarray, k_f16: np.ndarray, v_f16: np.ndarray, positions: np.ndarray,
+                         had: Tuple[int, int], base: float = 500000.0, bits: int = 4, clip: float = 1.0) -> QuantKV:
+    """RoPE on Q and K at their tokens' positions, rounded to fp16 (the
+    model's activations), then R3 and the KV quantizer as rotate_quant_kv."""
+    B, S, Hq, D = q_f16.shape
+    Hkv = k_f16.shape[2]
+    pos = np.asarray(positions, dtype=np.int64).reshape(B, S)
+    qp = rope(f16_to_f64(q_f16).reshape(-1, D), np.repeat(pos.reshape(-1), Hq), base)
+    kp = rope(f16_to_f64(k_f16).reshape(-1, D), np.repeat(pos.reshape(-1), Hkv), base)
+    return rotate_quant_kv(f64_to_f16(qp).reshape(B, S, Hq, D), f64_to_f16(kp).reshape(B, S, Hkv, D), v_f16, had,
+                           bits, clip)
+
+
+def decode_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, lens: Optional[np.ndarray] = None,
+                     scale: Optional[float] = None) -> np.ndarray:
+    """o[b, h] = sum_t softmax_t(scale q[b, h] . k[b, t, h / G]) v[b, t, h / G]
+    over t < lens[b] (double); q [B, Hq, D], k, v [B, S, Hkv, D]."""
+    q = _c(q, np.float64)
+    k = _c(k, np.float64)
+    v = _c(v, np.float64)
+    B, Hq, D = q.shape
+    S, Hkv = k.shape[1], k.shape[2]
+    sc = 1.0 / np.sqrt(D) if scale is None else float(scale)
+    L = None if lens is None else _c(lens, np.int64)
+    o = np.empty((B, Hq, D), dtype=np.float64)
+    _check(_load().oracle_decode_attention(_ptr(q), _ptr(k), _ptr(v), _ptr(L), B, S, Hq, Hkv, D, sc, _ptr(o)),
+           "decode_attention")
+    return o
+
+
+def dequant_kv(codes: np.ndarray, alpha: np.ndarray, beta: np.ndarray) -> np.ndarray:
+    """alpha u + beta per (token, kv head) group of Eq. 1 asymmetric codes."""
+    return dequantize_rows(codes.reshape(-1, codes.shape[-1]), alpha.reshape(-1), beta.reshape(-1)).reshape(codes.shape)

@@ -612,3 +612,75 @@ int oracle_fp8_gemm(const uint8_t* a_codes, const double* a_scale, const uint8_t
     }
   return OR_OK;
 }
+
+/* ------------------------------------------------------------------ */
+/* Decode attention over the 4-bit KV cache, and RoPE in front of R3   */
+/* (Sec. 3.1: R3 rotates Q and K over head_dim so that the KV cache    */
+/* quantizes to 4 bits; appendix "Latency measurement on GPU": decode  */
+/* time per token)                                                     */
+/* ------------------------------------------------------------------ */
+/* Rotary position embedding of one head vector (the rotate-half form of
+ * LLaMA): for i < D/2 with theta_i = base^(-2i/D) and angle p theta_i,
+ *   y_i = x_i cos - x_{i+D/2} sin,   y_{i+D/2} = x_i sin + x_{i+D/2} cos.
+ * rows x D values; pos[r] is the position of row r. */
+int oracle_rope(const double* x, const int64_t* pos, int64_t rows, int64_t D, double base, double* y) {
+  if (D <= 0 || D % 2 || rows < 0) return OR_EINVAL;
+  const int64_t h = D / 2;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t i = 0; i < h; ++i) {
+      const double th = pow(base, -2.0 * (double)i / (double)D);
+      const double ang = (double)pos[r] * th;
+      const double c = cos(ang), s = sin(ang);
+      const double a = x[r * D + i], b = x[r * D + i + h];
+      y[r * D + i] = a * c - b * s;
+      y[r * D + i + h] = a * s + b * c;
+    }
+  return OR_OK;
+}
+
+/* Attention of one decode query per (batch, query head) over a cache of
+ * dequantized keys and values:
+ *   s_t = scale * q . k_t,  p = softmax_t(s) over t < len_b,  o = sum_t p_t v_t,
+ * q [B][Hq][D], k, v [B][S][Hkv][D]; query head h reads kv head h / (Hq/Hkv). */
+int oracle_decode_attention(const double* q, const double* k, const double* v, const int64_t* lens, int64_t B,
+                            int64_t S, int64_t Hq, int64_t Hkv, int64_t D, double scale, double* o) {
+  if (B < 0 || S <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || D <= 0) return OR_EINVAL;
+  int err = 0;
+#pragma omp parallel for schedule(static) collapse(2)
+  for (int64_t b = 0; b < B; ++b)
+    for (int64_t h = 0; h < Hq; ++h) {
+      const int64_t L = lens ? lens[b] : S;
+      const int64_t hk = h / (Hq / Hkv);
+      double* out = o + (b * Hq + h) * D;
+      if (L <= 0 || L > S) {
+#pragma omp atomic write
+        err = 1;
+        continue;
+      }
+      double* s = (double*)malloc(sizeof(double) * L);
+      if (!s) {
+#pragma omp atomic write
+        err = 1;
+        continue;
+      }
+      const double* qh = q + (b * Hq + h) * D;
+      double mx = -INFINITY;
+      for (int64_t t = 0; t < L; ++t) {
+        const double* kt = k + ((b * S + t) * Hkv + hk) * D;
+        double acc = 0.0;
+        for (int64_t d = 0; d < D; ++d) acc += qh[d] * kt[d];
+        s[t] = scale * acc;
+        if (s[t] > mx) mx = s[t];
+      }
+      double den = 0.0;
+      for (int64_t t = 0; t < L; ++t) den += exp(s[t] - mx);
+      for (int64_t d = 0; d < D; ++d) out[d] = 0.0;
+      for (int64_t t = 0; t < L; ++t) {
+        const double p = exp(s[t] - mx) / den;
+        const double* vt = v + ((b * S + t) * Hkv + hk) * D;
+        for (int64_t d = 0; d < D; ++d) out[d] += p * vt[d];
+      }
+      free(s);
+    }
+  return err ? OR_EINVAL : OR_OK;
+}
