@@ -738,7 +738,56 @@ def run_configs(dev, hbm_peak, fp8_peak):
     torch.cuda.empty_cache()
     res.update(cayley_records(dev))
     res.update(variant8_records(dev, hbm_peak, fp8_peak))
+    res.update(attention_records(dev, hbm_peak))
     return res
+
+
+def attention_records(dev, hbm_peak):
+    """Config 4's KV path with RoPE in front of R3 (B 8, S 4096, 32 q / 8 kv
+    heads, D 128), and decode attention of one query per head over the 4-bit
+    cache it writes; both against HBM."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2405_16406_gb300 import spinq, synth
+    kv = synth.kv_case()
+    B, S, Hq, Hkv, Dd = kv.B, kv.S, kv.Hq, kv.Hkv, kv.D
+    th = 500000.0 ** (-2.0 * np.arange(Dd // 2) / Dd)
+    ang = np.arange(S)[:, None] * th[None, :]
+    cs = torch.from_numpy(np.stack([np.cos(ang), np.sin(ang)], -1).astype(np.float32)).to(dev)
+    pos = torch.arange(S, dtype=torch.int32, device=dev).repeat(B, 1)
+    q, k, v = (torch.from_numpy(t).to(dev) for t in (kv.q, kv.k, kv.v))
+    cache = spinq.rope_rotate_quant_kv(q, k, v, pos, cs)
+    rope_us = graph_us(lambda i: spinq.rope_rotate_quant_kv(q, k, v, pos, cs, out=cache), 1, reps=6)
+    rope_bytes = B * S * Hq * Dd * 4 + 2 * B * S * Hkv * (Dd * 2 + Dd // 2 + 8) + B * S * 4
+    rng = np.random.default_rng(11)
+    qd = torch.from_numpy((rng.standard_normal((B, Hq, Dd)) * 2).astype(np.float16)).to(dev)
+    outs = [torch.empty_like(qd) for _ in range(2)]
+    ws = torch.empty(spinq.spinq_decode_attention_workspace_bytes(B, S, Hq, Hkv, Dd), dtype=torch.uint8, device=dev)
+    att_us = graph_us(lambda i: spinq.decode_attention_kv4(qd, cache, out=outs[i], workspace=ws), 2)
+    torch.cuda.synchronize()
+    att_bytes = B * S * Hkv * (Dd + 16) + 2 * B * Hq * Dd * 2
+    # timed output of batch 0 against the oracle on the same codes
+    kc = oracle.unpack4(cache.k_codes[:1].cpu().numpy(), False)
+    vc = oracle.unpack4(cache.v_codes[:1].cpu().numpy(), False)
+    kd = oracle.dequant_kv(kc, cache.k_scale[:1].double().cpu().numpy(), cache.k_zero[:1].double().cpu().numpy())
+    vd = oracle.dequant_kv(vc, cache.v_scale[:1].double().cpu().numpy(), cache.v_zero[:1].double().cpu().numpy())
+    ref = oracle.decode_attention(qd[:1].double().cpu().numpy(), kd, vd)
+    got = outs[0][:1].double().cpu().numpy()
+    if not np.all(np.abs(got - ref) <= 2e-3 * np.abs(ref) + 2e-3 * np.abs(ref).max()):
+        raise RuntimeError("decode attention: timed output differs from the oracle")
+    del q, k, v, cache
+    torch.cuda.empty_cache()
+    return {
+        "f2_rope_r3_kv4_B8_S4096": {"us": round(rope_us, 2), "bytes": rope_bytes,
+                                     "frac_hbm": round(rope_bytes / rope_us / 1e3 / hbm_peak, 4),
+                                     "kernel": "rotate_quant_kv_kernel with the RoPE stage"},
+        "f2_decode_attention_kv4_B8_S4096_Hq32_Hkv8_D128": {
+            "us": round(att_us, 2), "bytes": att_bytes, "frac_hbm": round(att_bytes / att_us / 1e3 / hbm_peak, 4),
+            "chunks": int(ws.numel() // (B * Hq * (Dd + 2) * 4)),
+            "kernel": "attn_partial_kernel + attn_combine_kernel",
+            "checked": "batch 0's 32 heads vs the oracle on the same codes"}}
 
 
 def variant8_records(dev, hbm_peak, fp8_peak):

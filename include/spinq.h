@@ -289,6 +289,55 @@ int spinq_w4a4_gemm_plan(int64_t M, int64_t N, int64_t K);
 int spinq_w4a4_gemm_splitk_plan(int64_t M, int64_t N, int64_t K, int* nsplit);
 
 /*
+ * spinq_rope_rotate_quant_kv -- spinq_rotate_quant_kv with the rotary
+ * position embedding applied to Q and K first, in the same kernel: for each
+ * token at position p and i < D/2, with (cos, sin) of angle p theta_i taken
+ * from the caller's table,
+ *   x_i <- x_i cos - x_{i+D/2} sin,   x_{i+D/2} <- x_i sin + x_{i+D/2} cos
+ * (the rotate-half form), computed in fp32 and rounded to fp16 like the
+ * model's activations; then R3 (Sec. 3.1, the online Hadamard that follows
+ * RoPE on Q and K) and the KV quantizer exactly as spinq_rotate_quant_kv.
+ *   positions [B][S] int32, each in [0, max_pos) (others are clamped).
+ *   cos_sin   [max_pos][D/2] pairs (cos, sin) as fp32, 16-byte aligned; the
+ *             caller computes angle p theta_i, theta_i = base^(-2i/D),
+ *             accurately (e.g. in double) once.
+ * Other arguments, layouts and requirements as spinq_rotate_quant_kv.
+ */
+spinq_status spinq_rope_rotate_quant_kv(const void* q_in, void* q_out, const void* k_in, const void* v_in,
+                                        const int32_t* positions, const float* cos_sin, int64_t max_pos, int64_t B,
+                                        int64_t S, int64_t Hq, int64_t Hkv, int64_t D, const spinq_had_cfg* had,
+                                        const spinq_quant_cfg* kvq, uint8_t* k_codes, float* k_scale,
+                                        float* k_zero, uint8_t* v_codes, float* v_scale, float* v_zero,
+                                        void* stream);
+
+/*
+ * spinq_decode_attention_kv4 -- attention of one decode query per (batch,
+ * query head) over the 4-bit KV cache written by spinq_rotate_quant_kv (or
+ * its RoPE form), the consumer of R3 (Sec. 3.1: R3 rotates Q and K over
+ * head_dim so that Q K^T is unchanged while K quantizes to 4 bits):
+ *   s_t = softmax_scale * q . k_t,  k_t = k_scale * u_t + k_zero,
+ *   o   = sum_t softmax_t(s) v_t,     v_t = v_scale * u'_t + v_zero,
+ * over t < lens[b]; query head h reads kv head h / (Hq / Hkv).
+ *   q        [B][Hq][D] fp16, already rotated by R3 (the q_out of the call
+ *            above for the decode token).
+ *   k_codes, v_codes [B][S][Hkv][D/2]; k_scale, k_zero, v_scale, v_zero
+ *            [B][S][Hkv] fp32 (S is the cache capacity: the row stride).
+ *   lens     [B] int32 in [1, S] (device), or NULL for S everywhere.
+ *   out      [B][Hq][D] fp16.
+ *   workspace device buffer of spinq_decode_attention_workspace_bytes(B, S,
+ *            Hq, Hkv, D) bytes, 16-byte aligned (the per-chunk partial
+ *            results; no zeroing needed).
+ *   Supported: D = 64 or 128, Hq / Hkv in {1, 2, 4, 8}.  Arithmetic in
+ *   fp32; two kernels on `stream` (the chunks, then their merge).
+ */
+int64_t spinq_decode_attention_workspace_bytes(int64_t B, int64_t S, int64_t Hq, int64_t Hkv, int64_t D);
+spinq_status spinq_decode_attention_kv4(const void* q, const uint8_t* k_codes, const float* k_scale,
+                                        const float* k_zero, const uint8_t* v_codes, const float* v_scale,
+                                        const float* v_zero, const int32_t* lens, int64_t B, int64_t S, int64_t Hq,
+                                        int64_t Hkv, int64_t D, float softmax_scale, void* out, void* workspace,
+                                        int64_t workspace_bytes, void* stream);
+
+/*
  * 8-bit variants (main results table, W4A8 rows "4-8-x"; appendix "Latency
  * measurement on GPU": W-fp8-A-fp8 with the dequantization fused into the
  * GEMM epilogue).  They share the rotation convention above and run on the

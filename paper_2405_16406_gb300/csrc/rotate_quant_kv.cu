@@ -43,7 +43,7 @@ __device__ __forceinline__ uint32_t h16_pair(int k0, int k1, int n, bool hadamar
   return pack_half2_bits(v0, v1);
 }
 
-template <int D, bool CLAMP>
+template <int D, bool CLAMP, bool ROPE>
 __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) {
   constexpr int V = D / 32;  // 16-byte chunks per lane
   const int lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
@@ -87,6 +87,35 @@ __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) 
     uint4 in[V];
 #pragma unroll
     for (int v = 0; v < V; ++v) in[v] = valid ? __ldg(p + v) : make_uint4(0, 0, 0, 0);
+
+    if (ROPE && kind != 2) {
+      // Rotary embedding at the row's token position (rotate-half form), in
+      // fp32 from the caller's (cos, sin) table, rounded back to fp16 like the
+      // model's activations: y_i = x_i cos - x_{i+D/2} sin and
+      // y_{i+D/2} = x_i sin + x_{i+D/2} cos.  Lanes c and c ^ 2 of a quad hold
+      // the dimensions i and i + D/2 at the same register positions.
+      const int64_t H = kind == 0 ? a.Hq : a.Hkv;
+      int64_t pos = valid ? (int64_t)a.positions[row / H] : 0;
+      pos = pos < 0 ? 0 : (pos >= a.max_pos ? a.max_pos - 1 : pos);
+      const float2* cs = reinterpret_cast<const float2*>(a.cos_sin) + pos * (D / 2);
+      const bool first = c < 2;
+#pragma unroll
+      for (int v = 0; v < V; ++v) {
+        uint32_t w[4] = {in[v].x, in[v].y, in[v].z, in[v].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t pw = __shfl_xor_sync(0xffffffffu, w[j], 2);
+          const int f = (8 * V * c + 8 * v + 2 * j) & (D / 2 - 1);
+          const float4 t = valid ? __ldg(reinterpret_cast<const float4*>(cs + f)) : make_float4(1.f, 0.f, 1.f, 0.f);
+          const float2 x = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
+          const float2 o = __half22float2(*reinterpret_cast<const __half2*>(&pw));
+          const float y0 = first ? x.x * t.x - o.x * t.y : o.x * t.y + x.x * t.x;
+          const float y1 = first ? x.y * t.z - o.y * t.w : o.y * t.w + x.y * t.z;
+          w[j] = pack_half2_bits(y0, y1);
+        }
+        in[v] = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    }
 
     float y[V][8];
 #pragma unroll
@@ -194,7 +223,7 @@ __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) 
   }
 }
 
-template <int D, bool CLAMP>
+template <int D, bool CLAMP, bool ROPE>
 cudaError_t launch_t(const KVArgs& a, cudaStream_t stream) {
   const int64_t groups = (a.rows_q + 7) / 8 + 2 * ((a.rows_kv + 7) / 8);
   const int sms = device_sm_count();
@@ -202,8 +231,8 @@ cudaError_t launch_t(const KVArgs& a, cudaStream_t stream) {
   const int64_t cap = (int64_t)sms * 16;  // persistent-style cap: 16 blocks of 8 warps per SM
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  const cudaError_t e = launch_pdl(rotate_quant_kv_kernel<D, CLAMP>, dim3((unsigned)blocks), dim3(kWarps * 32), 0,
-                                   stream, 1, a);
+  const cudaError_t e = launch_pdl(rotate_quant_kv_kernel<D, CLAMP, ROPE>, dim3((unsigned)blocks),
+                                   dim3(kWarps * 32), 0, stream, 1, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -213,8 +242,13 @@ cudaError_t launch_t(const KVArgs& a, cudaStream_t stream) {
 cudaError_t launch_rotate_quant_kv(const KVArgs& a, cudaStream_t stream) {
   if (a.rows_q == 0 && a.rows_kv == 0) return cudaSuccess;
   const bool clamp = a.clip < 1.0f;
-  if (a.D == 128) return clamp ? launch_t<128, true>(a, stream) : launch_t<128, false>(a, stream);
-  if (a.D == 64) return clamp ? launch_t<64, true>(a, stream) : launch_t<64, false>(a, stream);
+  if (a.positions) {
+    if (a.D == 128) return clamp ? launch_t<128, true, true>(a, stream) : launch_t<128, false, true>(a, stream);
+    if (a.D == 64) return clamp ? launch_t<64, true, true>(a, stream) : launch_t<64, false, true>(a, stream);
+    return cudaErrorInvalidValue;
+  }
+  if (a.D == 128) return clamp ? launch_t<128, true, false>(a, stream) : launch_t<128, false, false>(a, stream);
+  if (a.D == 64) return clamp ? launch_t<64, true, false>(a, stream) : launch_t<64, false, false>(a, stream);
   return cudaErrorInvalidValue;
 }
 

@@ -289,6 +289,59 @@ spinq_status spinq_w4a8_gemm(const uint8_t* a_planes, const float* a_scale, cons
   return gemm8(true, a_planes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y_f16, acc_out, stream);
 }
 
+spinq_status spinq_rope_rotate_quant_kv(const void* q_in, void* q_out, const void* k_in, const void* v_in,
+                                        const int32_t* positions, const float* cos_sin, int64_t max_pos, int64_t B,
+                                        int64_t S, int64_t Hq, int64_t Hkv, int64_t D, const spinq_had_cfg* had,
+                                        const spinq_quant_cfg* kvq, uint8_t* k_codes, float* k_scale,
+                                        float* k_zero, uint8_t* v_codes, float* v_scale, float* v_zero,
+                                        void* stream) {
+  if (B * S > 0 && (!positions || !cos_sin || max_pos <= 0)) return SPINQ_EINVAL;
+  if (cos_sin && !aligned16(cos_sin)) return SPINQ_EINVAL;
+  if (!had || !kvq || B < 0 || S < 0 || Hq < 0 || Hkv < 0 || D <= 0) return SPINQ_EINVAL;
+  const int64_t rows_q = B * S * Hq, rows_kv = B * S * Hkv;
+  if (rows_q > 0 && (!q_in || !q_out)) return SPINQ_EINVAL;
+  if (rows_kv > 0 && (!k_in || !v_in || !k_codes || !k_scale || !k_zero || !v_codes || !v_scale || !v_zero))
+    return SPINQ_EINVAL;
+  if (!clip_ok(kvq->clip_ratio)) return SPINQ_EINVAL;
+  if (had->n_small != 1 || had->n_pow2 != D) return SPINQ_EINVAL;
+  for (const void* p : {q_in, (const void*)q_out, k_in, v_in, (const void*)k_codes, (const void*)v_codes})
+    if (p && !aligned16(p)) return SPINQ_EINVAL;
+  if (kvq->bits != 4 || kvq->symmetric != 0 || kvq->granularity != SPINQ_PER_GROUP || kvq->group_size != D)
+    return SPINQ_EUNSUPPORTED;
+  if (D != 64 && D != 128) return SPINQ_EUNSUPPORTED;
+  if (rows_q == 0 && rows_kv == 0) return SPINQ_OK;
+  KVArgs a{q_in, q_out, k_in, v_in, rows_q, rows_kv, (int)D, kvq->clip_ratio,
+           (float)(1.0 / std::sqrt((double)D)), k_codes, k_scale, k_zero, v_codes, v_scale, v_zero,
+           positions, cos_sin, max_pos, Hq, Hkv};
+  return from_cuda(launch_rotate_quant_kv(a, static_cast<cudaStream_t>(stream)));
+}
+
+int64_t spinq_decode_attention_workspace_bytes(int64_t B, int64_t S, int64_t Hq, int64_t Hkv, int64_t D) {
+  if (B <= 0 || S <= 0 || Hq <= 0 || Hkv <= 0 || D <= 0) return 0;
+  return B * Hq * (int64_t)decode_attention_chunks(B, S, Hkv) * (D + 2) * 4;
+}
+
+spinq_status spinq_decode_attention_kv4(const void* q, const uint8_t* k_codes, const float* k_scale,
+                                        const float* k_zero, const uint8_t* v_codes, const float* v_scale,
+                                        const float* v_zero, const int32_t* lens, int64_t B, int64_t S, int64_t Hq,
+                                        int64_t Hkv, int64_t D, float softmax_scale, void* out, void* workspace,
+                                        int64_t workspace_bytes, void* stream) {
+  if (B < 0 || S <= 0 || Hq <= 0 || Hkv <= 0 || D <= 0 || !std::isfinite(softmax_scale)) return SPINQ_EINVAL;
+  if (Hq % Hkv != 0) return SPINQ_EINVAL;
+  if (B > 0 && (!q || !k_codes || !k_scale || !k_zero || !v_codes || !v_scale || !v_zero || !out)) return SPINQ_EINVAL;
+  const int64_t need = spinq_decode_attention_workspace_bytes(B, S, Hq, Hkv, D);
+  if (B > 0 && (!workspace || !aligned16(workspace) || workspace_bytes < need)) return SPINQ_EINVAL;
+  for (const void* p : {q, (const void*)k_codes, (const void*)v_codes, (const void*)out})
+    if (p && !aligned16(p)) return SPINQ_EINVAL;
+  const int64_t G = Hq / Hkv;
+  if ((D != 64 && D != 128) || (G != 1 && G != 2 && G != 4 && G != 8)) return SPINQ_EUNSUPPORTED;
+  if (B > 65535 || Hkv > 65535 || S > INT32_MAX) return SPINQ_EUNSUPPORTED;
+  if (B == 0) return SPINQ_OK;
+  AttnArgs a{q, k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, lens, B, S, Hq, Hkv, (int)D, softmax_scale,
+             out, static_cast<float*>(workspace)};
+  return from_cuda(launch_decode_attention(a, decode_attention_chunks(B, S, Hkv), static_cast<cudaStream_t>(stream)));
+}
+
 int spinq_gemm_select_kernel(int kernel) { return w4a4_gemm_select(kernel); }
 
 int spinq_gemm_split_k(int n) { return w4a4_gemm_split_k(n); }

@@ -62,9 +62,35 @@ struct KVArgs {
   uint8_t* v_codes;
   float* v_scale;
   float* v_zero;
+  // rotary embedding ahead of R3 (positions == nullptr: none)
+  const int32_t* positions;  // [B*S] position of each token
+  const float* cos_sin;      // [max_pos][D/2] (cos, sin) pairs
+  int64_t max_pos;
+  int64_t Hq, Hkv;
 };
 
 cudaError_t launch_rotate_quant_kv(const KVArgs& a, cudaStream_t stream);
+
+struct AttnArgs {
+  const void* q;            // fp16 [B][Hq][D]
+  const uint8_t* k_codes;   // [B][S][Hkv][D/2]
+  const float* k_scale;     // [B][S][Hkv]
+  const float* k_zero;
+  const uint8_t* v_codes;
+  const float* v_scale;
+  const float* v_zero;
+  const int32_t* lens;      // [B] or nullptr (= S)
+  int64_t B, S, Hq, Hkv;
+  int D;
+  float scale;
+  void* out;                // fp16 [B][Hq][D]
+  float* workspace;
+};
+
+// Chunks of the cache length that the decode attention splits over (the
+// workspace holds B * Hq * chunks * (D + 2) floats).
+int decode_attention_chunks(int64_t B, int64_t S, int64_t Hkv);
+cudaError_t launch_decode_attention(const AttnArgs& a, int chunks, cudaStream_t stream);
 
 struct GemmArgs {
   const uint8_t* a_codes;

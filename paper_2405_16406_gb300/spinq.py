@@ -39,6 +39,7 @@ EXPORTED = (
     "spinq_w4a4_gemm_splitk", "spinq_w4a4_gemm_noalloc", "spinq_gemm_select_kernel", "spinq_gemm_split_k",
     "spinq_w4a4_gemm_plan", "spinq_w4a4_gemm_splitk_plan", "spinq_cayley_step",
     "spinq_rotate_quant_act8", "spinq_quant_weight8", "spinq_fp8_gemm", "spinq_w4a8_gemm",
+    "spinq_rope_rotate_quant_kv", "spinq_decode_attention_workspace_bytes", "spinq_decode_attention_kv4",
 )
 SPINQ_FMT_INT8_PLANES, SPINQ_FMT_E4M3, SPINQ_FMT_INT4_BYTES = 1, 2, 3
 
@@ -99,6 +100,15 @@ _lib.spinq_fp8_gemm.restype = ctypes.c_int
 _lib.spinq_fp8_gemm.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _P, _P]
 _lib.spinq_w4a8_gemm.restype = ctypes.c_int
 _lib.spinq_w4a8_gemm.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _P, _P]
+_lib.spinq_rope_rotate_quant_kv.restype = ctypes.c_int
+_lib.spinq_rope_rotate_quant_kv.argtypes = [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64, _I64,
+                                            ctypes.POINTER(HadCfg), ctypes.POINTER(QuantCfg),
+                                            _P, _P, _P, _P, _P, _P, _P]
+_lib.spinq_decode_attention_workspace_bytes.restype = ctypes.c_int64
+_lib.spinq_decode_attention_workspace_bytes.argtypes = [_I64, _I64, _I64, _I64, _I64]
+_lib.spinq_decode_attention_kv4.restype = ctypes.c_int
+_lib.spinq_decode_attention_kv4.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
+                                            ctypes.c_float, _P, _P, _I64, _P]
 _lib.spinq_cayley_step.restype = ctypes.c_int
 _lib.spinq_cayley_step.argtypes = [_P, _P, _I64, _I64, ctypes.c_float, ctypes.c_int32, _P, _P, _P]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
@@ -162,6 +172,22 @@ def spinq_fp8_gemm(a_codes, a_scale, w_codes, w_scale, M, N, K, y, stream) -> in
 
 def spinq_w4a8_gemm(a_planes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc, stream) -> int:
     return _lib.spinq_w4a8_gemm(a_planes, a_scale, a_zero, w_codes, w_scale, w_rowsum, M, N, K, y, acc, stream)
+
+
+def spinq_rope_rotate_quant_kv(q_in, q_out, k_in, v_in, positions, cos_sin, max_pos, B, S, Hq, Hkv, D, had, kvq,
+                               k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, stream) -> int:
+    return _lib.spinq_rope_rotate_quant_kv(q_in, q_out, k_in, v_in, positions, cos_sin, max_pos, B, S, Hq, Hkv, D,
+                                           had, kvq, k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, stream)
+
+
+def spinq_decode_attention_workspace_bytes(B, S, Hq, Hkv, D) -> int:
+    return int(_lib.spinq_decode_attention_workspace_bytes(B, S, Hq, Hkv, D))
+
+
+def spinq_decode_attention_kv4(q, k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, lens, B, S, Hq, Hkv, D,
+                               scale, out, ws, ws_bytes, stream) -> int:
+    return _lib.spinq_decode_attention_kv4(q, k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, lens, B, S, Hq,
+                                           Hkv, D, scale, out, ws, ws_bytes, stream)
 
 
 def spinq_cayley_step(R, grad, batch, n, alpha, iters, R_out, Y_out, stream) -> int:
@@ -406,3 +432,49 @@ def w4a8_gemm(a: ActCodes, w: WeightCodes, want_acc: bool = False, y: Optional[t
     _check(_lib.spinq_w4a8_gemm(_ptr(a.codes), _ptr(a.scale), _ptr(a.zero), _ptr(w.codes), _ptr(w.scale),
                                 _ptr(w.rowsum), M, N, K, _ptr(y), _ptr(acc), _stream(stream)), "spinq_w4a8_gemm")
     return (y, acc) if want_acc else y
+
+
+def rope_rotate_quant_kv(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, positions: torch.Tensor,
+                         cos_sin: torch.Tensor, clip: float = 1.0, in_place_q: bool = False,
+                         out: Optional[KVCodes] = None, stream: Optional[torch.cuda.Stream] = None) -> KVCodes:
+    """RoPE at ``positions`` [B, S] (int32) from ``cos_sin`` [max_pos, D/2, 2]
+    (fp32), then R3 and the 4-bit KV quantizer."""
+    B, S, Hq, D = q.shape
+    Hkv = k.shape[2]
+    dev = q.device
+    if out is None:
+        out = KVCodes(q if in_place_q else torch.empty_like(q),
+                      torch.empty((B, S, Hkv, D // 2), dtype=torch.uint8, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev),
+                      torch.empty((B, S, Hkv, D // 2), dtype=torch.uint8, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev),
+                      torch.empty((B, S, Hkv), dtype=torch.float32, device=dev))
+    kvq = quant_cfg(4, False, SPINQ_PER_GROUP, D, clip)
+    had = HadCfg(1, D)
+    _check(_lib.spinq_rope_rotate_quant_kv(_ptr(q), _ptr(out.q_out), _ptr(k), _ptr(v), _ptr(positions),
+                                           _ptr(cos_sin), cos_sin.shape[0], B, S, Hq, Hkv, D, ctypes.byref(had),
+                                           ctypes.byref(kvq), _ptr(out.k_codes), _ptr(out.k_scale),
+                                           _ptr(out.k_zero), _ptr(out.v_codes), _ptr(out.v_scale), _ptr(out.v_zero),
+                                           _stream(stream)), "spinq_rope_rotate_quant_kv")
+    return out
+
+
+def decode_attention_kv4(q: torch.Tensor, kv: KVCodes, lens: Optional[torch.Tensor] = None,
+                         scale: Optional[float] = None, out: Optional[torch.Tensor] = None,
+                         workspace: Optional[torch.Tensor] = None,
+                         stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """Decode attention of q [B, Hq, D] (fp16, rotated) over the 4-bit cache ``kv``."""
+    B, Hq, D = q.shape
+    S, Hkv = kv.k_codes.shape[1], kv.k_codes.shape[2]
+    if out is None:
+        out = torch.empty_like(q)
+    need = spinq_decode_attention_workspace_bytes(B, S, Hq, Hkv, D)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
+    sc = 1.0 / (D ** 0.5) if scale is None else float(scale)
+    _check(_lib.spinq_decode_attention_kv4(_ptr(q), _ptr(kv.k_codes), _ptr(kv.k_scale), _ptr(kv.k_zero),
+                                           _ptr(kv.v_codes), _ptr(kv.v_scale), _ptr(kv.v_zero), _ptr(lens), B, S, Hq,
+                                           Hkv, D, sc, _ptr(out), _ptr(workspace), workspace.numel(),
+                                           _stream(stream)), "spinq_decode_attention_kv4")
+    return out

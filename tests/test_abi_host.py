@@ -190,3 +190,24 @@ def test_8bit_entry_points_reject_invalid_arguments_on_the_host(lib):
     f = S.spinq_fp8_gemm
     assert f(fake, fake, fake, fake, 4, 32, 96, fake, None) == S.SPINQ_EINVAL
     assert f(fake, fake, fake, fake, 0, 32, 128, fake, None) == S.SPINQ_OK
+
+
+def test_attention_entry_points_reject_invalid_arguments_on_the_host(lib):
+    from paper_2405_16406_gb300 import spinq as S
+    fake = ctypes.c_void_p(1 << 20)
+    f = S.spinq_decode_attention_kv4
+    need = S.spinq_decode_attention_workspace_bytes(2, 64, 32, 8, 128)
+    assert need > 0 and S.spinq_decode_attention_workspace_bytes(0, 64, 32, 8, 128) == 0
+    args = [fake] * 7 + [None]
+    assert f(*args, 2, 64, 30, 8, 128, 0.1, fake, fake, need, None) == S.SPINQ_EINVAL          # Hq % Hkv
+    assert f(*args, 2, 64, 32, 8, 128, 0.1, fake, fake, need - 16, None) == S.SPINQ_EINVAL     # workspace
+    assert f(*args, 2, 64, 32, 8, 96, 0.1, fake, fake, 1 << 30, None) == S.SPINQ_EUNSUPPORTED  # D
+    assert f(*args, 2, 64, 48, 2, 128, 0.1, fake, fake, 1 << 30, None) == S.SPINQ_EUNSUPPORTED  # G = 24
+    assert f(*args, 0, 64, 32, 8, 128, 0.1, None, None, 0, None) == S.SPINQ_OK
+    g = S.spinq_rope_rotate_quant_kv
+    kvq = S.quant_cfg(4, False, S.SPINQ_PER_GROUP, 128, 1.0)
+    had = S.HadCfg(1, 128)
+    assert g(fake, fake, fake, fake, None, fake, 4096, 1, 4, 4, 2, 128, ctypes.byref(had), ctypes.byref(kvq),
+             fake, fake, fake, fake, fake, fake, None) == S.SPINQ_EINVAL                       # no positions
+    assert g(fake, fake, fake, fake, fake, ctypes.c_void_p((1 << 20) + 8), 4096, 1, 4, 4, 2, 128, ctypes.byref(had),
+             ctypes.byref(kvq), fake, fake, fake, fake, fake, fake, None) == S.SPINQ_EINVAL    # table alignment
