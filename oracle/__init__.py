@@ -239,14 +239,24 @@ class QuantAct:
 
 
 def rotate_quant_act(x_f16: np.ndarray, had: Optional[Tuple[int, int]], bits: int = 4,
-                     symmetric: bool = True, clip: float = 1.0) -> QuantAct:
+                     symmetric: bool = True, clip: float = 1.0, signs: Optional[np.ndarray] = None) -> QuantAct:
     """Sec. 3.1 R4: x' = x (H_s (x) H_P)/sqrt(K) (skipped if ``had`` is None),
-    then Eq. 1 per token (row)."""
+    then Eq. 1 per token (row).  ``signs`` (+-1 per input index, or None)
+    makes the rotation the random Hadamard S H of the Sec. 2.2 footnote:
+    x' = (x S) (H_s (x) H_P)/sqrt(K)."""
     x = f16_to_f64(x_f16)
+    if signs is not None:
+        x = x * _sign_vector(signs, x.shape[-1])
     xr = rotate(x, had[0], had[1]) if had is not None else x
     codes, alpha, beta = quantize_rows(xr, bits, symmetric, clip)
     return QuantAct(codes, pack4(codes) if bits == 4 else None, alpha,
                     None if symmetric else beta, xr)
+
+
+def _sign_vector(signs: np.ndarray, K: int) -> np.ndarray:
+    s = np.asarray(signs, dtype=np.float64).reshape(-1)
+    assert s.size == K and np.all(np.abs(s) == 1.0), "signs: one +-1 per input index"
+    return s
 
 
 @dataclass
@@ -259,10 +269,13 @@ class QuantWeight:
 
 
 def quant_weight(w_f16: np.ndarray, had: Optional[Tuple[int, int]], bits: int = 4,
-                 clip: float = 1.0) -> QuantWeight:
+                 clip: float = 1.0, signs: Optional[np.ndarray] = None) -> QuantWeight:
     """Sec. 3.1 invariance: W' = W R (each output row rotated like an
-    activation row), then Eq. 1 symmetric per output channel (RTN)."""
+    activation row), then Eq. 1 symmetric per output channel (RTN).  With
+    ``signs``, R = S H / sqrt(K) as for the activations (W' = W S H)."""
     w = f16_to_f64(w_f16)
+    if signs is not None:
+        w = w * _sign_vector(signs, w.shape[-1])
     wr = rotate(w, had[0], had[1]) if had is not None else w
     codes, scale, _ = quantize_rows(wr, bits, True, clip)
     return QuantWeight(codes, pack4(codes), scale, rowsum(codes), wr)

@@ -40,9 +40,11 @@ __device__ __forceinline__ float nib(uint32_t w, int i) {
 }
 
 template <int D, int G>
-__global__ void __launch_bounds__(kAttnWarps * 32) attn_partial_kernel(AttnArgs a, int chunk_len, int nchunk) {
-  constexpr int DPL = D / 32;   // dimensions per lane
-  constexpr int NT = 32 / G;    // tokens per block
+__global__ void __launch_bounds__(kAttnWarps * 32, 4) attn_partial_kernel(AttnArgs a, int chunk_len, int nchunk) {
+  constexpr int DPL = D / 32;                 // dimensions per lane
+  constexpr int NT = 32 / G < 8 ? 32 / G : 8; // tokens per block
+  constexpr int NV = NT * G;                  // dot products per block (8, 16 or 32)
+  constexpr int R = 32 / NV;                  // lanes that end up holding each of them
   __shared__ float p_s[kAttnWarps][32];
   __shared__ float c_s[kAttnWarps][G];
   __shared__ float m_s[kAttnWarps][G], l_s[kAttnWarps][G];
@@ -79,25 +81,47 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_partial_kernel(AttnArgs 
 #pragma unroll
     for (int i = 0; i < DPL; ++i) acc[h][i] = 0.f;
   }
-  // this lane's pair of the block: token jt = lane / G, head jh = lane % G
-  const int jt = lane / G, jh = lane % G;
+  // this lane's pair of the block: value vi = lane / R, token jt = vi / G,
+  // head jh = vi % G
+  const int vi = lane / R, jt = vi / G, jh = vi % G;
   const size_t kv_stride = (size_t)a.Hkv;   // rows between consecutive tokens
 
-  for (int64_t blk = t0 + (int64_t)warp * NT; blk < t1; blk += (int64_t)kAttnWarps * NT) {
-    // ---- scores: 32 dot products (token, head) of the block
-    uint32_t kw[NT];
+  // Every load of a block (key and value codes, their scales) is issued
+  // before any arithmetic on it: one memory round trip per block.
+  struct Blk {
+    uint32_t kw[NT], vw[NT];
+    float ka, kb;     // key scale / zero of token jt (this lane's pair)
+    float va, vb;     // value scale / zero of token (lane % NT)
+  };
+  auto load = [&](int64_t blk, Blk& x) {
 #pragma unroll
     for (int tt = 0; tt < NT; ++tt) {
       const int64_t t = blk + tt;
-      const uint8_t* kc = a.k_codes + (((size_t)b * a.S + t) * kv_stride + hk) * (D / 2) + (DPL / 2) * lane;
-      kw[tt] = t < t1 ? (DPL == 4 ? (uint32_t)*reinterpret_cast<const uint16_t*>(kc) : (uint32_t)*kc) : 0u;
+      const size_t r = ((size_t)b * a.S + t) * kv_stride + hk;
+      const uint8_t* kc = a.k_codes + r * (D / 2) + (DPL / 2) * lane;
+      const uint8_t* vc = a.v_codes + r * (D / 2) + (DPL / 2) * lane;
+      const bool in = t < t1;
+      x.kw[tt] = in ? (DPL == 4 ? (uint32_t)*reinterpret_cast<const uint16_t*>(kc) : (uint32_t)*kc) : 0u;
+      x.vw[tt] = in ? (DPL == 4 ? (uint32_t)*reinterpret_cast<const uint16_t*>(vc) : (uint32_t)*vc) : 0u;
     }
-    float v[32];
+    const int64_t tk = blk + jt, tv = blk + (lane % NT);
+    const size_t rk = ((size_t)b * a.S + tk) * kv_stride + hk, rv = ((size_t)b * a.S + tv) * kv_stride + hk;
+    x.ka = tk < t1 ? a.k_scale[rk] : 0.f;
+    x.kb = tk < t1 ? a.k_zero[rk] : 0.f;
+    x.va = tv < t1 ? a.v_scale[rv] : 0.f;
+    x.vb = tv < t1 ? a.v_zero[rv] : 0.f;
+  };
+  const int64_t step = (int64_t)kAttnWarps * NT;
+  Blk cur;
+  for (int64_t blk = t0 + (int64_t)warp * NT; blk < t1; blk += step) {
+    load(blk, cur);
+    // ---- scores: 32 dot products (token, head) of the block
+    float v[NV];
 #pragma unroll
     for (int tt = 0; tt < NT; ++tt) {
       float u[DPL];
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) u[i] = nib(kw[tt], i);
+      for (int i = 0; i < DPL; ++i) u[i] = nib(cur.kw[tt], i);
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         float d = 0.f;
@@ -106,9 +130,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_partial_kernel(AttnArgs 
         v[tt * G + h] = d;
       }
     }
-    // transpose-reduction: after it, lane j holds the warp sum of v[j]
+    // transpose-reduction: halving rounds over the top lane bits, then plain
+    // sums over the rest; after it, lane j holds the warp sum of v[j / R]
 #pragma unroll
-    for (int o = 16, n = 32; o >= 1; o >>= 1, n >>= 1) {
+    for (int o = 16, n = NV; n > 1; o >>= 1, n >>= 1) {
       const bool up = (lane & o) != 0;
 #pragma unroll
       for (int i = 0; i < n / 2; ++i) {
@@ -117,16 +142,14 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_partial_kernel(AttnArgs 
         v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
       }
     }
+#pragma unroll
+    for (int o = R / 2; o >= 1; o >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
     const int64_t tj = blk + jt;
-    float s = -FLT_MAX;
-    if (tj < t1) {
-      const size_t r = ((size_t)b * a.S + tj) * kv_stride + hk;
-      s = a.scale * fmaf(a.k_scale[r], v[0], a.k_zero[r] * qsum[jh]);
-    }
+    const float s = tj < t1 ? a.scale * fmaf(cur.ka, v[0], cur.kb * qsum[jh]) : -FLT_MAX;
     // block maximum and sum per head: lanes with the same head differ in the bits above log2(G)
     float mx = s;
 #pragma unroll
-    for (int o = G; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    for (int o = G * R; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     float mh = m[0];
 #pragma unroll
     for (int h = 1; h < G; ++h)
@@ -135,39 +158,33 @@ __global__ void __launch_bounds__(kAttnWarps * 32) attn_partial_kernel(AttnArgs 
     const float p = tj < t1 ? __expf(s - mnew) : 0.f;
     float ps = p;
 #pragma unroll
-    for (int o = G; o < 32; o <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
-    p_s[warp][lane] = p;
-    if (lane < G) c_s[warp][lane] = __expf(mh - mnew);   // lane h < G holds head h (jt = 0)
+    for (int o = G * R; o < 32; o <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
+    if (lane % R == 0) p_s[warp][vi] = p;
+    if (jt == 0 && lane % R == 0) c_s[warp][jh] = __expf(mh - mnew);   // lane h R holds head h
     __syncwarp();
     // new per-head state in every lane
 #pragma unroll
     for (int h = 0; h < G; ++h) {
       const float corr = c_s[warp][h];
-      const float m_h = __shfl_sync(0xffffffffu, mnew, h);
-      const float s_h = __shfl_sync(0xffffffffu, ps, h);
+      const float m_h = __shfl_sync(0xffffffffu, mnew, h * R);
+      const float s_h = __shfl_sync(0xffffffffu, ps, h * R);
       l[h] = l[h] * corr + s_h;
       m[h] = m_h;
 #pragma unroll
       for (int i = 0; i < DPL; ++i) acc[h][i] *= corr;
     }
-    // ---- values
-#pragma unroll 4
+    // ---- values (weights of masked tokens are 0, their codes 0)
+#pragma unroll
     for (int tt = 0; tt < NT; ++tt) {
-      const int64_t t = blk + tt;
-      if (t < t1) {
-        const size_t r = ((size_t)b * a.S + t) * kv_stride + hk;
-        const uint8_t* vc = a.v_codes + r * (D / 2) + (DPL / 2) * lane;
-        const uint32_t w = DPL == 4 ? *reinterpret_cast<const uint16_t*>(vc) : *vc;
-        const float al = a.v_scale[r], be = a.v_zero[r];
-        float vv[DPL];
+      const float al = __shfl_sync(0xffffffffu, cur.va, tt), be = __shfl_sync(0xffffffffu, cur.vb, tt);
+      float vv[DPL];
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) vv[i] = fmaf(al, nib(w, i), be);
+      for (int i = 0; i < DPL; ++i) vv[i] = fmaf(al, nib(cur.vw[tt], i), be);
 #pragma unroll
-        for (int h = 0; h < G; ++h) {
-          const float pw = p_s[warp][tt * G + h];
+      for (int h = 0; h < G; ++h) {
+        const float pw = p_s[warp][tt * G + h];
 #pragma unroll
-          for (int i = 0; i < DPL; ++i) acc[h][i] = fmaf(pw, vv[i], acc[h][i]);
-        }
+        for (int i = 0; i < DPL; ++i) acc[h][i] = fmaf(pw, vv[i], acc[h][i]);
       }
     }
     __syncwarp();
@@ -253,9 +270,9 @@ cudaError_t launch_d(const AttnArgs& a, int nchunk, cudaStream_t stream) {
 }  // namespace
 
 int decode_attention_chunks(int64_t B, int64_t S, int64_t Hkv) {
-  // about four CTAs per SM, at least 32 tokens per chunk
+  // about eight CTAs per SM, at least 32 tokens per chunk
   const int64_t pairs = B * Hkv > 0 ? B * Hkv : 1;
-  int64_t n = (4 * (int64_t)device_sm_count() + pairs - 1) / pairs;
+  int64_t n = (8 * (int64_t)device_sm_count() + pairs - 1) / pairs;
   const int64_t by_len = (S + 31) / 32;
   if (n > by_len) n = by_len;
   if (n > 1024) n = 1024;

@@ -34,7 +34,7 @@ __device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
   return r;
 }
 
-template <int FMT, bool SYM, bool CLAMP>
+template <int FMT, bool SYM, bool CLAMP, int NS>
 __global__ void __launch_bounds__(kThreads) rq8_rows_kernel(Rq8Args a) {
   extern __shared__ float s[];
   __shared__ float red_hi[kThreads / 32], red_lo[kThreads / 32];
@@ -73,14 +73,20 @@ __global__ void __launch_bounds__(kThreads) rq8_rows_kernel(Rq8Args a) {
         }
         __syncthreads();
       }
-      const int ns = a.n_small;
-      if (ns > 1) {
+      if constexpr (NS > 1) {
+        // the small factor, unrolled at its compile-time order (registers only)
+        uint32_t neg[NS];
+#pragma unroll
+        for (int ip = 0; ip < NS; ++ip) neg[ip] = a.hs.neg[ip];
         for (int j = tid; j < P; j += kThreads) {
-          float t[32];
-          for (int ip = 0; ip < ns; ++ip) t[ip] = s[ip * P + j];
-          for (int i = 0; i < ns; ++i) {
+          float t[NS];
+#pragma unroll
+          for (int ip = 0; ip < NS; ++ip) t[ip] = s[ip * P + j];
+#pragma unroll
+          for (int i = 0; i < NS; ++i) {
             float acc = 0.f;
-            for (int ip = 0; ip < ns; ++ip) acc += ((a.hs.neg[ip] >> i) & 1u) ? -t[ip] : t[ip];
+#pragma unroll
+            for (int ip = 0; ip < NS; ++ip) acc += ((neg[ip] >> i) & 1u) ? -t[ip] : t[ip];
             s[i * P + j] = acc;
           }
         }
@@ -190,10 +196,10 @@ __global__ void __launch_bounds__(kThreads) rq8_rows_kernel(Rq8Args a) {
   }
 }
 
-template <int FMT, bool SYM, bool CLAMP>
-cudaError_t launch_t(const Rq8Args& a, cudaStream_t stream) {
+template <int FMT, bool SYM, bool CLAMP, int NS>
+cudaError_t launch_ns(const Rq8Args& a, cudaStream_t stream) {
   const size_t smem = sizeof(float) * (size_t)a.K;
-  auto kern = rq8_rows_kernel<FMT, SYM, CLAMP>;
+  auto kern = rq8_rows_kernel<FMT, SYM, CLAMP, NS>;
   int per_sm = 0;
   cudaError_t e = prepare_launch(kern, kThreads, smem, &per_sm);
   if (e != cudaSuccess) return e;
@@ -202,6 +208,16 @@ cudaError_t launch_t(const Rq8Args& a, cudaStream_t stream) {
   e = launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), smem, stream, 1, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+template <int FMT, bool SYM, bool CLAMP>
+cudaError_t launch_t(const Rq8Args& a, cudaStream_t stream) {
+  switch (a.n_small) {
+    case 12: return launch_ns<FMT, SYM, CLAMP, 12>(a, stream);
+    case 20: return launch_ns<FMT, SYM, CLAMP, 20>(a, stream);
+    case 28: return launch_ns<FMT, SYM, CLAMP, 28>(a, stream);
+  }
+  return launch_ns<FMT, SYM, CLAMP, 1>(a, stream);
 }
 
 template <int FMT>
