@@ -117,6 +117,24 @@ spinq_status spinq_quant_weight(const void* w_f16, int64_t N, int64_t K, const s
                                 int32_t* rowsum, void* stream);
 
 /*
+ * Random-sign rotation (Sec. 2.2 footnote: a Hadamard matrix multiplied by a
+ * random +-1 diagonal S is again a rotation, a "random Hadamard matrix"):
+ * R = S (H_s (x) H_P) / sqrt(K), the signs acting on the input index k:
+ * x' = (x S) (H_s (x) H_P) / sqrt(K), and W' = W S H / sqrt(K) for the merged
+ * weights, so that x' W'^T = x W^T still holds.
+ *   signs  device bit mask [K/8] bytes: bit (k % 8) of byte k / 8 set means
+ *          s_k = -1.  Requires a Hadamard spec (had != NULL).
+ * Other arguments as spinq_rotate_quant_act / spinq_quant_weight.
+ */
+spinq_status spinq_rotate_quant_act_signed(const void* x_f16, int64_t M, int64_t K, int64_t ldx,
+                                           const spinq_had_cfg* had, const uint8_t* signs,
+                                           const spinq_quant_cfg* q, uint8_t* codes, float* scale, float* zero,
+                                           void* stream);
+spinq_status spinq_quant_weight_signed(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
+                                       const uint8_t* signs, const spinq_quant_cfg* q, uint8_t* codes,
+                                       float* scale, int32_t* rowsum, void* stream);
+
+/*
  * spinq_w4a4_gemm -- the W4A4 linear on Eq. 1 codes with an exact integer
  * accumulator and a fused per-token x per-channel dequantization epilogue.
  *   acc[m][n] = sum_k a_mk * q_nk, a = q (symmetric activations) or u - 8
@@ -208,6 +226,26 @@ spinq_status spinq_w4a4_gemm_noalloc(const uint8_t* a_codes, const float* a_scal
                                      const uint8_t* w_codes, const float* w_scale,
                                      const int32_t* w_rowsum, int64_t M, int64_t N, int64_t K,
                                      void* y_f16, int32_t* acc_out, void* stream);
+
+/*
+ * spinq_rotated_linear -- the down_proj of Sec. 3.1 in one call: the online
+ * rotation R4 (optionally with random signs, as spinq_rotate_quant_act_signed)
+ * fused with the per-token Eq. 1 quantizer, then the W4A4 GEMM on those codes
+ * against weights merged with the same rotation (spinq_quant_weight[_signed]).
+ * The two kernels run back to back on `stream` (the GEMM's prologue overlaps
+ * the quantizer's tail) and hand the codes over in `workspace`, which stays
+ * in L2 between them (14.7 MB for 2048 tokens of K = 14336).
+ *   x_f16 [M][ldx], had, signs (NULL = none), q (activation quantizer, 4
+ *   bits, per token) as spinq_rotate_quant_act(_signed); w_codes [N][K/2],
+ *   w_scale [N], w_rowsum [N], y_f16 [M][N] as spinq_w4a4_gemm.
+ *   workspace  device buffer of spinq_rotated_linear_workspace_bytes(M, K)
+ *              bytes, 16-byte aligned: the codes and scales in flight.
+ */
+int64_t spinq_rotated_linear_workspace_bytes(int64_t M, int64_t K);
+spinq_status spinq_rotated_linear(const void* x_f16, int64_t M, int64_t K, int64_t ldx, const spinq_had_cfg* had,
+                                  const uint8_t* signs, const spinq_quant_cfg* q, const uint8_t* w_codes,
+                                  const float* w_scale, const int32_t* w_rowsum, int64_t N, void* y_f16,
+                                  void* workspace, int64_t workspace_bytes, void* stream);
 
 /*
  * spinq_rotate_quant_kv -- R3 on Q and K over head_dim, then the 4-bit

@@ -108,7 +108,7 @@ struct Pow2Smem {
   static constexpr int BYTES = OFF_MISC + 16 + 2 * S::W * 4;
 };
 
-template <int LW, int L, bool SYM, bool CLAMP>
+template <int LW, int L, bool SYM, bool CLAMP, bool SG>
 __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
   using S = Pow2Shape<LW, L>;
   using SM = Pow2Smem<LW, L>;
@@ -136,6 +136,16 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
   pdl_wait();
   pdl_trigger();
   rs.prologue();
+  // Random signs (R = S H): chunk v of this lane is chunk ch of every row,
+  // whose 8 sign bits are byte ch of the bit mask; gathered once.
+  uint32_t sgb[(S::V + 3) / 4];
+#pragma unroll
+  for (int t = 0; t < (S::V + 3) / 4; ++t) sgb[t] = 0;
+  if constexpr (SG) {
+#pragma unroll
+    for (int v = 0; v < S::V; ++v)
+      sgb[v >> 2] |= (uint32_t)a.signs[lane + 32 * (w + S::W * v)] << (8 * (v & 3));
+  }
 
   // phase-2 fixed element bits of this thread: {L..2}, {3, 4}, v bits
   const uint32_t t_lo = (uint32_t)tid & ((1u << (3 - L)) - 1u);
@@ -154,7 +164,17 @@ __global__ void __launch_bounds__(32 << LW) rq_pow2_kernel(RotQuantArgs a) {
     const uint4* src = reinterpret_cast<const uint4*>(rs.stage(it));
     F2 y[S::V][4];  // y[v][q] = elements (2q, 2q + 1) of chunk v
 #pragma unroll
-    for (int v = 0; v < S::V; ++v) chunk_mma(src[lane + 32 * (w + S::W * v)], bh, y[v]);
+    for (int v = 0; v < S::V; ++v) {
+      uint4 in = src[lane + 32 * (w + S::W * v)];
+      if constexpr (SG) {   // negate the fp16 elements whose sign bit is set
+        const uint32_t B = sgb[v >> 2] >> (8 * (v & 3));
+        in.x ^= ((B & 1u) << 15) | ((B & 2u) << 30);
+        in.y ^= ((B & 4u) << 13) | ((B & 8u) << 28);
+        in.z ^= ((B & 16u) << 11) | ((B & 32u) << 26);
+        in.w ^= ((B & 64u) << 9) | ((B & 128u) << 24);
+      }
+      chunk_mma(in, bh, y[v]);
+    }
     rs.release_warp(it, release_count, S::W);  // the next copy into this stage overlaps the rest of the row
 #pragma unroll
     for (int v = 0; v < S::V; ++v) {  // e1
@@ -359,22 +379,22 @@ cudaError_t launch_rows(Kern kern, int threads, size_t smem, const RotQuantArgs&
   return cudaGetLastError();
 }
 
-template <int LW, int L, bool SYM, bool CLAMP>
+template <int LW, int L, bool SYM, bool CLAMP, bool SG>
 cudaError_t launch_pow2(const RotQuantArgs& a, cudaStream_t stream) {
   using S = Pow2Shape<LW, L>;
-  return launch_rows(rq_pow2_kernel<LW, L, SYM, CLAMP>, S::T, Pow2Smem<LW, L>::BYTES, a, stream);
+  return launch_rows(rq_pow2_kernel<LW, L, SYM, CLAMP, SG>, S::T, Pow2Smem<LW, L>::BYTES, a, stream);
 }
 
-template <bool SYM, bool CLAMP>
+template <bool SYM, bool CLAMP, bool SG = false>
 cudaError_t launch_pow2_for(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
   *handled = true;
   switch (a.n_pow2) {
-    case 512: return launch_pow2<0, 1, SYM, CLAMP>(a, stream);
-    case 1024: return launch_pow2<0, 2, SYM, CLAMP>(a, stream);
-    case 2048: return launch_pow2<1, 1, SYM, CLAMP>(a, stream);
-    case 4096: return launch_pow2<1, 2, SYM, CLAMP>(a, stream);
-    case 8192: return launch_pow2<2, 1, SYM, CLAMP>(a, stream);
-    case 16384: return launch_pow2<2, 2, SYM, CLAMP>(a, stream);
+    case 512: return launch_pow2<0, 1, SYM, CLAMP, SG>(a, stream);
+    case 1024: return launch_pow2<0, 2, SYM, CLAMP, SG>(a, stream);
+    case 2048: return launch_pow2<1, 1, SYM, CLAMP, SG>(a, stream);
+    case 4096: return launch_pow2<1, 2, SYM, CLAMP, SG>(a, stream);
+    case 8192: return launch_pow2<2, 1, SYM, CLAMP, SG>(a, stream);
+    case 16384: return launch_pow2<2, 2, SYM, CLAMP, SG>(a, stream);
   }
   *handled = false;
   return cudaSuccess;
@@ -408,6 +428,11 @@ cudaError_t launch_rotate_quant_act_fast(const RotQuantArgs& a, cudaStream_t str
     if (a.symmetric)
       return clamp ? launch_norot_for<true, true>(a, stream, handled) : launch_norot_for<true, false>(a, stream, handled);
     return clamp ? launch_norot_for<false, true>(a, stream, handled) : launch_norot_for<false, false>(a, stream, handled);
+  }
+  if (a.n_small == 1 && a.signs) {   // random signs: the unclipped forms (clipped ones take the generic kernel)
+    if (clamp) return cudaSuccess;
+    return a.symmetric ? launch_pow2_for<true, false, true>(a, stream, handled)
+                       : launch_pow2_for<false, false, true>(a, stream, handled);
   }
   if (a.n_small == 1) {
     if (a.symmetric)

@@ -120,7 +120,7 @@ __device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
-template <int NS, int LP, bool SYM, bool CLAMP>
+template <int NS, int LP, bool SYM, bool CLAMP, bool SG>
 __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
     rq_paley_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
   using S = PaleyShape<NS, LP>;
@@ -191,6 +191,31 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
         }
       }
     const uint32_t zero_addr = smem_u32(smem + S::OFF_ZERO);
+    // Random signs (R = S H): each fragment element below sits at the same
+    // row position for every row, so this lane gathers its sign bits once:
+    // bit ((v KS + ks) 4 + q) 2 + e is the sign of element e of fragment q.
+    constexpr int NSB = (4 * S::KS * 4 * 2 + 31) / 32;
+    uint32_t sgn[NSB];
+#pragma unroll
+    for (int t = 0; t < NSB; ++t) sgn[t] = 0;
+    if constexpr (SG) {
+#pragma unroll
+      for (int v = 0; v < 4; ++v)
+#pragma unroll
+        for (int ks = 0; ks < S::KS; ++ks)
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int ip = 8 * (q >> 1) + 16 * ks + 2 * c + e;
+              const int j = 16 * (w + W * v) + 8 * (q & 1) + g;
+              const int idx = ((v * S::KS + ks) * 4 + q) * 2 + e;
+              if (ip < NS) {
+                const int k = ip * P + j;
+                sgn[idx >> 5] |= (uint32_t)((a.signs[k >> 3] >> (k & 7)) & 1) << (idx & 31);
+              }
+            }
+    }
     // transpose-buffer position of j = 16 (w + W v) + 8 h + g, minus 8 h: bit 2
     // of j flips with v & 1, bit 4 (the low bit of w) with v >> 1
     int pos[4];
@@ -217,6 +242,14 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
               ip < NS ? stage_addr + (uint32_t)(line * 128 + ((((js & 63) >> 3) ^ (line & 7)) << 4)) : zero_addr;
           uint32_t af[4];
           ldmatrix_x4_trans(af, addr);
+          if constexpr (SG) {   // negate the fp16 elements whose sign bit is set
+#pragma unroll
+            for (int q2 = 0; q2 < 4; ++q2) {
+              const int idx = ((v * S::KS + ks) * 4 + q2) * 2;
+              const uint32_t bb = (sgn[idx >> 5] >> (idx & 31)) & 3u;
+              af[q2] ^= ((bb & 1u) << 15) | ((bb & 2u) << 30);
+            }
+          }
 #pragma unroll
           for (int nt = 0; nt < S::NT; ++nt) {
             if (ks == 0)
@@ -419,7 +452,7 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
   }
 }
 
-template <int NS, int LP, bool SYM, bool CLAMP>
+template <int NS, int LP, bool SYM, bool CLAMP, bool SG>
 cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
   using S = PaleyShape<NS, LP>;
   // rows as (j_lo, i, j_hi, row): one copy lands a row as 128-byte swizzled lines i + NS j_hi
@@ -434,7 +467,7 @@ cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorNotSupported;
-  auto kern = rq_paley_kernel<NS, LP, SYM, CLAMP>;
+  auto kern = rq_paley_kernel<NS, LP, SYM, CLAMP, SG>;
   int per_sm = 0;
   cudaError_t e = prepare_launch(kern, S::THREADS, S::BYTES, &per_sm);
   if (e != cudaSuccess) return e;
@@ -445,13 +478,13 @@ cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-template <int NS, bool SYM, bool CLAMP>
+template <int NS, bool SYM, bool CLAMP, bool SG>
 cudaError_t launch_ns(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
   *handled = true;
   switch (a.n_pow2) {
-    case 128: return launch_paley<NS, 7, SYM, CLAMP>(a, stream);
-    case 256: return launch_paley<NS, 8, SYM, CLAMP>(a, stream);
-    case 512: return launch_paley<NS, 9, SYM, CLAMP>(a, stream);
+    case 128: return launch_paley<NS, 7, SYM, CLAMP, SG>(a, stream);
+    case 256: return launch_paley<NS, 8, SYM, CLAMP, SG>(a, stream);
+    case 512: return launch_paley<NS, 9, SYM, CLAMP, SG>(a, stream);
   }
   *handled = false;
   return cudaSuccess;
@@ -477,7 +510,7 @@ SmallHadamard kron_h2(const SmallHadamard& h) {
   return r;
 }
 
-template <bool SYM, bool CLAMP>
+template <bool SYM, bool CLAMP, bool SG>
 cudaError_t launch_sc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
   if (a.n_small == 12 && a.n_pow2 == 256) {
     RotQuantArgs b = a;
@@ -485,12 +518,12 @@ cudaError_t launch_sc(const RotQuantArgs& a, cudaStream_t stream, bool* handled)
     b.n_small = 24;
     b.n_pow2 = 128;
     *handled = true;
-    return launch_paley<24, 7, SYM, CLAMP>(b, stream);
+    return launch_paley<24, 7, SYM, CLAMP, SG>(b, stream);
   }
   switch (a.n_small) {
-    case 12: return launch_ns<12, SYM, CLAMP>(a, stream, handled);
-    case 20: return launch_ns<20, SYM, CLAMP>(a, stream, handled);
-    case 28: return launch_ns<28, SYM, CLAMP>(a, stream, handled);
+    case 12: return launch_ns<12, SYM, CLAMP, SG>(a, stream, handled);
+    case 20: return launch_ns<20, SYM, CLAMP, SG>(a, stream, handled);
+    case 28: return launch_ns<28, SYM, CLAMP, SG>(a, stream, handled);
   }
   *handled = false;
   return cudaSuccess;
@@ -503,8 +536,14 @@ cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a, cudaStream_t st
   if (a.rows == 0 || a.rowsum || a.n_small <= 1) return cudaSuccess;
   if ((a.ldx * 2) % 16 != 0) return cudaSuccess;
   const bool clamp = a.clip < 1.0f;
-  if (a.symmetric) return clamp ? launch_sc<true, true>(a, stream, handled) : launch_sc<true, false>(a, stream, handled);
-  return clamp ? launch_sc<false, true>(a, stream, handled) : launch_sc<false, false>(a, stream, handled);
+  if (a.signs) {   // random signs: the unclipped forms (clipped ones take the generic kernel)
+    if (clamp) return cudaSuccess;
+    return a.symmetric ? launch_sc<true, false, true>(a, stream, handled)
+                       : launch_sc<false, false, true>(a, stream, handled);
+  }
+  if (a.symmetric)
+    return clamp ? launch_sc<true, true, false>(a, stream, handled) : launch_sc<true, false, false>(a, stream, handled);
+  return clamp ? launch_sc<false, true, false>(a, stream, handled) : launch_sc<false, false, false>(a, stream, handled);
 }
 
 }  // namespace spinq

@@ -56,11 +56,12 @@ __global__ void __launch_bounds__(kThreads) rotate_quant_rows_kernel(RotQuantArg
     for (int c = tid; c < K / 8; c += kThreads) {
       const uint4 v = __ldg(reinterpret_cast<const uint4*>(xr) + c);
       const __half2* h = reinterpret_cast<const __half2*>(&v);
+      const uint32_t sb = a.signs ? a.signs[c] : 0u;   // random signs of R = S H (bit e: element 8c + e)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const float2 f = __half22float2(h[e]);
-        s[8 * c + 2 * e] = f.x;
-        s[8 * c + 2 * e + 1] = f.y;
+        s[8 * c + 2 * e] = (sb >> (2 * e)) & 1u ? -f.x : f.x;
+        s[8 * c + 2 * e + 1] = (sb >> (2 * e + 1)) & 1u ? -f.y : f.y;
       }
     }
     __syncthreads();

@@ -55,10 +55,11 @@ const char* spinq_status_string(spinq_status s) {
 
 const char* spinq_version(void) { return "spinq-gb300 sm_103a 0.1"; }
 
-spinq_status spinq_rotate_quant_act(const void* x_f16, int64_t M, int64_t K, int64_t ldx,
-                                    const spinq_had_cfg* had, const spinq_quant_cfg* q,
-                                    uint8_t* codes, float* scale, float* zero, void* stream) {
+static spinq_status rqa(const void* x_f16, int64_t M, int64_t K, int64_t ldx, const spinq_had_cfg* had,
+                        const uint8_t* signs, const spinq_quant_cfg* q, uint8_t* codes, float* scale, float* zero,
+                        void* stream) {
   if (!q || M < 0 || K <= 0 || ldx < K) return SPINQ_EINVAL;
+  if (signs && !had) return SPINQ_EINVAL;
   if (M > 0 && (!x_f16 || !codes || !scale)) return SPINQ_EINVAL;
   if (!clip_ok(q->clip_ratio)) return SPINQ_EINVAL;
   if (q->symmetric != 0 && q->symmetric != 1) return SPINQ_EINVAL;
@@ -89,13 +90,28 @@ spinq_status spinq_rotate_quant_act(const void* x_f16, int64_t M, int64_t K, int
   a.scale = scale;
   a.zero = q->symmetric ? nullptr : zero;
   a.rowsum = nullptr;
+  a.signs = signs;
   return from_cuda(launch_rotate_quant_rows(a, static_cast<cudaStream_t>(stream)));
 }
 
-spinq_status spinq_quant_weight(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
-                                const spinq_quant_cfg* q, uint8_t* codes, float* scale,
-                                int32_t* rowsum, void* stream) {
+spinq_status spinq_rotate_quant_act(const void* x_f16, int64_t M, int64_t K, int64_t ldx,
+                                    const spinq_had_cfg* had, const spinq_quant_cfg* q,
+                                    uint8_t* codes, float* scale, float* zero, void* stream) {
+  return rqa(x_f16, M, K, ldx, had, nullptr, q, codes, scale, zero, stream);
+}
+
+spinq_status spinq_rotate_quant_act_signed(const void* x_f16, int64_t M, int64_t K, int64_t ldx,
+                                           const spinq_had_cfg* had, const uint8_t* signs,
+                                           const spinq_quant_cfg* q, uint8_t* codes, float* scale, float* zero,
+                                           void* stream) {
+  if (!signs || !had) return SPINQ_EINVAL;
+  return rqa(x_f16, M, K, ldx, had, signs, q, codes, scale, zero, stream);
+}
+
+static spinq_status qw(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had, const uint8_t* signs,
+                       const spinq_quant_cfg* q, uint8_t* codes, float* scale, int32_t* rowsum, void* stream) {
   if (!q || N < 0 || K <= 0) return SPINQ_EINVAL;
+  if (signs && !had) return SPINQ_EINVAL;
   if (N > 0 && (!w_f16 || !codes || !scale || !rowsum)) return SPINQ_EINVAL;
   if (!clip_ok(q->clip_ratio)) return SPINQ_EINVAL;
   if (K % 32 != 0 || !aligned16(w_f16) || !aligned16(codes)) return SPINQ_EINVAL;
@@ -124,7 +140,50 @@ spinq_status spinq_quant_weight(const void* w_f16, int64_t N, int64_t K, const s
   a.scale = scale;
   a.zero = nullptr;
   a.rowsum = rowsum;
+  a.signs = signs;
   return from_cuda(launch_rotate_quant_rows(a, static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_quant_weight(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
+                                const spinq_quant_cfg* q, uint8_t* codes, float* scale,
+                                int32_t* rowsum, void* stream) {
+  return qw(w_f16, N, K, had, nullptr, q, codes, scale, rowsum, stream);
+}
+
+spinq_status spinq_quant_weight_signed(const void* w_f16, int64_t N, int64_t K, const spinq_had_cfg* had,
+                                       const uint8_t* signs, const spinq_quant_cfg* q, uint8_t* codes,
+                                       float* scale, int32_t* rowsum, void* stream) {
+  if (!signs || !had) return SPINQ_EINVAL;
+  return qw(w_f16, N, K, had, signs, q, codes, scale, rowsum, stream);
+}
+
+// bytes of the codes / alpha / beta hand-off of spinq_rotated_linear, each
+// part 256-byte aligned
+static int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
+
+int64_t spinq_rotated_linear_workspace_bytes(int64_t M, int64_t K) {
+  if (M <= 0 || K <= 0) return 0;
+  return align256(M * (K / 2)) + 2 * align256(M * 4);
+}
+
+spinq_status spinq_rotated_linear(const void* x_f16, int64_t M, int64_t K, int64_t ldx, const spinq_had_cfg* had,
+                                  const uint8_t* signs, const spinq_quant_cfg* q, const uint8_t* w_codes,
+                                  const float* w_scale, const int32_t* w_rowsum, int64_t N, void* y_f16,
+                                  void* workspace, int64_t workspace_bytes, void* stream) {
+  if (!q || M < 0 || N < 0 || K <= 0) return SPINQ_EINVAL;
+  const int64_t need = spinq_rotated_linear_workspace_bytes(M, K);
+  if (M > 0 && (!workspace || !aligned16(workspace) || workspace_bytes < need)) return SPINQ_EINVAL;
+  if (K % 128 != 0 || N % 16 != 0) return SPINQ_EINVAL;
+  if (M > 0 && N > 0 && (!w_codes || !w_scale || !w_rowsum || !y_f16)) return SPINQ_EINVAL;
+  if (M == 0 || N == 0) return SPINQ_OK;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  uint8_t* codes = ws;
+  float* alpha = reinterpret_cast<float*>(ws + align256(M * (K / 2)));
+  float* beta = reinterpret_cast<float*>(ws + align256(M * (K / 2)) + align256(M * 4));
+  spinq_status st = rqa(x_f16, M, K, ldx, had, signs, q, codes, alpha, beta, stream);
+  if (st != SPINQ_OK) return st;
+  return spinq_w4a4_gemm(codes, alpha, q->symmetric ? nullptr : beta, w_codes, w_scale, w_rowsum, M, N, K, y_f16,
+                         nullptr, stream);
 }
 
 spinq_status spinq_w4a4_gemm(const uint8_t* a_codes, const float* a_scale, const float* a_zero,

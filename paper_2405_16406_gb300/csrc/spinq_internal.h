@@ -34,6 +34,7 @@ struct RotQuantArgs {
   float* scale;       // [rows]
   float* zero;        // [rows] or nullptr
   int32_t* rowsum;    // [rows] or nullptr (weights)
+  const uint8_t* signs;  // random signs S of R = S H: bit k set -> x_k negated; nullptr = none
 };
 
 cudaError_t launch_rotate_quant_rows(const RotQuantArgs& a, cudaStream_t stream);

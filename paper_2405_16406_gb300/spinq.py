@@ -40,6 +40,8 @@ EXPORTED = (
     "spinq_w4a4_gemm_plan", "spinq_w4a4_gemm_splitk_plan", "spinq_cayley_step",
     "spinq_rotate_quant_act8", "spinq_quant_weight8", "spinq_fp8_gemm", "spinq_w4a8_gemm",
     "spinq_rope_rotate_quant_kv", "spinq_decode_attention_workspace_bytes", "spinq_decode_attention_kv4",
+    "spinq_rotate_quant_act_signed", "spinq_quant_weight_signed", "spinq_rotated_linear_workspace_bytes",
+    "spinq_rotated_linear",
 )
 SPINQ_FMT_INT8_PLANES, SPINQ_FMT_E4M3, SPINQ_FMT_INT4_BYTES = 1, 2, 3
 
@@ -109,6 +111,17 @@ _lib.spinq_decode_attention_workspace_bytes.argtypes = [_I64, _I64, _I64, _I64, 
 _lib.spinq_decode_attention_kv4.restype = ctypes.c_int
 _lib.spinq_decode_attention_kv4.argtypes = [_P, _P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I64,
                                             ctypes.c_float, _P, _P, _I64, _P]
+_lib.spinq_rotate_quant_act_signed.restype = ctypes.c_int
+_lib.spinq_rotate_quant_act_signed.argtypes = [_P, _I64, _I64, _I64, ctypes.POINTER(HadCfg), _P,
+                                               ctypes.POINTER(QuantCfg), _P, _P, _P, _P]
+_lib.spinq_quant_weight_signed.restype = ctypes.c_int
+_lib.spinq_quant_weight_signed.argtypes = [_P, _I64, _I64, ctypes.POINTER(HadCfg), _P, ctypes.POINTER(QuantCfg),
+                                           _P, _P, _P, _P]
+_lib.spinq_rotated_linear_workspace_bytes.restype = ctypes.c_int64
+_lib.spinq_rotated_linear_workspace_bytes.argtypes = [_I64, _I64]
+_lib.spinq_rotated_linear.restype = ctypes.c_int
+_lib.spinq_rotated_linear.argtypes = [_P, _I64, _I64, _I64, ctypes.POINTER(HadCfg), _P, ctypes.POINTER(QuantCfg),
+                                      _P, _P, _P, _I64, _P, _P, _I64, _P]
 _lib.spinq_cayley_step.restype = ctypes.c_int
 _lib.spinq_cayley_step.argtypes = [_P, _P, _I64, _I64, ctypes.c_float, ctypes.c_int32, _P, _P, _P]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
@@ -188,6 +201,23 @@ def spinq_decode_attention_kv4(q, k_codes, k_scale, k_zero, v_codes, v_scale, v_
                                scale, out, ws, ws_bytes, stream) -> int:
     return _lib.spinq_decode_attention_kv4(q, k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, lens, B, S, Hq,
                                            Hkv, D, scale, out, ws, ws_bytes, stream)
+
+
+def spinq_rotate_quant_act_signed(x, M, K, ldx, had, signs, q, codes, scale, zero, stream) -> int:
+    return _lib.spinq_rotate_quant_act_signed(x, M, K, ldx, had, signs, q, codes, scale, zero, stream)
+
+
+def spinq_quant_weight_signed(w, N, K, had, signs, q, codes, scale, rowsum, stream) -> int:
+    return _lib.spinq_quant_weight_signed(w, N, K, had, signs, q, codes, scale, rowsum, stream)
+
+
+def spinq_rotated_linear_workspace_bytes(M, K) -> int:
+    return int(_lib.spinq_rotated_linear_workspace_bytes(M, K))
+
+
+def spinq_rotated_linear(x, M, K, ldx, had, signs, q, w_codes, w_scale, w_rowsum, N, y, ws, ws_bytes, stream) -> int:
+    return _lib.spinq_rotated_linear(x, M, K, ldx, had, signs, q, w_codes, w_scale, w_rowsum, N, y, ws, ws_bytes,
+                                     stream)
 
 
 def spinq_cayley_step(R, grad, batch, n, alpha, iters, R_out, Y_out, stream) -> int:
@@ -478,3 +508,60 @@ def decode_attention_kv4(q: torch.Tensor, kv: KVCodes, lens: Optional[torch.Tens
                                            Hkv, D, sc, _ptr(out), _ptr(workspace), workspace.numel(),
                                            _stream(stream)), "spinq_decode_attention_kv4")
     return out
+
+
+def sign_mask(signs) -> torch.Tensor:
+    """+-1 per input index -> the [K/8] byte bit mask of the signed entry
+    points (bit k % 8 of byte k / 8 set for s_k = -1), on the device."""
+    s = torch.as_tensor(signs).reshape(-1)
+    neg = (s < 0).to(torch.uint8).reshape(-1, 8)
+    bits = torch.zeros(neg.shape[0], dtype=torch.uint8)
+    for e in range(8):
+        bits |= neg[:, e].cpu() << e
+    return bits.cuda()
+
+
+def rotate_quant_act_signed(x: torch.Tensor, had: Tuple[int, int], signs: torch.Tensor, symmetric: bool = True,
+                            clip: float = 1.0, out: Optional[ActCodes] = None,
+                            stream: Optional[torch.cuda.Stream] = None) -> ActCodes:
+    """rotate_quant_act with R = S H / sqrt(K); ``signs`` is the device bit mask."""
+    M, K = x.shape
+    if out is None:
+        out = ActCodes(torch.empty((M, K // 2), dtype=torch.uint8, device=x.device),
+                       torch.empty(M, dtype=torch.float32, device=x.device),
+                       None if symmetric else torch.empty(M, dtype=torch.float32, device=x.device))
+    q = quant_cfg(4, symmetric, SPINQ_PER_TOKEN, 0, clip)
+    _check(_lib.spinq_rotate_quant_act_signed(_ptr(x), M, K, x.stride(0), _had(had), _ptr(signs), ctypes.byref(q),
+                                              _ptr(out.codes), _ptr(out.scale), _ptr(out.zero), _stream(stream)),
+           "spinq_rotate_quant_act_signed")
+    return out
+
+
+def quant_weight_signed(w: torch.Tensor, had: Tuple[int, int], signs: torch.Tensor, clip: float = 1.0,
+                        stream: Optional[torch.cuda.Stream] = None) -> WeightCodes:
+    N, K = w.shape
+    out = WeightCodes(torch.empty((N, K // 2), dtype=torch.uint8, device=w.device),
+                      torch.empty(N, dtype=torch.float32, device=w.device),
+                      torch.empty(N, dtype=torch.int32, device=w.device))
+    q = quant_cfg(4, True, SPINQ_PER_CHANNEL, 0, clip)
+    _check(_lib.spinq_quant_weight_signed(_ptr(w), N, K, _had(had), _ptr(signs), ctypes.byref(q), _ptr(out.codes),
+                                          _ptr(out.scale), _ptr(out.rowsum), _stream(stream)),
+           "spinq_quant_weight_signed")
+    return out
+
+
+def rotated_linear(x: torch.Tensor, had: Tuple[int, int], w: WeightCodes, signs: Optional[torch.Tensor] = None,
+                   symmetric: bool = True, clip: float = 1.0, y: Optional[torch.Tensor] = None,
+                   workspace: Optional[torch.Tensor] = None, stream: Optional[torch.cuda.Stream] = None):
+    """Online R4 (+ random signs) + act quant + W4A4 GEMM in one call."""
+    M, K = x.shape
+    N = w.codes.shape[0]
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float16, device=x.device)
+    if workspace is None:
+        workspace = torch.empty(spinq_rotated_linear_workspace_bytes(M, K), dtype=torch.uint8, device=x.device)
+    q = quant_cfg(4, symmetric, SPINQ_PER_TOKEN, 0, clip)
+    _check(_lib.spinq_rotated_linear(_ptr(x), M, K, x.stride(0), _had(had), _ptr(signs), ctypes.byref(q),
+                                     _ptr(w.codes), _ptr(w.scale), _ptr(w.rowsum), N, _ptr(y), _ptr(workspace),
+                                     workspace.numel(), _stream(stream)), "spinq_rotated_linear")
+    return y

@@ -211,3 +211,27 @@ def test_attention_entry_points_reject_invalid_arguments_on_the_host(lib):
              fake, fake, fake, fake, fake, fake, None) == S.SPINQ_EINVAL                       # no positions
     assert g(fake, fake, fake, fake, fake, ctypes.c_void_p((1 << 20) + 8), 4096, 1, 4, 4, 2, 128, ctypes.byref(had),
              ctypes.byref(kvq), fake, fake, fake, fake, fake, fake, None) == S.SPINQ_EINVAL    # table alignment
+
+
+def test_signed_and_fused_entry_points_reject_invalid_arguments_on_the_host(lib):
+    from paper_2405_16406_gb300 import spinq as S
+    fake = ctypes.c_void_p(1 << 20)
+    q = S.quant_cfg(4, True, S.SPINQ_PER_TOKEN, 0, 1.0)
+    had = S.HadCfg(28, 512)
+    # signs need a rotation and a mask
+    assert S.spinq_rotate_quant_act_signed(fake, 4, 14336, 14336, None, fake, ctypes.byref(q), fake, fake, None,
+                                           None) == S.SPINQ_EINVAL
+    assert S.spinq_rotate_quant_act_signed(fake, 4, 14336, 14336, ctypes.byref(had), None, ctypes.byref(q), fake,
+                                           fake, None, None) == S.SPINQ_EINVAL
+    qw = S.quant_cfg(4, True, S.SPINQ_PER_CHANNEL, 0, 1.0)
+    assert S.spinq_quant_weight_signed(fake, 4, 14336, None, fake, ctypes.byref(qw), fake, fake, fake,
+                                       None) == S.SPINQ_EINVAL
+    need = S.spinq_rotated_linear_workspace_bytes(2048, 14336)
+    assert need >= 2048 * 7168 + 2 * 2048 * 4
+    f = S.spinq_rotated_linear
+    assert f(fake, 2048, 14336, 14336, ctypes.byref(had), None, ctypes.byref(q), fake, fake, fake, 4096, fake,
+             fake, need - 256, None) == S.SPINQ_EINVAL          # workspace too small
+    assert f(fake, 2048, 14336, 14336, ctypes.byref(had), None, ctypes.byref(q), fake, fake, fake, 4100, fake,
+             fake, need, None) == S.SPINQ_EINVAL                 # N % 16
+    assert f(fake, 0, 14336, 14336, ctypes.byref(had), None, ctypes.byref(q), fake, fake, fake, 4096, fake,
+             None, 0, None) == S.SPINQ_OK
