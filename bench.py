@@ -739,7 +739,55 @@ def run_configs(dev, hbm_peak, fp8_peak):
     res.update(cayley_records(dev))
     res.update(variant8_records(dev, hbm_peak, fp8_peak))
     res.update(attention_records(dev, hbm_peak))
+    res.update(fused_down_proj_records(dev, fp8_peak))
     return res
+
+
+def fused_down_proj_records(dev, fp8_peak):
+    """Config 3's down_proj (2048 x 14336 -> 4096, online H28 (x) H512) as one
+    call (spinq_rotated_linear), plain and with random signs (R = S H), over
+    4 input sets, against the same two kernels called separately."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2405_16406_gb300 import spinq, synth
+    c = synth.llama3_8b_down_proj()
+    xt, wt = torch.from_numpy(c.x).to(dev), torch.from_numpy(c.w).to(dev)
+    xs = [xt] + [xt.clone() for _ in range(3)]
+    signs = np.random.default_rng(17).choice([-1.0, 1.0], c.K)
+    mask = spinq.sign_mask(signs)
+    out = {}
+    ops = 2.0 * c.M * c.N * c.K
+    for tag, m in (("plain", None), ("random_signs", mask)):
+        qw = spinq.quant_weight(wt, c.had) if m is None else spinq.quant_weight_signed(wt, c.had, m)
+        ws = [torch.empty(spinq.spinq_rotated_linear_workspace_bytes(c.M, c.K), dtype=torch.uint8, device=dev)
+              for _ in range(4)]
+        ys = [torch.empty(c.M, c.N, dtype=torch.float16, device=dev) for _ in range(4)]
+        us = graph_us(lambda i: spinq.rotated_linear(xs[i], c.had, qw, signs=m, y=ys[i], workspace=ws[i]), 4)
+        torch.cuda.synchronize()
+        # timed output of set 0, 2 rows, against the oracle's product of the handed-over codes
+        rows = np.array([5, 1500])
+        codes = ws[0][: c.M * c.K // 2].view(c.M, c.K // 2)[torch.as_tensor(rows, device=dev)].cpu().numpy()
+        alpha = ws[0][c.M * c.K // 2:].view(torch.float32)[: c.M][torch.as_tensor(rows, device=dev)]
+        ga, gw = oracle.unpack4(codes, True), oracle.unpack4(qw.codes.cpu().numpy(), True)
+        ref = oracle.w4a4_linear(oracle.QuantAct(ga, None, alpha.double().cpu().numpy(), None, None),
+                                 oracle.QuantWeight(gw, None, qw.scale.double().cpu().numpy(), gw.sum(1), None)).y
+        got = ys[0][torch.as_tensor(rows, device=dev)].double().cpu().numpy()
+        if not np.allclose(got, ref, rtol=2e-3, atol=1e-3 * np.abs(ref).max()):
+            raise RuntimeError(f"rotated_linear {tag}: timed output differs from the oracle")
+        rec = {"us": round(us, 2), "tops": round(ops / us / 1e6, 1), "frac_e4m3": round(ops / us / 1e6 / fp8_peak, 4)}
+        if m is None:
+            outs = [spinq.ActCodes(torch.empty(c.M, c.K // 2, dtype=torch.uint8, device=dev),
+                                   torch.empty(c.M, device=dev), None) for _ in range(4)]
+            rec["rotate_quant_alone_us"] = round(graph_us(lambda i: spinq.rotate_quant_act(xs[i], c.had, True, 1.0,
+                                                                                           out=outs[i]), 4), 2)
+            rec["gemm_alone_us"] = round(graph_us(lambda i: spinq.w4a4_gemm(outs[i], qw, y=ys[i]), 4), 2)
+        out[f"f1_rotated_linear_down_proj_{tag}"] = rec
+        del qw, ws, ys
+    del xs
+    torch.cuda.empty_cache()
+    return out
 
 
 def attention_records(dev, hbm_peak):

@@ -478,6 +478,30 @@ spinq_status spinq_w4a8_gemm(const uint8_t* a_planes, const float* a_scale, cons
 spinq_status spinq_cayley_step(const float* R, const float* grad, int64_t batch, int64_t n, float alpha,
                                int32_t iters, float* R_out, float* Y_out, void* stream);
 
+/*
+ * Testing controls of the failure paths (the paper has no counterpart).
+ * spinq_debug_set_wait_limit_ns -- time limit of the ordinary bounded waits
+ *   of the Paley rotate+quant, W4A4 and FP8 GEMM kernels on the current
+ *   device (2e9 ns by default; the drains of copies and MMAs in flight keep
+ *   their full limit).  A test lowers it so that those waits give up, checks
+ *   SPINQ_ETIMEOUT through spinq_device_status and sets it back.  Outputs of
+ *   a call that gave up are undefined.  SPINQ_EINVAL for ns <= 0.
+ * spinq_debug_stall_launches -- the next n launches of the Paley rotate+quant,
+ *   the W4A4 prefill (128- and 256-row tiles) and the FP8 GEMM kernels issue
+ *   no input copies, so the waits of their consumers run out of time (a
+ *   barrier that nothing completes): SPINQ_ETIMEOUT is recorded, every role
+ *   leaves its loop, MMAs in flight are drained and tensor memory is freed.
+ *   Lower the wait limit first so that this takes a millisecond, not 2 s.
+ *   Outputs of such a call are undefined.  Returns the previous count, or -1
+ *   for n < 0.
+ * spinq_debug_fail_launches -- the next n kernel launches of the library are
+ *   refused on the host (the call returns SPINQ_ECUDA; nothing reaches the
+ *   GPU).  Returns the previous count, or -1 for n < 0.
+ */
+spinq_status spinq_debug_set_wait_limit_ns(int64_t ns);
+int spinq_debug_stall_launches(int n);
+int spinq_debug_fail_launches(int n);
+
 /* Human-readable name of a status code (static storage). */
 const char* spinq_status_string(spinq_status s);
 

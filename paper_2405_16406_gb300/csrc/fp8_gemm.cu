@@ -48,6 +48,9 @@ constexpr int kStageBytes = kStageA + kStageB;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
+// limit of the ordinary waits (kWaitLimitNs unless a test lowers it); the
+// drains of copies and MMAs in flight always use kWaitLimitNs
+__device__ uint64_t g_wait_ns = kWaitLimitNs;
 constexpr int OFF_BAR = kStages * kStageBytes;                  // full[S] empty[S] accf[2] acce[2] drain
 constexpr int OFF_MISC = OFF_BAR + (2 * kStages + 5) * 8;       // tmem address, abort flag
 constexpr int kSmemBytes = OFF_MISC + 16 + 1024;                // + alignment slack
@@ -62,6 +65,7 @@ struct Fp8GemmParams {
   int* status;
   int M, N, K;             // K: the weights' reduction length
   int ksteps;              // K steps of the activation operand (planes * K / 128)
+  int debug_stall;         // issue no input copies, so the waits run out (tests)
 };
 
 __device__ __forceinline__ void set_timeout(int* status, int site) {
@@ -73,13 +77,14 @@ __device__ __forceinline__ void set_timeout(int* status, int site) {
 // raises the flag and records the site).
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status,
                                          int site) {
+  if (*abort_flag) return false;
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      if (globaltimer_ns() - t0 > g_wait_ns) {
         *abort_flag = 1;
         set_timeout(status, site);
         return false;
@@ -131,13 +136,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();
   pdl_trigger();
 
+  // the producer's last copy into each stage (for the drain after an abort)
+  int last_issued[kStages];
+  for (int s = 0; s < kStages; ++s) last_issued[s] = -1;
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer
       uint32_t g = 0;
-      int last_issued[kStages];
-      for (int s = 0; s < kStages; ++s) last_issued[s] = -1;
-      bool ok = true;
+      bool ok = !p.debug_stall;   // a test of the time-outs issues no copies
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
         const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
         for (int s = 0; s < p.ksteps; ++s, ++g) {
@@ -153,12 +159,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_2d(sa + kStageA, &tmB, &full[st], W4A8 ? ka % p.K : ka, n0);
           last_issued[st] = (int)g;
         }
-      }
-      if (*abort_flag) {
-        // let the copies still in flight land before the CTA can exit
-        for (int s = 0; s < kStages; ++s)
-          if (last_issued[s] >= 0)
-            mbar_wait_bounded(&full[s], ((uint32_t)last_issued[s] / kStages) & 1u, kWaitLimitNs);
       }
     }
   } else if (warp == 1) {
@@ -261,6 +261,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
+  // Every role has stopped, so the abort flag is final here.  After an abort
+  // the MMA may not have consumed the last copies: let them land before the
+  // CTA (and its shared memory) can go away.  Without an abort every copy
+  // was waited for by the MMA issuer.
+  if (warp == 0 && lane == 0 && *abort_flag)
+    for (int s = 0; s < kStages; ++s)
+      if (last_issued[s] >= 0) mbar_wait_bounded(&full[s], ((uint32_t)last_issued[s] / kStages) & 1u, kWaitLimitNs);
 }
 
 // E4M3 bytes [rows][cols], boxes of 128 bytes x box_rows with the 128-byte
@@ -291,13 +298,15 @@ cudaError_t launch_t(const Fp8GemmArgs& a, cudaStream_t stream) {
   const int64_t cap = device_sm_count();
   const int grid = (int)(tiles < cap ? tiles : cap);
   Fp8GemmParams p{a.a_scale, a.a_zero, a.w_scale, a.w_rowsum, a.y, a.acc_out, device_status_word(),
-                  (int)a.M, (int)a.N, (int)a.K, (int)(planes * a.K / BK)};
+                  (int)a.M, (int)a.N, (int)a.K, (int)(planes * a.K / BK), take_debug_stall() ? 1 : 0};
   e = launch_pdl(kern, dim3(grid), dim3(kThreads), kSmemBytes, stream, 1, tmA, tmB, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
 }  // namespace
+
+cudaError_t set_wait_limit_fp8(uint64_t ns) { return cudaMemcpyToSymbol(g_wait_ns, &ns, sizeof(ns)); }
 
 cudaError_t launch_fp8_gemm(const Fp8GemmArgs& a, cudaStream_t stream) {
   if (!a.w4a8) return launch_t<false, false>(a, stream);

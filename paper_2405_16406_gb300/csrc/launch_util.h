@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <map>
 #include <mutex>
 #include <tuple>
@@ -107,12 +108,20 @@ cudaError_t prepare_launch_tmem(Kern kern, int threads, size_t smem, int tmem_co
   return cudaSuccess;
 }
 
+// Launches still to be refused with cudaErrorLaunchOutOfResources without
+// reaching the driver (a host-side fake of a failing launch, set by tests
+// through spinq_debug_fail_launches; 0 in normal use).
+extern std::atomic<int> g_fail_launches;
+
 // Launch with programmatic stream serialization: the kernel may begin while
 // the previous kernel in the stream finishes (it waits with griddepcontrol
 // before touching global memory).  `cluster_x` > 1 adds a cluster dimension.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
                        int cluster_x, Args&&... args) {
+  if (g_fail_launches.load(std::memory_order_relaxed) > 0 &&
+      g_fail_launches.fetch_sub(1, std::memory_order_relaxed) > 0)
+    return cudaErrorLaunchOutOfResources;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;

@@ -56,6 +56,9 @@ namespace spinq {
 namespace {
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
+// limit of the ordinary waits (kWaitLimitNs unless a test lowers it); the
+// drain of copies in flight always uses kWaitLimitNs
+__device__ uint64_t g_wait_ns = kWaitLimitNs;
 constexpr int kSmemBudget = 232448;  // dynamic shared memory a CTA may opt into
 constexpr int kPhase2Bar = 1;        // named barrier of the phase-2 warps
 constexpr int kPhase1Bar = 2;        // named barrier of the phase-1 warps (exit only)
@@ -106,7 +109,7 @@ __device__ __forceinline__ bool combo_warp_idle(int cb, int ns) {
 // Bounded wait for the phase of `bar` with `parity`.  Returns false when the
 // abort flag is up or the limit expired (then it raises the flag).
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-  return mbar_wait_backoff(bar, parity, abort_flag, kWaitLimitNs);
+  return mbar_wait_backoff(bar, parity, abort_flag, g_wait_ns);
 }
 
 // bar.sync over `nthreads` threads whose result is the OR of `pred` over them.
@@ -165,7 +168,7 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
   __syncthreads();  // the last CTA-wide barrier: the roles part here
   pdl_wait();
   pdl_trigger();
-  if (tid == 0)
+  if (tid == 0 && !a.debug_stall)   // a test of the time-outs issues no copies
     for (int it = 0; it < NSTG && it < niter; ++it) issue(it);
 
   if (warp < W) {
@@ -310,6 +313,8 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
     // every phase-1 warp has stopped issuing; after an abort, let the copies
     // still in flight land before the CTA can exit
     named_bar_sync(kPhase1Bar, T);
+    if (*abort_flag && tid == 0 && a.status && atomicCAS(a.status, 0, (int)4 /* SPINQ_ETIMEOUT */) == 0)
+      atomicExch(a.status + 1, 20);   // wait site: the Paley rotate+quant kernel
     if (*abort_flag && tid == 0)
       for (int s = 0; s < NSTG; ++s)
         if (issued[s] >= 0) mbar_wait_bounded(&full[s], (uint32_t)(issued[s] / NSTG) & 1u, kWaitLimitNs);
@@ -473,7 +478,9 @@ cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const int64_t cap = (int64_t)device_sm_count() * per_sm;
   const int64_t grid = a.rows < cap ? a.rows : cap;
-  e = launch_pdl(kern, dim3((unsigned)grid), dim3(S::THREADS), S::BYTES, stream, 1, tmx, a);
+  RotQuantArgs la = a;
+  la.debug_stall = take_debug_stall() ? 1 : 0;
+  e = launch_pdl(kern, dim3((unsigned)grid), dim3(S::THREADS), S::BYTES, stream, 1, tmx, la);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -531,7 +538,12 @@ cudaError_t launch_sc(const RotQuantArgs& a, cudaStream_t stream, bool* handled)
 
 }  // namespace
 
-cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+cudaError_t set_wait_limit_paley(uint64_t ns) { return cudaMemcpyToSymbol(g_wait_ns, &ns, sizeof(ns)); }
+
+cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a0, cudaStream_t stream, bool* handled) {
+  RotQuantArgs a = a0;
+  a.status = device_status_word();
+  a.debug_stall = 0;
   *handled = false;
   if (a.rows == 0 || a.rowsum || a.n_small <= 1) return cudaSuccess;
   if ((a.ldx * 2) % 16 != 0) return cudaSuccess;

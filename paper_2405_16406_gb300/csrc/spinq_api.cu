@@ -4,12 +4,21 @@
 // documents that it does).
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 
 #include "../../include/spinq.h"
 #include "spinq_internal.h"
 
 using namespace spinq;
+
+namespace spinq {
+std::atomic<int> g_fail_launches{0};
+static std::atomic<int> g_debug_stall{0};
+bool take_debug_stall() {
+  return g_debug_stall.load(std::memory_order_relaxed) > 0 && g_debug_stall.fetch_sub(1) > 0;
+}
+}
 
 namespace {
 
@@ -399,6 +408,25 @@ spinq_status spinq_decode_attention_kv4(const void* q, const uint8_t* k_codes, c
   AttnArgs a{q, k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, lens, B, S, Hq, Hkv, (int)D, softmax_scale,
              out, static_cast<float*>(workspace)};
   return from_cuda(launch_decode_attention(a, decode_attention_chunks(B, S, Hkv), static_cast<cudaStream_t>(stream)));
+}
+
+spinq_status spinq_debug_set_wait_limit_ns(int64_t ns) {
+  if (ns <= 0) return SPINQ_EINVAL;
+  const uint64_t v = (uint64_t)ns;
+  if (set_wait_limit_paley(v) != cudaSuccess || set_wait_limit_gemm(v) != cudaSuccess ||
+      set_wait_limit_fp8(v) != cudaSuccess)
+    return SPINQ_ECUDA;
+  return SPINQ_OK;
+}
+
+int spinq_debug_stall_launches(int n) {
+  if (n < 0) return -1;
+  return g_debug_stall.exchange(n);
+}
+
+int spinq_debug_fail_launches(int n) {
+  if (n < 0) return -1;
+  return g_fail_launches.exchange(n);
 }
 
 int spinq_gemm_select_kernel(int kernel) { return w4a4_gemm_select(kernel); }

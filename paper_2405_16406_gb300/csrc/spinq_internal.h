@@ -35,6 +35,8 @@ struct RotQuantArgs {
   float* zero;        // [rows] or nullptr
   int32_t* rowsum;    // [rows] or nullptr (weights)
   const uint8_t* signs;  // random signs S of R = S H: bit k set -> x_k negated; nullptr = none
+  int* status;           // device status word (set by the launcher of kernels that record time-outs)
+  int debug_stall;       // issue no input copies, so the waits run out (tests; 0 normally)
 };
 
 cudaError_t launch_rotate_quant_rows(const RotQuantArgs& a, cudaStream_t stream);
@@ -103,6 +105,7 @@ struct GemmArgs {
   int64_t M, N, K;
   void* y;               // fp16 [M][N]
   int32_t* acc_out;      // optional
+  int debug_stall;       // prefill kernels: issue no input copies (tests; 0 normally)
 };
 
 // Returns cudaErrorNotSupported when the TMA descriptor cannot be encoded.
@@ -192,6 +195,17 @@ struct Fp8GemmArgs {
 // 8-bit linears on the E4M3 pipe; cudaErrorNotSupported when a tensor map
 // cannot be encoded.
 cudaError_t launch_fp8_gemm(const Fp8GemmArgs& a, cudaStream_t stream);
+
+// Launches of the Paley rotate+quant, W4A4 prefill and FP8 GEMM kernels still
+// to issue no input copies (spinq_debug_stall_launches); take_debug_stall()
+// consumes one.
+bool take_debug_stall();
+
+// Limit of the ordinary bounded waits of the Paley rotate+quant, W4A4 and
+// FP8 GEMM kernels (2 s by default; lowered only by tests).
+cudaError_t set_wait_limit_paley(uint64_t ns);
+cudaError_t set_wait_limit_gemm(uint64_t ns);
+cudaError_t set_wait_limit_fp8(uint64_t ns);
 
 // Device status word written by bounded waits that gave up.
 cudaError_t read_and_clear_device_status(int32_t* code, int32_t* detail);

@@ -67,6 +67,9 @@ constexpr int kThreads = (6 + kUnpackGroups * kUnpackWarps) * 32;
 constexpr int kFirstUnpackWarp = 6;
 constexpr int kFirstEpiWarp = 2;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
+// limit of the ordinary waits (kWaitLimitNs unless a test lowers it); the
+// drains of copies and MMAs in flight always use kWaitLimitNs
+__device__ uint64_t g_wait_ns = kWaitLimitNs;
 
 __device__ __forceinline__ void record_timeout(int site) {
   if (atomicCAS(&g_status[0], 0, (int)SPINQ_ETIMEOUT) == 0) atomicExch(&g_status[1], site);
@@ -85,7 +88,7 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+    if (globaltimer_ns() - t0 > g_wait_ns) {
       record_timeout(site);
       *abort_flag = 1;
       return false;
@@ -401,11 +404,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();
   pdl_trigger();
 
+  int prod_it = 0;   // copies the producer issued (for the drain after an abort)
   if (warp == 0) {
     // ------------------------------------------------ TMA producer
     if (lane == 0) {
-      int it = 0;
-      bool stop = false;
+      int& it = prod_it;
+      bool stop = args.debug_stall != 0;   // a test of the time-outs issues no copies
       for (int tile = blockIdx.x; tile < num_tiles && !stop; tile += gridDim.x) {
         const int32_t m0 = (tile % m_tiles) * BMT, n0 = (tile / m_tiles) * BN;
         for (int kt = 0; kt < num_k; ++kt, ++it) {
@@ -706,6 +710,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
+  // Every role has stopped, so the abort flag is final here.  After an abort
+  // the unpack warps may not have consumed the last copies (another role can
+  // abort after the producer issued them): let them land before the CTA and
+  // its shared memory go away.
+  if (warp == 0 && lane == 0 && *abort_flag)
+    for (int j = prod_it - NP < 0 ? 0 : prod_it - NP; j < prod_it; ++j) {
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(&full_p[j % NP], (j / NP) & 1) && globaltimer_ns() - t0 < kWaitLimitNs) {
+      }
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -811,9 +825,9 @@ __global__ void __launch_bounds__(kDecThreads, 2)
   pdl_wait();
   pdl_trigger();
 
+  int issued = 0;   // copies the producer issued (for the drain after an abort)
   if (warp == 0) {
     if (lane == 0) {
-      int issued = 0;
       for (int it = 0; it < nk; ++it) {
         const int s = it % NP;
         if (!wait_or_abort(&empty_p[s], ((it / NP) & 1) ^ 1, abort_flag, 11)) break;
@@ -1016,6 +1030,14 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     tc_fence_after();
     tmem_dealloc(tmem, L::tmem_cols);
   }
+  // the abort flag is final here: after an abort, let the producer's last
+  // copies land before the CTA goes away (see the prefill kernel)
+  if (warp == 0 && lane == 0 && *abort_flag)
+    for (int j = issued - NP < 0 ? 0 : issued - NP; j < issued; ++j) {
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(&full_p[j % NP], (j / NP) & 1) && globaltimer_ns() - t0 < kWaitLimitNs) {
+      }
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -1067,7 +1089,9 @@ cudaError_t launch_t(const GemmArgs& a, cudaStream_t stream) {
   const int n_tiles = (int)((a.N + BN - 1) / BN);
   const int tiles = m_tiles * n_tiles;
   const int grid = tiles < sms ? tiles : sms;
-  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, 1, tmA, tmB, a, (int)(a.K / 128), m_tiles,
+  GemmArgs la = a;
+  la.debug_stall = take_debug_stall() ? 1 : 0;
+  e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, 1, tmA, tmB, la, (int)(a.K / 128), m_tiles,
                  tiles);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
@@ -1316,6 +1340,8 @@ cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, int64_t 
   if (a.M <= 128) return launch_dec_mn<128>(a, ws_acc, ws_cnt, p.nsplit, stream);
   return launch_dec_mn<256>(a, ws_acc, ws_cnt, p.nsplit, stream);
 }
+
+cudaError_t set_wait_limit_gemm(uint64_t ns) { return cudaMemcpyToSymbol(g_wait_ns, &ns, sizeof(ns)); }
 
 int* device_status_word() {
   void* p = nullptr;

@@ -238,10 +238,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();
   pdl_trigger();
 
+  int prod_it = 0;   // copies the producer issued (for the drain after an abort)
   if (warp == 0) {
     // ------------------------------------------------ TMA producer (this CTA's halves)
     if (lane == 0) {
-      int it = 0;
+      int& it = prod_it;
       bool stop = false;
       for (int tile = cluster; tile < num_tiles && !stop; tile += nclusters) {
         const int32_t m0 = (tile % m_tiles) * 256 + 128 * (int)rank;
@@ -519,6 +520,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc_pair(tmem, 512);
   }
+  // every role of both CTAs has stopped, so the abort flag is final here:
+  // after an abort, let this CTA's last copies land before it goes away
+  // (another role may have aborted after the producer issued them)
+  if (warp == 0 && lane == 0 && *abort_flag)
+    for (int j = prod_it - NP < 0 ? 0 : prod_it - NP; j < prod_it; ++j) {
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(&full_p[j % NP], (j / NP) & 1) && globaltimer_ns() - t0 < kWaitLimitNs) {
+      }
+    }
 }
 
 // Co-resident clusters for this kernel (cached per device and kernel).

@@ -41,7 +41,8 @@ EXPORTED = (
     "spinq_rotate_quant_act8", "spinq_quant_weight8", "spinq_fp8_gemm", "spinq_w4a8_gemm",
     "spinq_rope_rotate_quant_kv", "spinq_decode_attention_workspace_bytes", "spinq_decode_attention_kv4",
     "spinq_rotate_quant_act_signed", "spinq_quant_weight_signed", "spinq_rotated_linear_workspace_bytes",
-    "spinq_rotated_linear",
+    "spinq_rotated_linear", "spinq_debug_set_wait_limit_ns", "spinq_debug_fail_launches",
+    "spinq_debug_stall_launches",
 )
 SPINQ_FMT_INT8_PLANES, SPINQ_FMT_E4M3, SPINQ_FMT_INT4_BYTES = 1, 2, 3
 
@@ -122,6 +123,12 @@ _lib.spinq_rotated_linear_workspace_bytes.argtypes = [_I64, _I64]
 _lib.spinq_rotated_linear.restype = ctypes.c_int
 _lib.spinq_rotated_linear.argtypes = [_P, _I64, _I64, _I64, ctypes.POINTER(HadCfg), _P, ctypes.POINTER(QuantCfg),
                                       _P, _P, _P, _I64, _P, _P, _I64, _P]
+_lib.spinq_debug_set_wait_limit_ns.restype = ctypes.c_int
+_lib.spinq_debug_set_wait_limit_ns.argtypes = [_I64]
+_lib.spinq_debug_stall_launches.restype = ctypes.c_int
+_lib.spinq_debug_stall_launches.argtypes = [ctypes.c_int]
+_lib.spinq_debug_fail_launches.restype = ctypes.c_int
+_lib.spinq_debug_fail_launches.argtypes = [ctypes.c_int]
 _lib.spinq_cayley_step.restype = ctypes.c_int
 _lib.spinq_cayley_step.argtypes = [_P, _P, _I64, _I64, ctypes.c_float, ctypes.c_int32, _P, _P, _P]
 _lib.spinq_rotate_quant_kv.restype = ctypes.c_int
@@ -218,6 +225,18 @@ def spinq_rotated_linear_workspace_bytes(M, K) -> int:
 def spinq_rotated_linear(x, M, K, ldx, had, signs, q, w_codes, w_scale, w_rowsum, N, y, ws, ws_bytes, stream) -> int:
     return _lib.spinq_rotated_linear(x, M, K, ldx, had, signs, q, w_codes, w_scale, w_rowsum, N, y, ws, ws_bytes,
                                      stream)
+
+
+def spinq_debug_set_wait_limit_ns(ns: int) -> int:
+    return int(_lib.spinq_debug_set_wait_limit_ns(ns))
+
+
+def spinq_debug_stall_launches(n: int) -> int:
+    return int(_lib.spinq_debug_stall_launches(n))
+
+
+def spinq_debug_fail_launches(n: int) -> int:
+    return int(_lib.spinq_debug_fail_launches(n))
 
 
 def spinq_cayley_step(R, grad, batch, n, alpha, iters, R_out, Y_out, stream) -> int:

@@ -235,3 +235,11 @@ def test_signed_and_fused_entry_points_reject_invalid_arguments_on_the_host(lib)
              fake, need, None) == S.SPINQ_EINVAL                 # N % 16
     assert f(fake, 0, 14336, 14336, ctypes.byref(had), None, ctypes.byref(q), fake, fake, fake, 4096, fake,
              None, 0, None) == S.SPINQ_OK
+
+
+def test_debug_controls_validate_on_the_host(lib):
+    from paper_2405_16406_gb300 import spinq as S
+    assert S.spinq_debug_set_wait_limit_ns(0) == S.SPINQ_EINVAL
+    assert S.spinq_debug_set_wait_limit_ns(-5) == S.SPINQ_EINVAL
+    assert S.spinq_debug_fail_launches(-1) == -1
+    assert S.spinq_debug_fail_launches(0) == 0
