@@ -77,7 +77,6 @@ __device__ __forceinline__ void set_timeout(int* status, int site) {
 // raises the flag and records the site).
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status,
                                          int site) {
-  if (*abort_flag) return false;
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {

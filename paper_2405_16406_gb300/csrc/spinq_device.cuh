@@ -212,11 +212,9 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 // Waits for the phase of `bar` with `parity`, sleeping between polls (32 ns
 // doubling to 1 us) so that waiting warps leave the issue slots to the warps
 // that work.  Returns false, and raises *abort_flag, after `limit_ns` of wall
-// time; returns false at once when *abort_flag is already up (checked before
-// the barrier, so an abort stops every role at its next wait).
+// time; returns false at once when *abort_flag is already up.
 __device__ __forceinline__ bool mbar_wait_backoff(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                                   uint64_t limit_ns) {
-  if (*abort_flag) return false;
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   uint32_t ns = 32;
