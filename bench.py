@@ -811,9 +811,13 @@ def attention_records(dev, hbm_peak):
     rope_bytes = B * S * Hq * Dd * 4 + 2 * B * S * Hkv * (Dd * 2 + Dd // 2 + 8) + B * S * 4
     rng = np.random.default_rng(11)
     qd = torch.from_numpy((rng.standard_normal((B, Hq, Dd)) * 2).astype(np.float16)).to(dev)
-    outs = [torch.empty_like(qd) for _ in range(2)]
+    # four caches (4 x 37.9 MB, more than the 129 MB L2): each timed call reads a cold cache
+    caches = [cache] + [spinq.KVCodes(None, *(t.clone() for t in (cache.k_codes, cache.k_scale, cache.k_zero,
+                                                                   cache.v_codes, cache.v_scale, cache.v_zero)))
+                        for _ in range(3)]
+    outs = [torch.empty_like(qd) for _ in range(4)]
     ws = torch.empty(spinq.spinq_decode_attention_workspace_bytes(B, S, Hq, Hkv, Dd), dtype=torch.uint8, device=dev)
-    att_us = graph_us(lambda i: spinq.decode_attention_kv4(qd, cache, out=outs[i], workspace=ws), 2)
+    att_us = graph_us(lambda i: spinq.decode_attention_kv4(qd, caches[i], out=outs[i], workspace=ws), 4)
     torch.cuda.synchronize()
     att_bytes = B * S * Hkv * (Dd + 16) + 2 * B * Hq * Dd * 2
     # timed output of batch 0 against the oracle on the same codes
@@ -825,7 +829,7 @@ def attention_records(dev, hbm_peak):
     got = outs[0][:1].double().cpu().numpy()
     if not np.all(np.abs(got - ref) <= 2e-3 * np.abs(ref) + 2e-3 * np.abs(ref).max()):
         raise RuntimeError("decode attention: timed output differs from the oracle")
-    del q, k, v, cache
+    del q, k, v, cache, caches
     torch.cuda.empty_cache()
     return {
         "f2_rope_r3_kv4_B8_S4096": {"us": round(rope_us, 2), "bytes": rope_bytes,
@@ -1053,6 +1057,76 @@ def relaunch(args_n):
     return subprocess.call(cmd)
 
 
+PROFILE_CASES = ("attention", "rope_kv", "fp8_gemm", "w4a8_gemm", "rq8_paley", "cayley", "paley", "gemm")
+
+
+def profile_case(name, reps):
+    """One kernel family on its bench workload, `reps` launches, for a
+    profiler (`ncu -k ... python bench.py --profile-case NAME`): no timing,
+    prints the device status.  attention: decode attention over the
+    B 8, S 4096, 32/8-head, D 128 cache; rope_kv: RoPE + R3 + KV4 on B 2 of
+    that cache; fp8_gemm / w4a8_gemm: the gate_up projection 2048 x 4096 ->
+    14336 with E4M3 codes / 4-bit weights and 8-bit activation planes;
+    rq8_paley: the 8-bit quantizer with H28 x H512 on 2048 x 14336; cayley:
+    152 rotations of 128 x 128, 2 iterations; paley: the 4-bit R4 kernel on
+    2048 x 14336; gemm: the W4A4 down_proj 2048 x 14336 -> 4096."""
+    import numpy as np
+    import torch
+
+    from paper_2405_16406_gb300 import spinq, synth
+    dev = torch.device("cuda", 0)
+    if name == "attention":
+        kv = synth.kv_case()
+        cache = spinq.rotate_quant_kv(torch.from_numpy(kv.q).to(dev), torch.from_numpy(kv.k).to(dev),
+                                      torch.from_numpy(kv.v).to(dev))
+        qd = (torch.randn(kv.B, kv.Hq, kv.D, device=dev) * 2).half()
+        fn = lambda: spinq.decode_attention_kv4(qd, cache)
+    elif name == "rope_kv":
+        kv = synth.kv_case(B=2)
+        th = 500000.0 ** (-2.0 * np.arange(kv.D // 2) / kv.D)
+        ang = np.arange(kv.S)[:, None] * th[None, :]
+        cs = torch.from_numpy(np.stack([np.cos(ang), np.sin(ang)], -1).astype(np.float32)).to(dev)
+        pos = torch.arange(kv.S, dtype=torch.int32, device=dev).repeat(kv.B, 1)
+        q, k, v = (torch.from_numpy(t).to(dev) for t in (kv.q, kv.k, kv.v))
+        fn = lambda: spinq.rope_rotate_quant_kv(q, k, v, pos, cs)
+    elif name in ("fp8_gemm", "w4a8_gemm"):
+        c = synth.llama3_8b_gate_up()
+        x, w = torch.from_numpy(c.x).to(dev), torch.from_numpy(c.w).to(dev)
+        if name == "fp8_gemm":
+            qa = spinq.rotate_quant_act8(x, None, spinq.SPINQ_FMT_E4M3, True)
+            qw = spinq.quant_weight8(w, None, spinq.SPINQ_FMT_E4M3)
+            fn = lambda: spinq.fp8_gemm(qa, qw)
+        else:
+            qa = spinq.rotate_quant_act8(x, None, spinq.SPINQ_FMT_INT8_PLANES, False)
+            qw = spinq.quant_weight8(w, None, spinq.SPINQ_FMT_INT4_BYTES)
+            fn = lambda: spinq.w4a8_gemm(qa, qw)
+    elif name in ("rq8_paley", "paley", "gemm"):
+        c = synth.llama3_8b_down_proj()
+        x = torch.from_numpy(c.x).to(dev)
+        if name == "rq8_paley":
+            fn = lambda: spinq.rotate_quant_act8(x, c.had, spinq.SPINQ_FMT_E4M3, True)
+        elif name == "paley":
+            fn = lambda: spinq.rotate_quant_act(x, c.had)
+        else:
+            qa = spinq.rotate_quant_act(x, c.had)
+            qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), c.had)
+            fn = lambda: spinq.w4a4_gemm(qa, qw)
+    elif name == "cayley":
+        rng = np.random.default_rng(0)
+        R = np.stack([np.linalg.qr(rng.standard_normal((128, 128)))[0] for _ in range(152)]).astype(np.float32)
+        Rt = torch.from_numpy(R).to(dev)
+        G = torch.from_numpy((rng.standard_normal((152, 128, 128)) * 0.5).astype(np.float32)).to(dev)
+        fn = lambda: spinq.cayley_step(Rt, G, 0.01, 2)
+    else:
+        raise ValueError(f"unknown profile case {name}")
+    for _ in range(reps):
+        fn()
+    torch.cuda.synchronize()
+    st = spinq.spinq_device_status()
+    print(json.dumps({"profile_case": name, "reps": reps, "device_status": list(st)}))
+    return 0 if st[0] == spinq.SPINQ_OK else 1
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -1065,8 +1139,13 @@ def main():
     ap.add_argument("--no-configs", action="store_true", help="skip the per-config full-size runs")
     ap.add_argument("--launch-check", action="store_true",
                     help="only start the ranks, join the process group and report them (no kernels)")
+    ap.add_argument("--profile-case", choices=PROFILE_CASES,
+                    help="run one kernel family on its bench workload --reps times and exit (for a profiler)")
+    ap.add_argument("--reps", type=int, default=3, help="launches of --profile-case")
     args = ap.parse_args()
 
+    if args.profile_case:
+        sys.exit(profile_case(args.profile_case, args.reps))
     if args.gpus < 1:
         ap.error("--gpus must be at least 1")
     if "WORLD_SIZE" not in os.environ and args.gpus > 1:

@@ -358,15 +358,21 @@ spinq_status spinq_rope_rotate_quant_kv(const void* q_in, void* q_out, const voi
  * over t < lens[b]; query head h reads kv head h / (Hq / Hkv).
  *   q        [B][Hq][D] fp16, already rotated by R3 (the q_out of the call
  *            above for the decode token).
- *   k_codes, v_codes [B][S][Hkv][D/2]; k_scale, k_zero, v_scale, v_zero
- *            [B][S][Hkv] fp32 (S is the cache capacity: the row stride).
+ *   k_codes, v_codes [B][S][Hkv][D/2], 16-byte aligned; k_scale, k_zero,
+ *            v_scale, v_zero [B][S][Hkv] fp32 (S is the cache capacity: the
+ *            row stride).
  *   lens     [B] int32 in [1, S] (device), or NULL for S everywhere.
  *   out      [B][Hq][D] fp16.
  *   workspace device buffer of spinq_decode_attention_workspace_bytes(B, S,
  *            Hq, Hkv, D) bytes, 16-byte aligned (the per-chunk partial
  *            results; no zeroing needed).
- *   Supported: D = 64 or 128, Hq / Hkv in {1, 2, 4, 8}.  Arithmetic in
- *   fp32; two kernels on `stream` (the chunks, then their merge).
+ *   Supported: D = 64 or 128, Hq / Hkv in {1, 2, 4, 8}, S * Hkv * D / 2 <
+ *   2^31 (one batch's codes within 2 GiB).  Both products run
+ *   on the tensor core with fp32 accumulation: q . u on the fp16 query and
+ *   the exact codes, the value sum on the codes and fp16 weights
+ *   p * v_scale / max(v_scale) (relative rounding 2^-11 per weight); the
+ *   softmax and the scales in fp32.  Two kernels on `stream` (the chunks,
+ *   then their merge).
  */
 int64_t spinq_decode_attention_workspace_bytes(int64_t B, int64_t S, int64_t Hq, int64_t Hkv, int64_t D);
 spinq_status spinq_decode_attention_kv4(const void* q, const uint8_t* k_codes, const float* k_scale,

@@ -404,6 +404,7 @@ spinq_status spinq_decode_attention_kv4(const void* q, const uint8_t* k_codes, c
   const int64_t G = Hq / Hkv;
   if ((D != 64 && D != 128) || (G != 1 && G != 2 && G != 4 && G != 8)) return SPINQ_EUNSUPPORTED;
   if (B > 65535 || Hkv > 65535 || S > INT32_MAX) return SPINQ_EUNSUPPORTED;
+  if (S * Hkv * (D / 2) > INT32_MAX) return SPINQ_EUNSUPPORTED;   // one batch's cache within 2 GiB
   if (B == 0) return SPINQ_OK;
   AttnArgs a{q, k_codes, k_scale, k_zero, v_codes, v_scale, v_zero, lens, B, S, Hq, Hkv, (int)D, softmax_scale,
              out, static_cast<float*>(workspace)};

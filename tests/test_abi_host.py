@@ -203,6 +203,7 @@ def test_attention_entry_points_reject_invalid_arguments_on_the_host(lib):
     assert f(*args, 2, 64, 32, 8, 128, 0.1, fake, fake, need - 16, None) == S.SPINQ_EINVAL     # workspace
     assert f(*args, 2, 64, 32, 8, 96, 0.1, fake, fake, 1 << 30, None) == S.SPINQ_EUNSUPPORTED  # D
     assert f(*args, 2, 64, 48, 2, 128, 0.1, fake, fake, 1 << 30, None) == S.SPINQ_EUNSUPPORTED  # G = 24
+    assert f(*args, 1, 1 << 23, 32, 8, 128, 0.1, fake, fake, 1 << 40, None) == S.SPINQ_EUNSUPPORTED  # 4 GiB batch
     assert f(*args, 0, 64, 32, 8, 128, 0.1, None, None, 0, None) == S.SPINQ_OK
     g = S.spinq_rope_rotate_quant_kv
     kvq = S.quant_cfg(4, False, S.SPINQ_PER_GROUP, 128, 1.0)

@@ -8,8 +8,12 @@ the elements), which moves every R3 output of that row by at most
 ulp16(max|x|) / sqrt(D); with the R3 bound of the plain KV path this gives
 |dq| <= ulp16(q) + 2^-20 |x| + 2 ulp16(max|x|) / sqrt(D).  Attention: the
 oracle runs on the GPU's own codes and scales (dequantized in double), so the
-kernel is compared on identical inputs; fp32 scores and sums against double
-plus the fp16 output rounding: elementwise within 2e-3 |o| + 2e-3 max|o|."""
+kernel is compared on identical inputs; tensor-core products with fp32
+accumulation (exact fp16 query times exact code), fp16 weights p v_scale / r
+(relative rounding 2^-12 each) and the fp16 output rounding against double:
+elementwise within 2e-3 |o| + 2e-3 max|o|."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -120,6 +124,42 @@ def test_decode_attention_matches_oracle(B, S, Hq, Hkv, D, lens):
     got = o.cpu().numpy().astype(np.float64)
     assert rel_frob(got, ref) <= 2e-3
     assert np.all(np.abs(got - ref) <= 2e-3 * np.abs(ref) + 2e-3 * np.abs(ref).max())
+    assert spinq.spinq_device_status()[0] == spinq.SPINQ_OK
+
+
+@pytest.mark.parametrize("v_mag", [1e-4, 30.0])
+def test_decode_attention_value_scale_range(v_mag):
+    """Values far below and above 1 (outputs up to ~2600, within fp16): the
+    fp16 weights p v_scale / r are scaled by the running maximum r of the
+    value scales, so they stay in [0, 1] and clear of the subnormal range."""
+    from paper_2405_16406_gb300 import spinq
+    B, S, Hq, Hkv, D = 2, 777, 16, 4, 128
+    cache, q, _ = _attention_case(5, B, S, Hq, Hkv, D)
+    cache = dataclasses.replace(cache, v_scale=cache.v_scale * v_mag, v_zero=cache.v_zero * v_mag)
+    o = spinq.decode_attention_kv4(torch.from_numpy(q).cuda(), cache)
+    torch.cuda.synchronize()
+    ref = _oracle_attention(cache, q, None, D)
+    got = o.cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(got))
+    assert np.all(np.abs(got - ref) <= 2e-3 * np.abs(ref) + 2e-3 * np.abs(ref).max())
+
+
+def test_decode_attention_one_chunk_long_cache():
+    """B * Hkv large enough that each (batch, kv head) runs as one chunk over
+    a long cache (many steps per warp, the online rescaling over thousands of
+    tokens)."""
+    from paper_2405_16406_gb300 import spinq
+    B, S, Hq, Hkv, D = 80, 1500, 64, 8, 64
+    cache, q, _ = _attention_case(9, B, S, Hq, Hkv, D)
+    assert spinq.spinq_decode_attention_workspace_bytes(B, S, Hq, Hkv, D) == B * Hq * (D + 2) * 4
+    o = spinq.decode_attention_kv4(torch.from_numpy(q).cuda(), cache)
+    torch.cuda.synchronize()
+    got = o.cpu().numpy().astype(np.float64)
+    for b in (0, 41, 79):
+        sub = spinq.KVCodes(None, cache.k_codes[b:b + 1], cache.k_scale[b:b + 1], cache.k_zero[b:b + 1],
+                            cache.v_codes[b:b + 1], cache.v_scale[b:b + 1], cache.v_zero[b:b + 1])
+        ref = _oracle_attention(sub, q[b:b + 1], None, D)[0]
+        assert np.all(np.abs(got[b] - ref) <= 2e-3 * np.abs(ref) + 2e-3 * np.abs(ref).max())
     assert spinq.spinq_device_status()[0] == spinq.SPINQ_OK
 
 
