@@ -20,28 +20,28 @@
 // Phase 1 of row r + 1 runs while phase 2 of row r runs, and the copies of
 // the next rows are in flight meanwhile.
 //
-// Phase 1 (tensor core, raw fp16).  Y[i][j] = sum_i' X[i'][j] H_s[i'][i] is an
-// m16n8k16 MMA per 16 consecutive j: A[m = j][k = i'] comes straight from the
-// staged fp16 rows with ldmatrix.trans, B = H_s (+-1, zero-padded to 16/32).
-// Lane (g, c) of phase-1 warp w receives j = 16 (w + W v) + 8 h + g for h in
-// {0, 1}, v in 0..3 and i = 2c + {0, 1} + 8 nt.  Radix-2 butterflies inside
-// the lane cover the j bits of h and v, on packed fp32 pairs (i, i + 1).
+// Phase 1 (tensor core, raw fp16).  Y^T[i][j] = sum_i' H_s[i'][i] X[i'][j]
+// is an m16n8k16 MMA per 16 Paley rows i and 8 consecutive j: A = H_s^T (+-1,
+// zero outside NS), B[k = i'][n = j] straight from the staged fp16 row with
+// ldmatrix.trans.  Warp w takes j in [64 w, 64 w + 64); lane (g, c) receives
+// the pairs (j, j + 1), j = 64 w + 8 nt + 2c, of rows i = 16 mt + 8 h + g, and
+// finishes j bit 0 inside each pair and j bits 3..5 (nt) across its registers.
 //
-// Transpose.  Y goes to an fp32 buffer with row stride P + 4 in which j is
-// stored at j ^ (bit (4 + log2 W) of j) << 2 ^ (bit (5 + log2 W) of j) << 4:
-// the scalar stores here and the 16-byte loads of phase 2 are both free of
-// bank conflicts.
+// Transpose.  Y goes to an fp32 buffer with row stride P + 8 in which j sits
+// at j with bit 2 flipped by bit 5: the 8-byte pair stores here and the
+// 16-byte loads of phase 2 are both free of bank conflicts.
 //
 // Phase 2.  A thread owns, for one i, the 8 consecutive j of bits 0..2 for
-// each value of the phase-1 warp bits (8 W values), finishes the butterflies
-// over those bits on pairs of consecutive elements and joins the row-wide
-// range reduction (one named barrier over the phase-2 warps).  The 8 lanes of
-// a quarter warp share i, so a warp writes 4 whole segments of codes: lane
-// pairs swap packed words so that each lane stores 16 contiguous bytes.
+// each value of the bits above 5 (8 W values), finishes the butterflies over
+// j bits 1, 2 and 6.. on packed pairs and joins the row-wide range reduction
+// (one named barrier over the phase-2 warps).  The 8 lanes of a quarter warp
+// share i, so each of their 4-byte code words lands next to the others
+// (32 contiguous bytes per store instruction and quarter warp).
 // Eq. 1 runs on the unnormalised row; alpha and beta carry 1/sqrt(K).
 //
-// Every wait is bounded in time.  A warp that gives up raises the CTA's abort
-// flag; the others see it in their own waits, the phase-2 warps agree on it
+// Every wait is bounded in time (suspended in hardware until the phase
+// completes, the limit checked every ~20 us).  A warp that gives up raises the
+// CTA's abort flag; the others see it in their own waits, the phase-2 warps agree on it
 // through a barrier reduction before any global store, and the phase-1 warps
 // let the copies in flight land before they exit.
 #include <cuda_fp16.h>
@@ -70,29 +70,36 @@ struct PaleyShape {
   static constexpr int T = 32 * W;                 // threads per compute role
   static constexpr int THREADS = 2 * T;            // phase-1 warps, then phase-2 warps
   static constexpr int KS = (NS + 15) / 16;        // k16 steps over i'
-  static constexpr int NT = (NS + 7) / 8;          // n8 tiles over i
+  static constexpr int MT = (NS + 15) / 16;        // m16 tiles over i
   static constexpr int NSP = NS <= 16 ? 16 : 32;   // phase-2 row slots
   static constexpr int NCOMBO = NSP * 8;           // phase-2 (i slot, j group) combos
   static constexpr int NCB = (NCOMBO + T - 1) / T; // combos per thread
-  static constexpr int PS = P + 4;                 // fp32 row stride
+  static constexpr int PS = P + 8;                 // fp32 row stride (8 mod 32: see the layout note)
   static constexpr int ROWB = NS * P * 2;          // staged row (bytes, a multiple of 1024)
   static constexpr int F32B = NS * PS * 4;         // one transpose buffer (bytes)
-  static constexpr int MISC = 16 + 4 * 8 + 16 + 2 * 2 * W * 4;  // zero chunk, 4 barriers, flag, range scratch
+  static constexpr int MISC = 4 * 8 + 16 + 2 * 2 * W * 4;  // 4 barriers, flag, range scratch
   static constexpr int NSTG_FIT = (kSmemBudget - 1024 - 2 * F32B - MISC) / (ROWB + 16);  // 16: barrier + counters
   static constexpr int NSTG = NSTG_FIT < 4 ? NSTG_FIT : 4;   // staged rows
   static_assert(NSTG >= 2, "two staged rows must fit");
   static_assert(ROWB % 1024 == 0, "stages keep the 1024-byte alignment of the swizzle pattern");
+  static_assert(NS % 4 == 0, "phase-2 warps hold 4 whole Paley rows");
   // shared memory layout (bytes from the 1024-aligned base)
   static constexpr int OFF_STAGE = 0;
   static constexpr int OFF_F32 = NSTG * ROWB;
-  static constexpr int OFF_ZERO = OFF_F32 + 2 * F32B;
-  static constexpr int OFF_BAR = OFF_ZERO + 16;    // full[NSTG] bfull[2] bempty[2]
+  static constexpr int OFF_BAR = OFF_F32 + 2 * F32B;   // full[NSTG] bfull[2] bempty[2]
   static constexpr int OFF_CNT = OFF_BAR + (NSTG + 4) * 8;   // int readers[NSTG], int issued[NSTG]
   static constexpr int OFF_FLAG = OFF_CNT + NSTG * 8;
   static constexpr int OFF_RED = OFF_FLAG + 16;    // [2 rows][hi W, lo W]
   static constexpr int BYTES = OFF_RED + 2 * 2 * W * 4 + 1024;  // + alignment slack
   static_assert(BYTES <= kSmemBudget, "shared memory");
 };
+
+// Transpose-buffer position (floats from the row start) of element j: j with
+// bit 2 flipped by bit 5.  With the row stride P + 8 (8 mod 32) this keeps
+// both the phase-1 stores (8-byte pairs (j, j + 1) of 4 Paley rows x 4 lane
+// columns per half warp) and the phase-2 loads (16-byte quads of the 8 j
+// groups of one Paley row per quarter warp) free of bank conflicts.
+__host__ __device__ constexpr int tpos(int j) { return j ^ (((j >> 5) & 1) << 2); }
 
 // Paley row slot of phase-2 combo cb: the 8 lanes of a quarter warp share
 // it (cb & 7 is the j group), so a warp covers 4 consecutive slots
@@ -109,7 +116,7 @@ __device__ __forceinline__ bool combo_warp_idle(int cb, int ns) {
 // Bounded wait for the phase of `bar` with `parity`.  Returns false when the
 // abort flag is up or the limit expired (then it raises the flag).
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-  return mbar_wait_backoff(bar, parity, abort_flag, g_wait_ns);
+  return mbar_wait_suspend(bar, parity, abort_flag, g_wait_ns);
 }
 
 // bar.sync over `nthreads` threads whose result is the OR of `pred` over them.
@@ -127,7 +134,7 @@ template <int NS, int LP, bool SYM, bool CLAMP, bool SG>
 __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
     rq_paley_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
   using S = PaleyShape<NS, LP>;
-  constexpr int P = S::P, W = S::W, T = S::T, NSTG = S::NSTG;
+  constexpr int P = S::P, W = S::W, T = S::T, NSTG = S::NSTG, PS = S::PS;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-aligned base, derived from the shared array itself so that every
   // access below stays in the shared address space
@@ -160,7 +167,6 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
       mbar_init(&bfull[b], W);   // one arrival per warp, after __syncwarp
       mbar_init(&bempty[b], W);
     }
-    *reinterpret_cast<uint4*>(smem + S::OFF_ZERO) = make_uint4(0, 0, 0, 0);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmx);
@@ -173,95 +179,105 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
 
   if (warp < W) {
     // ---------------- phase 1: H_s on the tensor core, first butterflies
+    // Y^T = H_s^T X as m16n8k16 MMAs: M = i (the Paley index, S::MT tiles),
+    // N = 8 consecutive j, K = i'.  Warp w takes j in [64 w, 64 w + 64) (8
+    // n-tiles); lane (g, c) ends up with the pairs (j, j + 1) for
+    // j = 64 w + 8 nt + 2c and i = 16 mt + 8 h + g.
     const int w = warp, g = lane >> 2, c = lane & 3;
-    // B fragments of H_s (k = i', n = i), zero outside NS
-    uint32_t bs[S::KS][S::NT][2];
+    // A fragments of H_s^T: A[i][i'] = H_s[i'][i], zero outside NS (so the
+    // padding rows of the B operand, which read a real row, add nothing)
+    uint32_t ah[S::MT][S::KS][4];
 #pragma unroll
-    for (int ks = 0; ks < S::KS; ++ks)
+    for (int mt = 0; mt < S::MT; ++mt)
 #pragma unroll
-      for (int nt = 0; nt < S::NT; ++nt) {
-        const int n = g + 8 * nt;
+      for (int ks = 0; ks < S::KS; ++ks)
 #pragma unroll
-        for (int hb = 0; hb < 2; ++hb) {
-          const int k0 = 2 * c + 8 * hb + 16 * ks;
+        for (int q = 0; q < 4; ++q) {
+          const int i = 16 * mt + g + 8 * (q & 1), k0 = 16 * ks + 2 * c + 8 * (q >> 1);
           float v[2];
 #pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int k = k0 + e;
-            v[e] = (k < NS && n < NS) ? (((a.hs.neg[k] >> n) & 1u) ? -1.f : 1.f) : 0.f;
-          }
-          bs[ks][nt][hb] = pack_half2_bits(v[0], v[1]);
+          for (int e = 0; e < 2; ++e)
+            v[e] = (i < NS && k0 + e < NS) ? (((a.hs.neg[k0 + e] >> i) & 1u) ? -1.f : 1.f) : 0.f;
+          ah[mt][ks][q] = pack_half2_bits(v[0], v[1]);
         }
-      }
-    const uint32_t zero_addr = smem_u32(smem + S::OFF_ZERO);
-    // Random signs (R = S H): each fragment element below sits at the same
-    // row position for every row, so this lane gathers its sign bits once:
-    // bit ((v KS + ks) 4 + q) 2 + e is the sign of element e of fragment q.
-    constexpr int NSB = (4 * S::KS * 4 * 2 + 31) / 32;
+    // ldmatrix.x4.trans row addresses (from the stage base): matrix q of
+    // (ks, ntp) holds i' = 16 ks + 8 (q & 1) + 0..7 (rows) at j = 64 w + 8 nt
+    // + 0..7 (columns), nt = 2 ntp + (q >> 1); lane 8q + r gives row r.  The
+    // stage holds 128-byte lines l = i' + NS j_hi with chunk c at c ^ (l % 8).
+    uint32_t loff[S::KS][4];
+    {
+      const int q = lane >> 3, r = lane & 7;
+#pragma unroll
+      for (int ks = 0; ks < S::KS; ++ks)
+#pragma unroll
+        for (int ntp = 0; ntp < 4; ++ntp) {
+          int ip = 16 * ks + 8 * (q & 1) + r;
+          ip = ip < NS ? ip : NS - 1;
+          const int nt = 2 * ntp + (q >> 1), line = ip + NS * w;
+          loff[ks][ntp] = (uint32_t)(line * 128 + ((nt ^ (line & 7)) << 4));
+        }
+    }
+    // Random signs (R = S H): element e of register q of the (ks, ntp)
+    // fragment is x[i'][j] with i' = 16 ks + 8 (q & 1) + 2c + e and
+    // j = 64 w + 8 (2 ntp + (q >> 1)) + g, the same for every row: this lane
+    // gathers those sign bits once, bit ((ks 4 + ntp) 4 + q) 2 + e.
+    constexpr int NSB = (S::KS * 4 * 4 * 2 + 31) / 32;
     uint32_t sgn[NSB];
 #pragma unroll
     for (int t = 0; t < NSB; ++t) sgn[t] = 0;
     if constexpr (SG) {
 #pragma unroll
-      for (int v = 0; v < 4; ++v)
+      for (int ks = 0; ks < S::KS; ++ks)
 #pragma unroll
-        for (int ks = 0; ks < S::KS; ++ks)
+        for (int ntp = 0; ntp < 4; ++ntp)
 #pragma unroll
           for (int q = 0; q < 4; ++q)
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-              const int ip = 8 * (q >> 1) + 16 * ks + 2 * c + e;
-              const int j = 16 * (w + W * v) + 8 * (q & 1) + g;
-              const int idx = ((v * S::KS + ks) * 4 + q) * 2 + e;
+              const int ip = 16 * ks + 8 * (q & 1) + 2 * c + e;
+              const int j = 64 * w + 8 * (2 * ntp + (q >> 1)) + g;
+              const int idx = ((ks * 4 + ntp) * 4 + q) * 2 + e;
               if (ip < NS) {
                 const int k = ip * P + j;
                 sgn[idx >> 5] |= (uint32_t)((a.signs[k >> 3] >> (k & 7)) & 1) << (idx & 31);
               }
             }
     }
-    // transpose-buffer position of j = 16 (w + W v) + 8 h + g, minus 8 h: bit 2
-    // of j flips with v & 1, bit 4 (the low bit of w) with v >> 1
-    int pos[4];
-#pragma unroll
-    for (int v = 0; v < 4; ++v) pos[v] = 16 * ((w ^ (v >> 1)) + W * v) + (g ^ ((v & 1) << 2));
+    // transpose-buffer float offsets of this lane's pairs: row g, column
+    // tpos(64 w + 8 nt + 2c) = 64 w + 8 nt + (2c ^ 4 (nt >> 2))
+    const int sb0 = g * PS + 64 * w + 2 * c, sb1 = g * PS + 64 * w + ((2 * c) ^ 4);
     for (int it = 0; it < niter; ++it) {
       const int s = it % NSTG;
       // warp-uniform decision: the MMAs below need every lane
       if (!__all_sync(0xffffffffu, wait_or_abort(&full[s], (uint32_t)(it / NSTG) & 1u, abort_flag))) break;
       const uint32_t stage_addr = smem_u32(smem + S::OFF_STAGE + s * S::ROWB);
-      // y[nt][h][v] = the pair of outputs i = 2c + 8 nt + {0, 1} at
-      // j = 16 (w + W v) + 8 h + g
-      F2 y[S::NT][2][4];
+      // y[mt][h][nt] = the pair (j, j + 1), j = 64 w + 8 nt + 2c, of row i = 16 mt + 8 h + g
+      F2 y[S::MT][2][8];
 #pragma unroll
-      for (int v = 0; v < 4; ++v) {
-        const int jb = 16 * (w + W * v);
+      for (int ks = 0; ks < S::KS; ++ks)
 #pragma unroll
-        for (int ks = 0; ks < S::KS; ++ks) {
-          const int q = lane >> 3, r = lane & 7;
-          const int ip = r + 8 * (q >> 1) + 16 * ks;
-          const int js = jb + 8 * (q & 1);
-          const int line = ip + NS * (js >> 6);
-          const uint32_t addr =
-              ip < NS ? stage_addr + (uint32_t)(line * 128 + ((((js & 63) >> 3) ^ (line & 7)) << 4)) : zero_addr;
-          uint32_t af[4];
-          ldmatrix_x4_trans(af, addr);
+        for (int ntp = 0; ntp < 4; ++ntp) {
+          uint32_t bf[4];
+          ldmatrix_x4_trans(bf, stage_addr + loff[ks][ntp]);
           if constexpr (SG) {   // negate the fp16 elements whose sign bit is set
 #pragma unroll
-            for (int q2 = 0; q2 < 4; ++q2) {
-              const int idx = ((v * S::KS + ks) * 4 + q2) * 2;
+            for (int q = 0; q < 4; ++q) {
+              const int idx = ((ks * 4 + ntp) * 4 + q) * 2;
               const uint32_t bb = (sgn[idx >> 5] >> (idx & 31)) & 3u;
-              af[q2] ^= ((bb & 1u) << 15) | ((bb & 2u) << 30);
+              bf[q] ^= ((bb & 1u) << 15) | ((bb & 2u) << 30);
             }
           }
 #pragma unroll
-          for (int nt = 0; nt < S::NT; ++nt) {
-            if (ks == 0)
-              mma_16816_f16_f32_pairs(y[nt][0][v], y[nt][1][v], af, bs[ks][nt][0], bs[ks][nt][1]);
-            else
-              mma_16816_f16_f32_pairs_acc(y[nt][0][v], y[nt][1][v], af, bs[ks][nt][0], bs[ks][nt][1]);
-          }
+          for (int mt = 0; mt < S::MT; ++mt)
+#pragma unroll
+            for (int hn = 0; hn < 2; ++hn) {
+              const int nt = 2 * ntp + hn;
+              if (ks == 0)
+                mma_16816_f16_f32_pairs(y[mt][0][nt], y[mt][1][nt], ah[mt][ks], bf[2 * hn], bf[2 * hn + 1]);
+              else
+                mma_16816_f16_f32_pairs_acc(y[mt][0][nt], y[mt][1][nt], ah[mt][ks], bf[2 * hn], bf[2 * hn + 1]);
+            }
         }
-      }
       __syncwarp();
       if (lane == 0) {
         // this warp no longer reads the stage; the last one refills it
@@ -271,42 +287,39 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
           if (it + NSTG < niter) issue(it + NSTG);
         }
       }
-      // butterflies over h (j bit 3) and v (the two highest j bits)
+      // butterflies over j bit 0 (inside each pair) and j bits 3, 4, 5 (nt);
+      // row halves wholly past NS hold zeros and are skipped
 #pragma unroll
-      for (int nt = 0; nt < S::NT; ++nt) {
+      for (int mt = 0; mt < S::MT; ++mt)
 #pragma unroll
-        for (int v = 0; v < 4; ++v) f2_bfly(y[nt][0][v], y[nt][1][v]);
+        for (int h = 0; h < 2; ++h) {
+          if (16 * mt + 8 * h >= NS) continue;
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
+          for (int nt = 0; nt < 8; ++nt) f2_bfly_inner(y[mt][h][nt]);
 #pragma unroll
-          for (int bit = 1; bit < 4; bit <<= 1)
+          for (int bit = 1; bit < 8; bit <<= 1)
 #pragma unroll
-            for (int v = 0; v < 4; ++v)
-              if (!(v & bit)) f2_bfly(y[nt][h][v], y[nt][h][v | bit]);
-      }
+            for (int nt = 0; nt < 8; ++nt)
+              if (!(nt & bit)) f2_bfly(y[mt][h][nt], y[mt][h][nt | bit]);
+        }
       const int b = it & 1;
       if (it >= 2 &&
           !__all_sync(0xffffffffu, wait_or_abort(&bempty[b], (uint32_t)((it >> 1) - 1) & 1u, abort_flag)))
         break;
-      // transpose through shared memory (NS is even: both outputs of a pair
-      // are real or both are padding)
+      // transpose through shared memory: one 8-byte store per pair
       float* sf = reinterpret_cast<float*>(smem + S::OFF_F32 + b * S::F32B);
 #pragma unroll
-      for (int nt = 0; nt < S::NT; ++nt) {
-        const int i = 2 * c + 8 * nt;
-        if (i < NS) {
+      for (int mt = 0; mt < S::MT; ++mt)
 #pragma unroll
-          for (int h = 0; h < 2; ++h)
+        for (int h = 0; h < 2; ++h) {
+          if (16 * mt + 8 * h >= NS) continue;
+          if (16 * mt + 8 * h + g < NS) {
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              float lo, hi;
-              f2_split(y[nt][h][v], lo, hi);
-              float* dst = sf + i * S::PS + pos[v] + 8 * h;
-              dst[0] = lo;
-              dst[S::PS] = hi;
-            }
+            for (int nt = 0; nt < 8; ++nt)
+              *reinterpret_cast<unsigned long long*>(sf + (nt < 4 ? sb0 : sb1) + (16 * mt + 8 * h) * PS + 8 * nt) =
+                  y[mt][h][nt].u;
+          }
         }
-      }
       __syncwarp();
       if (lane == 0) mbar_arrive(&bfull[b]);  // release: the warp's stores above are ordered before it
     }
@@ -322,41 +335,39 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
   }
 
   // ---------------- phase 2: remaining butterflies, range, Eq. 1, codes
+  // Combo cb = (Paley row i, j group jg = j bits 3..5): the thread holds the
+  // 8 consecutive j of bits 0..2 for each value wv of the bits above 5, as
+  // z[k][wv][q] = the pair (j, j + 1), j = 64 wv + 8 jg + 2q.  The 8 lanes of
+  // a quarter warp share i, so a warp holds 4 whole Paley rows.
   const int t2 = tid - T, w2 = warp - W;
   float* red = reinterpret_cast<float*>(smem + S::OFF_RED);
+  int ld0[S::NCB], ld1[S::NCB];   // float offsets of the quads hh = 0, 1 at wv = 0
+#pragma unroll
+  for (int k = 0; k < S::NCB; ++k) {
+    const int cb = t2 + T * k, i2 = combo_i(cb), jg = cb & 7;
+    ld0[k] = i2 * PS + tpos(8 * jg);
+    ld1[k] = i2 * PS + tpos(8 * jg + 4);
+  }
   for (int it = 0; it < niter; ++it) {
     const int64_t row = r0 + (int64_t)it * G;
     const int b = it & 1;
     // on a failed wait the buffer is read anyway (in bounds, discarded below)
     const bool ok = wait_or_abort(&bfull[b], (uint32_t)(it >> 1) & 1u, abort_flag);
     const float* sf = reinterpret_cast<const float*>(smem + S::OFF_F32 + b * S::F32B);
-    // z[k][wv][q] = elements e = 2q, 2q + 1 of the 8 consecutive j at
-    // jf + 16 wv of combo k
     F2 z[S::NCB][W][4];
 #pragma unroll
     for (int k = 0; k < S::NCB; ++k) {
       const int cb = t2 + T * k;
-      const int i2 = combo_i(cb), jc = cb & 7;
-      const int jf = 8 * (jc & 1) + 16 * W * (jc >> 1);
-      // position of j = jf + 16 wv + 4 u in the transpose buffer: bits 2 and 4
-      // of j flip with the two high bits of jc
-      const int xr = (((jc >> 1) & 1) << 2) | ((jc >> 2) << 4);
-      if (cb < S::NCOMBO && i2 < NS) {
+      if (cb < S::NCOMBO && !combo_warp_idle(cb, NS)) {
 #pragma unroll
         for (int wv = 0; wv < W; ++wv) {
-          const float* rowp = sf + i2 * S::PS + jf;
-          const ulonglong2 u0 = *reinterpret_cast<const ulonglong2*>(rowp + ((16 * wv) ^ xr));
-          const ulonglong2 u1 = *reinterpret_cast<const ulonglong2*>(rowp + ((16 * wv + 4) ^ xr));
+          const ulonglong2 u0 = *reinterpret_cast<const ulonglong2*>(sf + ld0[k] + 64 * wv);
+          const ulonglong2 u1 = *reinterpret_cast<const ulonglong2*>(sf + ld1[k] + 64 * wv);
           z[k][wv][0].u = u0.x;
           z[k][wv][1].u = u0.y;
           z[k][wv][2].u = u1.x;
           z[k][wv][3].u = u1.y;
         }
-      } else {
-#pragma unroll
-        for (int wv = 0; wv < W; ++wv)
-#pragma unroll
-          for (int q = 0; q < 4; ++q) z[k][wv][q].u = 0ull;
       }
     }
     __syncwarp();
@@ -365,31 +376,26 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
 #pragma unroll
     for (int k = 0; k < S::NCB; ++k) {
       const int cb = t2 + T * k;
-      const bool act = cb < S::NCOMBO && combo_i(cb) < NS;
       if (cb >= S::NCOMBO || combo_warp_idle(cb, NS)) continue;
 #pragma unroll
       for (int wv = 0; wv < W; ++wv) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) f2_bfly_inner(z[k][wv][q]);  // e bit 0
-#pragma unroll
-        for (int bit = 1; bit < 4; bit <<= 1)                     // e bits 1, 2
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            if (!(q & bit)) f2_bfly(z[k][wv][q], z[k][wv][q | bit]);
+        f2_bfly(z[k][wv][0], z[k][wv][1]);   // j bit 1
+        f2_bfly(z[k][wv][2], z[k][wv][3]);
+        f2_bfly(z[k][wv][0], z[k][wv][2]);   // j bit 2
+        f2_bfly(z[k][wv][1], z[k][wv][3]);
       }
 #pragma unroll
-      for (int bit = 1; bit < W; bit <<= 1)
+      for (int bit = 1; bit < W; bit <<= 1)   // j bits 6 ..
 #pragma unroll
         for (int wv = 0; wv < W; ++wv)
           if (!(wv & bit)) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) f2_bfly(z[k][wv][q], z[k][wv | bit][q]);
           }
-      if (act)
 #pragma unroll
-        for (int wv = 0; wv < W; ++wv)
+      for (int wv = 0; wv < W; ++wv)
 #pragma unroll
-          for (int q = 0; q < 4; ++q) rg.add_pair(z[k][wv][q]);
+        for (int q = 0; q < 4; ++q) rg.add_pair(z[k][wv][q]);
     }
     // row range over the phase-2 warps (scratch alternates between rows, so
     // one barrier per row suffices); the same barrier settles the abort
@@ -409,45 +415,20 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
       if (!SYM) rg.lo = fminf(rg.lo, rd[W + i]);
     }
     const QParams<SYM> qp(rg, a.clip);
-    uint8_t* out = a.codes + row * (a.K / 2);
+    uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
 #pragma unroll
     for (int k = 0; k < S::NCB; ++k) {
       const int cb = t2 + T * k;
-      const int i2 = combo_i(cb), jc = cb & 7;
-      const bool act = cb < S::NCOMBO && i2 < NS;
       if (cb >= S::NCOMBO || combo_warp_idle(cb, NS)) continue;
-      // wd[wv] = codes of j = jf + 16 wv .. + 7: word (jc & 1) + 2 W (jc >> 1) + 2 wv of segment i2
-      uint32_t wd[W];
+      // word 8 wv + jg of segment i2 holds the codes of j = 64 wv + 8 jg .. + 7;
+      // a quarter warp writes 32 contiguous bytes per wv
+      uint32_t* seg = out + combo_i(cb) * (P / 8) + (cb & 7);
 #pragma unroll
       for (int wv = 0; wv < W; ++wv) {
         uint32_t rb[8];
 #pragma unroll
         for (int q = 0; q < 4; ++q) qp.template code_bits2<CLAMP>(z[k][wv][q], rb[2 * q], rb[2 * q + 1]);
-        wd[wv] = pack8_nibbles(rb);
-      }
-      // The pair (jc, jc ^ 1) (lanes l, l ^ 1) holds 2 W consecutive words,
-      // interleaved.  Cut them into chunks of CW words; the even lane stores
-      // the even chunks, the odd lane the odd ones, after swapping halves.
-      constexpr int CW = W >= 4 ? 4 : 2, NCH = 2 * W / CW, HV = CW / 2;
-      const bool odd = jc & 1;
-      uint32_t* seg = reinterpret_cast<uint32_t*>(out + i2 * (P / 2)) + 2 * W * (jc >> 1);
-#pragma unroll
-      for (int kk = 0; kk < NCH / 2; ++kk) {
-        uint32_t own[HV], oth[HV];
-#pragma unroll
-        for (int t = 0; t < HV; ++t) {
-          const uint32_t e = wd[(2 * kk) * HV + t], o = wd[(2 * kk + 1) * HV + t];
-          own[t] = odd ? o : e;
-          oth[t] = __shfl_xor_sync(0xffffffffu, odd ? e : o, 1);
-        }
-        uint32_t* dst = seg + (2 * kk + (odd ? 1 : 0)) * CW;
-        if (act) {
-          if constexpr (CW == 4)
-            *reinterpret_cast<uint4*>(dst) = odd ? make_uint4(oth[0], own[0], oth[HV - 1], own[HV - 1])
-                                                 : make_uint4(own[0], oth[0], own[HV - 1], oth[HV - 1]);
-          else
-            *reinterpret_cast<uint2*>(dst) = odd ? make_uint2(oth[0], own[0]) : make_uint2(own[0], oth[0]);
-        }
+        seg[8 * wv] = pack8_nibbles(rb);
       }
     }
     if (t2 == 0) {
