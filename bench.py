@@ -708,7 +708,7 @@ def run_configs(dev, hbm_peak, fp8_peak):
         return r
 
     res["c1_tiny_16x256x512_h256"] = linear(synth.tiny_linear(), "config 1", "latency")
-    for Mr in (1, 16, 128, 8192):
+    for Mr in (1, 8, 16, 128, 8192):
         bound = "tensor" if Mr >= 2048 else "hbm"
         res[f"c5_up_M{Mr}_h12xh256"] = linear(synth.llama32_3b_up(M=Mr), f"config 5 up M={Mr}", bound)
         res[f"c5_down_M{Mr}_h8192"] = linear(synth.llama32_3b_down(M=Mr), f"config 5 down M={Mr}", bound)

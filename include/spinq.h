@@ -282,7 +282,13 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
  *                       weights; calls it cannot serve use AUTO;
  *   SPINQ_GEMM_SPLITK   the split-K kernel on the _splitk / _noalloc entry
  *                       points for every M <= 256 (GEMV and prefill kernels
- *                       excluded); spinq_w4a4_gemm treats it as AUTO.
+ *                       excluded); spinq_w4a4_gemm treats it as AUTO;
+ *   SPINQ_GEMM_TCGEMV   (M <= 16, on every entry point; AUTO picks it for 5 to
+ *                       8 tokens) a CTA per 16 output channels streams their
+ *                       packed weights through shared memory and takes the
+ *                       products on the tensor core (fp16 m16n8k16 on the
+ *                       exact codes), no workspace; calls it cannot serve use
+ *                       AUTO.
  * All kernels compute bit-identical outputs; this is a tuning and testing
  * control.  Returns the previous selection, or -1 (and changes nothing) for
  * an unknown value.  Not synchronized with GEMM calls in other threads.
@@ -293,7 +299,8 @@ typedef enum {
   SPINQ_GEMM_TILE256 = 2,
   SPINQ_GEMM_PAIR = 3,
   SPINQ_GEMM_GEMV = 4,
-  SPINQ_GEMM_SPLITK = 5
+  SPINQ_GEMM_SPLITK = 5,
+  SPINQ_GEMM_TCGEMV = 6
 } spinq_gemm_kernel;
 
 int spinq_gemm_select_kernel(int kernel);
@@ -309,8 +316,8 @@ int spinq_gemm_select_kernel(int kernel);
 int spinq_gemm_split_k(int n);
 
 /*
- * spinq_w4a4_gemm_plan -- the kernel (SPINQ_GEMM_TILE128, _TILE256, _PAIR or
- * _GEMV) that spinq_w4a4_gemm runs for an M x N x K call on the current CUDA
+ * spinq_w4a4_gemm_plan -- the kernel (SPINQ_GEMM_TILE128, _TILE256, _PAIR,
+ * _GEMV or _TCGEMV) that spinq_w4a4_gemm runs for an M x N x K call on the current CUDA
  * device under the current selection; -1 for shapes the call rejects.
  * Launches nothing.
  */

@@ -132,6 +132,16 @@ inline bool w4a4_gemv_fits(int64_t M, int64_t K) {
 }
 cudaError_t launch_w4a4_gemv(const GemmArgs& a, cudaStream_t stream, bool* handled);
 
+// Tensor-core GEMV for M <= kGemvTcMaxM tokens: a CTA per 16 output
+// channels over the whole K, weights streamed into registers, m16n8k32 e4m3
+// MMAs, no workspace.  Sets *handled = false when the shape is out of range.
+constexpr int64_t kGemvTcMaxM = 16;
+inline bool w4a4_gemv_tc_fits(int64_t M, int64_t N, int64_t K) {
+  return M >= 1 && M <= kGemvTcMaxM && N >= 16 && N % 16 == 0 && K >= 128 && K % 128 == 0 && K <= 65536 &&
+         N / 16 <= 0x7FFFFFFF;
+}
+cudaError_t launch_w4a4_gemv_tc(const GemmArgs& a, cudaStream_t stream, bool* handled);
+
 // Decode GEMM for M <= kDecodeMaxM (launch_w4a4_gemm above): the GEMV kernel,
 // the split-K kernel or the prefill kernels, as a fitted cost model predicts
 // fastest.  `workspace` holds `workspace_bytes` bytes that are zero before

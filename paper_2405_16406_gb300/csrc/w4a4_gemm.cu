@@ -1157,7 +1157,7 @@ int dec_per_sm_for(int64_t M, int* mn) {
 std::atomic<int> g_gemm_kernel{SPINQ_GEMM_AUTO};
 
 int w4a4_gemm_select(int kernel) {
-  if (kernel < SPINQ_GEMM_AUTO || kernel > SPINQ_GEMM_SPLITK) return -1;
+  if (kernel < SPINQ_GEMM_AUTO || kernel > SPINQ_GEMM_TCGEMV) return -1;
   return g_gemm_kernel.exchange(kernel);
 }
 
@@ -1200,10 +1200,24 @@ PrefillChoice choose_prefill(int64_t M, int64_t N, int64_t K, bool allow_pair) {
   return c;
 }
 
+// The tensor-core GEMV serves every entry point for the shapes it fits when
+// it is selected, and 5 to 8 tokens under the automatic choice: measured on
+// GB300 over K x N in {3072 x 8192, 8192 x 3072, 4096 x 14336, 14336 x 4096},
+// it takes 5.8 / 6.5 / 14.2 / 10.2 us at 8 tokens against 9.1 / 9.0 / 14.2 /
+// 13.3 us for the split-K kernel; from 1 to 4 tokens the GEMV kernel is
+// faster, from 9 on the split-K kernel.
+constexpr int64_t kGemvTcAutoLo = 5, kGemvTcAutoHi = 8;
+bool tcgemv_serves(int64_t M, int64_t N, int64_t K) {
+  const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
+  if (!w4a4_gemv_tc_fits(M, N, K)) return false;
+  return forced == SPINQ_GEMM_TCGEMV || (forced == SPINQ_GEMM_AUTO && M >= kGemvTcAutoLo && M <= kGemvTcAutoHi);
+}
+
 }  // namespace
 
 int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K) {
   const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
+  if (tcgemv_serves(M, N, K)) return SPINQ_GEMM_TCGEMV;
   // a handful of tokens: the product streams the weights, no tile kernel fits
   // (the split-K selection concerns the other entry point only)
   if ((forced == SPINQ_GEMM_AUTO || forced == SPINQ_GEMM_GEMV || forced == SPINQ_GEMM_SPLITK) &&
@@ -1218,6 +1232,11 @@ int plan_w4a4_gemm(int64_t M, int64_t N, int64_t K) {
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
   const int kind = plan_w4a4_gemm(a.M, a.N, a.K);
+  if (kind == SPINQ_GEMM_TCGEMV) {
+    bool handled = false;
+    const cudaError_t e = launch_w4a4_gemv_tc(a, stream, &handled);
+    if (e != cudaSuccess || handled) return e;
+  }
   if (kind == SPINQ_GEMM_GEMV) {
     bool handled = false;
     const cudaError_t e = launch_w4a4_gemv(a, stream, &handled);
@@ -1304,7 +1323,7 @@ bool gemv_serves(int64_t M, int64_t K) {
 
 int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K) {
   // only split K slices sum through the workspace
-  if (M <= 0 || N <= 0 || M > kDecodeMaxM || gemv_serves(M, K)) return 0;
+  if (M <= 0 || N <= 0 || M > kDecodeMaxM || gemv_serves(M, K) || tcgemv_serves(M, N, K)) return 0;
   const DecodePlan p = plan_splitk_entry(M, N, K, true);
   if (p.prefill || p.nsplit <= 1) return 0;
   return split_workspace_bytes(M, N);
@@ -1313,6 +1332,7 @@ int64_t w4a4_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K) {
 int plan_w4a4_gemm_splitk(int64_t M, int64_t N, int64_t K, int* nsplit) {
   *nsplit = 0;
   if (M > kDecodeMaxM) return plan_w4a4_gemm(M, N, K);
+  if (tcgemv_serves(M, N, K)) return SPINQ_GEMM_TCGEMV;
   if (gemv_serves(M, K)) return SPINQ_GEMM_GEMV;
   const DecodePlan p = plan_splitk_entry(M, N, K, true);
   if (p.prefill) return plan_w4a4_gemm(M, N, K);
@@ -1324,6 +1344,11 @@ cudaError_t launch_w4a4_gemm_splitk(const GemmArgs& a, void* workspace, int64_t 
                                     cudaStream_t stream) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
   if (a.M > kDecodeMaxM) return launch_w4a4_gemm(a, stream);
+  if (tcgemv_serves(a.M, a.N, a.K)) {
+    bool handled = false;
+    const cudaError_t et = launch_w4a4_gemv_tc(a, stream, &handled);
+    if (et != cudaSuccess || handled) return et;
+  }
   if (gemv_serves(a.M, a.K)) {
     bool handled = false;
     const cudaError_t eg = launch_w4a4_gemv(a, stream, &handled);

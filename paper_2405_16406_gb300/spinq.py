@@ -31,7 +31,7 @@ _lib = ctypes.CDLL(LIB_PATH)
 SPINQ_OK, SPINQ_EINVAL, SPINQ_EUNSUPPORTED, SPINQ_ECUDA, SPINQ_ETIMEOUT, SPINQ_ESCRATCH = range(6)
 SPINQ_NOALLOC_SCRATCH_BYTES = 8 << 20   # include/spinq.h
 SPINQ_PER_TOKEN, SPINQ_PER_CHANNEL, SPINQ_PER_GROUP = range(3)
-SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR, SPINQ_GEMM_GEMV, SPINQ_GEMM_SPLITK = range(6)
+SPINQ_GEMM_AUTO, SPINQ_GEMM_TILE128, SPINQ_GEMM_TILE256, SPINQ_GEMM_PAIR, SPINQ_GEMM_GEMV, SPINQ_GEMM_SPLITK, SPINQ_GEMM_TCGEMV = range(7)
 
 EXPORTED = (
     "spinq_rotate_quant_act", "spinq_quant_weight", "spinq_w4a4_gemm", "spinq_rotate_quant_kv",

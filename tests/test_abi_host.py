@@ -108,7 +108,7 @@ def test_gemm_controls_validate_on_the_host(lib):
     """The kernel selection, the K-slice control and the plan queries check
     their arguments on the host; rejected values change nothing."""
     from paper_2405_16406_gb300 import spinq as S
-    for bad in (-1, S.SPINQ_GEMM_SPLITK + 1, 99):
+    for bad in (-1, S.SPINQ_GEMM_TCGEMV + 1, 99):
         assert S.spinq_gemm_select_kernel(bad) == -1
     prev = S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TILE256)
     try:

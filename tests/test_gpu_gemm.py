@@ -123,7 +123,7 @@ def test_gemm_each_kernel_same_bits(S, gemm_kernel):
 
 
 def test_gemm_select_kernel_rejects_unknown(S):
-    assert S.spinq_gemm_select_kernel(7) == -1
+    assert S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TCGEMV + 1) == -1
     assert S.spinq_gemm_select_kernel(-1) == -1
     assert S.spinq_gemm_select_kernel(0) == 0
 
@@ -144,7 +144,7 @@ def test_gemm_plan_follows_selection(S):
     assert S.spinq_w4a4_gemm_plan(2048, 14336, 4096) in (1, 2, 3)
     assert S.spinq_w4a4_gemm_plan(4, 14336, 4096) == 4      # a handful of tokens: GEMV
     assert S.spinq_w4a4_gemm_plan(5, 14336, 4096) != 4
-    assert S.spinq_gemm_select_kernel(6) == -1
+    assert S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TCGEMV + 1) == -1
 
 
 @pytest.mark.parametrize("symmetric", [True, False])
@@ -376,7 +376,7 @@ def test_splitk_plan_covers_every_route(S):
     routes = set()
     for M, N, K in shapes:
         kind, nsplit = S.spinq_w4a4_gemm_splitk_plan(M, N, K)
-        assert kind in (1, 2, 3, 4, 5)
+        assert kind in (1, 2, 3, 4, 5, 6)
         assert (nsplit >= 1) == (kind == S.SPINQ_GEMM_SPLITK)
         routes.add("sliced" if nsplit > 1 else "whole_k" if nsplit == 1 else kind)
         # the workspace exists exactly for K slices
@@ -455,6 +455,84 @@ def test_gemv_extreme_codes_long_k(S):
         al, ws_ = np.full(M, 0.5), np.full(N, 0.25)
         y, acc = run_splitk(S, ac, al, None, wc, ws_)
         assert np.array_equal(acc, oracle_full(ac, al, None, wc, ws_).acc)
+
+
+def _with_kernel(S, kind, fn):
+    prev = S.spinq_gemm_select_kernel(kind)
+    try:
+        return fn()
+    finally:
+        S.spinq_gemm_select_kernel(prev)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 16, 128), (5, 48, 256), (8, 272, 1152), (9, 512, 1024), (16, 3072, 8192),
+                                   (13, 1040, 4224), (16, 4096, 14336), (3, 8192, 3072), (12, 16, 40960)])
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_tcgemv_random_codes_exact(S, M, N, K, symmetric):
+    """The tensor-core GEMV (M <= 16) through both entry points: exact acc,
+    y within the GEMM bars; K block counts that leave the 8 warps' last
+    rounds partly empty."""
+    rng = np.random.default_rng(M * 131 + N + K + symmetric)
+    ac, al, be, wc, ws_ = random_codes(rng, M, N, K, symmetric)
+    ref = oracle_full(ac, al, be, wc, ws_)
+
+    def go():
+        assert S.spinq_w4a4_gemm_plan(M, N, K) == S.SPINQ_GEMM_TCGEMV
+        assert S.spinq_w4a4_gemm_splitk_plan(M, N, K) == (S.SPINQ_GEMM_TCGEMV, 0)
+        assert S.spinq_w4a4_gemm_workspace_bytes(M, N, K) == 0
+        return [run_splitk(S, ac, al, be, wc, ws_), run(S, ac, al, be, wc, ws_)]
+    for y, acc in _with_kernel(S, S.SPINQ_GEMM_TCGEMV, go):
+        assert np.array_equal(acc, ref.acc)
+        assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
+        assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
+
+
+@pytest.mark.parametrize("M", [3, 11, 16])
+def test_tcgemv_same_bits_as_the_other_decode_kernels(S, M):
+    """y and acc bit for bit against the kernel the cost model picks."""
+    rng = np.random.default_rng(M)
+    N, K = 1296, 3072
+    ac, al, be, wc, ws_ = random_codes(rng, M, N, K, False)
+    y0, acc0 = run_splitk(S, ac, al, be, wc, ws_)
+    y1, acc1 = _with_kernel(S, S.SPINQ_GEMM_TCGEMV, lambda: run_splitk(S, ac, al, be, wc, ws_))
+    assert np.array_equal(acc0, acc1)
+    assert np.array_equal(y0.view(np.uint16), y1.view(np.uint16))
+
+
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_tcgemv_extreme_codes_long_k(S, symmetric):
+    """K = 65536 with every code at an extreme: the e4m3 accumulator reaches
+    225 K 2^-18 (just below 2^6) and must stay exact."""
+    M, N, K = 16, 32, 65536
+    pairs = ((7, 7), (-8, -8), (7, -8)) if symmetric else ((15, 7), (0, -8), (15, -8))
+    for aval, wval in pairs:
+        ac = np.full((M, K), aval, dtype=np.int32)
+        wc = np.full((N, K), wval, dtype=np.int32)
+        al, ws_ = np.full(M, 0.5), np.full(N, 0.25)
+        be = None if symmetric else np.full(M, -1.0)
+        y, acc = _with_kernel(S, S.SPINQ_GEMM_TCGEMV, lambda: run_splitk(S, ac, al, be, wc, ws_))
+        assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc), (aval, wval)
+
+
+def test_auto_plan_takes_tcgemv_for_five_to_eight_tokens(S):
+    for M, want in ((4, S.SPINQ_GEMM_GEMV), (5, S.SPINQ_GEMM_TCGEMV), (8, S.SPINQ_GEMM_TCGEMV)):
+        assert S.spinq_w4a4_gemm_plan(M, 8192, 3072) == want
+        assert S.spinq_w4a4_gemm_splitk_plan(M, 8192, 3072) == (want, 0)
+    assert S.spinq_w4a4_gemm_splitk_plan(9, 8192, 3072)[0] == S.SPINQ_GEMM_SPLITK
+    # a forced split-K selection keeps the split-K kernel
+    prev = S.spinq_gemm_select_kernel(S.SPINQ_GEMM_SPLITK)
+    try:
+        assert S.spinq_w4a4_gemm_splitk_plan(6, 8192, 3072)[0] == S.SPINQ_GEMM_SPLITK
+    finally:
+        S.spinq_gemm_select_kernel(prev)
+
+
+def test_tcgemv_plan_falls_back_beyond_its_range(S):
+    def go():
+        assert S.spinq_w4a4_gemm_plan(17, 4096, 4096) != S.SPINQ_GEMM_TCGEMV
+        assert S.spinq_w4a4_gemm_splitk_plan(17, 4096, 4096)[0] != S.SPINQ_GEMM_TCGEMV
+        assert S.spinq_w4a4_gemm_plan(16, 4096, 4096) == S.SPINQ_GEMM_TCGEMV
+    _with_kernel(S, S.SPINQ_GEMM_TCGEMV, go)
 
 
 def test_splitk_workspace_reused_and_left_zero(S):
