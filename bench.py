@@ -1057,7 +1057,8 @@ def relaunch(args_n):
     return subprocess.call(cmd)
 
 
-PROFILE_CASES = ("attention", "rope_kv", "fp8_gemm", "w4a8_gemm", "rq8_paley", "cayley", "paley", "gemm")
+PROFILE_CASES = ("attention", "rope_kv", "fp8_gemm", "w4a8_gemm", "rq8_paley", "cayley", "paley", "gemm",
+                 "decode_gemm")
 
 
 def profile_case(name, reps):
@@ -1069,7 +1070,8 @@ def profile_case(name, reps):
     14336 with E4M3 codes / 4-bit weights and 8-bit activation planes;
     rq8_paley: the 8-bit quantizer with H28 x H512 on 2048 x 14336; cayley:
     152 rotations of 128 x 128, 2 iterations; paley: the 4-bit R4 kernel on
-    2048 x 14336; gemm: the W4A4 down_proj 2048 x 14336 -> 4096."""
+    2048 x 14336; gemm: the W4A4 down_proj 2048 x 14336 -> 4096;
+    decode_gemm: 8 tokens through 4096 -> 14336 on the automatic route."""
     import numpy as np
     import torch
 
@@ -1111,6 +1113,11 @@ def profile_case(name, reps):
             qa = spinq.rotate_quant_act(x, c.had)
             qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), c.had)
             fn = lambda: spinq.w4a4_gemm(qa, qw)
+    elif name == "decode_gemm":
+        c = synth.llama3_8b_gate_up(M=8)
+        qa = spinq.rotate_quant_act(torch.from_numpy(c.x).to(dev), None, False)
+        qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), None)
+        fn = lambda: spinq.w4a4_gemm_splitk(qa, qw)
     elif name == "cayley":
         rng = np.random.default_rng(0)
         R = np.stack([np.linalg.qr(rng.standard_normal((128, 128)))[0] for _ in range(152)]).astype(np.float32)
