@@ -231,6 +231,10 @@ cudaError_t launch_fmt(const Rq8Args& a, cudaStream_t stream) {
 
 cudaError_t launch_rotate_quant_8bit(const Rq8Args& a, cudaStream_t stream) {
   if (a.rows == 0) return cudaSuccess;
+  // a Paley rotation with the unclipped activation formats: the Paley kernel
+  bool handled = false;
+  const cudaError_t ep = launch_rotate_quant_8bit_paley(a, stream, &handled);
+  if (ep != cudaSuccess || handled) return ep;
   switch (a.format) {
     case kFmtInt8Planes: return launch_fmt<kFmtInt8Planes>(a, stream);
     case kFmtE4M3: return a.symmetric ? launch_fmt<kFmtE4M3>(a, stream) : cudaErrorInvalidValue;

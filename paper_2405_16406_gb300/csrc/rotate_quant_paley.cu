@@ -130,7 +130,72 @@ __device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
-template <int NS, int LP, bool SYM, bool CLAMP, bool SG>
+__device__ __forceinline__ uint32_t e4m3x2_bits(float lo, float hi) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// The 8-bit quantizers of rotate_quant_8bit.cu (unclipped forms) on a row
+// range: E4M3 codes x / alpha with alpha = max|x| / 448; int8 codes
+// c = rint(x / alpha) (symmetric, alpha = max|x| / 127) or rint((x - beta) /
+// alpha) - 128 (asymmetric, alpha = (max - min) / 255), stored as the planes
+// E4M3(16 floor(c / 16)) and E4M3(c mod 16).  rint is the 1.5 2^23 rounding
+// (to nearest even, as the other kernel's conversion), floor(c / 16) is
+// rint((c - 7.5) / 16), exact for integer c; every value is exact in E4M3.
+template <bool SYM>
+struct Quant8 {
+  float inv, off, alpha, beta;
+  __device__ __forceinline__ Quant8(const Range<SYM>& r, float clip, bool e4m3) {
+    off = 0.f;
+    beta = 0.f;
+    if (e4m3) {
+      const float m = clip * r.hi;
+      alpha = m * (1.f / 448.f);
+      inv = m > 0.f ? 448.f / m : 0.f;
+    } else if (SYM) {
+      const float m = clip * r.hi;
+      alpha = m / 127.f;
+      inv = m > 0.f ? 127.f / m : 0.f;
+    } else {
+      const float h2 = clip * r.hi, l2 = clip * r.lo;
+      alpha = (h2 - l2) / 255.f;
+      inv = h2 > l2 ? 255.f / (h2 - l2) : 0.f;
+      beta = l2;
+      off = -l2 * inv;
+    }
+  }
+  // the codes of 8 consecutive elements (4 pairs): E4M3 bytes in `hi`, or the
+  // two planes in `hi` (16 floor(c / 16)) and `lo` (c mod 16)
+  template <int F8>
+  __device__ __forceinline__ void codes8(const F2 (&v)[4], uint2& hi, uint2& lo) const {
+    uint32_t hb[4], lb[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float x0, x1;
+      f2_split(v[q], x0, x1);
+      if (F8 == kFmtE4M3) {
+        hb[q] = e4m3x2_bits(fmaf(x0, inv, off), fmaf(x1, inv, off));
+        lb[q] = 0;
+      } else {
+        float c0 = (fmaf(x0, inv, off) + kRoundMagic) - kRoundMagic;
+        float c1 = (fmaf(x1, inv, off) + kRoundMagic) - kRoundMagic;
+        if (!SYM) c0 -= 128.f, c1 -= 128.f;
+        const float q0 = (fmaf(c0, 0.0625f, -0.46875f) + kRoundMagic) - kRoundMagic;
+        const float q1 = (fmaf(c1, 0.0625f, -0.46875f) + kRoundMagic) - kRoundMagic;
+        hb[q] = e4m3x2_bits(16.f * q0, 16.f * q1);
+        lb[q] = e4m3x2_bits(fmaf(-16.f, q0, c0), fmaf(-16.f, q1, c1));
+      }
+    }
+    hi = make_uint2(hb[0] | (hb[1] << 16), hb[2] | (hb[3] << 16));
+    lo = make_uint2(lb[0] | (lb[1] << 16), lb[2] | (lb[3] << 16));
+  }
+};
+
+// F8 = 0: 4-bit codes (Eq. 1, N = 4); F8 = kFmtInt8Planes / kFmtE4M3: the
+// 8-bit quantizers of the 8-bit linears (codes laid out as in
+// rotate_quant_8bit.cu), on the same rotation.
+template <int NS, int LP, bool SYM, bool CLAMP, bool SG, int F8 = 0>
 __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
     rq_paley_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
   using S = PaleyShape<NS, LP>;
@@ -414,31 +479,55 @@ __global__ void __launch_bounds__(PaleyShape<NS, LP>::THREADS, 1)
       rg.hi = fmaxf(rg.hi, rd[i]);
       if (!SYM) rg.lo = fminf(rg.lo, rd[W + i]);
     }
-    const QParams<SYM> qp(rg, a.clip);
-    uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
+    if constexpr (F8 == 0) {
+      const QParams<SYM> qp(rg, a.clip);
+      uint32_t* out = reinterpret_cast<uint32_t*>(a.codes + row * (a.K / 2));
 #pragma unroll
-    for (int k = 0; k < S::NCB; ++k) {
-      const int cb = t2 + T * k;
-      if (cb >= S::NCOMBO || combo_warp_idle(cb, NS)) continue;
-      // word 8 wv + jg of segment i2 holds the codes of j = 64 wv + 8 jg .. + 7;
-      // a quarter warp writes 32 contiguous bytes per wv
-      uint32_t* seg = out + combo_i(cb) * (P / 8) + (cb & 7);
+      for (int k = 0; k < S::NCB; ++k) {
+        const int cb = t2 + T * k;
+        if (cb >= S::NCOMBO || combo_warp_idle(cb, NS)) continue;
+        // word 8 wv + jg of segment i2 holds the codes of j = 64 wv + 8 jg .. + 7;
+        // a quarter warp writes 32 contiguous bytes per wv
+        uint32_t* seg = out + combo_i(cb) * (P / 8) + (cb & 7);
 #pragma unroll
-      for (int wv = 0; wv < W; ++wv) {
-        uint32_t rb[8];
+        for (int wv = 0; wv < W; ++wv) {
+          uint32_t rb[8];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) qp.template code_bits2<CLAMP>(z[k][wv][q], rb[2 * q], rb[2 * q + 1]);
-        seg[8 * wv] = pack8_nibbles(rb);
+          for (int q = 0; q < 4; ++q) qp.template code_bits2<CLAMP>(z[k][wv][q], rb[2 * q], rb[2 * q + 1]);
+          seg[8 * wv] = pack8_nibbles(rb);
+        }
       }
-    }
-    if (t2 == 0) {
-      a.scale[row] = qp.alpha * a.norm;
-      if (!SYM) a.zero[row] = qp.beta * a.norm;
+      if (t2 == 0) {
+        a.scale[row] = qp.alpha * a.norm;
+        if (!SYM) a.zero[row] = qp.beta * a.norm;
+      }
+    } else {
+      static_assert(!CLAMP, "the 8-bit quantizers run here unclipped");
+      const Quant8 q8(rg, a.clip, F8 == kFmtE4M3);
+      uint8_t* out = a.codes + row * (F8 == kFmtInt8Planes ? 2 * a.K : a.K);
+#pragma unroll
+      for (int k = 0; k < S::NCB; ++k) {
+        const int cb = t2 + T * k;
+        if (cb >= S::NCOMBO || combo_warp_idle(cb, NS)) continue;
+        // the 8 bytes of j = 64 wv + 8 jg .. + 7 of segment i2
+        uint8_t* seg = out + combo_i(cb) * P + 8 * (cb & 7);
+#pragma unroll
+        for (int wv = 0; wv < W; ++wv) {
+          uint2 hi, lo;
+          q8.template codes8<F8>(z[k][wv], hi, lo);
+          *reinterpret_cast<uint2*>(seg + 64 * wv) = hi;
+          if (F8 == kFmtInt8Planes) *reinterpret_cast<uint2*>(seg + a.K + 64 * wv) = lo;
+        }
+      }
+      if (t2 == 0) {
+        a.scale[row] = q8.alpha * a.norm;
+        if (!SYM && F8 == kFmtInt8Planes) a.zero[row] = q8.beta * a.norm;
+      }
     }
   }
 }
 
-template <int NS, int LP, bool SYM, bool CLAMP, bool SG>
+template <int NS, int LP, bool SYM, bool CLAMP, bool SG, int F8 = 0>
 cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
   using S = PaleyShape<NS, LP>;
   // rows as (j_lo, i, j_hi, row): one copy lands a row as 128-byte swizzled lines i + NS j_hi
@@ -453,7 +542,7 @@ cudaError_t launch_paley(const RotQuantArgs& a, cudaStream_t stream) {
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorNotSupported;
-  auto kern = rq_paley_kernel<NS, LP, SYM, CLAMP, SG>;
+  auto kern = rq_paley_kernel<NS, LP, SYM, CLAMP, SG, F8>;
   int per_sm = 0;
   cudaError_t e = prepare_launch(kern, S::THREADS, S::BYTES, &per_sm);
   if (e != cudaSuccess) return e;
@@ -517,7 +606,61 @@ cudaError_t launch_sc(const RotQuantArgs& a, cudaStream_t stream, bool* handled)
   return cudaSuccess;
 }
 
+// The 8-bit quantizers on a Paley rotation (unclipped forms, no random signs).
+template <int F8, bool SYM>
+cudaError_t launch8_sc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = true;
+  if (a.n_small == 12 && a.n_pow2 == 256) {
+    RotQuantArgs b = a;
+    b.hs = kron_h2(a.hs);
+    b.n_small = 24;
+    b.n_pow2 = 128;
+    return launch_paley<24, 7, SYM, false, false, F8>(b, stream);
+  }
+#define SPINQ_P8(NS_)                                                      \
+  switch (a.n_pow2) {                                                      \
+    case 128: return launch_paley<NS_, 7, SYM, false, false, F8>(a, stream); \
+    case 256: return launch_paley<NS_, 8, SYM, false, false, F8>(a, stream); \
+    case 512: return launch_paley<NS_, 9, SYM, false, false, F8>(a, stream); \
+  }                                                                        \
+  break;
+  switch (a.n_small) {
+    case 12: SPINQ_P8(12)
+    case 20: SPINQ_P8(20)
+    case 28: SPINQ_P8(28)
+  }
+#undef SPINQ_P8
+  *handled = false;
+  return cudaSuccess;
+}
+
 }  // namespace
+
+cudaError_t launch_rotate_quant_8bit_paley(const Rq8Args& a, cudaStream_t stream, bool* handled) {
+  *handled = false;
+  if (a.rows == 0 || a.n_small <= 1 || a.clip < 1.0f) return cudaSuccess;
+  if (a.format != kFmtE4M3 && a.format != kFmtInt8Planes) return cudaSuccess;
+  if (a.format == kFmtE4M3 && !a.symmetric) return cudaSuccess;
+  if ((a.ldx * 2) % 16 != 0) return cudaSuccess;
+  RotQuantArgs b{};
+  b.x = a.x;
+  b.rows = a.rows;
+  b.K = a.K;
+  b.ldx = a.ldx;
+  b.n_small = a.n_small;
+  b.n_pow2 = a.n_pow2;
+  b.hs = a.hs;
+  b.symmetric = a.symmetric;
+  b.clip = a.clip;
+  b.norm = a.norm;
+  b.codes = a.codes;
+  b.scale = a.scale;
+  b.zero = a.zero;
+  b.status = device_status_word();
+  if (a.format == kFmtE4M3) return launch8_sc<kFmtE4M3, true>(b, stream, handled);
+  return a.symmetric ? launch8_sc<kFmtInt8Planes, true>(b, stream, handled)
+                     : launch8_sc<kFmtInt8Planes, false>(b, stream, handled);
+}
 
 cudaError_t set_wait_limit_paley(uint64_t ns) { return cudaMemcpyToSymbol(g_wait_ns, &ns, sizeof(ns)); }
 

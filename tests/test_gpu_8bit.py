@@ -43,6 +43,8 @@ ACT_CASES = [
     ("h28x512", (28, 512), 14336),
     ("h8192", (1, 8192), 8192),
     ("h12x256", (12, 256), 3072),
+    ("h20x256", (20, 256), 5120),
+    ("h28x128", (28, 128), 3584),
     ("h256", (1, 256), 256),
 ]
 
