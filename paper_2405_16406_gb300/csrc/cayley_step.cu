@@ -22,9 +22,10 @@
 //   D_{k+1} = M + (a/2) Y D_k        ping-pong between buf0 and buf2
 //   R_out = R + D_iters              (R re-read from global memory)
 //
-// Thread (rg, cg) owns rows i0 = TR rg .. and columns j0 = 8 cg .. of every
-// product; the products run on packed fp32 pairs (fma.rn.f32x2), the column
-// pairs of a row in one register pair.
+// Thread (rg, cg) owns rows i0 = TR rg .. and columns 4 cg .. 4 cg + 3 and
+// N/2 + 4 cg .. + 3 of every product (so that the 16-byte operand loads of a
+// quarter warp are contiguous); the products run on packed fp32 pairs
+// (fma.rn.f32x2), the column pairs of a row in one register pair.
 #include <cuda_runtime.h>
 
 #include "launch_util.h"
@@ -49,10 +50,10 @@ struct CayleyShape {
 template <int N>
 using Acc = F2[CayleyShape<N>::TR][4];
 
-// acc[r][c] += sum_k X(i0 + r, k) * B[k][j0 + 2c .. j0 + 2c + 1], with
+// acc[r][c] += sum_k X(i0 + r, k) * B[k][col 2c, 2c + 1 of the thread], with
 // X(i, k) = X[i][k], or X[k][i] when XT.
 template <int N, bool XT>
-__device__ __forceinline__ void mm_acc(const float* X, const float* B, int i0, int j0, Acc<N>& acc) {
+__device__ __forceinline__ void mm_acc(const float* X, const float* B, int i0, int ja, int jb, Acc<N>& acc) {
   using S = CayleyShape<N>;
 #pragma unroll 2
   for (int k = 0; k < N; ++k) {
@@ -71,8 +72,8 @@ __device__ __forceinline__ void mm_acc(const float* X, const float* B, int i0, i
 #pragma unroll
       for (int r = 0; r < S::TR; ++r) xv[r] = X[(i0 + r) * S::S + k];
     }
-    const float4 b0 = *reinterpret_cast<const float4*>(B + k * S::S + j0);
-    const float4 b1 = *reinterpret_cast<const float4*>(B + k * S::S + j0 + 4);
+    const float4 b0 = *reinterpret_cast<const float4*>(B + k * S::S + ja);
+    const float4 b1 = *reinterpret_cast<const float4*>(B + k * S::S + jb);
     const F2 bp[4] = {f2_make(b0.x, b0.y), f2_make(b0.z, b0.w), f2_make(b1.x, b1.y), f2_make(b1.z, b1.w)};
 #pragma unroll
     for (int r = 0; r < S::TR; ++r) {
@@ -92,15 +93,15 @@ __device__ __forceinline__ void acc_zero(Acc<N>& acc) {
 }
 
 template <int N>
-__device__ __forceinline__ void tile_store(float* dst, int i0, int j0, const Acc<N>& acc) {
+__device__ __forceinline__ void tile_store(float* dst, int i0, int ja, int jb, const Acc<N>& acc) {
   using S = CayleyShape<N>;
 #pragma unroll
   for (int r = 0; r < S::TR; ++r) {
     float v[8];
 #pragma unroll
     for (int c = 0; c < 4; ++c) f2_split(acc[r][c], v[2 * c], v[2 * c + 1]);
-    *reinterpret_cast<float4*>(dst + (i0 + r) * S::S + j0) = make_float4(v[0], v[1], v[2], v[3]);
-    *reinterpret_cast<float4*>(dst + (i0 + r) * S::S + j0 + 4) = make_float4(v[4], v[5], v[6], v[7]);
+    *reinterpret_cast<float4*>(dst + (i0 + r) * S::S + ja) = make_float4(v[0], v[1], v[2], v[3]);
+    *reinterpret_cast<float4*>(dst + (i0 + r) * S::S + jb) = make_float4(v[4], v[5], v[6], v[7]);
   }
 }
 
@@ -115,7 +116,9 @@ __global__ void __launch_bounds__(CayleyShape<N>::THREADS, 1)
   float* buf2 = sm + 2 * S::BUF;
   const int tid = threadIdx.x;
   const int cg = tid % S::CG, rg = tid / S::CG;
-  const int i0 = rg * S::TR, j0 = cg * 8;
+  // columns 4 cg .. + 3 and N/2 + 4 cg .. + 3: the 16-byte operand loads of
+  // a quarter warp (cg = 0..7, one rg) cover 128 contiguous bytes
+  const int i0 = rg * S::TR, ja = 4 * cg, jb = N / 2 + 4 * cg;
   const size_t base = (size_t)blockIdx.x * N * N;
   pdl_wait();
   pdl_trigger();
@@ -123,43 +126,43 @@ __global__ void __launch_bounds__(CayleyShape<N>::THREADS, 1)
   // buf0 = R^T, buf1 = G = -grad
 #pragma unroll
   for (int r = 0; r < S::TR; ++r) {
-    const float4 a0 = *reinterpret_cast<const float4*>(R + base + (size_t)(i0 + r) * N + j0);
-    const float4 a1 = *reinterpret_cast<const float4*>(R + base + (size_t)(i0 + r) * N + j0 + 4);
+    const float4 a0 = *reinterpret_cast<const float4*>(R + base + (size_t)(i0 + r) * N + ja);
+    const float4 a1 = *reinterpret_cast<const float4*>(R + base + (size_t)(i0 + r) * N + jb);
     const float v[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
 #pragma unroll
-    for (int c = 0; c < 8; ++c) buf0[(j0 + c) * S::S + i0 + r] = v[c];
-    const float4 g0 = *reinterpret_cast<const float4*>(grad + base + (size_t)(i0 + r) * N + j0);
-    const float4 g1 = *reinterpret_cast<const float4*>(grad + base + (size_t)(i0 + r) * N + j0 + 4);
-    *reinterpret_cast<float4*>(buf1 + (i0 + r) * S::S + j0) = make_float4(-g0.x, -g0.y, -g0.z, -g0.w);
-    *reinterpret_cast<float4*>(buf1 + (i0 + r) * S::S + j0 + 4) = make_float4(-g1.x, -g1.y, -g1.z, -g1.w);
+    for (int c = 0; c < 8; ++c) buf0[(c < 4 ? ja + c : jb + c - 4) * S::S + i0 + r] = v[c];
+    const float4 g0 = *reinterpret_cast<const float4*>(grad + base + (size_t)(i0 + r) * N + ja);
+    const float4 g1 = *reinterpret_cast<const float4*>(grad + base + (size_t)(i0 + r) * N + jb);
+    *reinterpret_cast<float4*>(buf1 + (i0 + r) * S::S + ja) = make_float4(-g0.x, -g0.y, -g0.z, -g0.w);
+    *reinterpret_cast<float4*>(buf1 + (i0 + r) * S::S + jb) = make_float4(-g1.x, -g1.y, -g1.z, -g1.w);
   }
   __syncthreads();
 
   Acc<N> acc;
   // A = G R^T -> buf2
   acc_zero<N>(acc);
-  mm_acc<N, false>(buf1, buf0, i0, j0, acc);
-  tile_store<N>(buf2, i0, j0, acc);
+  mm_acc<N, false>(buf1, buf0, i0, ja, jb, acc);
+  tile_store<N>(buf2, i0, ja, jb, acc);
   __syncthreads();
   // C = R^T A -> buf1
   acc_zero<N>(acc);
-  mm_acc<N, false>(buf0, buf2, i0, j0, acc);
-  tile_store<N>(buf1, i0, j0, acc);
+  mm_acc<N, false>(buf0, buf2, i0, ja, jb, acc);
+  tile_store<N>(buf1, i0, ja, jb, acc);
   __syncthreads();
   // G_hat = A - 1/2 R C -> buf2
   acc_zero<N>(acc);
-  mm_acc<N, true>(buf0, buf1, i0, j0, acc);
+  mm_acc<N, true>(buf0, buf1, i0, ja, jb, acc);
   const F2 mhalf = f2_make(-0.5f, -0.5f);
 #pragma unroll
   for (int r = 0; r < S::TR; ++r) {
-    const float* at = buf2 + (i0 + r) * S::S + j0;   // this thread's own tile of A
-    const float4 t0 = *reinterpret_cast<const float4*>(at);
-    const float4 t1 = *reinterpret_cast<const float4*>(at + 4);
+    const float* at = buf2 + (i0 + r) * S::S;   // this thread's own tile of A
+    const float4 t0 = *reinterpret_cast<const float4*>(at + ja);
+    const float4 t1 = *reinterpret_cast<const float4*>(at + jb);
     const F2 av[4] = {f2_make(t0.x, t0.y), f2_make(t0.z, t0.w), f2_make(t1.x, t1.y), f2_make(t1.z, t1.w)};
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[r][c] = f2_fma(acc[r][c], mhalf, av[c]);
   }
-  tile_store<N>(buf2, i0, j0, acc);
+  tile_store<N>(buf2, i0, ja, jb, acc);
   __syncthreads();
   // Y = G_hat - G_hat^T -> buf1 (and Y_out); buf0 transposed in place to R
 #pragma unroll
@@ -168,7 +171,7 @@ __global__ void __launch_bounds__(CayleyShape<N>::THREADS, 1)
     float y[8];
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
-      const int j = j0 + c;
+      const int j = c < 4 ? ja + c : jb + c - 4;
       y[c] = buf2[i * S::S + j] - buf2[j * S::S + i];
       buf1[i * S::S + j] = y[c];
       if (i < j) {
@@ -178,33 +181,33 @@ __global__ void __launch_bounds__(CayleyShape<N>::THREADS, 1)
       }
     }
     if (Y_out) {
-      *reinterpret_cast<float4*>(Y_out + base + (size_t)i * N + j0) = make_float4(y[0], y[1], y[2], y[3]);
-      *reinterpret_cast<float4*>(Y_out + base + (size_t)i * N + j0 + 4) = make_float4(y[4], y[5], y[6], y[7]);
+      *reinterpret_cast<float4*>(Y_out + base + (size_t)i * N + ja) = make_float4(y[0], y[1], y[2], y[3]);
+      *reinterpret_cast<float4*>(Y_out + base + (size_t)i * N + jb) = make_float4(y[4], y[5], y[6], y[7]);
     }
   }
   __syncthreads();
   // M = a Y R (registers), D_0 = M -> buf2
   Acc<N> m;
   acc_zero<N>(acc);
-  mm_acc<N, false>(buf1, buf0, i0, j0, acc);
+  mm_acc<N, false>(buf1, buf0, i0, ja, jb, acc);
   const F2 a2 = f2_make(alpha, alpha), h2 = f2_make(0.5f * alpha, 0.5f * alpha), zero2 = f2_make(0.f, 0.f);
 #pragma unroll
   for (int r = 0; r < S::TR; ++r)
 #pragma unroll
     for (int c = 0; c < 4; ++c) m[r][c] = f2_fma(acc[r][c], a2, zero2);
-  if (iters > 0) tile_store<N>(buf2, i0, j0, m);
+  if (iters > 0) tile_store<N>(buf2, i0, ja, jb, m);
   // D_{k+1} = M + (a/2) Y D_k, left in acc (D_0 = M when iters = 0)
   float* cur = buf2;
   float* nxt = buf0;
   for (int k = 0; k < iters; ++k) {
     __syncthreads();
     acc_zero<N>(acc);
-    mm_acc<N, false>(buf1, cur, i0, j0, acc);
+    mm_acc<N, false>(buf1, cur, i0, ja, jb, acc);
 #pragma unroll
     for (int r = 0; r < S::TR; ++r)
 #pragma unroll
       for (int c = 0; c < 4; ++c) acc[r][c] = f2_fma(acc[r][c], h2, m[r][c]);
-    if (k + 1 < iters) tile_store<N>(nxt, i0, j0, acc);
+    if (k + 1 < iters) tile_store<N>(nxt, i0, ja, jb, acc);
     float* t = cur;
     cur = nxt;
     nxt = t;
@@ -218,14 +221,14 @@ __global__ void __launch_bounds__(CayleyShape<N>::THREADS, 1)
   // R' = R + D
 #pragma unroll
   for (int r = 0; r < S::TR; ++r) {
-    const size_t off = base + (size_t)(i0 + r) * N + j0;
-    const float4 a0 = *reinterpret_cast<const float4*>(R + off);
-    const float4 a1 = *reinterpret_cast<const float4*>(R + off + 4);
+    const size_t off = base + (size_t)(i0 + r) * N;
+    const float4 a0 = *reinterpret_cast<const float4*>(R + off + ja);
+    const float4 a1 = *reinterpret_cast<const float4*>(R + off + jb);
     float v[8];
 #pragma unroll
     for (int c = 0; c < 4; ++c) f2_split(acc[r][c], v[2 * c], v[2 * c + 1]);
-    *reinterpret_cast<float4*>(R_out + off) = make_float4(a0.x + v[0], a0.y + v[1], a0.z + v[2], a0.w + v[3]);
-    *reinterpret_cast<float4*>(R_out + off + 4) = make_float4(a1.x + v[4], a1.y + v[5], a1.z + v[6], a1.w + v[7]);
+    *reinterpret_cast<float4*>(R_out + off + ja) = make_float4(a0.x + v[0], a0.y + v[1], a0.z + v[2], a0.w + v[3]);
+    *reinterpret_cast<float4*>(R_out + off + jb) = make_float4(a1.x + v[4], a1.y + v[5], a1.z + v[6], a1.w + v[7]);
   }
 }
 
