@@ -524,6 +524,9 @@ def run_ours(args, rank, world, local_rank):
             "achieved": round(gemm_tops, 1), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
             "frac": round(gemm_tops / fp8_peak, 4),
             "traffic": gemm_traffic_from_profile(f"w4a4_gemm_gate_up_M{M}_K{K}_N{N}.md", GEMM_KERNELS[kind1][1]),
+            "traffic_note": "dram__bytes_read.sum + dram__bytes_write.sum per launch from the committed ncu "
+                            "summary in profiles/ (not measured in this run); null when the kernel source "
+                            "hash differs from the one the counters were taken with",
             "peak_note": f"e4m3 dense = 2 x {peak_kind} bf16 ({bf16_peak} TFLOP/s); "
                          "int4 codes carried as e4m3 on tcgen05 kind::f8f6f4",
         },
@@ -1058,7 +1061,7 @@ def relaunch(args_n):
 
 
 PROFILE_CASES = ("attention", "rope_kv", "fp8_gemm", "w4a8_gemm", "rq8_paley", "cayley", "paley", "gemm",
-                 "decode_gemm")
+                 "gemm_gate_up", "decode_gemm")
 
 
 def profile_case(name, reps):
@@ -1070,7 +1073,8 @@ def profile_case(name, reps):
     14336 with E4M3 codes / 4-bit weights and 8-bit activation planes;
     rq8_paley: the 8-bit quantizer with H28 x H512 on 2048 x 14336; cayley:
     152 rotations of 128 x 128, 2 iterations; paley: the 4-bit R4 kernel on
-    2048 x 14336; gemm: the W4A4 down_proj 2048 x 14336 -> 4096;
+    2048 x 14336; gemm: the W4A4 down_proj 2048 x 14336 -> 4096; gemm_gate_up:
+    the W4A4 gate_up 2048 x 4096 -> 14336 (asymmetric activations);
     decode_gemm: 8 tokens through 4096 -> 14336 on the automatic route."""
     import numpy as np
     import torch
@@ -1113,6 +1117,11 @@ def profile_case(name, reps):
             qa = spinq.rotate_quant_act(x, c.had)
             qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), c.had)
             fn = lambda: spinq.w4a4_gemm(qa, qw)
+    elif name == "gemm_gate_up":
+        c = synth.llama3_8b_gate_up()
+        qa = spinq.rotate_quant_act(torch.from_numpy(c.x).to(dev), None, False)
+        qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), None)
+        fn = lambda: spinq.w4a4_gemm(qa, qw)
     elif name == "decode_gemm":
         c = synth.llama3_8b_gate_up(M=8)
         qa = spinq.rotate_quant_act(torch.from_numpy(c.x).to(dev), None, False)

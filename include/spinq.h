@@ -276,19 +276,23 @@ spinq_status spinq_rotate_quant_kv(const void* q_in, void* q_out, const void* k_
  *   SPINQ_GEMM_TILE256  one CTA per 256 x 256 output tile;
  *   SPINQ_GEMM_PAIR     two CTAs (an SM pair) per 256 x 256 tile; calls it
  *                       cannot serve (M <= 128, no pair resident) use AUTO;
- *   SPINQ_GEMM_GEMV     (M <= 4 with M * K <= 160 KiB; AUTO picks it there,
- *                       on the _splitk / _noalloc entry points too) each warp
+ *   SPINQ_GEMM_GEMV     (M <= 4 with M * K <= 160 KiB; AUTO picks it there
+ *                       unless SPINQ_GEMM_TCGEMV takes the tokens, on the
+ *                       _splitk / _noalloc entry points too) each warp
  *                       owns whole output channels and streams their packed
  *                       weights; calls it cannot serve use AUTO;
  *   SPINQ_GEMM_SPLITK   the split-K kernel on the _splitk / _noalloc entry
  *                       points for every M <= 256 (GEMV and prefill kernels
  *                       excluded); spinq_w4a4_gemm treats it as AUTO;
- *   SPINQ_GEMM_TCGEMV   (M <= 16, on every entry point; AUTO picks it for 5 to
- *                       8 tokens) a CTA per 16 output channels streams their
- *                       packed weights through shared memory and takes the
- *                       products on the tensor core (fp16 m16n8k16 on the
- *                       exact codes), no workspace; calls it cannot serve use
- *                       AUTO.
+ *   SPINQ_GEMM_TCGEMV   (M <= 16, on every entry point; AUTO picks it for 3 to
+ *                       16 tokens when K / 128 = NKW W with NKW in {1, 2, 4,
+ *                       8} and W <= 16, else for 5 to 8 tokens) the products
+ *                       on the tensor core (fp16 m16n8k16 on the exact codes),
+ *                       no workspace: for such K, one CTA per SM whose W
+ *                       warps split K and stream the packed weights straight
+ *                       into registers; else a CTA per 16 output channels
+ *                       that stages them through shared memory; calls it
+ *                       cannot serve use AUTO.
  * All kernels compute bit-identical outputs; this is a tuning and testing
  * control.  Returns the previous selection, or -1 (and changes nothing) for
  * an unknown value.  Not synchronized with GEMM calls in other threads.

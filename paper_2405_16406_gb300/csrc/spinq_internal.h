@@ -132,15 +132,20 @@ inline bool w4a4_gemv_fits(int64_t M, int64_t K) {
 }
 cudaError_t launch_w4a4_gemv(const GemmArgs& a, cudaStream_t stream, bool* handled);
 
-// Tensor-core GEMV for M <= kGemvTcMaxM tokens: a CTA per 16 output
-// channels over the whole K, weights streamed into registers, m16n8k32 e4m3
-// MMAs, no workspace.  Sets *handled = false when the shape is out of range.
+// Tensor-core GEMV for M <= kGemvTcMaxM tokens: fp16 m16n8k16 MMAs on the
+// exact codes, no workspace.  Where w4a4_gemv_tc_streamed(K) holds, warps
+// split K and stream the weights straight into registers (one CTA per SM);
+// else each CTA owns 16 channels and stages them through shared memory.
+// Sets *handled = false when the shape is out of range.
 constexpr int64_t kGemvTcMaxM = 16;
 inline bool w4a4_gemv_tc_fits(int64_t M, int64_t N, int64_t K) {
   return M >= 1 && M <= kGemvTcMaxM && N >= 16 && N % 16 == 0 && K >= 128 && K % 128 == 0 && K <= 65536 &&
          N / 16 <= 0x7FFFFFFF;
 }
 cudaError_t launch_w4a4_gemv_tc(const GemmArgs& a, cudaStream_t stream, bool* handled);
+// True when the register-streamed form takes K (K / 128 = NKW W with NKW in
+// {1, 2, 4, 8} and W <= 16 warps).
+bool w4a4_gemv_tc_streamed(int64_t K);
 
 // Decode GEMM for M <= kDecodeMaxM (launch_w4a4_gemm above): the GEMV kernel,
 // the split-K kernel or the prefill kernels, as a fitted cost model predicts

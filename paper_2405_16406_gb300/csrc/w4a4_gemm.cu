@@ -1201,16 +1201,24 @@ PrefillChoice choose_prefill(int64_t M, int64_t N, int64_t K, bool allow_pair) {
 }
 
 // The tensor-core GEMV serves every entry point for the shapes it fits when
-// it is selected, and 5 to 8 tokens under the automatic choice: measured on
-// GB300 over K x N in {3072 x 8192, 8192 x 3072, 4096 x 14336, 14336 x 4096},
-// it takes 5.8 / 6.5 / 14.2 / 10.2 us at 8 tokens against 9.1 / 9.0 / 14.2 /
-// 13.3 us for the split-K kernel; from 1 to 4 tokens the GEMV kernel is
-// faster, from 9 on the split-K kernel.
-constexpr int64_t kGemvTcAutoLo = 5, kGemvTcAutoHi = 8;
+// it is selected.  Under the automatic choice it takes 3 to 16 tokens where
+// its register-streamed form covers K, else 5 to 8 tokens.  Measured on GB300
+// over K x N in {3072 x 8192, 8192 x 3072, 4096 x 14336, 14336 x 4096}
+// (graphs of 40 calls over 8 weight sets), register-streamed form against
+// the GEMV kernel / the split-K kernel:
+//   3 tokens:  ~5.2 / 5.5 / 9.7 / 8.8 us against 5.8 / 6.6 / 9.1 / 10.9 (GEMV)
+//   8 tokens:  5.4 / 6.1 / 9.9 / 9.2 us against 9.1 / 9.0 / 14.2 / 13.3 (split-K)
+//   16 tokens: 7.9 / 8.2 / 13.9 / 12.8 us against 9.8 / 9.7 / 14.8 / 14.1 (split-K)
+// and 1 or 2 tokens stay on the GEMV kernel (3.6 / 3.6 / 5.6 / 7.9 us at 1).
+constexpr int64_t kGemvTcAutoLo = 5, kGemvTcAutoHi = 8;          // the shared-memory stage form
+constexpr int64_t kGemvTcStreamLo = 3, kGemvTcStreamHi = 16;     // the register-streamed form
 bool tcgemv_serves(int64_t M, int64_t N, int64_t K) {
   const int forced = g_gemm_kernel.load(std::memory_order_relaxed);
   if (!w4a4_gemv_tc_fits(M, N, K)) return false;
-  return forced == SPINQ_GEMM_TCGEMV || (forced == SPINQ_GEMM_AUTO && M >= kGemvTcAutoLo && M <= kGemvTcAutoHi);
+  if (forced == SPINQ_GEMM_TCGEMV) return true;
+  if (forced != SPINQ_GEMM_AUTO) return false;
+  if (w4a4_gemv_tc_streamed(K)) return M >= kGemvTcStreamLo && M <= kGemvTcStreamHi;
+  return M >= kGemvTcAutoLo && M <= kGemvTcAutoHi;
 }
 
 }  // namespace

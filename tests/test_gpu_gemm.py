@@ -142,8 +142,8 @@ def test_gemm_plan_follows_selection(S):
             S.spinq_gemm_select_kernel(prev)
     assert S.spinq_w4a4_gemm_plan(128, 14336, 4096) in (1, 2)
     assert S.spinq_w4a4_gemm_plan(2048, 14336, 4096) in (1, 2, 3)
-    assert S.spinq_w4a4_gemm_plan(4, 14336, 4096) == 4      # a handful of tokens: GEMV
-    assert S.spinq_w4a4_gemm_plan(5, 14336, 4096) != 4
+    assert S.spinq_w4a4_gemm_plan(2, 14336, 4096) == 4      # one or two tokens: GEMV
+    assert S.spinq_w4a4_gemm_plan(3, 14336, 4096) == 6      # 3 to 16: the tensor-core GEMV
     assert S.spinq_gemm_select_kernel(S.SPINQ_GEMM_TCGEMV + 1) == -1
 
 
@@ -388,21 +388,21 @@ def test_splitk_plan_covers_every_route(S):
 
 
 def test_splitk_workspace_follows_the_plan(S):
-    for M in (1, 3, 4):
+    for M, kind in ((1, S.SPINQ_GEMM_GEMV), (2, S.SPINQ_GEMM_GEMV), (3, S.SPINQ_GEMM_TCGEMV), (16, S.SPINQ_GEMM_TCGEMV)):
         assert S.spinq_w4a4_gemm_workspace_bytes(M, 8192, 3072) == 0
         assert S.gemm_workspace(M, 8192, 3072) is None
-        assert S.spinq_w4a4_gemm_splitk_plan(M, 8192, 3072) == (S.SPINQ_GEMM_GEMV, 0)
-    # few tokens, narrow outputs, long K: every SM streams a slice of the weights
-    kind, nsplit = S.spinq_w4a4_gemm_splitk_plan(16, 3072, 8192)
+        assert S.spinq_w4a4_gemm_splitk_plan(M, 8192, 3072) == (kind, 0)
+    # a few dozen tokens, narrow outputs, long K: every SM streams a slice of the weights
+    kind, nsplit = S.spinq_w4a4_gemm_splitk_plan(32, 3072, 8192)
     assert kind == S.SPINQ_GEMM_SPLITK and nsplit > 1
-    assert S.spinq_w4a4_gemm_workspace_bytes(16, 3072, 8192) == 16 * 3072 * 4 + 24 * 4
+    assert S.spinq_w4a4_gemm_workspace_bytes(32, 3072, 8192) == 32 * 3072 * 4 + 24 * 4
     # the tokens no longer fit in the GEMV kernel's shared memory
     assert S.spinq_w4a4_gemm_splitk_plan(4, 8192, 65536)[0] == S.SPINQ_GEMM_SPLITK
     # no slices, no workspace
     prev = S.spinq_gemm_split_k(1)
     try:
-        assert S.spinq_w4a4_gemm_workspace_bytes(16, 3072, 8192) == 0
-        assert S.spinq_w4a4_gemm_splitk_plan(16, 3072, 8192) == (S.SPINQ_GEMM_SPLITK, 1)
+        assert S.spinq_w4a4_gemm_workspace_bytes(32, 3072, 8192) == 0
+        assert S.spinq_w4a4_gemm_splitk_plan(32, 3072, 8192) == (S.SPINQ_GEMM_SPLITK, 1)
     finally:
         S.spinq_gemm_split_k(prev)
     assert S.spinq_gemm_split_k(65) == -1 and S.spinq_gemm_split_k(-1) == -1
@@ -422,19 +422,19 @@ def test_splitk_workspace_follows_the_plan(S):
                                    (4, 8192, 8192), (3, 100 * 16, 14336), (1, 8192, 40960)])
 @pytest.mark.parametrize("symmetric", [True, False])
 def test_gemv_random_codes_exact(S, M, N, K, symmetric):
-    """The GEMV kernel (M <= 4) through both entry points."""
+    """The GEMV kernel (M <= 4, selected: AUTO gives 3 and 4 tokens to the
+    tensor-core GEMV where it covers K) through both entry points."""
     rng = np.random.default_rng(M * 31 + N + K + symmetric)
     ac, al, be, wc, ws_ = random_codes(rng, M, N, K, symmetric)
     ref = oracle_full(ac, al, be, wc, ws_)
-    for entry in ("splitk", "gemm"):
-        if entry == "splitk":
-            y, acc = run_splitk(S, ac, al, be, wc, ws_)
-        else:
-            y, acc = run(S, ac, al, be, wc, ws_)
+
+    def go():
+        assert S.spinq_w4a4_gemm_plan(M, N, K) == S.SPINQ_GEMM_GEMV
+        return [run_splitk(S, ac, al, be, wc, ws_), run(S, ac, al, be, wc, ws_)]
+    for entry, (y, acc) in zip(("splitk", "gemm"), _with_kernel(S, S.SPINQ_GEMM_GEMV, go)):
         assert np.array_equal(acc, ref.acc), entry
         assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
         assert np.allclose(y.astype(np.float64), ref.y, rtol=2e-3, atol=1e-3 * np.abs(ref.y).max())
-    assert S.spinq_w4a4_gemm_plan(M, N, K) == 4
 
 
 def test_gemv_shared_memory_sizes_in_any_order(S):
@@ -443,7 +443,7 @@ def test_gemv_shared_memory_sizes_in_any_order(S):
     rng = np.random.default_rng(5)
     for (M, N, K) in [(4, 256, 32768), (3, 256, 14336), (4, 256, 32768), (2, 256, 1024), (4, 256, 32768)]:
         ac, al, be, wc, ws_ = random_codes(rng, M, N, K, False)
-        y, acc = run_splitk(S, ac, al, be, wc, ws_)
+        y, acc = _with_kernel(S, S.SPINQ_GEMM_GEMV, lambda: run_splitk(S, ac, al, be, wc, ws_))
         assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc)
 
 
@@ -453,7 +453,7 @@ def test_gemv_extreme_codes_long_k(S):
         ac = np.full((M, K), aval, dtype=np.int32)
         wc = np.full((N, K), wval, dtype=np.int32)
         al, ws_ = np.full(M, 0.5), np.full(N, 0.25)
-        y, acc = run_splitk(S, ac, al, None, wc, ws_)
+        y, acc = _with_kernel(S, S.SPINQ_GEMM_GEMV, lambda: run_splitk(S, ac, al, None, wc, ws_))
         assert np.array_equal(acc, oracle_full(ac, al, None, wc, ws_).acc)
 
 
@@ -514,11 +514,47 @@ def test_tcgemv_extreme_codes_long_k(S, symmetric):
         assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc), (aval, wval)
 
 
-def test_auto_plan_takes_tcgemv_for_five_to_eight_tokens(S):
-    for M, want in ((4, S.SPINQ_GEMM_GEMV), (5, S.SPINQ_GEMM_TCGEMV), (8, S.SPINQ_GEMM_TCGEMV)):
+@pytest.mark.parametrize("symmetric", [True, False])
+def test_tcgemv_register_streamed_extreme_codes(S, symmetric):
+    """The register-streamed form at its longest K (16 warps of 8 K blocks):
+    every code at an extreme, 2^-44 units up to 225 K."""
+    M, N, K = 16, 4096, 16384
+    pairs = ((7, 7), (-8, -8), (7, -8)) if symmetric else ((15, 7), (0, -8), (15, -8))
+    for aval, wval in pairs:
+        ac = np.full((M, K), aval, dtype=np.int32)
+        wc = np.full((N, K), wval, dtype=np.int32)
+        al, ws_ = np.full(M, 0.5), np.full(N, 0.25)
+        be = None if symmetric else np.full(M, -1.0)
+        y, acc = _with_kernel(S, S.SPINQ_GEMM_TCGEMV, lambda: run_splitk(S, ac, al, be, wc, ws_))
+        assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc), (aval, wval)
+
+
+@pytest.mark.parametrize("M,N,K", [(2, 8192, 3072), (16, 3072, 8192), (7, 14336, 4096), (16, 4096, 14336),
+                                   (1, 1216, 2048), (4, 64, 1536), (16, 14592, 1024), (11, 20480, 384)])
+def test_tcgemv_register_streamed_shapes(S, M, N, K):
+    """The decode shapes of both configs, K block counts of 1, 2, 4 and 8 per
+    warp, and 6 to 9 tiles per CTA (every reduction slot reused): exact acc
+    against the oracle on random codes."""
+    rng = np.random.default_rng(M * 7 + N + K)
+    ac, al, be, wc, ws_ = random_codes(rng, M, N, K, M % 2 == 0)
+    ref = oracle_full(ac, al, be, wc, ws_)
+    y, acc = _with_kernel(S, S.SPINQ_GEMM_TCGEMV, lambda: run_splitk(S, ac, al, be, wc, ws_))
+    assert np.array_equal(acc, ref.acc)
+    assert pu.rel_frob(y, ref.y) <= pu.Y_REL_FROB
+
+
+def test_auto_plan_takes_tcgemv_for_three_to_sixteen_tokens(S):
+    """Automatic choice: the GEMV kernel up to 2 tokens, the tensor-core GEMV
+    from 3 to 16 where its register-streamed form covers K (3072 = 24 K
+    blocks), else from 5 to 8 (4224 = 33 K blocks); split-K beyond."""
+    for M, want in ((1, S.SPINQ_GEMM_GEMV), (2, S.SPINQ_GEMM_GEMV), (3, S.SPINQ_GEMM_TCGEMV),
+                    (8, S.SPINQ_GEMM_TCGEMV), (16, S.SPINQ_GEMM_TCGEMV)):
         assert S.spinq_w4a4_gemm_plan(M, 8192, 3072) == want
         assert S.spinq_w4a4_gemm_splitk_plan(M, 8192, 3072) == (want, 0)
-    assert S.spinq_w4a4_gemm_splitk_plan(9, 8192, 3072)[0] == S.SPINQ_GEMM_SPLITK
+    assert S.spinq_w4a4_gemm_splitk_plan(17, 8192, 3072)[0] == S.SPINQ_GEMM_SPLITK
+    for M, want in ((4, S.SPINQ_GEMM_GEMV), (5, S.SPINQ_GEMM_TCGEMV), (8, S.SPINQ_GEMM_TCGEMV)):
+        assert S.spinq_w4a4_gemm_plan(M, 8192, 4224) == want
+    assert S.spinq_w4a4_gemm_splitk_plan(9, 8192, 4224)[0] == S.SPINQ_GEMM_SPLITK
     # a forced split-K selection keeps the split-K kernel
     prev = S.spinq_gemm_select_kernel(S.SPINQ_GEMM_SPLITK)
     try:
@@ -536,15 +572,20 @@ def test_tcgemv_plan_falls_back_beyond_its_range(S):
 
 
 def test_splitk_workspace_reused_and_left_zero(S):
+    """The split-K kernel (selected: AUTO gives 16 tokens to the tensor-core
+    GEMV) slices K here; its workspace is reused and left zero."""
     rng = np.random.default_rng(21)
     M, N, K = 16, 1024, 2048
-    ws = S.gemm_workspace(M, N, K)
-    assert ws is not None   # the plan slices K here
-    for rep in range(3):
-        ac, al, be, wc, ws_ = random_codes(rng, M, N, K, rep % 2 == 0)
-        y, acc = run_splitk(S, ac, al, be, wc, ws_, workspace=ws)
-        assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc)
-        assert int(torch.count_nonzero(ws)) == 0
+
+    def go():
+        ws = S.gemm_workspace(M, N, K)
+        assert ws is not None   # the plan slices K here
+        for rep in range(3):
+            ac, al, be, wc, ws_ = random_codes(rng, M, N, K, rep % 2 == 0)
+            y, acc = run_splitk(S, ac, al, be, wc, ws_, workspace=ws)
+            assert np.array_equal(acc, oracle_full(ac, al, be, wc, ws_).acc)
+            assert int(torch.count_nonzero(ws)) == 0
+    _with_kernel(S, S.SPINQ_GEMM_SPLITK, go)
 
 
 @pytest.mark.parametrize("splitk_route", ["sliced", "whole_k"], indirect=True)
