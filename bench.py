@@ -1061,7 +1061,7 @@ def relaunch(args_n):
 
 
 PROFILE_CASES = ("attention", "rope_kv", "fp8_gemm", "w4a8_gemm", "rq8_paley", "cayley", "paley", "gemm",
-                 "gemm_gate_up", "decode_gemm")
+                 "gemm_gate_up", "decode_gemm", "decode_gemm16")
 
 
 def profile_case(name, reps):
@@ -1075,7 +1075,8 @@ def profile_case(name, reps):
     152 rotations of 128 x 128, 2 iterations; paley: the 4-bit R4 kernel on
     2048 x 14336; gemm: the W4A4 down_proj 2048 x 14336 -> 4096; gemm_gate_up:
     the W4A4 gate_up 2048 x 4096 -> 14336 (asymmetric activations);
-    decode_gemm: 8 tokens through 4096 -> 14336 on the automatic route."""
+    decode_gemm: 8 tokens through 4096 -> 14336 on the automatic route;
+    decode_gemm16: 16 tokens through 3072 -> 8192 on the automatic route."""
     import numpy as np
     import torch
 
@@ -1126,6 +1127,11 @@ def profile_case(name, reps):
         c = synth.llama3_8b_gate_up(M=8)
         qa = spinq.rotate_quant_act(torch.from_numpy(c.x).to(dev), None, False)
         qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), None)
+        fn = lambda: spinq.w4a4_gemm_splitk(qa, qw)
+    elif name == "decode_gemm16":
+        c = synth.llama32_3b_up(M=16)
+        qa = spinq.rotate_quant_act(torch.from_numpy(c.x).to(dev), c.had, c.act_symmetric)
+        qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), c.had)
         fn = lambda: spinq.w4a4_gemm_splitk(qa, qw)
     elif name == "cayley":
         rng = np.random.default_rng(0)

@@ -338,6 +338,20 @@ __global__ void __launch_bounds__(kRsMaxWarps * 32, 1) w4a4_decode_rs_kernel(Gem
       ra[d] = ldg_stream(p);
       rb[d] = ldg_stream(p + r8);
     }
+  // the channel constants of every tile of this CTA: loaded now, stored
+  // after the token words below, so that the two loads' latencies overlap
+  const int nch = 16 * nt_cta;
+  float csn[2];
+  int crw[2];
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int e = threadIdx.x + k * blockDim.x;
+    if (e < nch) {
+      const int64_t n = 16 * (blockIdx.x + (int64_t)(e >> 4) * G) + (e & 15);
+      csn[k] = __ldg(a.w_scale + n);
+      crw[k] = __ldg(a.w_rowsum + n);
+    }
+  }
   // this warp's token words: token 8 nt + g, its K blocks, chunk c; made
   // unsigned (u = code ^ 8 for two's complement codes) and nibble-swapped;
   // tokens past M are zero
@@ -371,7 +385,15 @@ __global__ void __launch_bounds__(kRsMaxWarps * 32, 1) w4a4_decode_rs_kernel(Gem
   // the channel constants of every tile of this CTA
   float* sn_s = reinterpret_cast<float*>(tok_s + (size_t)W * NKW * NT * 32);
   int* rw_s = reinterpret_cast<int*>(sn_s + 16 * nt_cta);
-  for (int e = threadIdx.x; e < 16 * nt_cta; e += blockDim.x) {
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int e = threadIdx.x + k * blockDim.x;
+    if (e < nch) {
+      sn_s[e] = csn[k];
+      rw_s[e] = crw[k];
+    }
+  }
+  for (int e = threadIdx.x + 2 * blockDim.x; e < nch; e += blockDim.x) {
     const int64_t n = 16 * (blockIdx.x + (int64_t)(e >> 4) * G) + (e & 15);
     sn_s[e] = __ldg(a.w_scale + n);
     rw_s[e] = __ldg(a.w_rowsum + n);
