@@ -43,6 +43,8 @@
 // the outputs are bit-identical.
 #include <cuda_fp16.h>
 
+#include <utility>
+
 #include "../../include/spinq.h"
 #include "launch_util.h"
 #include "spinq_device.cuh"
@@ -410,93 +412,113 @@ __global__ void __launch_bounds__(kRsMaxWarps * 32, 1) w4a4_decode_rs_kernel(Gem
 #pragma unroll
     for (int e = 0; e < 4; ++e) d0[nt][e] = d1[nt][e] = 0.f;
   const uint8_t* wp = w0 + (size_t)TG * tstride;          // tile ti + TG
-  bool ok = true;
-  for (int t = 0; t < nt_cta && ok; t += TG) {
+  // One tile: its K blocks (ring slots from the compile-time position U of
+  // the tile in the ring's turn), then its share of the reduction.  `refill`
+  // is false only for the last TG tiles (nothing further to load).
+  auto do_tile = [&](auto U, int ti, bool refill) -> bool {
+    constexpr int u = decltype(U)::value;
 #pragma unroll
-    for (int u = 0; u < TG; ++u) {
-      const int ti = t + u;
-      if (ti >= nt_cta || !ok) break;   // warp-uniform
-      const bool next_tile = ti + TG < nt_cta;
+    for (int j = 0; j < NKW; ++j) {
+      const int dd = (u * NKW + j) % D;
+      const uint4 wa = ra[dd], wb = rb[dd];
+      uint4 tv[NT];
 #pragma unroll
-      for (int j = 0; j < NKW; ++j) {
-        const int dd = (u * NKW + j) % D;
-        const uint4 wa = ra[dd], wb = rb[dd];
-        uint4 tv[NT];
+      for (int nt = 0; nt < NT; ++nt) tv[nt] = tw[(j * NT + nt) * 32];
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) tv[nt] = tw[(j * NT + nt) * 32];
+      for (int s = 0; s < 4; ++s) {
+        const uint32_t x0 = word(wa, s), x1 = word(wb, s), y0 = x0 >> 8, y1 = x1 >> 8;
+        const uint32_t a1[4] = {and_xor(x0, mlo, flo), and_xor(x1, mlo, flo), and_xor(x0, mhi, fhi),
+                                and_xor(x1, mhi, fhi)};
+        const uint32_t a2[4] = {and_xor(y0, mlo, flo), and_xor(y1, mlo, flo), and_xor(y0, mhi, fhi),
+                                and_xor(y1, mhi, fhi)};
 #pragma unroll
-        for (int s = 0; s < 4; ++s) {
-          const uint32_t x0 = word(wa, s), x1 = word(wb, s), y0 = x0 >> 8, y1 = x1 >> 8;
-          const uint32_t a1[4] = {and_xor(x0, mlo, flo), and_xor(x1, mlo, flo), and_xor(x0, mhi, fhi),
-                                  and_xor(x1, mhi, fhi)};
-          const uint32_t a2[4] = {and_xor(y0, mlo, flo), and_xor(y1, mlo, flo), and_xor(y0, mhi, fhi),
-                                  and_xor(y1, mhi, fhi)};
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            const uint32_t t0 = word(tv[nt], s), t8 = t0 >> 8;
-            mma_16816_f16_f32_acc(d0[nt], a1, t0 & 0x00F000F0u, t0 & 0x000F000Fu);
-            mma_16816_f16_f32_acc(d1[nt], a2, t8 & 0x00F000F0u, t8 & 0x000F000Fu);
-          }
-        }
-        // refill the slot with the block D ahead: tile ti + TG, block j (RT);
-        // block j + D of this tile, or block j + D - NKW of the next one
-        const uint8_t* q = RT ? wp + j * 64 : (j + D < NKW ? wp - tstride + (j + D) * 64 : wp + (j + D - NKW) * 64);
-        if (__builtin_expect(RT ? next_tile : (j + D < NKW || next_tile), 1)) {
-          ra[dd] = ldg_stream(q);
-          rb[dd] = ldg_stream(q + r8);
+        for (int nt = 0; nt < NT; ++nt) {
+          const uint32_t t0 = word(tv[nt], s), t8 = t0 >> 8;
+          mma_16816_f16_f32_acc(d0[nt], a1, t0 & 0x00F000F0u, t0 & 0x000F000Fu);
+          mma_16816_f16_f32_acc(d1[nt], a2, t8 & 0x00F000F0u, t8 & 0x000F000Fu);
         }
       }
-      wp += tstride;
-      // ---- this warp's share of tile ti is done
-      const int slot = ti & (kRsSlots - 1);
-      if (ti >= kRsSlots)
-        ok = mbar_wait_suspend(&empty[slot], (uint32_t)((ti / kRsSlots) - 1) & 1u, abort_flag, kRsWaitNs);
-      if (!__all_sync(0xffffffffu, ok)) {
-        ok = false;
-        break;
-      }
-      // lane (g, c): channels g and g + 8, tokens 8 nt + 2c and 8 nt + 2c + 1;
-      // exact integers (whole numbers of 2^-44 below 2^24 of them)
-      const float unit = 17592186044416.0f;   // 2^44
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int m = 8 * nt + 2 * c + (e & 1);
-          if (m < M)
-            atomicAdd(&acc_s[slot][m * 16 + g + 8 * (e >> 1)], __float2int_rn((d0[nt][e] + d1[nt][e]) * unit));
-          d0[nt][e] = d1[nt][e] = 0.f;
-        }
-      // the last warp to finish the tile applies the epilogue (the fence
-      // orders each warp's adds before its count)
-      __threadfence_block();
-      __syncwarp();
-      int last = 0;
-      if (lane == 0) last = atomicAdd(&cnt_s[slot], 1) == W - 1;
-      if (!__shfl_sync(0xffffffffu, last, 0)) continue;
-      __threadfence_block();
-      const int ch = lane & 15;
-      const int64_t n = 16 * (blockIdx.x + (int64_t)ti * G) + ch;
-      const float sn = sn_s[16 * ti + ch];
-      const int rw = rw_s[16 * ti + ch];
-#pragma unroll
-      for (int q = 0; q < TOK / 2; ++q) {
-        const int idx = lane + 32 * q, m = idx >> 4;
-        const int v = acc_s[slot][idx];
-        acc_s[slot][idx] = 0;
-        if (m < M) {
-          const int accm = v - 8 * sa_s[m] - 8 * rw;
-          reinterpret_cast<__half*>(a.y)[(int64_t)m * a.N + n] =
-              __float2half_rn(sn * fmaf(al_s[m], (float)accm, bp_s[m] * (float)rw));
-          if (ACC_OUT) a.acc_out[(int64_t)m * a.N + n] = accm;
-        }
-      }
-      __syncwarp();
-      if (lane == 0) {
-        cnt_s[slot] = 0;
-        mbar_arrive(&empty[slot]);   // release: the cleared slot is ordered before it
+      // refill the slot with the block D ahead: tile ti + TG, block j (RT);
+      // block j + D of this tile, or block j + D - NKW of the next one
+      const uint8_t* q = RT ? wp + j * 64 : (j + D < NKW ? wp - tstride + (j + D) * 64 : wp + (j + D - NKW) * 64);
+      if ((!RT && j + D < NKW) || refill) {
+        ra[dd] = ldg_stream(q);
+        rb[dd] = ldg_stream(q + r8);
       }
     }
+    wp += tstride;
+    // ---- this warp's share of tile ti is done
+    const int slot = ti & (kRsSlots - 1);
+    if (ti >= kRsSlots &&
+        !__all_sync(0xffffffffu, mbar_wait_suspend(&empty[slot], (uint32_t)((ti / kRsSlots) - 1) & 1u, abort_flag,
+                                                   kRsWaitNs)))
+      return false;
+    // lane (g, c): channels g and g + 8, tokens 8 nt + 2c and 8 nt + 2c + 1;
+    // exact integers (whole numbers of 2^-44 below 2^24 of them); the sums
+    // of tokens past M are zero (their words are), so every lane adds
+    const float unit = 17592186044416.0f;   // 2^44
+    int* accp = &acc_s[slot][(2 * c) * 16 + g];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        atomicAdd(accp + (8 * nt + (e & 1)) * 16 + 8 * (e >> 1), __float2int_rn((d0[nt][e] + d1[nt][e]) * unit));
+        d0[nt][e] = d1[nt][e] = 0.f;
+      }
+    // the last warp to finish the tile applies the epilogue (the fence
+    // orders each warp's adds before its count)
+    __threadfence_block();
+    __syncwarp();
+    int last = 0;
+    if (lane == 0) last = atomicAdd(&cnt_s[slot], 1) == W - 1;
+    if (!__shfl_sync(0xffffffffu, last, 0)) return true;
+    __threadfence_block();
+    const int ch = lane & 15;
+    const int64_t n = 16 * (blockIdx.x + (int64_t)ti * G) + ch;
+    const float sn = sn_s[16 * ti + ch];
+    const int rw = rw_s[16 * ti + ch];
+#pragma unroll
+    for (int q = 0; q < TOK / 2; ++q) {
+      const int idx = lane + 32 * q, m = idx >> 4;
+      const int v = acc_s[slot][idx];
+      acc_s[slot][idx] = 0;
+      if (m < M) {
+        const int accm = v - 8 * sa_s[m] - 8 * rw;
+        reinterpret_cast<__half*>(a.y)[(int64_t)m * a.N + n] =
+            __float2half_rn(sn * fmaf(al_s[m], (float)accm, bp_s[m] * (float)rw));
+        if (ACC_OUT) a.acc_out[(int64_t)m * a.N + n] = accm;
+      }
+    }
+    __syncwarp();
+    if (lane == 0) {
+      cnt_s[slot] = 0;
+      mbar_arrive(&empty[slot]);   // release: the cleared slot is ordered before it
+    }
+    return true;
+  };
+  bool ok = true;
+  int t = 0;
+  static_assert(TG <= 4, "tiles per turn of the ring");
+  // tile U of the turn starting at t (U < TG); `tail`: the last turns, where
+  // tiles past nt_cta are skipped and the last TG load nothing more
+  auto turn_tile = [&](auto U, bool tail) {
+    constexpr int u = decltype(U)::value;
+    if constexpr (u < TG) {
+      if (ok && (!tail || t + u < nt_cta)) ok = do_tile(U, t + u, !tail || t + u + TG < nt_cta);
+    }
+  };
+  // whole turns of the ring whose tiles all refill it
+  for (; t + 2 * TG <= nt_cta && ok; t += TG) {
+    turn_tile(std::integral_constant<int, 0>{}, false);
+    turn_tile(std::integral_constant<int, 1>{}, false);
+    turn_tile(std::integral_constant<int, 2>{}, false);
+    turn_tile(std::integral_constant<int, 3>{}, false);
+  }
+  for (; t < nt_cta && ok; t += TG) {
+    turn_tile(std::integral_constant<int, 0>{}, true);
+    turn_tile(std::integral_constant<int, 1>{}, true);
+    turn_tile(std::integral_constant<int, 2>{}, true);
+    turn_tile(std::integral_constant<int, 3>{}, true);
   }
   if (!ok && threadIdx.x % 32 == 0 && status && atomicCAS(status, 0, (int)SPINQ_ETIMEOUT) == 0)
     atomicExch(status + 1, kRsSite);
