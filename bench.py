@@ -537,7 +537,7 @@ def run_ours(args, rank, world, local_rank):
             "traffic": gemm_traffic_from_profile(f"w4a4_gemm_down_proj_M{M}_K{K2}_N{N2}.md", GEMM_KERNELS[kind2][1]),
         },
         "rotate_quant_roofline": {
-            "bound": "hbm", "kernel": "rq_paley_kernel (R4 = H28 (x) H512 + act quant, 2048 x 14336, sym)",
+            "bound": "hbm", "kernel": "rq_paley_tc_kernel (R4 = H28 (x) H512 + act quant on tcgen05, 2048 x 14336, sym)",
             "achieved": round(rq2_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
             "frac": round(rq2_gbs / hbm_peak, 4), "us": round(t_rq2 * 1e6, 2),
             "isolated_us": round(iso["r4_quant"] * 1e6, 2),

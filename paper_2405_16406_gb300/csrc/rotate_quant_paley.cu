@@ -662,7 +662,10 @@ cudaError_t launch_rotate_quant_8bit_paley(const Rq8Args& a, cudaStream_t stream
                      : launch8_sc<kFmtInt8Planes, false>(b, stream, handled);
 }
 
-cudaError_t set_wait_limit_paley(uint64_t ns) { return cudaMemcpyToSymbol(g_wait_ns, &ns, sizeof(ns)); }
+cudaError_t set_wait_limit_paley(uint64_t ns) {
+  const cudaError_t e = cudaMemcpyToSymbol(g_wait_ns, &ns, sizeof(ns));
+  return e != cudaSuccess ? e : set_wait_limit_paley_tc(ns);
+}
 
 cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a0, cudaStream_t stream, bool* handled) {
   RotQuantArgs a = a0;
@@ -671,6 +674,10 @@ cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a0, cudaStream_t s
   *handled = false;
   if (a.rows == 0 || a.rowsum || a.n_small <= 1) return cudaSuccess;
   if ((a.ldx * 2) % 16 != 0) return cudaSuccess;
+  {
+    const cudaError_t e = launch_rotate_quant_act_paley_tc(a, stream, handled);
+    if (*handled || e != cudaSuccess) return e;
+  }
   const bool clamp = a.clip < 1.0f;
   if (a.signs) {   // random signs: the unclipped forms (clipped ones take the generic kernel)
     if (clamp) return cudaSuccess;

@@ -1,0 +1,364 @@
+// rotate_quant_paley_tc.cu -- spinq_rotate_quant_act for R = (H_s (x) H_512)
+// / sqrt(K), K = 512 n_s, n_s in {12, 20, 28} (Sec. 3.1, R4 of non-power-of-
+// two size), fused with the per-token Eq. 1 4-bit quantizer, on the 5th-
+// generation tensor core.  Element k = i 512 + j (i: Paley index).
+//
+// The Sylvester H_512 is H_4 on the top two bits of j (jh = j / 128) times
+// H_128 on the rest (jl = j % 128), so with the row written as the matrix
+// X[(i, jh)][jl] (MR = 4 n_s rows of 128 columns)
+//
+//   Y[(i, jh)][jl] = sum_jl' ( sum_(i',jh') T[(i, jh)][(i', jh')] X[(i', jh')][jl'] ) H_128[jl'][jl],
+//   T[(i, jh)][(i', jh')] = H_s[i'][i] H_4[jh'][jh].
+//
+// The inner sum is one tcgen05 MMA per row on the raw fp16 input (M = 128
+// rows of T, the first MR of them non-zero; N = 128 columns jl; K = MR in
+// K steps of 16): entries +-1, so the products are exact and the sums are
+// fp32 sums of fp16 values, as for the H_s stage of the mma.sync kernel.  The
+// accumulator lands in tensor memory with row (i, jh) on lane 4 i + jh and
+// the 128 columns jl across 128 columns, so one thread reads the whole
+// 128-point vector of its row: the 7 stages of H_128 are butterflies inside
+// the thread (no shared-memory transpose), then the row range (over the
+// threads of the row), Eq. 1 and 64 contiguous bytes of codes per thread
+// (lane m writes the codes of elements 128 m .. 128 m + 127).
+//
+// Warp roles (one CTA per SM, rows r0, r0 + G, ...):
+//  * warp 0: one thread copies each row into a ring of NSTG stages with one
+//    TMA tensor copy (the tensor map views the row as (jl % 64, jh, i,
+//    jl / 64): two 64-column atoms of MR 128-byte rows, 128-byte swizzle,
+//    the canonical MN-major layout of the MMA's B operand);
+//  * warp 1: one thread issues the MMAs of a row into one of NBUF tensor
+//    memory accumulators (128 columns each) and commits them to the stage's
+//    `free` barrier and the accumulator's `full` barrier;
+//  * NGRP groups of 4 warps (one per tensor-memory lane quadrant) take rows
+//    in turn: read the accumulator (releasing it for the next MMA), the
+//    butterflies, the range (a named barrier per group), Eq. 1 and the codes.
+// T is written once per CTA into shared memory (K-major, 128-byte swizzle).
+//
+// Every wait is bounded in time (suspended in hardware, the limit checked
+// every ~20 us); a wait that gives up raises the CTA's abort flag, the
+// others see it at their next wait, the MMA thread drains its MMAs and the
+// copy thread lets its copies land before tensor memory is released.
+#include <cuda_fp16.h>
+
+#include "../../include/spinq.h"
+#include "launch_util.h"
+#include "quant_common.cuh"
+#include "spinq_device.cuh"
+#include "spinq_internal.h"
+#include "tensor_map.h"
+
+namespace spinq {
+namespace {
+
+constexpr uint64_t kTcWaitLimitNs = 2000000000ull;
+// limit of the ordinary waits (kTcWaitLimitNs unless a test lowers it); the
+// drains of copies and MMAs in flight always use kTcWaitLimitNs
+__device__ uint64_t g_tc_wait_ns = kTcWaitLimitNs;
+constexpr int kTcSmemBudget = 232448;
+constexpr int kTcSite = 21;   // wait site recorded on a time-out
+
+template <int NS>
+struct PaleyTc {
+  static constexpr int MR = 4 * NS;               // rows (i, jh) of the row matrix
+  static constexpr int KS = MR / 16;              // MMA K steps
+  static constexpr int ATOMB = MR * 128;          // one 64-column atom of a staged row
+  static constexpr int ROWB = 2 * ATOMB;          // a staged row (= NS 512 fp16)
+  static constexpr int NGRP = 2;                  // row groups of GW warps
+  static constexpr int GW = 4;                    // one warp per tensor-memory lane quadrant
+  static constexpr int NBUF = 4;                  // tensor-memory accumulators (128 columns each)
+  static constexpr int TMEM_COLS = NBUF * 128 <= 256 ? 256 : 512;   // allocated (a power of two)
+  static constexpr int THREADS = 32 * (2 + GW * NGRP);
+  static constexpr int TB = 2 * 128 * 128;        // T: two 64-column K atoms of 128 rows (fp16)
+  static constexpr int MISC = 1024;               // barriers, flags, range scratch
+  static constexpr int NSTG_FIT = (kTcSmemBudget - 1024 - TB - MISC) / ROWB;
+  static constexpr int NSTG = NSTG_FIT < 6 ? NSTG_FIT : 6;   // staged rows
+  static_assert(MR % 16 == 0 && ATOMB % 1024 == 0, "atoms keep the 1024-byte swizzle period");
+  static_assert(NSTG >= 2, "two staged rows must fit");
+  static_assert(NGRP <= NBUF && NBUF % NGRP == 0, "each accumulator belongs to one group");
+  // shared memory (bytes from the 1024-aligned base)
+  static constexpr int OFF_T = 0;
+  static constexpr int OFF_STG = TB;
+  static constexpr int OFF_BAR = OFF_STG + NSTG * ROWB;   // full[NSTG] sfree[NSTG] dfull[NBUF] dfree[NBUF] drain
+  static constexpr int OFF_MISC = OFF_BAR + (2 * NSTG + 2 * NBUF + 1) * 8;   // tmem slot, abort flag, issued[NSTG]
+  static constexpr int OFF_RED = OFF_MISC + 8 + 4 * NSTG;                   // [NGRP][row parity][hi GW, lo GW]
+  static constexpr int BYTES = OFF_RED + NGRP * 2 * 2 * GW * 4 + 1024;
+  static_assert(OFF_RED + NGRP * 2 * 2 * GW * 4 <= OFF_BAR + MISC, "misc area");
+  static_assert(BYTES <= kTcSmemBudget, "shared memory");
+};
+
+// byte offset of byte b of row r in a block of 128-byte rows with the 128-byte swizzle
+__device__ __forceinline__ uint32_t sw128(uint32_t r, uint32_t b) {
+  return r * 128 + ((((b >> 4) ^ (r & 7)) << 4) | (b & 15));
+}
+
+__device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+  return mbar_wait_suspend(bar, parity, abort_flag, g_tc_wait_ns);
+}
+
+// bar.sync over `nthreads` threads whose result is the OR of `pred` over them.
+__device__ __forceinline__ bool tc_bar_or(int id, int nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
+template <int NS, bool SYM, bool CLAMP>
+__global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
+    rq_paley_tc_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
+  using S = PaleyTc<NS>;
+  constexpr int MR = S::MR, KS = S::KS, NSTG = S::NSTG, NBUF = S::NBUF, NGRP = S::NGRP;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-aligned base, derived from the shared array itself
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);   // row landed in stage s
+  uint64_t* sfree = full + NSTG;                                       // stage s read by its MMAs
+  uint64_t* dfull = sfree + NSTG;                                      // accumulator b written
+  uint64_t* dfree = dfull + NBUF;                                      // accumulator b read out (4 warps)
+  uint64_t* drain = dfree + NBUF;                                      // every MMA issued has completed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + S::OFF_MISC + 4);
+  int* issued = reinterpret_cast<int*>(smem + S::OFF_MISC + 8);      // last iteration copied into stage s
+  float* red = reinterpret_cast<float*>(smem + S::OFF_RED);           // [group][row parity][hi 4, lo 4]
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t r0 = blockIdx.x, G = gridDim.x;
+  const int niter = a.rows > r0 ? (int)((a.rows - r0 + G - 1) / G) : 0;
+
+  // T = H_s^T (x) H_4^T in the MMA's A layout (K-major, 128-byte swizzle):
+  // element (m, k) at K atom k / 64, row m, bytes 2 (k % 64); zero outside MR
+  for (int e = tid; e < 128 * 64; e += S::THREADS) {
+    const int m = e >> 6, k = (e & 63) * 2;
+    float v[2];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int kk = k + q;
+      float t = 0.f;
+      if (m < MR && kk < MR) {
+        const int i = m >> 2, jh = m & 3, ip = kk >> 2, jhp = kk & 3;
+        const uint32_t neg = ((a.hs.neg[ip] >> i) & 1u) ^ (uint32_t)(__popc(jh & jhp) & 1);
+        t = neg ? -1.f : 1.f;
+      }
+      v[q] = t;
+    }
+    *reinterpret_cast<uint32_t*>(smem + S::OFF_T + (k >> 6) * 16384 + sw128(m, (k & 63) * 2)) =
+        pack_half2_bits(v[0], v[1]);
+  }
+  if (tid == 0) {
+    for (int s = 0; s < NSTG; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&sfree[s], 1);
+      issued[s] = -1;
+    }
+    for (int b = 0; b < NBUF; ++b) {
+      mbar_init(&dfull[b], 1);
+      mbar_init(&dfree[b], S::GW);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmx);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, S::TMEM_COLS);
+    tmem_relinquish();
+  }
+  fence_proxy_async_smem();   // T, written by ordinary stores, is read by the tensor core
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    // ---------------- copies: one TMA tensor copy per row
+    if (lane == 0 && !a.debug_stall) {   // a test of the time-outs issues no copies
+      for (int it = 0; it < niter; ++it) {
+        const int s = it % NSTG;
+        if (it >= NSTG && !tc_wait(&sfree[s], (uint32_t)((it / NSTG) - 1) & 1u, abort_flag)) break;
+        mbar_arrive_expect_tx(&full[s], (uint32_t)S::ROWB);
+        tma_load_5d(smem + S::OFF_STG + s * S::ROWB, &tmx, &full[s], 0, 0, 0, 0, (int32_t)(r0 + (int64_t)it * G));
+        issued[s] = it;
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMAs: T (x) the staged row into accumulator it % NBUF
+    if (lane == 0) {
+      constexpr uint32_t idesc = umma_idesc_f16_f32_bmn(128, 128);
+      const uint32_t tb = smem_u32(smem + S::OFF_T), sb0 = smem_u32(smem + S::OFF_STG);
+      for (int it = 0; it < niter; ++it) {
+        const int s = it % NSTG, b = it % NBUF;
+        if (!tc_wait(&full[s], (uint32_t)(it / NSTG) & 1u, abort_flag)) break;
+        if (it >= NBUF && !tc_wait(&dfree[b], (uint32_t)((it / NBUF) - 1) & 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t sb = sb0 + (uint32_t)(s * S::ROWB);
+        // E = T [X0 | X1]: columns 0..63 E0 = T X0, columns 64..127 E1 = T X1
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks)
+          tc_mma_f16(tmem + (uint32_t)(b * 128), umma_desc_sw128(tb + (ks >> 2) * 16384 + (ks & 3) * 32),
+                     umma_desc_sw128_mn(sb + ks * 2048, S::ATOMB, 1024), idesc, ks > 0 ? 1u : 0u);
+        tc_commit(&sfree[s]);   // the stage may be refilled once these MMAs have read it
+        tc_commit(&dfull[b]);
+      }
+      // tensor memory is released only after every MMA issued has completed
+      tc_commit(drain);
+      mbar_wait_bounded(drain, 0, kTcWaitLimitNs);
+    }
+  } else {
+    // ---------------- groups of GW = 4 warps (one per tensor-memory lane
+    // quadrant): butterflies, range, Eq. 1, codes
+    constexpr int GW = S::GW;
+    const int gw = warp - 2, grp = gw / GW, quad = warp & 3;
+    const int m = quad * 32 + lane;   // this thread's row (i, jh) = (m / 4, m % 4)
+    const bool live = m < MR;
+    for (int it = grp; it < niter; it += NGRP) {
+      const int b = it % NBUF;
+      const int64_t row = r0 + (int64_t)it * G;
+      // on a failed wait the accumulator is read anyway (in bounds, discarded below)
+      const bool ok = tc_wait(&dfull[b], (uint32_t)(it / NBUF) & 1u, abort_flag);
+      __syncwarp();   // the tensor-memory loads below are warp-collective
+      tc_fence_after();
+      uint32_t r[128];
+      const uint32_t ta = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(b * 128);
+#pragma unroll
+      for (int q = 0; q < 128; q += 32) tmem_ld_32x32b_x32(ta + q, r + q);
+#pragma unroll
+      for (int q = 0; q < 128; q += 16) tmem_ld_wait(r + q);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0 && ok) mbar_arrive(&dfree[b]);   // the accumulator is in registers
+      // H_128 over jl: bit 0 inside each pair (jl, jl + 1), bits 1..6 across pairs
+      F2 z[64];
+#pragma unroll
+      for (int p = 0; p < 64; ++p) {
+        z[p] = f2_from_bits(r[2 * p], r[2 * p + 1]);
+        f2_bfly_inner(z[p]);
+      }
+#pragma unroll
+      for (int h = 1; h < 64; h <<= 1)
+#pragma unroll
+        for (int p = 0; p < 64; ++p)
+          if (!(p & h)) f2_bfly(z[p], z[p | h]);
+      // row range: four partial ranges (short dependency chains), then the
+      // warp and the group's warps (scratch alternates between the group's
+      // rows, so one barrier per row suffices); the same barrier settles the
+      // abort decision for every thread of the group
+      Range<SYM> rg[4];
+      if (live) {
+#pragma unroll
+        for (int p = 0; p < 64; ++p) rg[p & 3].add_pair(z[p]);
+      }
+#pragma unroll
+      for (int q = 1; q < 4; ++q) {
+        rg[0].hi = fmaxf(rg[0].hi, rg[q].hi);
+        if (!SYM) rg[0].lo = fminf(rg[0].lo, rg[q].lo);
+      }
+      rg[0].warp_reduce();
+      float* rd = red + (grp * 2 + ((it / NGRP) & 1)) * 2 * GW;
+      if (lane == 0) {
+        rd[quad] = rg[0].hi;
+        rd[GW + quad] = rg[0].lo;
+      }
+      if (tc_bar_or(1 + grp, 32 * GW, !ok || *abort_flag)) break;
+      Range<SYM> rr;
+      rr.hi = rd[0];
+      rr.lo = rd[GW];
+#pragma unroll
+      for (int q = 1; q < GW; ++q) {
+        rr.hi = fmaxf(rr.hi, rd[q]);
+        if (!SYM) rr.lo = fminf(rr.lo, rd[GW + q]);
+      }
+      const QParams<SYM> qp(rr, a.clip);
+      if (live) {
+        // codes of elements 128 m .. 128 m + 127: 64 contiguous bytes
+        uint4* out = reinterpret_cast<uint4*>(a.codes + row * (a.K / 2) + (int64_t)m * 64);
+#pragma unroll
+        for (int w4 = 0; w4 < 4; ++w4) {
+          uint32_t wd[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t rb[8];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) qp.template code_bits2<CLAMP>(z[16 * w4 + 4 * q + t], rb[2 * t], rb[2 * t + 1]);
+            wd[q] = pack8_nibbles(rb);
+          }
+          out[w4] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        }
+      }
+      if (m == 0) {
+        a.scale[row] = qp.alpha * a.norm;
+        if (!SYM) a.zero[row] = qp.beta * a.norm;
+      }
+    }
+  }
+  // after an abort the copies still in flight land before the CTA exits
+  if (warp == 0 && lane == 0 && *abort_flag)
+    for (int s = 0; s < NSTG; ++s)
+      if (issued[s] >= 0) mbar_wait_bounded(&full[s], (uint32_t)(issued[s] / NSTG) & 1u, kTcWaitLimitNs);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (*abort_flag && tid == 0 && a.status && atomicCAS(a.status, 0, (int)SPINQ_ETIMEOUT) == 0)
+    atomicExch(a.status + 1, kTcSite);
+  if (warp == 1) tmem_dealloc(tmem, S::TMEM_COLS);
+}
+
+template <int NS, bool SYM, bool CLAMP>
+cudaError_t launch_tc(const RotQuantArgs& a, cudaStream_t stream) {
+  using S = PaleyTc<NS>;
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return cudaErrorNotSupported;
+  // a row as (jl % 64, jh, i, jl / 64): two 64-column atoms of MR 128-byte rows (i, jh)
+  CUtensorMap tmx;
+  const cuuint64_t gdim[5] = {64, 4, (cuuint64_t)NS, 2, (cuuint64_t)a.rows};
+  const cuuint64_t gstride[4] = {256, 1024, 128, (cuuint64_t)(a.ldx * 2)};
+  const cuuint32_t box[5] = {64, 4, (cuuint32_t)NS, 2, 1};
+  const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  if (enc(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<void*>(a.x), gdim, gstride, box, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorNotSupported;
+  auto kern = rq_paley_tc_kernel<NS, SYM, CLAMP>;
+  int per_sm = 0;
+  cudaError_t e = prepare_launch_tmem(kern, S::THREADS, S::BYTES, S::TMEM_COLS, &per_sm);
+  if (e != cudaSuccess) return e;
+  const int64_t cap = (int64_t)device_sm_count() * per_sm;
+  const int64_t grid = a.rows < cap ? a.rows : cap;
+  RotQuantArgs la = a;
+  la.debug_stall = take_debug_stall() ? 1 : 0;
+  e = launch_pdl(kern, dim3((unsigned)grid), dim3(S::THREADS), S::BYTES, stream, 1, tmx, la);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+template <bool SYM, bool CLAMP>
+cudaError_t launch_tc_ns(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = true;
+  switch (a.n_small) {
+    case 12: return launch_tc<12, SYM, CLAMP>(a, stream);
+    case 20: return launch_tc<20, SYM, CLAMP>(a, stream);
+    case 28: return launch_tc<28, SYM, CLAMP>(a, stream);
+  }
+  *handled = false;
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t set_wait_limit_paley_tc(uint64_t ns) { return cudaMemcpyToSymbol(g_tc_wait_ns, &ns, sizeof(ns)); }
+
+cudaError_t launch_rotate_quant_act_paley_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = false;
+  if (a.rows == 0 || a.rowsum || a.signs || a.n_pow2 != 512) return cudaSuccess;
+  if (a.n_small != 12 && a.n_small != 20 && a.n_small != 28) return cudaSuccess;
+  if ((a.ldx * 2) % 16 != 0 || a.K != (int64_t)a.n_small * 512) return cudaSuccess;
+  const bool clamp = a.clip < 1.0f;
+  if (a.symmetric)
+    return clamp ? launch_tc_ns<true, true>(a, stream, handled) : launch_tc_ns<true, false>(a, stream, handled);
+  return clamp ? launch_tc_ns<false, true>(a, stream, handled) : launch_tc_ns<false, false>(a, stream, handled);
+}
+
+}  // namespace spinq

@@ -353,6 +353,15 @@ __device__ __forceinline__ void tma_load_4d(void* smem_dst, const void* tmap, ui
       : "memory");
 }
 
+__device__ __forceinline__ void tma_load_5d(void* smem_dst, const void* tmap, uint64_t* bar, int32_t c0,
+                                            int32_t c1, int32_t c2, int32_t c3, int32_t c4) {
+  asm volatile(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+      "%3, %4, %5, %6}], [%7];\n" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(smem_u32(bar))
+      : "memory");
+}
+
 // Bulk (non-tensor) copy global -> shared, completion on an mbarrier.  Both
 // addresses 16-byte aligned, `bytes` a multiple of 16.
 __device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
@@ -555,6 +564,41 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t addr) {
   d |= (uint64_t)1 << 46;                        // descriptor version (sm_100 family)
   d |= (uint64_t)2 << 61;                        // layout: 128-byte swizzle
   return d;
+}
+
+// Shared-memory matrix descriptor for an MN-major operand stored with the
+// 128-byte swizzle: 64-element atoms along M/N, each 8 K-rows of 128 bytes
+// (chunk c of row r at chunk c ^ (r % 8)); `lbo` bytes between atoms along
+// M/N, `sbo` bytes between 8-row groups along K.  Base 1024-byte aligned.
+__device__ __forceinline__ uint64_t umma_desc_sw128_mn(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr >> 4) & 0x3FFF);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// D[tmem] (+)= A[smem] * B[smem], 16-bit floating point operands (kind::f16).
+__device__ __forceinline__ void tc_mma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Instruction descriptor for kind::f16, FP16 x FP16 -> F32, A K-major, B
+// MN-major (bit 16).
+__host__ __device__ constexpr uint32_t umma_idesc_f16_f32_bmn(int M, int N) {
+  return (1u << 4)                          // D format: F32
+         | (0u << 7)                        // A format: F16
+         | (0u << 10)                       // B format: F16
+         | (1u << 16)                       // B MN-major
+         | ((uint32_t)(N >> 3) << 17)       // N / 8
+         | ((uint32_t)(M >> 4) << 24);      // M / 16
 }
 
 // Instruction descriptor for kind::f8f6f4, E4M3 x E4M3 -> F32, both K-major.

@@ -49,6 +49,12 @@ cudaError_t launch_rotate_quant_act_fast(const RotQuantArgs& a, cudaStream_t str
 // {128, 256, 512}).  Sets *handled = false for other shapes.
 cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
 
+// The same for P = 512 without random signs on the 5th-generation tensor
+// core (rotate_quant_paley_tc.cu); launch_rotate_quant_act_paley tries it
+// first.  Sets *handled = false for other shapes.
+cudaError_t launch_rotate_quant_act_paley_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
+cudaError_t set_wait_limit_paley_tc(uint64_t ns);
+
 struct KVArgs {
   const void* q_in;
   void* q_out;

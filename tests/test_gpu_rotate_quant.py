@@ -72,11 +72,12 @@ def test_act_shapes_and_modes(S, had, symmetric):
     check_act(S, x, had, symmetric, 1.0, f"had={had} sym={symmetric}")
 
 
+@pytest.mark.parametrize("had", [(12, 256), (28, 512)])
 @pytest.mark.parametrize("symmetric,clip", [(True, 0.9), (False, 0.9), (False, 0.5)])
-def test_act_clipping(S, symmetric, clip):
+def test_act_clipping(S, had, symmetric, clip):
     rng = np.random.default_rng(9)
-    x = synth.activations(rng, 64, 3072, outlier_frac=0.01, factor=30.0)
-    check_act(S, x, (12, 256), symmetric, clip, f"clip={clip}")
+    x = synth.activations(rng, 64, had[0] * had[1], outlier_frac=0.01, factor=30.0)
+    check_act(S, x, had, symmetric, clip, f"had={had} clip={clip}")
 
 
 def test_act_degenerate_rows(S):
