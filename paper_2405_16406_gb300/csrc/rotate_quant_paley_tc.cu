@@ -34,8 +34,8 @@
 //    butterflies, the range (a named barrier per group), Eq. 1 and the codes.
 // T is written once per CTA into shared memory (K-major, 128-byte swizzle).
 //
-// Every wait is bounded in time (suspended in hardware, the limit checked
-// every ~20 us); a wait that gives up raises the CTA's abort flag, the
+// Every wait is bounded in time (polled, the limit checked every 256
+// polls); a wait that gives up raises the CTA's abort flag, the
 // others see it at their next wait, the MMA thread drains its MMAs and the
 // copy thread lets its copies land before tensor memory is released.
 #include <cuda_fp16.h>
@@ -57,12 +57,20 @@ __device__ uint64_t g_tc_wait_ns = kTcWaitLimitNs;
 constexpr int kTcSmemBudget = 232448;
 constexpr int kTcSite = 21;   // wait site recorded on a time-out
 
-template <int NS>
-struct PaleyTc {
-  static constexpr int MR = 4 * NS;               // rows (i, jh) of the row matrix
+// NS > 0: the Paley rotation H_NS (x) H_512, one row per MMA, MR = 4 NS rows
+// (i, jh).  NS = 0: the Sylvester rotation H_P = H_JH (x) H_128, P = 128 JH
+// in {8192, 16384}: RPS = 128 / JH rows per MMA (T = I_RPS (x) H_JH), MR =
+// 128 rows (r, jh).
+template <int NS, int JH>
+struct RqTc {
+  static constexpr bool PALEY = NS > 0;
+  static constexpr int MR = PALEY ? 4 * NS : 128;   // live rows of the MMA (lanes)
+  static constexpr int RPS = PALEY ? 1 : 128 / JH;  // input rows per MMA
+  static constexpr int LPR = PALEY ? MR : JH;       // tensor-memory lanes per input row
   static constexpr int KS = MR / 16;              // MMA K steps
-  static constexpr int ATOMB = MR * 128;          // one 64-column atom of a staged row
-  static constexpr int ROWB = 2 * ATOMB;          // a staged row (= NS 512 fp16)
+  static constexpr int ATOMB = MR * 128;          // one 64-column atom of a stage
+  static constexpr int ROWB = 2 * ATOMB;          // a stage (RPS rows of K fp16)
+  static_assert(PALEY || JH == 64 || JH == 128, "Sylvester factors H_64 and H_128");
   static constexpr int NGRP = 2;                  // row groups of GW warps
   static constexpr int GW = 4;                    // one warp per tensor-memory lane quadrant
   static constexpr int NBUF = 4;                  // tensor-memory accumulators (128 columns each)
@@ -91,8 +99,34 @@ __device__ __forceinline__ uint32_t sw128(uint32_t r, uint32_t b) {
   return r * 128 + ((((b >> 4) ^ (r & 7)) << 4) | (b & 15));
 }
 
+// Non-blocking probe of the phase with `parity` (never suspends the thread).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait that polls: a suspended wait woke up to ~0.5 us after the
+// phase completed (measured on the row pipeline of this kernel: 40.8 against
+// 36.7 us for H_8192 on 8192 rows), which the quantizer groups pay once per
+// row.  The abort flag and the time limit are checked every 256 polls.
 __device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-  return mbar_wait_suspend(bar, parity, abort_flag, g_tc_wait_ns);
+  if (mbar_test_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t k = 1;; ++k) {
+    if (mbar_test_wait(bar, parity)) return true;
+    if ((k & 255u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > g_tc_wait_ns) {
+        *abort_flag = 1;
+        return false;
+      }
+    }
+  }
 }
 
 // bar.sync over `nthreads` threads whose result is the OR of `pred` over them.
@@ -106,10 +140,10 @@ __device__ __forceinline__ bool tc_bar_or(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
-template <int NS, bool SYM, bool CLAMP>
-__global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
+template <int NS, int JH, bool SYM, bool CLAMP>
+__global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
     rq_paley_tc_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
-  using S = PaleyTc<NS>;
+  using S = RqTc<NS, JH>;
   constexpr int MR = S::MR, KS = S::KS, NSTG = S::NSTG, NBUF = S::NBUF, NGRP = S::NGRP;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-aligned base, derived from the shared array itself
@@ -125,10 +159,12 @@ __global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
   float* red = reinterpret_cast<float*>(smem + S::OFF_RED);           // [group][row parity][hi 4, lo 4]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t r0 = blockIdx.x, G = gridDim.x;
-  const int niter = a.rows > r0 ? (int)((a.rows - r0 + G - 1) / G) : 0;
+  const int64_t units = a.rows / S::RPS;   // MMAs (RPS rows each)
+  const int niter = units > r0 ? (int)((units - r0 + G - 1) / G) : 0;
 
-  // T = H_s^T (x) H_4^T in the MMA's A layout (K-major, 128-byte swizzle):
-  // element (m, k) at K atom k / 64, row m, bytes 2 (k % 64); zero outside MR
+  // T in the MMA's A layout (K-major, 128-byte swizzle): element (m, k) at K
+  // atom k / 64, row m, bytes 2 (k % 64); zero outside MR.  Paley: T =
+  // H_s^T (x) H_4^T, m = 4 i + jh; Sylvester: T = I_RPS (x) H_JH, m = JH r + jh
   for (int e = tid; e < 128 * 64; e += S::THREADS) {
     const int m = e >> 6, k = (e & 63) * 2;
     float v[2];
@@ -137,9 +173,13 @@ __global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
       const int kk = k + q;
       float t = 0.f;
       if (m < MR && kk < MR) {
-        const int i = m >> 2, jh = m & 3, ip = kk >> 2, jhp = kk & 3;
-        const uint32_t neg = ((a.hs.neg[ip] >> i) & 1u) ^ (uint32_t)(__popc(jh & jhp) & 1);
-        t = neg ? -1.f : 1.f;
+        if constexpr (S::PALEY) {
+          const int i = m >> 2, jh = m & 3, ip = kk >> 2, jhp = kk & 3;
+          const uint32_t neg = ((a.hs.neg[ip] >> i) & 1u) ^ (uint32_t)(__popc(jh & jhp) & 1);
+          t = neg ? -1.f : 1.f;
+        } else if (m / JH == kk / JH) {
+          t = (__popc((m % JH) & (kk % JH)) & 1) ? -1.f : 1.f;
+        }
       }
       v[q] = t;
     }
@@ -212,11 +252,14 @@ __global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
     // quadrant): butterflies, range, Eq. 1, codes
     constexpr int GW = S::GW;
     const int gw = warp - 2, grp = gw / GW, quad = warp & 3;
-    const int m = quad * 32 + lane;   // this thread's row (i, jh) = (m / 4, m % 4)
+    const int m = quad * 32 + lane;   // this thread's lane: (i, jh) = (m / 4, m % 4) or (r, jh) = (m / JH, m % JH)
     const bool live = m < MR;
+    const int rr_ = m / S::LPR;       // its input row within the MMA
+    // the lane quadrants holding that row
+    const int q_lo = (rr_ * S::LPR) / 32, q_hi = ((rr_ + 1) * S::LPR - 1) / 32;
     for (int it = grp; it < niter; it += NGRP) {
       const int b = it % NBUF;
-      const int64_t row = r0 + (int64_t)it * G;
+      const int64_t row = (r0 + (int64_t)it * G) * S::RPS + rr_;
       // on a failed wait the accumulator is read anyway (in bounds, discarded below)
       const bool ok = tc_wait(&dfull[b], (uint32_t)(it / NBUF) & 1u, abort_flag);
       __syncwarp();   // the tensor-memory loads below are warp-collective
@@ -264,17 +307,18 @@ __global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
       }
       if (tc_bar_or(1 + grp, 32 * GW, !ok || *abort_flag)) break;
       Range<SYM> rr;
-      rr.hi = rd[0];
-      rr.lo = rd[GW];
+      rr.hi = rd[q_lo];
+      rr.lo = rd[GW + q_lo];
 #pragma unroll
-      for (int q = 1; q < GW; ++q) {
-        rr.hi = fmaxf(rr.hi, rd[q]);
-        if (!SYM) rr.lo = fminf(rr.lo, rd[GW + q]);
-      }
+      for (int q = 0; q < GW; ++q)
+        if (q > q_lo && q <= q_hi) {
+          rr.hi = fmaxf(rr.hi, rd[q]);
+          if (!SYM) rr.lo = fminf(rr.lo, rd[GW + q]);
+        }
       const QParams<SYM> qp(rr, a.clip);
       if (live) {
-        // codes of elements 128 m .. 128 m + 127: 64 contiguous bytes
-        uint4* out = reinterpret_cast<uint4*>(a.codes + row * (a.K / 2) + (int64_t)m * 64);
+        // codes of elements 128 (m % LPR) .. + 127 of the row: 64 contiguous bytes
+        uint4* out = reinterpret_cast<uint4*>(a.codes + row * (a.K / 2) + (int64_t)(m % S::LPR) * 64);
 #pragma unroll
         for (int w4 = 0; w4 < 4; ++w4) {
           uint32_t wd[4];
@@ -288,7 +332,7 @@ __global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
           out[w4] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
         }
       }
-      if (m == 0) {
+      if (live && m % S::LPR == 0) {
         a.scale[row] = qp.alpha * a.norm;
         if (!SYM) a.zero[row] = qp.beta * a.norm;
       }
@@ -306,27 +350,34 @@ __global__ void __launch_bounds__(PaleyTc<NS>::THREADS, 1)
   if (warp == 1) tmem_dealloc(tmem, S::TMEM_COLS);
 }
 
-template <int NS, bool SYM, bool CLAMP>
+template <int NS, int JH, bool SYM, bool CLAMP>
 cudaError_t launch_tc(const RotQuantArgs& a, cudaStream_t stream) {
-  using S = PaleyTc<NS>;
+  using S = RqTc<NS, JH>;
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return cudaErrorNotSupported;
-  // a row as (jl % 64, jh, i, jl / 64): two 64-column atoms of MR 128-byte rows (i, jh)
+  // Paley: a row as (jl % 64, jh, i, jl / 64); Sylvester: RPS rows as
+  // (jl % 64, jh, r, jl / 64): two 64-column atoms of MR 128-byte rows
   CUtensorMap tmx;
-  const cuuint64_t gdim[5] = {64, 4, (cuuint64_t)NS, 2, (cuuint64_t)a.rows};
-  const cuuint64_t gstride[4] = {256, 1024, 128, (cuuint64_t)(a.ldx * 2)};
-  const cuuint32_t box[5] = {64, 4, (cuuint32_t)NS, 2, 1};
+  const cuuint64_t ld = (cuuint64_t)(a.ldx * 2);
+  const cuuint64_t gdim_p[5] = {64, 4, (cuuint64_t)NS, 2, (cuuint64_t)a.rows};
+  const cuuint64_t gstr_p[4] = {256, 1024, 128, ld};
+  const cuuint32_t box_p[5] = {64, 4, (cuuint32_t)NS, 2, 1};
+  const cuuint64_t gdim_s[5] = {64, (cuuint64_t)JH, (cuuint64_t)S::RPS, 2, (cuuint64_t)(a.rows / S::RPS)};
+  const cuuint64_t gstr_s[4] = {256, ld, 128, ld * S::RPS};
+  const cuuint32_t box_s[5] = {64, (cuuint32_t)JH, (cuuint32_t)S::RPS, 2, 1};
   const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-  if (enc(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<void*>(a.x), gdim, gstride, box, estr,
-          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  if (enc(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<void*>(a.x), S::PALEY ? gdim_p : gdim_s,
+          S::PALEY ? gstr_p : gstr_s, S::PALEY ? box_p : box_s, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorNotSupported;
-  auto kern = rq_paley_tc_kernel<NS, SYM, CLAMP>;
+  auto kern = rq_paley_tc_kernel<NS, JH, SYM, CLAMP>;
   int per_sm = 0;
   cudaError_t e = prepare_launch_tmem(kern, S::THREADS, S::BYTES, S::TMEM_COLS, &per_sm);
   if (e != cudaSuccess) return e;
+  const int64_t units = a.rows / S::RPS;
   const int64_t cap = (int64_t)device_sm_count() * per_sm;
-  const int64_t grid = a.rows < cap ? a.rows : cap;
+  const int64_t grid = units < cap ? units : cap;
   RotQuantArgs la = a;
   la.debug_stall = take_debug_stall() ? 1 : 0;
   e = launch_pdl(kern, dim3((unsigned)grid), dim3(S::THREADS), S::BYTES, stream, 1, tmx, la);
@@ -338,9 +389,20 @@ template <bool SYM, bool CLAMP>
 cudaError_t launch_tc_ns(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
   *handled = true;
   switch (a.n_small) {
-    case 12: return launch_tc<12, SYM, CLAMP>(a, stream);
-    case 20: return launch_tc<20, SYM, CLAMP>(a, stream);
-    case 28: return launch_tc<28, SYM, CLAMP>(a, stream);
+    case 12: return launch_tc<12, 0, SYM, CLAMP>(a, stream);
+    case 20: return launch_tc<20, 0, SYM, CLAMP>(a, stream);
+    case 28: return launch_tc<28, 0, SYM, CLAMP>(a, stream);
+  }
+  *handled = false;
+  return cudaSuccess;
+}
+
+template <bool SYM, bool CLAMP>
+cudaError_t launch_tc_pow2(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = true;
+  switch (a.n_pow2) {
+    case 8192: return launch_tc<0, 64, SYM, CLAMP>(a, stream);
+    case 16384: return launch_tc<0, 128, SYM, CLAMP>(a, stream);
   }
   *handled = false;
   return cudaSuccess;
@@ -359,6 +421,18 @@ cudaError_t launch_rotate_quant_act_paley_tc(const RotQuantArgs& a, cudaStream_t
   if (a.symmetric)
     return clamp ? launch_tc_ns<true, true>(a, stream, handled) : launch_tc_ns<true, false>(a, stream, handled);
   return clamp ? launch_tc_ns<false, true>(a, stream, handled) : launch_tc_ns<false, false>(a, stream, handled);
+}
+
+cudaError_t launch_rotate_quant_act_pow2_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = false;
+  if (a.rows == 0 || a.rowsum || a.signs || a.n_small != 1) return cudaSuccess;
+  if (a.n_pow2 != 8192 && a.n_pow2 != 16384) return cudaSuccess;
+  const int64_t rps = 16384 / a.n_pow2;   // rows per MMA
+  if (a.rows % rps != 0 || (a.ldx * 2) % 16 != 0 || a.K != a.n_pow2) return cudaSuccess;
+  const bool clamp = a.clip < 1.0f;
+  if (a.symmetric)
+    return clamp ? launch_tc_pow2<true, true>(a, stream, handled) : launch_tc_pow2<true, false>(a, stream, handled);
+  return clamp ? launch_tc_pow2<false, true>(a, stream, handled) : launch_tc_pow2<false, false>(a, stream, handled);
 }
 
 }  // namespace spinq

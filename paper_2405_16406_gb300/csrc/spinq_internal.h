@@ -54,6 +54,10 @@ cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a, cudaStream_t st
 // first.  Sets *handled = false for other shapes.
 cudaError_t launch_rotate_quant_act_paley_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
 cudaError_t set_wait_limit_paley_tc(uint64_t ns);
+// A Sylvester rotation of 8192 or 16384 points (rows a multiple of
+// 16384 / P, no random signs) on the same kernel; launch_rotate_quant_act_fast
+// tries it first.  Sets *handled = false for other shapes.
+cudaError_t launch_rotate_quant_act_pow2_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
 
 struct KVArgs {
   const void* q_in;
