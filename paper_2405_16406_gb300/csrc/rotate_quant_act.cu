@@ -435,7 +435,7 @@ cudaError_t launch_rotate_quant_act_fast(const RotQuantArgs& a, cudaStream_t str
                        : launch_pow2_for<false, false, true>(a, stream, handled);
   }
   if (a.n_small == 1) {
-    const cudaError_t e = launch_rotate_quant_act_pow2_tc(a, stream, handled);
+    const cudaError_t e = launch_rotate_quant_act_tc(a, stream, handled);
     if (*handled || e != cudaSuccess) return e;
     if (a.symmetric)
       return clamp ? launch_pow2_for<true, true>(a, stream, handled) : launch_pow2_for<true, false>(a, stream, handled);

@@ -664,7 +664,7 @@ cudaError_t launch_rotate_quant_8bit_paley(const Rq8Args& a, cudaStream_t stream
 
 cudaError_t set_wait_limit_paley(uint64_t ns) {
   const cudaError_t e = cudaMemcpyToSymbol(g_wait_ns, &ns, sizeof(ns));
-  return e != cudaSuccess ? e : set_wait_limit_paley_tc(ns);
+  return e != cudaSuccess ? e : set_wait_limit_rq_tc(ns);
 }
 
 cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a0, cudaStream_t stream, bool* handled) {
@@ -675,7 +675,7 @@ cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a0, cudaStream_t s
   if (a.rows == 0 || a.rowsum || a.n_small <= 1) return cudaSuccess;
   if ((a.ldx * 2) % 16 != 0) return cudaSuccess;
   {
-    const cudaError_t e = launch_rotate_quant_act_paley_tc(a, stream, handled);
+    const cudaError_t e = launch_rotate_quant_act_tc(a, stream, handled);
     if (*handled || e != cudaSuccess) return e;
   }
   const bool clamp = a.clip < 1.0f;

@@ -1,37 +1,39 @@
-// rotate_quant_paley_tc.cu -- spinq_rotate_quant_act for R = (H_s (x) H_512)
-// / sqrt(K), K = 512 n_s, n_s in {12, 20, 28} (Sec. 3.1, R4 of non-power-of-
-// two size), fused with the per-token Eq. 1 4-bit quantizer, on the 5th-
-// generation tensor core.  Element k = i 512 + j (i: Paley index).
+// rotate_quant_paley_tc.cu -- spinq_rotate_quant_act for plain rotations R =
+// (H_s (x) H_P) / sqrt(K) (Sec. 3.1, R4; H_s a Paley factor, or n_s = 1 for a
+// Sylvester rotation of P points), fused with the per-token Eq. 1 4-bit
+// quantizer, on the 5th-generation tensor core.  Element k = i P + j.
 //
-// The Sylvester H_512 is H_4 on the top two bits of j (jh = j / 128) times
+// The Sylvester H_P is H_(P/128) on the top bits of j (jh = j / 128) times
 // H_128 on the rest (jl = j % 128), so with the row written as the matrix
-// X[(i, jh)][jl] (MR = 4 n_s rows of 128 columns)
+// X[a][jl], a = i (P / 128) + jh (F = n_s P / 128 rows of 128 columns),
 //
-//   Y[(i, jh)][jl] = sum_jl' ( sum_(i',jh') T[(i, jh)][(i', jh')] X[(i', jh')][jl'] ) H_128[jl'][jl],
-//   T[(i, jh)][(i', jh')] = H_s[i'][i] H_4[jh'][jh].
+//   Y[a][jl] = sum_jl' ( sum_a' T[a][a'] X[a'][jl'] ) H_128[jl'][jl],
+//   T[a][a'] = H_s[i'][i] H_(P/128)[jh'][jh].
 //
-// The inner sum is one tcgen05 MMA per row on the raw fp16 input (M = 128
-// rows of T, the first MR of them non-zero; N = 128 columns jl; K = MR in
-// K steps of 16): entries +-1, so the products are exact and the sums are
-// fp32 sums of fp16 values, as for the H_s stage of the mma.sync kernel.  The
-// accumulator lands in tensor memory with row (i, jh) on lane 4 i + jh and
-// the 128 columns jl across 128 columns, so one thread reads the whole
-// 128-point vector of its row: the 7 stages of H_128 are butterflies inside
-// the thread (no shared-memory transpose), then the row range (over the
-// threads of the row), Eq. 1 and 64 contiguous bytes of codes per thread
-// (lane m writes the codes of elements 128 m .. 128 m + 127).
+// The inner sum is one tcgen05 MMA for RPS = 128 / F rows at once (T =
+// I_RPS (x) T on the MMA's M = 128 rows, the first MR = RPS F of them
+// non-zero; N = 128 columns jl; K = MR in K steps of 16) on the raw fp16
+// input: entries +-1, so the products are exact and the sums are fp32 sums of
+// fp16 values, as for the H_s stage of the mma.sync kernel.  The accumulator
+// lands in tensor memory with (r, a) on lane F r + a and the 128 columns jl
+// across 128 columns, so one thread reads the whole 128-point vector of its
+// block: the 7 stages of H_128 are butterflies inside the thread (no
+// shared-memory transpose), then the row range (over the row's lanes),
+// Eq. 1 and 64 contiguous bytes of codes per thread (the codes of elements
+// 128 a .. 128 a + 127 of row r).
 //
 // Warp roles (one CTA per SM, rows r0, r0 + G, ...):
-//  * warp 0: one thread copies each row into a ring of NSTG stages with one
-//    TMA tensor copy (the tensor map views the row as (jl % 64, jh, i,
-//    jl / 64): two 64-column atoms of MR 128-byte rows, 128-byte swizzle,
-//    the canonical MN-major layout of the MMA's B operand);
-//  * warp 1: one thread issues the MMAs of a row into one of NBUF tensor
+//  * warp 0: one thread copies each MMA's RPS rows into a ring of NSTG
+//    stages with one TMA tensor copy (the tensor map views them as (jl % 64,
+//    a, r, jl / 64): two 64-column atoms of MR 128-byte rows, 128-byte
+//    swizzle, the canonical MN-major layout of the MMA's B operand);
+//  * warp 1: one thread issues the MMAs of a stage into one of NBUF tensor
 //    memory accumulators (128 columns each) and commits them to the stage's
 //    `free` barrier and the accumulator's `full` barrier;
-//  * NGRP groups of 4 warps (one per tensor-memory lane quadrant) take rows
-//    in turn: read the accumulator (releasing it for the next MMA), the
-//    butterflies, the range (a named barrier per group), Eq. 1 and the codes.
+//  * NGRP groups of 4 warps (one per tensor-memory lane quadrant) take the
+//    accumulators in turn: read one (releasing it for the next MMA), the
+//    butterflies, the ranges (shared-memory atomics and a named barrier per
+//    group), Eq. 1 and the codes.
 // T is written once per CTA into shared memory (K-major, 128-byte swizzle).
 //
 // Every wait is bounded in time (polled, the limit checked every 256
@@ -39,6 +41,8 @@
 // others see it at their next wait, the MMA thread drains its MMAs and the
 // copy thread lets its copies land before tensor memory is released.
 #include <cuda_fp16.h>
+
+#include <climits>
 
 #include "../../include/spinq.h"
 #include "launch_util.h"
@@ -57,42 +61,50 @@ __device__ uint64_t g_tc_wait_ns = kTcWaitLimitNs;
 constexpr int kTcSmemBudget = 232448;
 constexpr int kTcSite = 21;   // wait site recorded on a time-out
 
-// NS > 0: the Paley rotation H_NS (x) H_512, one row per MMA, MR = 4 NS rows
-// (i, jh).  NS = 0: the Sylvester rotation H_P = H_JH (x) H_128, P = 128 JH
-// in {8192, 16384}: RPS = 128 / JH rows per MMA (T = I_RPS (x) H_JH), MR =
-// 128 rows (r, jh).
-template <int NS, int JH>
+// A row of K = n_s P elements (n_s = 1 for a Sylvester rotation) is the
+// matrix X[a][jl] of F = n_s P / 128 rows a = i (P / 128) + jh (i the Paley
+// index, jh = j / 128) and 128 columns jl = j % 128; R = H_s (x) H_P with
+// H_P = H_(P/128) (x) H_128, so the factor H_f = H_s (x) H_(P/128) acts on a and
+// H_128 on jl.  RPS rows share one MMA: T = I_RPS (x) H_f^T, MR = RPS F lanes.
+template <int F, int RPS>
 struct RqTc {
-  static constexpr bool PALEY = NS > 0;
-  static constexpr int MR = PALEY ? 4 * NS : 128;   // live rows of the MMA (lanes)
-  static constexpr int RPS = PALEY ? 1 : 128 / JH;  // input rows per MMA
-  static constexpr int LPR = PALEY ? MR : JH;       // tensor-memory lanes per input row
+  static constexpr int MR = F * RPS;              // live lanes: rows (r, a) of the MMA
   static constexpr int KS = MR / 16;              // MMA K steps
   static constexpr int ATOMB = MR * 128;          // one 64-column atom of a stage
   static constexpr int ROWB = 2 * ATOMB;          // a stage (RPS rows of K fp16)
-  static_assert(PALEY || JH == 64 || JH == 128, "Sylvester factors H_64 and H_128");
+  static_assert(MR <= 128 && MR % 16 == 0 && ATOMB % 1024 == 0, "MMA shape and the swizzle period");
   static constexpr int NGRP = 2;                  // row groups of GW warps
   static constexpr int GW = 4;                    // one warp per tensor-memory lane quadrant
   static constexpr int NBUF = 4;                  // tensor-memory accumulators (128 columns each)
   static constexpr int TMEM_COLS = NBUF * 128 <= 256 ? 256 : 512;   // allocated (a power of two)
   static constexpr int THREADS = 32 * (2 + GW * NGRP);
   static constexpr int TB = 2 * 128 * 128;        // T: two 64-column K atoms of 128 rows (fp16)
-  static constexpr int MISC = 1024;               // barriers, flags, range scratch
+  static constexpr int MISC = 1024;               // barriers, flags, range slots
   static constexpr int NSTG_FIT = (kTcSmemBudget - 1024 - TB - MISC) / ROWB;
-  static constexpr int NSTG = NSTG_FIT < 6 ? NSTG_FIT : 6;   // staged rows
-  static_assert(MR % 16 == 0 && ATOMB % 1024 == 0, "atoms keep the 1024-byte swizzle period");
-  static_assert(NSTG >= 2, "two staged rows must fit");
+  static constexpr int NSTG = NSTG_FIT < 6 ? NSTG_FIT : 6;   // staged MMA inputs
+  static_assert(NSTG >= 2, "two stages must fit");
   static_assert(NGRP <= NBUF && NBUF % NGRP == 0, "each accumulator belongs to one group");
   // shared memory (bytes from the 1024-aligned base)
   static constexpr int OFF_T = 0;
   static constexpr int OFF_STG = TB;
   static constexpr int OFF_BAR = OFF_STG + NSTG * ROWB;   // full[NSTG] sfree[NSTG] dfull[NBUF] dfree[NBUF] drain
   static constexpr int OFF_MISC = OFF_BAR + (2 * NSTG + 2 * NBUF + 1) * 8;   // tmem slot, abort flag, issued[NSTG]
-  static constexpr int OFF_RED = OFF_MISC + 8 + 4 * NSTG;                   // [NGRP][row parity][hi GW, lo GW]
-  static constexpr int BYTES = OFF_RED + NGRP * 2 * 2 * GW * 4 + 1024;
-  static_assert(OFF_RED + NGRP * 2 * 2 * GW * 4 <= OFF_BAR + MISC, "misc area");
+  // each warp's lanes belong to one row: per-quadrant partials; else atomics
+  static constexpr bool QUADS = RPS == 1 || F % 32 == 0;
+  static constexpr int OFF_RED = OFF_MISC + 8 + 4 * NSTG;   // QUADS: float [NGRP][2][hi GW, lo GW]; else int [NGRP][3][RPS][hi, lo]
+  static constexpr int REDB = QUADS ? NGRP * 2 * 2 * GW * 4 : NGRP * 3 * RPS * 2 * 4;
+  static constexpr int BYTES = OFF_RED + REDB + 1024;
+  static_assert(OFF_RED + REDB <= OFF_BAR + MISC, "misc area");
   static_assert(BYTES <= kTcSmemBudget, "shared memory");
 };
+
+// Order-preserving map between float bit patterns and signed ints (an
+// involution), so that atomicMax / atomicMin on ints give the float max / min.
+__device__ __forceinline__ int f2ord(float f) {
+  const int b = __float_as_int(f);
+  return b >= 0 ? b : b ^ 0x7FFFFFFF;
+}
+__device__ __forceinline__ float ord2f(int b) { return __int_as_float(b >= 0 ? b : b ^ 0x7FFFFFFF); }
 
 // byte offset of byte b of row r in a block of 128-byte rows with the 128-byte swizzle
 __device__ __forceinline__ uint32_t sw128(uint32_t r, uint32_t b) {
@@ -140,10 +152,10 @@ __device__ __forceinline__ bool tc_bar_or(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
-template <int NS, int JH, bool SYM, bool CLAMP>
-__global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
-    rq_paley_tc_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
-  using S = RqTc<NS, JH>;
+template <int F, int RPS, bool SYM, bool CLAMP>
+__global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
+    rq_tc_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
+  using S = RqTc<F, RPS>;
   constexpr int MR = S::MR, KS = S::KS, NSTG = S::NSTG, NBUF = S::NBUF, NGRP = S::NGRP;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-aligned base, derived from the shared array itself
@@ -156,15 +168,18 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + S::OFF_MISC + 4);
   int* issued = reinterpret_cast<int*>(smem + S::OFF_MISC + 8);      // last iteration copied into stage s
-  float* red = reinterpret_cast<float*>(smem + S::OFF_RED);           // [group][row parity][hi 4, lo 4]
+  int* rslot = reinterpret_cast<int*>(smem + S::OFF_RED);            // [group][row % 3][r][hi, lo]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t r0 = blockIdx.x, G = gridDim.x;
-  const int64_t units = a.rows / S::RPS;   // MMAs (RPS rows each)
+  const int64_t units = a.rows / RPS;   // MMAs (RPS rows each)
   const int niter = units > r0 ? (int)((units - r0 + G - 1) / G) : 0;
 
-  // T in the MMA's A layout (K-major, 128-byte swizzle): element (m, k) at K
-  // atom k / 64, row m, bytes 2 (k % 64); zero outside MR.  Paley: T =
-  // H_s^T (x) H_4^T, m = 4 i + jh; Sylvester: T = I_RPS (x) H_JH, m = JH r + jh
+  // T = I_RPS (x) H_f^T in the MMA's A layout (K-major, 128-byte swizzle):
+  // element (m, k) at K atom k / 64, row m, bytes 2 (k % 64); m = F r + a,
+  // a = i JHB + jh; T[(r, a)][(r, a')] = H_s[i'][i] H_JHB[jh'][jh], zero
+  // between different rows r and outside MR
+  const int lj = __ffs(a.n_pow2) - 8;   // log2(P / 128): P is a power of two
+  const int jm = (1 << lj) - 1;
   for (int e = tid; e < 128 * 64; e += S::THREADS) {
     const int m = e >> 6, k = (e & 63) * 2;
     float v[2];
@@ -172,14 +187,11 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
     for (int q = 0; q < 2; ++q) {
       const int kk = k + q;
       float t = 0.f;
-      if (m < MR && kk < MR) {
-        if constexpr (S::PALEY) {
-          const int i = m >> 2, jh = m & 3, ip = kk >> 2, jhp = kk & 3;
-          const uint32_t neg = ((a.hs.neg[ip] >> i) & 1u) ^ (uint32_t)(__popc(jh & jhp) & 1);
-          t = neg ? -1.f : 1.f;
-        } else if (m / JH == kk / JH) {
-          t = (__popc((m % JH) & (kk % JH)) & 1) ? -1.f : 1.f;
-        }
+      if (m < MR && kk < MR && m / F == kk / F) {
+        const int am = m % F, ak = kk % F;
+        const int i = am >> lj, jh = am & jm, ip = ak >> lj, jhp = ak & jm;
+        const uint32_t ps = a.n_small > 1 ? (a.hs.neg[ip] >> i) & 1u : 0u;
+        t = (ps ^ (uint32_t)(__popc(jh & jhp) & 1)) ? -1.f : 1.f;
       }
       v[q] = t;
     }
@@ -197,6 +209,11 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
       mbar_init(&dfree[b], S::GW);
     }
     mbar_init(drain, 1);
+    if (!S::QUADS)
+      for (int e = 0; e < S::REDB / 8; ++e) {   // every slot at its identity
+        rslot[2 * e] = SYM ? 0 : INT_MIN;
+        rslot[2 * e + 1] = INT_MAX;
+      }
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmx);
@@ -252,14 +269,12 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
     // quadrant): butterflies, range, Eq. 1, codes
     constexpr int GW = S::GW;
     const int gw = warp - 2, grp = gw / GW, quad = warp & 3;
-    const int m = quad * 32 + lane;   // this thread's lane: (i, jh) = (m / 4, m % 4) or (r, jh) = (m / JH, m % JH)
+    const int m = quad * 32 + lane;   // this thread's lane: row r = m / F, block a = m % F
     const bool live = m < MR;
-    const int rr_ = m / S::LPR;       // its input row within the MMA
-    // the lane quadrants holding that row
-    const int q_lo = (rr_ * S::LPR) / 32, q_hi = ((rr_ + 1) * S::LPR - 1) / 32;
+    const int rr_ = live ? m / F : 0;  // its input row within the MMA
     for (int it = grp; it < niter; it += NGRP) {
       const int b = it % NBUF;
-      const int64_t row = (r0 + (int64_t)it * G) * S::RPS + rr_;
+      const int64_t row = (r0 + (int64_t)it * G) * RPS + rr_;
       // on a failed wait the accumulator is read anyway (in bounds, discarded below)
       const bool ok = tc_wait(&dfull[b], (uint32_t)(it / NBUF) & 1u, abort_flag);
       __syncwarp();   // the tensor-memory loads below are warp-collective
@@ -285,10 +300,9 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
 #pragma unroll
         for (int p = 0; p < 64; ++p)
           if (!(p & h)) f2_bfly(z[p], z[p | h]);
-      // row range: four partial ranges (short dependency chains), then the
-      // warp and the group's warps (scratch alternates between the group's
-      // rows, so one barrier per row suffices); the same barrier settles the
-      // abort decision for every thread of the group
+      // row range: four partial ranges per thread (short dependency chains),
+      // then over the row's lanes; the group barrier also settles the abort
+      // decision for every thread of the group
       Range<SYM> rg[4];
       if (live) {
 #pragma unroll
@@ -299,26 +313,67 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
         rg[0].hi = fmaxf(rg[0].hi, rg[q].hi);
         if (!SYM) rg[0].lo = fminf(rg[0].lo, rg[q].lo);
       }
-      rg[0].warp_reduce();
-      float* rd = red + (grp * 2 + ((it / NGRP) & 1)) * 2 * GW;
-      if (lane == 0) {
-        rd[quad] = rg[0].hi;
-        rd[GW + quad] = rg[0].lo;
-      }
-      if (tc_bar_or(1 + grp, 32 * GW, !ok || *abort_flag)) break;
+      const int qrow = it / NGRP;
       Range<SYM> rr;
-      rr.hi = rd[q_lo];
-      rr.lo = rd[GW + q_lo];
-#pragma unroll
-      for (int q = 0; q < GW; ++q)
-        if (q > q_lo && q <= q_hi) {
-          rr.hi = fmaxf(rr.hi, rd[q]);
-          if (!SYM) rr.lo = fminf(rr.lo, rd[GW + q]);
+      if constexpr (S::QUADS) {
+        // one warp reduction, the partials of the quadrants holding the row
+        // (scratch alternates between the group's rows: one barrier per row)
+        rg[0].warp_reduce();
+        float* rd = reinterpret_cast<float*>(rslot) + (grp * 2 + (qrow & 1)) * 2 * GW;
+        if (lane == 0) {
+          rd[quad] = rg[0].hi;
+          rd[GW + quad] = rg[0].lo;
         }
+        if (tc_bar_or(1 + grp, 32 * GW, !ok || *abort_flag)) break;
+        const int q_lo = (rr_ * F) / 32, q_hi = ((rr_ + 1) * F - 1) / 32;
+        rr.hi = rd[q_lo];
+        rr.lo = rd[GW + q_lo];
+#pragma unroll
+        for (int q = 0; q < GW; ++q)
+          if (q > q_lo && q <= q_hi && q * 32 < MR) {
+            rr.hi = fmaxf(rr.hi, rd[q]);
+            if (!SYM) rr.lo = fminf(rr.lo, rd[GW + q]);
+          }
+      } else {
+        // rows share warps: masked warp reductions per row the warp's lanes
+        // span, then shared-memory atomics on order-preserving ints (slot
+        // sets rotate over three rows: set q + 1 is reset before this row's
+        // barrier, after every thread has read it for row q - 2)
+        int* set = rslot + (grp * 3 + qrow % 3) * RPS * 2;
+        if (gw % GW == 0 && lane == 0) {
+          int* nxt = rslot + (grp * 3 + (qrow + 1) % 3) * RPS * 2;
+          for (int r = 0; r < RPS; ++r) {
+            nxt[2 * r] = SYM ? 0 : INT_MIN;
+            nxt[2 * r + 1] = INT_MAX;
+          }
+        }
+        constexpr int NRW = F >= 32 ? 2 : 3;
+        const int row0 = (quad * 32) / F;
+#pragma unroll
+        for (int k = 0; k < NRW; ++k) {
+          const int rk = row0 + k;
+          const bool mine = live && rr_ == rk;
+          Range<SYM> w;
+          if (mine) w = rg[0];
+          w.warp_reduce();
+          const bool any = __any_sync(0xffffffffu, mine);
+          if (lane == 0 && any) {
+            if (SYM) {
+              atomicMax(&set[2 * rk], __float_as_int(w.hi));   // hi >= 0
+            } else {
+              atomicMax(&set[2 * rk], f2ord(w.hi));
+              atomicMin(&set[2 * rk + 1], f2ord(w.lo));
+            }
+          }
+        }
+        if (tc_bar_or(1 + grp, 32 * GW, !ok || *abort_flag)) break;
+        rr.hi = SYM ? __int_as_float(set[2 * rr_]) : ord2f(set[2 * rr_]);
+        if (!SYM) rr.lo = ord2f(set[2 * rr_ + 1]);
+      }
       const QParams<SYM> qp(rr, a.clip);
       if (live) {
-        // codes of elements 128 (m % LPR) .. + 127 of the row: 64 contiguous bytes
-        uint4* out = reinterpret_cast<uint4*>(a.codes + row * (a.K / 2) + (int64_t)(m % S::LPR) * 64);
+        // codes of elements 128 a .. 128 a + 127 of row r: 64 contiguous bytes
+        uint4* out = reinterpret_cast<uint4*>(a.codes + row * (a.K / 2) + (int64_t)(m % F) * 64);
 #pragma unroll
         for (int w4 = 0; w4 < 4; ++w4) {
           uint32_t wd[4];
@@ -332,7 +387,7 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
           out[w4] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
         }
       }
-      if (live && m % S::LPR == 0) {
+      if (live && m % F == 0) {
         a.scale[row] = qp.alpha * a.norm;
         if (!SYM) a.zero[row] = qp.beta * a.norm;
       }
@@ -350,32 +405,28 @@ __global__ void __launch_bounds__(RqTc<NS, JH>::THREADS, 1)
   if (warp == 1) tmem_dealloc(tmem, S::TMEM_COLS);
 }
 
-template <int NS, int JH, bool SYM, bool CLAMP>
+template <int F, int RPS, bool SYM, bool CLAMP>
 cudaError_t launch_tc(const RotQuantArgs& a, cudaStream_t stream) {
-  using S = RqTc<NS, JH>;
+  using S = RqTc<F, RPS>;
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return cudaErrorNotSupported;
-  // Paley: a row as (jl % 64, jh, i, jl / 64); Sylvester: RPS rows as
-  // (jl % 64, jh, r, jl / 64): two 64-column atoms of MR 128-byte rows
+  // RPS rows as (jl % 64, a, r, jl / 64): two 64-column atoms of MR
+  // 128-byte rows (r, a) (a indexes the row's 128-element blocks)
   CUtensorMap tmx;
   const cuuint64_t ld = (cuuint64_t)(a.ldx * 2);
-  const cuuint64_t gdim_p[5] = {64, 4, (cuuint64_t)NS, 2, (cuuint64_t)a.rows};
-  const cuuint64_t gstr_p[4] = {256, 1024, 128, ld};
-  const cuuint32_t box_p[5] = {64, 4, (cuuint32_t)NS, 2, 1};
-  const cuuint64_t gdim_s[5] = {64, (cuuint64_t)JH, (cuuint64_t)S::RPS, 2, (cuuint64_t)(a.rows / S::RPS)};
-  const cuuint64_t gstr_s[4] = {256, ld, 128, ld * S::RPS};
-  const cuuint32_t box_s[5] = {64, (cuuint32_t)JH, (cuuint32_t)S::RPS, 2, 1};
+  const cuuint64_t gdim[5] = {64, (cuuint64_t)F, (cuuint64_t)RPS, 2, (cuuint64_t)(a.rows / RPS)};
+  const cuuint64_t gstr[4] = {256, ld, 128, ld * RPS};
+  const cuuint32_t box[5] = {64, (cuuint32_t)F, (cuuint32_t)RPS, 2, 1};
   const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-  if (enc(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<void*>(a.x), S::PALEY ? gdim_p : gdim_s,
-          S::PALEY ? gstr_p : gstr_s, S::PALEY ? box_p : box_s, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  if (enc(&tmx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<void*>(a.x), gdim, gstr, box, estr,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorNotSupported;
-  auto kern = rq_paley_tc_kernel<NS, JH, SYM, CLAMP>;
+  auto kern = rq_tc_kernel<F, RPS, SYM, CLAMP>;
   int per_sm = 0;
   cudaError_t e = prepare_launch_tmem(kern, S::THREADS, S::BYTES, S::TMEM_COLS, &per_sm);
   if (e != cudaSuccess) return e;
-  const int64_t units = a.rows / S::RPS;
+  const int64_t units = a.rows / RPS;
   const int64_t cap = (int64_t)device_sm_count() * per_sm;
   const int64_t grid = units < cap ? units : cap;
   RotQuantArgs la = a;
@@ -385,54 +436,32 @@ cudaError_t launch_tc(const RotQuantArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-template <bool SYM, bool CLAMP>
-cudaError_t launch_tc_ns(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
-  *handled = true;
-  switch (a.n_small) {
-    case 12: return launch_tc<12, 0, SYM, CLAMP>(a, stream);
-    case 20: return launch_tc<20, 0, SYM, CLAMP>(a, stream);
-    case 28: return launch_tc<28, 0, SYM, CLAMP>(a, stream);
-  }
-  *handled = false;
-  return cudaSuccess;
-}
-
-template <bool SYM, bool CLAMP>
-cudaError_t launch_tc_pow2(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
-  *handled = true;
-  switch (a.n_pow2) {
-    case 8192: return launch_tc<0, 64, SYM, CLAMP>(a, stream);
-    case 16384: return launch_tc<0, 128, SYM, CLAMP>(a, stream);
-  }
-  *handled = false;
-  return cudaSuccess;
+template <int F, int RPS>
+cudaError_t launch_tc_f(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+  *handled = a.rows % RPS == 0;
+  if (!*handled) return cudaSuccess;
+  const bool clamp = a.clip < 1.0f;
+  if (a.symmetric) return clamp ? launch_tc<F, RPS, true, true>(a, stream) : launch_tc<F, RPS, true, false>(a, stream);
+  return clamp ? launch_tc<F, RPS, false, true>(a, stream) : launch_tc<F, RPS, false, false>(a, stream);
 }
 
 }  // namespace
 
-cudaError_t set_wait_limit_paley_tc(uint64_t ns) { return cudaMemcpyToSymbol(g_tc_wait_ns, &ns, sizeof(ns)); }
+cudaError_t set_wait_limit_rq_tc(uint64_t ns) { return cudaMemcpyToSymbol(g_tc_wait_ns, &ns, sizeof(ns)); }
 
-cudaError_t launch_rotate_quant_act_paley_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
+cudaError_t launch_rotate_quant_act_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
   *handled = false;
-  if (a.rows == 0 || a.rowsum || a.signs || a.n_pow2 != 512) return cudaSuccess;
-  if (a.n_small != 12 && a.n_small != 20 && a.n_small != 28) return cudaSuccess;
-  if ((a.ldx * 2) % 16 != 0 || a.K != (int64_t)a.n_small * 512) return cudaSuccess;
-  const bool clamp = a.clip < 1.0f;
-  if (a.symmetric)
-    return clamp ? launch_tc_ns<true, true>(a, stream, handled) : launch_tc_ns<true, false>(a, stream, handled);
-  return clamp ? launch_tc_ns<false, true>(a, stream, handled) : launch_tc_ns<false, false>(a, stream, handled);
-}
-
-cudaError_t launch_rotate_quant_act_pow2_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled) {
-  *handled = false;
-  if (a.rows == 0 || a.rowsum || a.signs || a.n_small != 1) return cudaSuccess;
-  if (a.n_pow2 != 8192 && a.n_pow2 != 16384) return cudaSuccess;
-  const int64_t rps = 16384 / a.n_pow2;   // rows per MMA
-  if (a.rows % rps != 0 || (a.ldx * 2) % 16 != 0 || a.K != a.n_pow2) return cudaSuccess;
-  const bool clamp = a.clip < 1.0f;
-  if (a.symmetric)
-    return clamp ? launch_tc_pow2<true, true>(a, stream, handled) : launch_tc_pow2<true, false>(a, stream, handled);
-  return clamp ? launch_tc_pow2<false, true>(a, stream, handled) : launch_tc_pow2<false, false>(a, stream, handled);
+  if (a.rows == 0 || a.rowsum || a.signs || a.n_small < 1 || a.n_pow2 < 128 || a.n_pow2 % 128 != 0) return cudaSuccess;
+  if ((a.ldx * 2) % 16 != 0 || a.K != (int64_t)a.n_small * a.n_pow2) return cudaSuccess;
+  // the block counts F = n_s P / 128 with an instance (RPS rows per MMA)
+  switch (a.n_small * (a.n_pow2 / 128)) {
+    case 112: return launch_tc_f<112, 1>(a, stream, handled);   // H_28 (x) H_512
+    case 80: return launch_tc_f<80, 1>(a, stream, handled);     // H_20 (x) H_512
+    case 48: return launch_tc_f<48, 2>(a, stream, handled);     // H_12 (x) H_512
+    case 64: return a.n_small == 1 ? launch_tc_f<64, 2>(a, stream, handled) : cudaSuccess;     // H_8192
+    case 128: return a.n_small == 1 ? launch_tc_f<128, 1>(a, stream, handled) : cudaSuccess;   // H_16384
+  }
+  return cudaSuccess;
 }
 
 }  // namespace spinq

@@ -49,15 +49,12 @@ cudaError_t launch_rotate_quant_act_fast(const RotQuantArgs& a, cudaStream_t str
 // {128, 256, 512}).  Sets *handled = false for other shapes.
 cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
 
-// The same for P = 512 without random signs on the 5th-generation tensor
-// core (rotate_quant_paley_tc.cu); launch_rotate_quant_act_paley tries it
-// first.  Sets *handled = false for other shapes.
-cudaError_t launch_rotate_quant_act_paley_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
-cudaError_t set_wait_limit_paley_tc(uint64_t ns);
-// A Sylvester rotation of 8192 or 16384 points (rows a multiple of
-// 16384 / P, no random signs) on the same kernel; launch_rotate_quant_act_fast
-// tries it first.  Sets *handled = false for other shapes.
-cudaError_t launch_rotate_quant_act_pow2_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
+// Rotate+quant on the 5th-generation tensor core (rotate_quant_paley_tc.cu)
+// for plain rotations H_s (x) H_P whose block count n_s P / 128 has an
+// instance (H_28, H_20, H_12 with P = 512; Sylvester 8192 and 16384) and a row count those rows-per-MMA divide; the Paley and
+// power-of-two launchers try it first.  Sets *handled = false otherwise.
+cudaError_t launch_rotate_quant_act_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
+cudaError_t set_wait_limit_rq_tc(uint64_t ns);
 
 struct KVArgs {
   const void* q_in;

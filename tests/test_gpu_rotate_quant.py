@@ -72,7 +72,7 @@ def test_act_shapes_and_modes(S, had, symmetric):
     check_act(S, x, had, symmetric, 1.0, f"had={had} sym={symmetric}")
 
 
-@pytest.mark.parametrize("had,rows", [((1, 8192), 38), ((1, 8192), 2), ((1, 16384), 37), ((12, 512), 5),
+@pytest.mark.parametrize("had,rows", [((1, 8192), 38), ((1, 8192), 2), ((1, 16384), 37), ((12, 512), 6), ((12, 512), 5),
                                       ((20, 512), 64)])
 @pytest.mark.parametrize("symmetric", [True, False])
 def test_act_tensor_core_rotation_shapes(S, had, rows, symmetric):
