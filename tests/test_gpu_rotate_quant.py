@@ -72,23 +72,25 @@ def test_act_shapes_and_modes(S, had, symmetric):
     check_act(S, x, had, symmetric, 1.0, f"had={had} sym={symmetric}")
 
 
-@pytest.mark.parametrize("had,rows", [((1, 8192), 38), ((1, 8192), 2), ((1, 16384), 37), ((12, 512), 6), ((12, 512), 5),
-                                      ((20, 512), 64)])
+@pytest.mark.parametrize("had,rows", [((1, 8192), 306), ((1, 8192), 2), ((1, 16384), 153), ((12, 512), 306),
+                                      ((12, 512), 305), ((20, 512), 160)])
 @pytest.mark.parametrize("symmetric", [True, False])
 def test_act_tensor_core_rotation_shapes(S, had, rows, symmetric):
-    """The tcgen05 rotate+quant kernel: Sylvester 8192 (two rows per MMA, an
-    even row count) and 16384, Paley factors with few and many lanes."""
+    """The tcgen05 rotate+quant kernel (at least one MMA per SM): Sylvester
+    8192 (two rows per MMA) and 16384, Paley factors with few and many lanes
+    (H_12 (x) H_512: two rows per MMA sharing warps); odd and small row
+    counts take the other kernels."""
     K = had[0] * had[1]
     rng = np.random.default_rng(K + rows + symmetric)
     x = synth.activations(rng, rows, K, outlier_frac=0.02, factor=25.0)
     check_act(S, x, had, symmetric, 1.0, f"had={had} rows={rows} sym={symmetric}")
 
 
-@pytest.mark.parametrize("had", [(12, 256), (28, 512), (1, 8192)])
+@pytest.mark.parametrize("had,rows", [((12, 256), 64), ((28, 512), 64), ((28, 512), 160), ((1, 8192), 320)])
 @pytest.mark.parametrize("symmetric,clip", [(True, 0.9), (False, 0.9), (False, 0.5)])
-def test_act_clipping(S, had, symmetric, clip):
+def test_act_clipping(S, had, rows, symmetric, clip):
     rng = np.random.default_rng(9)
-    x = synth.activations(rng, 64, had[0] * had[1], outlier_frac=0.01, factor=30.0)
+    x = synth.activations(rng, rows, had[0] * had[1], outlier_frac=0.01, factor=30.0)
     check_act(S, x, had, symmetric, clip, f"had={had} clip={clip}")
 
 
