@@ -537,7 +537,7 @@ def run_ours(args, rank, world, local_rank):
             "traffic": gemm_traffic_from_profile(f"w4a4_gemm_down_proj_M{M}_K{K2}_N{N2}.md", GEMM_KERNELS[kind2][1]),
         },
         "rotate_quant_roofline": {
-            "bound": "hbm", "kernel": "rq_paley_tc_kernel (R4 = H28 (x) H512 + act quant on tcgen05, 2048 x 14336, sym)",
+            "bound": "hbm", "kernel": "rq_tc_kernel (R4 = H28 (x) H512 + act quant on tcgen05, 2048 x 14336, sym)",
             "achieved": round(rq2_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
             "frac": round(rq2_gbs / hbm_peak, 4), "us": round(t_rq2 * 1e6, 2),
             "isolated_us": round(iso["r4_quant"] * 1e6, 2),
@@ -1061,7 +1061,7 @@ def relaunch(args_n):
 
 
 PROFILE_CASES = ("attention", "rope_kv", "fp8_gemm", "w4a8_gemm", "rq8_paley", "cayley", "paley", "gemm",
-                 "gemm_gate_up", "decode_gemm", "decode_gemm16")
+                 "gemm_gate_up", "decode_gemm", "decode_gemm16", "rq_h8192")
 
 
 def profile_case(name, reps):
@@ -1076,7 +1076,8 @@ def profile_case(name, reps):
     2048 x 14336; gemm: the W4A4 down_proj 2048 x 14336 -> 4096; gemm_gate_up:
     the W4A4 gate_up 2048 x 4096 -> 14336 (asymmetric activations);
     decode_gemm: 8 tokens through 4096 -> 14336 on the automatic route;
-    decode_gemm16: 16 tokens through 3072 -> 8192 on the automatic route."""
+    decode_gemm16: 16 tokens through 3072 -> 8192 on the automatic route;
+    rq_h8192: the 4-bit R4 kernel with H8192 on 8192 x 8192 (asymmetric)."""
     import numpy as np
     import torch
 
@@ -1118,6 +1119,10 @@ def profile_case(name, reps):
             qa = spinq.rotate_quant_act(x, c.had)
             qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), c.had)
             fn = lambda: spinq.w4a4_gemm(qa, qw)
+    elif name == "rq_h8192":
+        c = synth.llama32_3b_down(M=8192)
+        x8 = torch.from_numpy(c.x).to(dev)
+        fn = lambda: spinq.rotate_quant_act(x8, c.had, c.act_symmetric)
     elif name == "gemm_gate_up":
         c = synth.llama3_8b_gate_up()
         qa = spinq.rotate_quant_act(torch.from_numpy(c.x).to(dev), None, False)
