@@ -36,10 +36,13 @@
 //    group), Eq. 1 and the codes.
 // T is written once per CTA into shared memory (K-major, 128-byte swizzle).
 //
-// Every wait is bounded in time (polled, the limit checked every 256
-// polls); a wait that gives up raises the CTA's abort flag, the
-// others see it at their next wait, the MMA thread drains its MMAs and the
-// copy thread lets its copies land before tensor memory is released.
+// Every wait is bounded in time; a wait that gives up raises the CTA's abort
+// flag, the others see it at their next wait, the MMA thread drains its MMAs
+// and the copy thread lets its copies land before tensor memory is released.
+// The quantizer groups poll (a suspended wait woke up late); the copy thread,
+// which runs rows ahead, sleeps between polls and leaves the issue slots to
+// the groups on its sub-partition, and so does the MMA thread where an MMA
+// covers two rows.
 #include <cuda_fp16.h>
 
 #include <climits>
@@ -93,8 +96,9 @@ struct RqTc {
   static constexpr bool QUADS = RPS == 1 || F % 32 == 0;
   static constexpr int OFF_RED = OFF_MISC + 8 + 4 * NSTG;   // QUADS: float [NGRP][2][hi GW, lo GW]; else int [NGRP][3][RPS][hi, lo]
   static constexpr int REDB = QUADS ? NGRP * 2 * 2 * GW * 4 : NGRP * 3 * RPS * 2 * 4;
-  static constexpr int BYTES = OFF_RED + REDB + 1024;
-  static_assert(OFF_RED + REDB <= OFF_BAR + MISC, "misc area");
+  static constexpr int OFF_NEG = OFF_RED + REDB;   // the Paley sign words hs.neg[32]
+  static constexpr int BYTES = OFF_NEG + 128 + 1024;
+  static_assert(OFF_NEG + 128 <= OFF_BAR + MISC, "misc area");
   static_assert(BYTES <= kTcSmemBudget, "shared memory");
 };
 
@@ -169,35 +173,18 @@ __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + S::OFF_MISC + 4);
   int* issued = reinterpret_cast<int*>(smem + S::OFF_MISC + 8);      // last iteration copied into stage s
   int* rslot = reinterpret_cast<int*>(smem + S::OFF_RED);            // [group][row % 3][r][hi, lo]
+  uint32_t* neg_s = reinterpret_cast<uint32_t*>(smem + S::OFF_NEG);  // H_s sign words (0 for n_s = 1)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t r0 = blockIdx.x, G = gridDim.x;
   const int64_t units = a.rows / RPS;   // MMAs (RPS rows each)
   const int niter = units > r0 ? (int)((units - r0 + G - 1) / G) : 0;
 
-  // T = I_RPS (x) H_f^T in the MMA's A layout (K-major, 128-byte swizzle):
-  // element (m, k) at K atom k / 64, row m, bytes 2 (k % 64); m = F r + a,
-  // a = i JHB + jh; T[(r, a)][(r, a')] = H_s[i'][i] H_JHB[jh'][jh], zero
-  // between different rows r and outside MR
-  const int lj = __ffs(a.n_pow2) - 8;   // log2(P / 128): P is a power of two
-  const int jm = (1 << lj) - 1;
-  for (int e = tid; e < 128 * 64; e += S::THREADS) {
-    const int m = e >> 6, k = (e & 63) * 2;
-    float v[2];
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const int kk = k + q;
-      float t = 0.f;
-      if (m < MR && kk < MR && m / F == kk / F) {
-        const int am = m % F, ak = kk % F;
-        const int i = am >> lj, jh = am & jm, ip = ak >> lj, jhp = ak & jm;
-        const uint32_t ps = a.n_small > 1 ? (a.hs.neg[ip] >> i) & 1u : 0u;
-        t = (ps ^ (uint32_t)(__popc(jh & jhp) & 1)) ? -1.f : 1.f;
-      }
-      v[q] = t;
-    }
-    *reinterpret_cast<uint32_t*>(smem + S::OFF_T + (k >> 6) * 16384 + sw128(m, (k & 63) * 2)) =
-        pack_half2_bits(v[0], v[1]);
-  }
+  // one TMA tensor copy: the RPS rows of iteration `it` into stage s
+  auto copy_row = [&](int it, int s) {
+    mbar_arrive_expect_tx(&full[s], (uint32_t)S::ROWB);
+    tma_load_5d(smem + S::OFF_STG + s * S::ROWB, &tmx, &full[s], 0, 0, 0, 0, (int32_t)(r0 + (int64_t)it * G));
+    issued[s] = it;
+  };
   if (tid == 0) {
     for (int s = 0; s < NSTG; ++s) {
       mbar_init(&full[s], 1);
@@ -214,6 +201,10 @@ __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
         rslot[2 * e] = SYM ? 0 : INT_MIN;
         rslot[2 * e + 1] = INT_MAX;
       }
+    // constant indexes: a lane-dependent index into the parameter space
+    // would serialize over the distinct words
+#pragma unroll
+    for (int q = 0; q < 32; ++q) neg_s[q] = a.n_small > 1 ? a.hs.neg[q] : 0u;
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmx);
@@ -221,6 +212,46 @@ __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
   if (warp == 1) {
     tmem_alloc(tmem_slot, S::TMEM_COLS);
     tmem_relinquish();
+  }
+  __syncthreads();   // barriers and sign words
+  // the first pass over the ring is issued before T is built, so the first
+  // rows land while the CTA sets up (measured: issuing two first and the
+  // rest once row 0 is in was slower, 18.3 against 17.3 us on 2048 x 14336)
+  const int it0 = a.debug_stall ? 0 : (niter < NSTG ? niter : NSTG);
+  if (tid == 0) {
+    pdl_wait();
+    for (int it = 0; it < it0; ++it) copy_row(it, it);
+  }
+
+  // T = I_RPS (x) H_f^T in the MMA's A layout (K-major, 128-byte swizzle):
+  // element (m, k) at K atom k / 64, row m, bytes 2 (k % 64); m = F r + a,
+  // a = i JHB + jh; T[(r, a)][(r, a')] = H_s[i'][i] H_JHB[jh'][jh], zero
+  // between different rows r and outside MR.  A warp writes one row m per
+  // step, lane l the four k = 4 l .. 4 l + 3 (their terms fixed per lane).
+  {
+    const int lj = __ffs(a.n_pow2) - 8;   // log2(P / 128): P is a power of two
+    const int jm = (1 << lj) - 1;
+    uint32_t wk[4];
+    int jk[4], rk[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int kk = 4 * lane + q, ak = kk % F;
+      wk[q] = neg_s[ak >> lj];
+      jk[q] = ak & jm;
+      rk[q] = kk < MR ? kk / F : -1;
+    }
+    uint8_t* tl = smem + S::OFF_T + (lane >> 4) * 16384;
+    for (int m = warp; m < 128; m += S::THREADS / 32) {
+      const int am = m % F, rm = m < MR ? m / F : -2;
+      const int i = am >> lj, jh = am & jm;
+      uint32_t h[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t sg = ((wk[q] >> i) ^ (uint32_t)__popc(jh & jk[q])) & 1u;
+        h[q] = rk[q] == rm ? (0x3C00u | (sg << 15)) : 0u;   // fp16 +-1 or 0
+      }
+      *reinterpret_cast<uint2*>(tl + sw128(m, (lane & 15) * 8)) = make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
+    }
   }
   fence_proxy_async_smem();   // T, written by ordinary stores, is read by the tensor core
   tc_fence_before();
@@ -233,12 +264,10 @@ __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
   if (warp == 0) {
     // ---------------- copies: one TMA tensor copy per row
     if (lane == 0 && !a.debug_stall) {   // a test of the time-outs issues no copies
-      for (int it = 0; it < niter; ++it) {
+      for (int it = it0; it < niter; ++it) {
         const int s = it % NSTG;
-        if (it >= NSTG && !tc_wait(&sfree[s], (uint32_t)((it / NSTG) - 1) & 1u, abort_flag)) break;
-        mbar_arrive_expect_tx(&full[s], (uint32_t)S::ROWB);
-        tma_load_5d(smem + S::OFF_STG + s * S::ROWB, &tmx, &full[s], 0, 0, 0, 0, (int32_t)(r0 + (int64_t)it * G));
-        issued[s] = it;
+        if (!mbar_wait_backoff(&sfree[s], (uint32_t)((it / NSTG) - 1) & 1u, abort_flag, g_tc_wait_ns)) break;
+        copy_row(it, s);
       }
     }
   } else if (warp == 1) {
@@ -246,10 +275,16 @@ __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = umma_idesc_f16_f32_bmn(128, 128);
       const uint32_t tb = smem_u32(smem + S::OFF_T), sb0 = smem_u32(smem + S::OFF_STG);
+      // with two rows per MMA this thread sleeps between polls (H_8192 on
+      // 8192 x 8192: 33.2 against 36.8 us polling); with one it polls
+      // (H_28 (x) H_512 on 2048 x 14336: 17.3 against 17.8 us sleeping)
+      auto mma_wait = [&](uint64_t* bar, uint32_t parity) {
+        return RPS > 1 ? mbar_wait_backoff(bar, parity, abort_flag, g_tc_wait_ns) : tc_wait(bar, parity, abort_flag);
+      };
       for (int it = 0; it < niter; ++it) {
         const int s = it % NSTG, b = it % NBUF;
-        if (!tc_wait(&full[s], (uint32_t)(it / NSTG) & 1u, abort_flag)) break;
-        if (it >= NBUF && !tc_wait(&dfree[b], (uint32_t)((it / NBUF) - 1) & 1u, abort_flag)) break;
+        if (!mma_wait(&full[s], (uint32_t)(it / NSTG) & 1u)) break;
+        if (it >= NBUF && !mma_wait(&dfree[b], (uint32_t)((it / NBUF) - 1) & 1u)) break;
         tc_fence_after();
         const uint32_t sb = sb0 + (uint32_t)(s * S::ROWB);
         // E = T [X0 | X1]: columns 0..63 E0 = T X0, columns 64..127 E1 = T X1
