@@ -496,6 +496,7 @@ cudaError_t launch_rotate_quant_act_tc(const RotQuantArgs& a, cudaStream_t strea
     case 112: return launch_tc_f<112, 1>(a, stream, handled);   // H_28 (x) H_512
     case 80: return launch_tc_f<80, 1>(a, stream, handled);     // H_20 (x) H_512
     case 48: return launch_tc_f<48, 2>(a, stream, handled);     // H_12 (x) H_512
+    case 24: return launch_tc_f<24, 4>(a, stream, handled);     // H_12 (x) H_256 (19.6 against 20.2 us on 8192 x 3072)
     case 64: return a.n_small == 1 ? launch_tc_f<64, 2>(a, stream, handled) : cudaSuccess;     // H_8192
     case 128: return a.n_small == 1 ? launch_tc_f<128, 1>(a, stream, handled) : cudaSuccess;   // H_16384
   }

@@ -51,10 +51,10 @@ cudaError_t launch_rotate_quant_act_paley(const RotQuantArgs& a, cudaStream_t st
 
 // Rotate+quant on the 5th-generation tensor core (rotate_quant_paley_tc.cu)
 // for plain rotations H_s (x) H_P whose block count n_s P / 128 has an
-// instance (H_28, H_20, H_12 with P = 512; Sylvester 8192 and 16384) and a
-// row count those rows-per-MMA divide into at least one MMA per SM; the
-// Paley and power-of-two launchers try it first.  Sets *handled = false
-// otherwise.
+// instance (H_28, H_20, H_12 with P = 512; H_12 with P = 256; Sylvester 8192
+// and 16384) and a row count those rows-per-MMA divide into at least one MMA
+// per SM; the Paley and power-of-two launchers try it first.  Sets
+// *handled = false otherwise.
 cudaError_t launch_rotate_quant_act_tc(const RotQuantArgs& a, cudaStream_t stream, bool* handled);
 cudaError_t set_wait_limit_rq_tc(uint64_t ns);
 

@@ -73,7 +73,7 @@ def test_act_shapes_and_modes(S, had, symmetric):
 
 
 @pytest.mark.parametrize("had,rows", [((1, 8192), 306), ((1, 8192), 2), ((1, 16384), 153), ((12, 512), 306),
-                                      ((12, 512), 305), ((20, 512), 160)])
+                                      ((12, 512), 305), ((20, 512), 160), ((12, 256), 612), ((12, 256), 610)])
 @pytest.mark.parametrize("symmetric", [True, False])
 def test_act_tensor_core_rotation_shapes(S, had, rows, symmetric):
     """The tcgen05 rotate+quant kernel (at least one MMA per SM): Sylvester
