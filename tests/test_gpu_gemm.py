@@ -295,6 +295,48 @@ def test_rotated_linear_end_to_end(S, name, builder, kw):
     assert np.array_equal(acc2.cpu().numpy(), ref2.acc)
 
 
+FULL_CHAIN = [
+    ("gate_up", synth.llama3_8b_gate_up, {}),
+    ("down_proj", synth.llama3_8b_down_proj, {}),
+]
+
+
+@pytest.mark.parametrize("name,builder,kw", FULL_CHAIN, ids=[c[0] for c in FULL_CHAIN])
+def test_rotated_linear_chain_full_size(S, name, builder, kw):
+    """The whole chain at the configs' own size (2048 tokens; gate_up
+    4096 -> 14336 with no online rotation, down_proj 14336 -> 4096 with R4 =
+    H28 (x) H512): GPU rotate+quant of the activations, GPU weight quant, GPU
+    GEMM.  On sampled rows and channels: the codes against the oracle's (the
+    +-1 tie bar), the accumulator exactly and y (fp16) against the oracle's
+    product of the GPU's own codes.  (y against the oracle chain is not a
+    usable bar on a sample: with gate_up's coarse asymmetric codes one allowed
+    tie flip moves a row of y by ~0.7 %.)"""
+    c = builder(**kw)
+    x = torch.from_numpy(c.x).cuda()
+    w = torch.from_numpy(c.w).cuda()
+    qa = S.rotate_quant_act(x, c.had, c.act_symmetric, c.clip)
+    qw = S.quant_weight(w, c.had)
+    y, acc = S.w4a4_gemm(qa, qw, want_acc=True)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(11)
+    ms = np.unique(np.concatenate([rng.integers(0, c.M, 24), [0, c.M - 1]]))
+    ns = np.unique(np.concatenate([rng.integers(0, c.N, 48), [0, c.N - 1]]))
+    ms_t = torch.as_tensor(ms, device="cuda")
+    ns_t = torch.as_tensor(ns, device="cuda")
+    got_a = pu.gpu_codes(qa.codes[ms_t].cpu().numpy(), c.act_symmetric)
+    got_w = pu.gpu_codes(qw.codes[ns_t].cpu().numpy(), True)
+    ra = oracle.rotate_quant_act(c.x[ms], c.had, 4, c.act_symmetric, c.clip)
+    rw = oracle.quant_weight(c.w[ns], c.had)
+    pu.assert_codes_close(got_a, ra.codes, name + " activation codes")
+    pu.assert_codes_close(got_w, rw.codes, name + " weight codes")
+    ref = oracle.w4a4_linear(
+        oracle.QuantAct(got_a, None, qa.scale[ms_t].cpu().numpy().astype(np.float64),
+                        None if qa.zero is None else qa.zero[ms_t].cpu().numpy().astype(np.float64), None),
+        oracle.QuantWeight(got_w, None, qw.scale[ns_t].cpu().numpy().astype(np.float64), got_w.sum(1), None))
+    assert np.array_equal(acc.cpu().numpy()[np.ix_(ms, ns)], ref.acc)
+    assert pu.rel_frob(y.cpu().numpy()[np.ix_(ms, ns)], ref.y) <= 2e-3
+
+
 def test_rotation_reduces_quantization_error(S):
     """Sec. 2 / Fig. 2 and Sec. 3.1 on the device: with R4 the per-token int4
     activation error on outlier-channel inputs drops sharply (Fig. 2(b)), and

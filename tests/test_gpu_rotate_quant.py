@@ -50,6 +50,7 @@ CASES = [
     ("l32_up_M128", synth.llama32_3b_up, {"M": 128}),
     ("l32_up_M8192", synth.llama32_3b_up, {"M": 8192}),
     ("l32_down_M1", synth.llama32_3b_down, {"M": 1}),
+    ("l32_down_M16", synth.llama32_3b_down, {"M": 16}),
     ("l32_down_M128", synth.llama32_3b_down, {"M": 128}),
     ("l32_down_M8192", synth.llama32_3b_down, {"M": 8192}),
 ]
