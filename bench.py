@@ -1061,7 +1061,7 @@ def relaunch(args_n):
 
 
 PROFILE_CASES = ("attention", "rope_kv", "fp8_gemm", "w4a8_gemm", "rq8_paley", "cayley", "paley", "gemm",
-                 "gemm_gate_up", "decode_gemm", "decode_gemm16", "rq_h8192")
+                 "gemm_gate_up", "decode_gemm", "decode_gemm16", "rq_h8192", "kv2048", "act_quant")
 
 
 def profile_case(name, reps):
@@ -1077,7 +1077,10 @@ def profile_case(name, reps):
     the W4A4 gate_up 2048 x 4096 -> 14336 (asymmetric activations);
     decode_gemm: 8 tokens through 4096 -> 14336 on the automatic route;
     decode_gemm16: 16 tokens through 3072 -> 8192 on the automatic route;
-    rq_h8192: the 4-bit R4 kernel with H8192 on 8192 x 8192 (asymmetric)."""
+    rq_h8192: the 4-bit R4 kernel with H8192 on 8192 x 8192 (asymmetric);
+    kv2048: R3 + KV4 on the step's 2048 tokens (32 / 8 heads, D 128);
+    act_quant: the step's gate_up activation quantizer (2048 x 4096, no
+    rotation, asymmetric)."""
     import numpy as np
     import torch
 
@@ -1138,6 +1141,14 @@ def profile_case(name, reps):
         qa = spinq.rotate_quant_act(torch.from_numpy(c.x).to(dev), c.had, c.act_symmetric)
         qw = spinq.quant_weight(torch.from_numpy(c.w).to(dev), c.had)
         fn = lambda: spinq.w4a4_gemm_splitk(qa, qw)
+    elif name == "kv2048":
+        kv = synth.kv_case(B=1, S=2048)
+        q, k, v = (torch.from_numpy(t).to(dev) for t in (kv.q, kv.k, kv.v))
+        fn = lambda: spinq.rotate_quant_kv(q, k, v)
+    elif name == "act_quant":
+        c = synth.llama3_8b_gate_up()
+        x = torch.from_numpy(c.x).to(dev)
+        fn = lambda: spinq.rotate_quant_act(x, None, False)
     elif name == "cayley":
         rng = np.random.default_rng(0)
         R = np.stack([np.linalg.qr(rng.standard_normal((128, 128)))[0] for _ in range(152)]).astype(np.float32)

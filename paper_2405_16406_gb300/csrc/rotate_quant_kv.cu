@@ -98,19 +98,21 @@ __global__ void __launch_bounds__(kWarps * 32) rotate_quant_kv_kernel(KVArgs a) 
       int64_t pos = valid ? (int64_t)a.positions[row / H] : 0;
       pos = pos < 0 ? 0 : (pos >= a.max_pos ? a.max_pos - 1 : pos);
       const float2* cs = reinterpret_cast<const float2*>(a.cos_sin) + pos * (D / 2);
-      const bool first = c < 2;
+      // the partner's value enters with sign -1 in the first half and +1 in
+      // the second: y = x cos + (-+x') sin, the sign flipped on its fp16 bits
+      const uint32_t nsign = c < 2 ? 0x80008000u : 0u;
 #pragma unroll
       for (int v = 0; v < V; ++v) {
         uint32_t w[4] = {in[v].x, in[v].y, in[v].z, in[v].w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          const uint32_t pw = __shfl_xor_sync(0xffffffffu, w[j], 2);
+          const uint32_t pw = __shfl_xor_sync(0xffffffffu, w[j], 2) ^ nsign;
           const int f = (8 * V * c + 8 * v + 2 * j) & (D / 2 - 1);
           const float4 t = valid ? __ldg(reinterpret_cast<const float4*>(cs + f)) : make_float4(1.f, 0.f, 1.f, 0.f);
           const float2 x = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
           const float2 o = __half22float2(*reinterpret_cast<const __half2*>(&pw));
-          const float y0 = first ? x.x * t.x - o.x * t.y : o.x * t.y + x.x * t.x;
-          const float y1 = first ? x.y * t.z - o.y * t.w : o.y * t.w + x.y * t.z;
+          const float y0 = __fadd_rn(__fmul_rn(x.x, t.x), __fmul_rn(o.x, t.y));
+          const float y1 = __fadd_rn(__fmul_rn(x.y, t.z), __fmul_rn(o.y, t.w));
           w[j] = pack_half2_bits(y0, y1);
         }
         in[v] = make_uint4(w[0], w[1], w[2], w[3]);
