@@ -900,7 +900,9 @@ def variant8_records(dev, hbm_peak, fp8_peak):
             out[f"f3_{variant}_{tag}_{Mr}x{Kr}x{Nr}"] = {
                 "rotate_quant": {"us": round(rq_us, 2), "bytes": rq_bytes,
                                  "frac_hbm": round(rq_bytes / rq_us / 1e3 / hbm_peak, 4),
-                                 "kernel": "rq8_rows_kernel (one CTA per row)"},
+                                 "kernel": ("rq8_rows_kernel (one CTA per row)" if case.had is None else
+                                            "rq_tc_kernel (tcgen05, E4M3 epilogue)" if variant == "fp8" else
+                                            "rq_paley_kernel (int8 planes epilogue)")},
                 "gemm": {"us": round(g_us, 2), "tops": round(ops / g_us / 1e6, 1),
                          "tensor_frac_e4m3": round(planes * ops / g_us / 1e6 / fp8_peak, 4),
                          "kernel": "fp8_gemm_kernel" + (" (two activation planes, K' = 2K)" if planes == 2 else "")},

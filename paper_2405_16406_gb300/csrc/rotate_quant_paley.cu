@@ -130,68 +130,6 @@ __device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
-__device__ __forceinline__ uint32_t e4m3x2_bits(float lo, float hi) {
-  uint16_t r;
-  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
-  return r;
-}
-
-// The 8-bit quantizers of rotate_quant_8bit.cu (unclipped forms) on a row
-// range: E4M3 codes x / alpha with alpha = max|x| / 448; int8 codes
-// c = rint(x / alpha) (symmetric, alpha = max|x| / 127) or rint((x - beta) /
-// alpha) - 128 (asymmetric, alpha = (max - min) / 255), stored as the planes
-// E4M3(16 floor(c / 16)) and E4M3(c mod 16).  rint is the 1.5 2^23 rounding
-// (to nearest even, as the other kernel's conversion), floor(c / 16) is
-// rint((c - 7.5) / 16), exact for integer c; every value is exact in E4M3.
-template <bool SYM>
-struct Quant8 {
-  float inv, off, alpha, beta;
-  __device__ __forceinline__ Quant8(const Range<SYM>& r, float clip, bool e4m3) {
-    off = 0.f;
-    beta = 0.f;
-    if (e4m3) {
-      const float m = clip * r.hi;
-      alpha = m * (1.f / 448.f);
-      inv = m > 0.f ? 448.f / m : 0.f;
-    } else if (SYM) {
-      const float m = clip * r.hi;
-      alpha = m / 127.f;
-      inv = m > 0.f ? 127.f / m : 0.f;
-    } else {
-      const float h2 = clip * r.hi, l2 = clip * r.lo;
-      alpha = (h2 - l2) / 255.f;
-      inv = h2 > l2 ? 255.f / (h2 - l2) : 0.f;
-      beta = l2;
-      off = -l2 * inv;
-    }
-  }
-  // the codes of 8 consecutive elements (4 pairs): E4M3 bytes in `hi`, or the
-  // two planes in `hi` (16 floor(c / 16)) and `lo` (c mod 16)
-  template <int F8>
-  __device__ __forceinline__ void codes8(const F2 (&v)[4], uint2& hi, uint2& lo) const {
-    uint32_t hb[4], lb[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      float x0, x1;
-      f2_split(v[q], x0, x1);
-      if (F8 == kFmtE4M3) {
-        hb[q] = e4m3x2_bits(fmaf(x0, inv, off), fmaf(x1, inv, off));
-        lb[q] = 0;
-      } else {
-        float c0 = (fmaf(x0, inv, off) + kRoundMagic) - kRoundMagic;
-        float c1 = (fmaf(x1, inv, off) + kRoundMagic) - kRoundMagic;
-        if (!SYM) c0 -= 128.f, c1 -= 128.f;
-        const float q0 = (fmaf(c0, 0.0625f, -0.46875f) + kRoundMagic) - kRoundMagic;
-        const float q1 = (fmaf(c1, 0.0625f, -0.46875f) + kRoundMagic) - kRoundMagic;
-        hb[q] = e4m3x2_bits(16.f * q0, 16.f * q1);
-        lb[q] = e4m3x2_bits(fmaf(-16.f, q0, c0), fmaf(-16.f, q1, c1));
-      }
-    }
-    hi = make_uint2(hb[0] | (hb[1] << 16), hb[2] | (hb[3] << 16));
-    lo = make_uint2(lb[0] | (lb[1] << 16), lb[2] | (lb[3] << 16));
-  }
-};
-
 // F8 = 0: 4-bit codes (Eq. 1, N = 4); F8 = kFmtInt8Planes / kFmtE4M3: the
 // 8-bit quantizers of the 8-bit linears (codes laid out as in
 // rotate_quant_8bit.cu), on the same rotation.
@@ -657,6 +595,10 @@ cudaError_t launch_rotate_quant_8bit_paley(const Rq8Args& a, cudaStream_t stream
   b.scale = a.scale;
   b.zero = a.zero;
   b.status = device_status_word();
+  {
+    const cudaError_t e = launch_rotate_quant_8bit_tc(b, a.format, stream, handled);
+    if (*handled || e != cudaSuccess) return e;
+  }
   if (a.format == kFmtE4M3) return launch8_sc<kFmtE4M3, true>(b, stream, handled);
   return a.symmetric ? launch8_sc<kFmtInt8Planes, true>(b, stream, handled)
                      : launch8_sc<kFmtInt8Planes, false>(b, stream, handled);

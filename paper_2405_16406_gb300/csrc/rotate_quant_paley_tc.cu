@@ -156,7 +156,13 @@ __device__ __forceinline__ bool tc_bar_or(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
-template <int F, int RPS, bool SYM, bool CLAMP>
+// F8 = 0: the 4-bit codes (Eq. 1); F8 = kFmtE4M3: the per-row FP8 quantizer
+// of the 8-bit linears (unclipped), codes laid out as in rotate_quant_8bit.cu
+// (the int8-planes epilogue is written for F8 = kFmtInt8Planes too, but it
+// is not instantiated: its two roundings and two conversions per element on
+// the quantizer groups made H_28 (x) H_512 slower here, 43.3 against 34.4 us
+// on the Paley kernel, while E4M3 went 26.0 -> 19.0 us).
+template <int F, int RPS, bool SYM, bool CLAMP, int F8 = 0>
 __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
     rq_tc_kernel(const __grid_constant__ CUtensorMap tmx, RotQuantArgs a) {
   using S = RqTc<F, RPS>;
@@ -405,6 +411,29 @@ __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
         rr.hi = SYM ? __int_as_float(set[2 * rr_]) : ord2f(set[2 * rr_]);
         if (!SYM) rr.lo = ord2f(set[2 * rr_ + 1]);
       }
+      if constexpr (F8 != 0) {
+        // 128 codes of elements 128 a .. 128 a + 127 of row r: one E4M3 byte
+        // each, or one byte in each of the two int8 planes (row stride 2K)
+        const Quant8<SYM> q8(rr, a.clip, F8 == kFmtE4M3);
+        if (live) {
+          uint8_t* base = a.codes + row * (F8 == kFmtE4M3 ? a.K : 2 * a.K) + (int64_t)(m % F) * 128;
+#pragma unroll
+          for (int g = 0; g < 16; g += 2) {
+            uint2 h0, l0, h1, l1;
+            const F2 v0[4] = {z[4 * g], z[4 * g + 1], z[4 * g + 2], z[4 * g + 3]};
+            const F2 v1[4] = {z[4 * g + 4], z[4 * g + 5], z[4 * g + 6], z[4 * g + 7]};
+            q8.template codes8<F8>(v0, h0, l0);
+            q8.template codes8<F8>(v1, h1, l1);
+            *reinterpret_cast<uint4*>(base + g * 8) = make_uint4(h0.x, h0.y, h1.x, h1.y);
+            if (F8 == kFmtInt8Planes) *reinterpret_cast<uint4*>(base + a.K + g * 8) = make_uint4(l0.x, l0.y, l1.x, l1.y);
+          }
+        }
+        if (live && m % F == 0) {
+          a.scale[row] = q8.alpha * a.norm;
+          if (!SYM) a.zero[row] = q8.beta * a.norm;
+        }
+        continue;
+      }
       const QParams<SYM> qp(rr, a.clip);
       if (live) {
         // codes of elements 128 a .. 128 a + 127 of row r: 64 contiguous bytes
@@ -440,7 +469,7 @@ __global__ void __launch_bounds__(RqTc<F, RPS>::THREADS, 1)
   if (warp == 1) tmem_dealloc(tmem, S::TMEM_COLS);
 }
 
-template <int F, int RPS, bool SYM, bool CLAMP>
+template <int F, int RPS, bool SYM, bool CLAMP, int F8 = 0>
 cudaError_t launch_tc(const RotQuantArgs& a, cudaStream_t stream) {
   using S = RqTc<F, RPS>;
   EncodeTiledFn enc = get_encode_fn();
@@ -457,7 +486,7 @@ cudaError_t launch_tc(const RotQuantArgs& a, cudaStream_t stream) {
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorNotSupported;
-  auto kern = rq_tc_kernel<F, RPS, SYM, CLAMP>;
+  auto kern = rq_tc_kernel<F, RPS, SYM, CLAMP, F8>;
   int per_sm = 0;
   cudaError_t e = prepare_launch_tmem(kern, S::THREADS, S::BYTES, S::TMEM_COLS, &per_sm);
   if (e != cudaSuccess) return e;
@@ -484,6 +513,18 @@ cudaError_t launch_tc_f(const RotQuantArgs& a, cudaStream_t stream, bool* handle
 }
 
 }  // namespace
+
+cudaError_t launch_rotate_quant_8bit_tc(const RotQuantArgs& a, int format, cudaStream_t stream, bool* handled) {
+  // the FP8 quantizer on the tcgen05 kernel for H_28 (x) H_512 (the 8-bit
+  // linears' down_proj): symmetric, unclipped, no random signs, at least one
+  // row per SM
+  *handled = false;
+  if (format != kFmtE4M3 || !a.symmetric) return cudaSuccess;
+  if (a.rows < device_sm_count() || a.signs || a.rowsum || a.clip < 1.0f) return cudaSuccess;
+  if (a.n_small != 28 || a.n_pow2 != 512 || a.K != 14336 || (a.ldx * 2) % 16 != 0) return cudaSuccess;
+  *handled = true;
+  return launch_tc<112, 1, true, false, kFmtE4M3>(a, stream);
+}
 
 cudaError_t set_wait_limit_rq_tc(uint64_t ns) { return cudaMemcpyToSymbol(g_tc_wait_ns, &ns, sizeof(ns)); }
 

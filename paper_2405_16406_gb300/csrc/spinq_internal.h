@@ -205,6 +205,10 @@ cudaError_t launch_rotate_quant_8bit(const Rq8Args& a, cudaStream_t stream);
 // The 8-bit quantizers (int8 planes, E4M3; unclipped) on a Paley rotation,
 // in the Paley rotate+quant kernel.  Sets *handled = false for other shapes.
 cudaError_t launch_rotate_quant_8bit_paley(const Rq8Args& a, cudaStream_t stream, bool* handled);
+// The FP8 quantizer (kFmtE4M3, symmetric, unclipped) on the tcgen05
+// rotate+quant kernel, for H_28 (x) H_512 with at least one row per SM
+// (rotate_quant_paley_tc.cu).  Sets *handled = false for other requests.
+cudaError_t launch_rotate_quant_8bit_tc(const RotQuantArgs& a, int format, cudaStream_t stream, bool* handled);
 
 struct Fp8GemmArgs {
   bool w4a8;              // false: FP8 x FP8; true: W4A8 (activation planes [M][2K])

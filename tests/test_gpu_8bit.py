@@ -78,6 +78,34 @@ def test_fp8_quantizer(name, had, K):
     assert_scale_close(out.scale.cpu().numpy(), ref.alpha, "alpha")
 
 
+@pytest.mark.parametrize("fmt,sym", [("e4m3", True), ("planes", True), ("planes", False)])
+def test_8bit_quantizers_on_the_tensor_core_rotation(fmt, sym):
+    """H28 (x) H512 with at least one row per SM: the FP8 quantizer runs on
+    the tcgen05 rotate+quant kernel, the int8 planes on the Paley kernel;
+    160 rows (more than the 152 SMs, not a multiple), every row against the
+    oracle."""
+    from paper_2405_16406_gb300 import spinq
+    rng = np.random.default_rng(160 + sym)
+    x = synth.activations(rng, 160, 14336, outlier_frac=0.01, factor=30.0)
+    x[7] = 0
+    xt = torch.from_numpy(x).cuda()
+    if fmt == "e4m3":
+        out = spinq.rotate_quant_act8(xt, (28, 512), spinq.SPINQ_FMT_E4M3, True)
+        torch.cuda.synchronize()
+        ref = oracle.rotate_quant_act_fp8(x, (28, 512))
+        _assert_e4m3_close(out.codes.cpu().numpy(), ref.codes, "fp8 tcgen05")
+    else:
+        out = spinq.rotate_quant_act8(xt, (28, 512), spinq.SPINQ_FMT_INT8_PLANES, sym)
+        torch.cuda.synchronize()
+        ref = oracle.rotate_quant_act(x, (28, 512), 8, sym, 1.0)
+        c = _planes_to_codes(out.codes, 14336)
+        assert_codes_close(c if sym else c + 128, ref.codes, "int8 tcgen05")
+        if not sym:
+            assert_zero_close(out.zero.cpu().numpy(), ref.beta, ref.alpha, "beta")
+    assert_scale_close(out.scale.cpu().numpy(), ref.alpha, "alpha")
+    assert spinq.spinq_device_status()[0] == spinq.SPINQ_OK
+
+
 def test_clipped_quantizers_saturate_like_the_oracle():
     from paper_2405_16406_gb300 import spinq
     rng = np.random.default_rng(5)
