@@ -20,7 +20,8 @@
 // block: the 7 stages of H_128 are butterflies inside the thread (no
 // shared-memory transpose), then the row range (over the row's lanes),
 // Eq. 1 and 64 contiguous bytes of codes per thread (the codes of elements
-// 128 a .. 128 a + 127 of row r).
+// 128 a .. 128 a + 127 of row r); or, for the 8-bit linears, the per-row FP8
+// quantizer and 128 bytes of E4M3 codes per thread.
 //
 // Warp roles (one CTA per SM, rows r0, r0 + G, ...):
 //  * warp 0: one thread copies each MMA's RPS rows into a ring of NSTG
@@ -32,9 +33,12 @@
 //    `free` barrier and the accumulator's `full` barrier;
 //  * NGRP groups of 4 warps (one per tensor-memory lane quadrant) take the
 //    accumulators in turn: read one (releasing it for the next MMA), the
-//    butterflies, the ranges (shared-memory atomics and a named barrier per
-//    group), Eq. 1 and the codes.
-// T is written once per CTA into shared memory (K-major, 128-byte swizzle).
+//    butterflies, the ranges (per-quadrant partials, or shared-memory
+//    atomics where rows share warps, and a named barrier per group), Eq. 1
+//    and the codes.
+// T is written once per CTA into shared memory (K-major, 128-byte swizzle),
+// from the Paley sign words staged in shared memory, after the copy thread
+// has issued the first pass over the ring.
 //
 // Every wait is bounded in time; a wait that gives up raises the CTA's abort
 // flag, the others see it at their next wait, the MMA thread drains its MMAs
